@@ -1,0 +1,306 @@
+"""CPU oracle for the LionMuon optimizer step (arXiv 2605.19811).
+
+TEST INFRASTRUCTURE ONLY.  This module is the slow, plain restatement of the
+paper's update that the CUDA library is checked against.  Only the test suite,
+``__graft_entry__.smoke()`` and the ``cpu_baseline`` / ``--impl reference`` legs
+of ``bench.py`` may import it.  It shares no code with the CUDA path and never
+imports the product package.
+
+Everything is numpy in float64 unless a function says otherwise.  Each function
+names the passage of the paper it restates:
+
+* Algorithm 1 ("LionMuon and SignMuon for a single 2D parameter"): the
+  interpolated direction G_hat from the *pre-update* buffer M_{t-1}, the
+  branch on ``t mod P``, the Muon step with NS_{K_NS}, the Lion sign step,
+  decoupled weight decay on both branches, and the momentum update on every
+  step.
+* Section 2 (Related works, "Spectral methods" / "Approximating the matrix
+  sign") and the Notations of Section 2.1: msign(X) = U V^T, computed by an
+  odd-polynomial Newton-Schulz iteration.
+* Table 5 (full experimental configuration): K_NS = 5 and the NS output
+  scaling 0.2 * sqrt(max(m, n)).
+* Section 3, Implementation notes: one persisted buffer per parameter.
+
+Readings taken where the paper is silent (each listed in the design doc):
+
+* NS coefficients: the paper gives none; the default is the widely used
+  quintic (a, b, c) = (3.4445, -4.7750, 2.0315), constant over iterations.
+* The NS input is pre-normalised as X / (||X||_F + eps), eps = 1e-7.
+* For a tall matrix (m > n) the iteration runs on X^T and the result is
+  transposed back; p(X X^T) X = X p(X^T X) makes this the same function.
+* The 0.2*sqrt(max(m,n)) factor multiplies the NS output inside the eta_M
+  bracket; the decay term is not scaled.
+* sign(0) = 0 and sign(NaN) = NaN.
+* 1-D parameters (vectors) take the Lion step on every step.
+* P = infinity is encoded as ``period = 0``.
+
+Parity status: the fp64 update rules are pinned by closed forms and
+invariants in tests/test_oracle_pins.py.  The end-to-end trajectory values are
+pinned only through those invariants: the paper prints no worked example of
+an update, so the exact trajectory of the paper's implementation (whose NS
+coefficients it does not state) is "parity unpinned".
+"""
+
+from __future__ import annotations
+
+import dataclasses
+import math
+from typing import List, Optional, Sequence, Tuple
+
+import numpy as np
+
+# Quintic Newton-Schulz coefficients used as the default reading (the paper
+# cites the Muon iteration but prints no coefficients).
+NS_QUINTIC = (3.4445, -4.7750, 2.0315)
+# Classic cubic Newton-Schulz iteration X <- 1.5 X - 0.5 X X^T X, which
+# converges to msign(X) for ||X||_2 < sqrt(3).
+NS_CUBIC = (1.5, -0.5, 0.0)
+
+
+@dataclasses.dataclass
+class Config:
+    """Hyper-parameters named in the Require line of Algorithm 1."""
+
+    beta1: float = 0.9
+    beta2: float = 0.99
+    eta_muon: float = 3e-3
+    eta_lion: float = 2e-5
+    weight_decay: float = 0.1
+    period: int = 2            # P >= 1; 0 encodes P = infinity (never Muon)
+    ns_steps: int = 5          # K_NS (Table 5)
+    ns_a: float = NS_QUINTIC[0]
+    ns_b: float = NS_QUINTIC[1]
+    ns_c: float = NS_QUINTIC[2]
+    ns_eps: float = 1e-7
+    shape_scale: float = 0.2   # NS scaling 0.2*sqrt(max(m,n)) (Table 5)
+
+
+# ---------------------------------------------------------------------------
+# Scalar building blocks
+# ---------------------------------------------------------------------------
+
+def sign(x: np.ndarray) -> np.ndarray:
+    """Element-wise sign, the l_inf LMO of Section 2.1 (up to the minus sign).
+
+    sign(+-0) = 0, sign(NaN) = NaN (numpy's definition, written out so the
+    choice is visible)."""
+    x = np.asarray(x)
+    out = np.where(x > 0, 1.0, np.where(x < 0, -1.0, 0.0)).astype(x.dtype)
+    return np.where(np.isnan(x), x, out)
+
+
+def is_muon_step(t: int, period: int) -> bool:
+    """Branch condition of Algorithm 1: Muon iff ``t mod P == 0``.
+
+    P = infinity (``period == 0``) never takes the Muon branch."""
+    if t < 0:
+        raise ValueError("t must be >= 0")
+    if period < 0:
+        raise ValueError("period must be >= 0 (0 encodes infinity)")
+    return period != 0 and t % period == 0
+
+
+def interpolated_direction(M_prev, G, beta1):
+    """G_hat_t = beta1 * M_{t-1} + (1 - beta1) * G_t (Algorithm 1, uses the
+    buffer *before* this step's momentum update)."""
+    return beta1 * M_prev + (1.0 - beta1) * G
+
+
+def momentum_update(M_prev, G, beta2):
+    """M_t = beta2 * M_{t-1} + (1 - beta2) * G_t (Algorithm 1, every step)."""
+    return beta2 * M_prev + (1.0 - beta2) * G
+
+
+# ---------------------------------------------------------------------------
+# Matrix sign
+# ---------------------------------------------------------------------------
+
+def ns_polynomial(G: np.ndarray, steps: int, a: float, b: float, c: float,
+                  eps: float = 1e-7) -> np.ndarray:
+    """NS_K(G): odd-polynomial Newton-Schulz approximation of msign(G).
+
+    Section 2 ("Spectral methods", "Approximating the matrix sign") names the
+    iteration; the polynomial form used is, per step,
+        A = X X^T,  B = b A + c A A,  X <- a X + B X,
+    which maps every singular value s of X to a s + b s^3 + c s^5.
+    The input is first divided by (||G||_F + eps).  A tall input (m > n) is
+    iterated in its transposed (wide) orientation and transposed back.
+    """
+    X = np.array(G, dtype=np.float64)
+    if X.ndim != 2:
+        raise ValueError("NS needs a 2-D matrix")
+    transposed = X.shape[0] > X.shape[1]
+    if transposed:
+        X = X.T.copy()
+    X = X / (np.linalg.norm(X) + eps)
+    for _ in range(steps):
+        A = X @ X.T
+        B = b * A + c * (A @ A)
+        X = a * X + B @ X
+    return X.T.copy() if transposed else X
+
+
+def msign_svd(G: np.ndarray) -> np.ndarray:
+    """Exact msign(G) = U V^T from the thin SVD G = U S V^T (Section 2,
+    "msign(X) = U V^T"; Section 2.1, LMO of the spectral norm).  Zero singular
+    values contribute nothing (the minimum-norm element of the subdifferential).
+    LAPACK's SVD is the library primitive."""
+    G = np.asarray(G, dtype=np.float64)
+    U, s, Vt = np.linalg.svd(G, full_matrices=False)
+    tol = s.max(initial=0.0) * max(G.shape) * np.finfo(np.float64).eps
+    keep = s > tol
+    return (U[:, keep] @ Vt[keep, :])
+
+
+def ns_scalar_map(x: np.ndarray, steps: int, a: float, b: float, c: float) -> np.ndarray:
+    """phi^K(x) with phi(x) = a x + b x^3 + c x^5: what NS does to each
+    normalised singular value."""
+    x = np.array(x, dtype=np.float64)
+    for _ in range(steps):
+        x = a * x + b * x ** 3 + c * x ** 5
+    return x
+
+
+# ---------------------------------------------------------------------------
+# The two update rules of Algorithm 1 (fp64)
+# ---------------------------------------------------------------------------
+
+def lion_update(W, G_hat, eta_lion, weight_decay):
+    """Lion branch of Algorithm 1: W <- W - eta_L (sign(G_hat) + lambda W)."""
+    return W - eta_lion * (sign(G_hat) + weight_decay * W)
+
+
+def muon_update(W, G_hat, cfg: Config):
+    """Muon branch of Algorithm 1 with Table 5's NS scaling:
+    W <- W - eta_M (0.2 sqrt(max(m,n)) NS_K(G_hat) + lambda W)."""
+    O = ns_polynomial(G_hat, cfg.ns_steps, cfg.ns_a, cfg.ns_b, cfg.ns_c, cfg.ns_eps)
+    scale = cfg.shape_scale * math.sqrt(max(W.shape))
+    return W - cfg.eta_muon * (scale * O + cfg.weight_decay * W)
+
+
+def is_matrix(shape: Sequence[int]) -> bool:
+    """A parameter is a hidden matrix (takes Muon steps) unless it is a vector
+    (one of its two dimensions is 1)."""
+    return len(shape) == 2 and shape[0] > 1 and shape[1] > 1
+
+
+def lionmuon_param_step(W, G, M_prev, t: int, cfg: Config):
+    """One iteration of Algorithm 1 for one parameter, fp64, exact.
+
+    Returns (W_{t+1}, M_t)."""
+    W = np.asarray(W, dtype=np.float64)
+    G = np.asarray(G, dtype=np.float64)
+    M_prev = np.asarray(M_prev, dtype=np.float64)
+    G_hat = interpolated_direction(M_prev, G, cfg.beta1)
+    if is_matrix(W.shape) and is_muon_step(t, cfg.period):
+        W_new = muon_update(W, G_hat, cfg)
+    else:
+        W_new = lion_update(W, G_hat, cfg.eta_lion, cfg.weight_decay)
+    M_new = momentum_update(M_prev, G, cfg.beta2)
+    return W_new, M_new
+
+
+# ---------------------------------------------------------------------------
+# Storage modelling (bf16 / fp32 rounding of the persisted state)
+# ---------------------------------------------------------------------------
+
+def bf16_round(x: np.ndarray) -> np.ndarray:
+    """Round to the nearest bfloat16 value, ties to even, returned as float32.
+
+    Written from the IEEE-754 binary32 layout: bfloat16 keeps the top 16 bits.
+    Adding 0x7FFF plus the lowest kept bit to the 32-bit pattern and
+    truncating rounds to nearest with ties to even; the carry into the
+    exponent handles overflow to infinity.  NaN stays NaN (quiet)."""
+    f = np.ascontiguousarray(np.asarray(x, dtype=np.float32))
+    u = f.view(np.uint32).astype(np.uint64)
+    lsb = (u >> 16) & 1
+    r = ((u + 0x7FFF + lsb) >> 16) << 16
+    out = (r & 0xFFFFFFFF).astype(np.uint32).view(np.float32)
+    return np.where(np.isnan(f), np.float32(np.nan), out).astype(np.float32)
+
+
+def round_to_storage(x: np.ndarray, dtype: str) -> np.ndarray:
+    """Round fp64 values to what a buffer of ``dtype`` ('bf16' or 'f32') holds,
+    returned as float64 for further fp64 arithmetic."""
+    if dtype == "f32":
+        return np.asarray(x, dtype=np.float32).astype(np.float64)
+    if dtype == "bf16":
+        return bf16_round(np.asarray(x, dtype=np.float64).astype(np.float32)).astype(np.float64)
+    raise ValueError(f"unknown storage dtype {dtype!r}")
+
+
+def lionmuon_step(params: List[np.ndarray], grads: List[np.ndarray],
+                  moms: List[np.ndarray], t: int, cfg: Config,
+                  param_dtypes: Optional[List[str]] = None):
+    """One LionMuon step over a list of parameters (Algorithm 1 applied to
+    each parameter; vectors take the Lion step every step).
+
+    With ``param_dtypes`` given, the new weights are rounded to their storage
+    dtype and the momentum to float32 (storage-modelled mode); otherwise the
+    state stays in fp64 (exact mode).  Returns (new_params, new_moms)."""
+    if not (len(params) == len(grads) == len(moms)):
+        raise ValueError("params, grads and moms must have equal length")
+    new_p, new_m = [], []
+    for i, (W, G, M) in enumerate(zip(params, grads, moms)):
+        if np.shape(W) != np.shape(G) or np.shape(W) != np.shape(M):
+            raise ValueError(f"shape mismatch at parameter {i}")
+        W1, M1 = lionmuon_param_step(W, G, M, t, cfg)
+        if param_dtypes is not None:
+            W1 = round_to_storage(W1, param_dtypes[i])
+            M1 = round_to_storage(M1, "f32")
+        new_p.append(W1)
+        new_m.append(M1)
+    return new_p, new_m
+
+
+# ---------------------------------------------------------------------------
+# Same-order float32 Lion step (bit-level reference)
+# ---------------------------------------------------------------------------
+
+def lion_constants_f32(beta1, beta2, eta_lion, weight_decay):
+    """The six float32 constants of the Lion step, each rounded once from
+    float64: (beta1, 1-beta1, beta2, 1-beta2, eta_L, lambda)."""
+    f = np.float32
+    return (f(beta1), f(1.0 - beta1), f(beta2), f(1.0 - beta2), f(eta_lion), f(weight_decay))
+
+
+def lion_step_f32(w: np.ndarray, g: np.ndarray, m: np.ndarray, beta1, beta2,
+                  eta_lion, weight_decay, w_dtype: str = "bf16"):
+    """Lion branch + momentum update of Algorithm 1 evaluated in float32 with a
+    fixed operation order, every product and sum rounded separately (no fused
+    multiply-add):
+
+        gh = b1*m + c1*g ;  u = sign(gh)
+        w  = w - eL*(u + lam*w)      (then bf16 round-to-nearest-even if bf16)
+        m  = b2*m + c2*g
+
+    ``w`` and ``g`` hold the stored values (bf16 values as float32), ``m`` is
+    float32.  numpy evaluates each float32 operation with one rounding, which
+    is what makes this a bit-level reference.  Returns (w_new, m_new) as
+    float32 arrays."""
+    b1, c1, b2, c2, eL, lam = lion_constants_f32(beta1, beta2, eta_lion, weight_decay)
+    w = np.asarray(w, dtype=np.float32)
+    g = np.asarray(g, dtype=np.float32)
+    m = np.asarray(m, dtype=np.float32)
+    gh = (b1 * m) + (c1 * g)
+    u = sign(gh).astype(np.float32)
+    w_new = w - eL * (u + lam * w)
+    m_new = (b2 * m) + (c2 * g)
+    if w_dtype == "bf16":
+        w_new = bf16_round(w_new)
+    elif w_dtype != "f32":
+        raise ValueError(f"unknown w dtype {w_dtype!r}")
+    return w_new.astype(np.float32), m_new.astype(np.float32)
+
+
+# ---------------------------------------------------------------------------
+# Cost model (for reporting; FLOP counts of the method's contractions)
+# ---------------------------------------------------------------------------
+
+def ns_flops(m: int, n: int, steps: int, symmetric: bool = True) -> float:
+    """FLOPs of NS_K on an m x n matrix, s = min, l = max.  Per iteration:
+    X X^T (s^2 l with the symmetric half, 2 s^2 l dense), A A (s^3 / 2 s^3),
+    B X (2 s^2 l)."""
+    s, l = min(m, n), max(m, n)
+    per = (3 * s * s * l + s ** 3) if symmetric else (4 * s * s * l + 2 * s ** 3)
+    return float(steps) * per
