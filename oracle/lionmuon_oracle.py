@@ -184,9 +184,13 @@ def is_matrix(shape: Sequence[int]) -> bool:
     return len(shape) == 2 and shape[0] > 1 and shape[1] > 1
 
 
-def lionmuon_param_step(W, G, M_prev, t: int, cfg: Config):
-    """One iteration of Algorithm 1 for one parameter, fp64, exact.
+def lionmuon_param_step(W, G, M_prev, t: int, cfg: Config, sign_in_f32: bool = False):
+    """One iteration of Algorithm 1 for one parameter, fp64.
 
+    With ``sign_in_f32`` the Lion branch decides sign(G_hat) on the float32
+    value of G_hat formed as fl(fl(b1*M) + fl(c1*G)) with float32 constants
+    (the order the CUDA library uses), so both sides take the same integer
+    decision near ties; the update itself stays fp64.
     Returns (W_{t+1}, M_t)."""
     W = np.asarray(W, dtype=np.float64)
     G = np.asarray(G, dtype=np.float64)
@@ -195,7 +199,11 @@ def lionmuon_param_step(W, G, M_prev, t: int, cfg: Config):
     if is_matrix(W.shape) and is_muon_step(t, cfg.period):
         W_new = muon_update(W, G_hat, cfg)
     else:
-        W_new = lion_update(W, G_hat, cfg.eta_lion, cfg.weight_decay)
+        direction = G_hat
+        if sign_in_f32:
+            b1, c1 = np.float32(cfg.beta1), np.float32(1.0 - cfg.beta1)
+            direction = (b1 * M_prev.astype(np.float32)) + (c1 * G.astype(np.float32))
+        W_new = W - cfg.eta_lion * (sign(direction).astype(np.float64) + cfg.weight_decay * W)
     M_new = momentum_update(M_prev, G, cfg.beta2)
     return W_new, M_new
 
@@ -236,15 +244,16 @@ def lionmuon_step(params: List[np.ndarray], grads: List[np.ndarray],
     each parameter; vectors take the Lion step every step).
 
     With ``param_dtypes`` given, the new weights are rounded to their storage
-    dtype and the momentum to float32 (storage-modelled mode); otherwise the
-    state stays in fp64 (exact mode).  Returns (new_params, new_moms)."""
+    dtype, the momentum to float32, and Lion signs are decided on the float32
+    G_hat (storage-modelled mode); otherwise the state stays in fp64 (exact
+    mode).  Returns (new_params, new_moms)."""
     if not (len(params) == len(grads) == len(moms)):
         raise ValueError("params, grads and moms must have equal length")
     new_p, new_m = [], []
     for i, (W, G, M) in enumerate(zip(params, grads, moms)):
         if np.shape(W) != np.shape(G) or np.shape(W) != np.shape(M):
             raise ValueError(f"shape mismatch at parameter {i}")
-        W1, M1 = lionmuon_param_step(W, G, M, t, cfg)
+        W1, M1 = lionmuon_param_step(W, G, M, t, cfg, sign_in_f32=param_dtypes is not None)
         if param_dtypes is not None:
             W1 = round_to_storage(W1, param_dtypes[i])
             M1 = round_to_storage(M1, "f32")

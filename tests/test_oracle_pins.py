@@ -455,3 +455,26 @@ def test_lion_f32_order_is_separately_rounded():
 def test_ns_flop_count():
     assert O.ns_flops(128, 256, 1, symmetric=False) == 4 * 128 * 128 * 256 + 2 * 128 ** 3
     assert O.ns_flops(256, 128, 5, symmetric=True) == 5 * (3 * 128 * 128 * 256 + 128 ** 3)
+
+
+def test_storage_mode_sign_decision_matches_f32_lion():
+    """Storage-modelled mode decides Lion signs on the float32 G_hat: its
+    weights then agree with the same-order float32 Lion step to within the
+    final bf16 rounding (one bf16 ulp), including near-tie entries."""
+    r = np.random.default_rng(21)
+    n = 20000
+    w = O.bf16_round(r.standard_normal(n).astype(np.float32) * np.float32(0.02))
+    g = O.bf16_round(r.standard_normal(n).astype(np.float32) * np.float32(1e-3))
+    m = (r.standard_normal(n) * 1e-3).astype(np.float32)
+    # near ties: G_hat almost exactly 0 in float64 but not in float32
+    g[:100] = O.bf16_round(np.float32(-9.0) * m[:100])
+    cfg = O.Config(beta1=0.9, beta2=0.99, eta_lion=1e-2, weight_decay=0.1, period=0)
+    P, M = O.lionmuon_step([w.astype(np.float64)], [g.astype(np.float64)], [m.astype(np.float64)], 1,
+                           cfg, param_dtypes=["bf16"])
+    w32, m32 = O.lion_step_f32(w, g, m, 0.9, 0.99, 1e-2, 0.1, w_dtype="bf16")
+    ulp = np.spacing(np.abs(w32)) * 65536.0
+    assert np.all(np.abs(P[0] - w32) <= ulp)
+    # fp64 EMA rounded once vs the float32 same-order EMA: within two ulps of
+    # the larger addend
+    mag = np.maximum(np.abs(m), np.abs(g)).astype(np.float32)
+    assert np.all(np.abs(M[0] - m32.astype(np.float64)) <= 2 * np.spacing(mag).astype(np.float64))
