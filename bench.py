@@ -1,0 +1,443 @@
+#!/usr/bin/env python
+"""Benchmark of the LionMuon optimizer step on one GB300 per rank.
+
+A step is one lm_step over the whole parameter set (a Muon step when
+t mod P == 0, otherwise a Lion step).  The headline value is the
+period-averaged optimizer time per step (P = 2 by default) on the 720M-shaped
+GPT parameter set, inputs resident in HBM, timed with CUDA events over whole
+periods.  Prints one JSON line (rank 0).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Under torchrun every rank runs an independent replica (the optimizer step
+has no exchange between parameter sets: weak scaling); the time is the max
+over ranks.  ``--impl reference`` times the CPU oracle on bounded samples of
+the same workload instead (rank 0 only).
+"""
+
+from __future__ import annotations
+
+import argparse
+import ctypes
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = ("period-averaged optimizer ms/step (P=2) per param set; Lion HBM GB/s; "
+          "NS tensor-pipe %")
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=8)
+    ap.add_argument("--warmup", type=int, default=4)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--set", default="gpt_720m")
+    ap.add_argument("--period", type=int, default=2)
+    ap.add_argument("--precision", choices=["bf16", "f32"], default="bf16")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    return ap.parse_args()
+
+
+# ---------------------------------------------------------------------------
+# workload description (shared by both arms)
+# ---------------------------------------------------------------------------
+
+def workload(name):
+    from paper_2605_19811_gb300 import synth
+    ps = synth.PARAM_SETS[name]
+    shapes = [tuple(s) for s in ps.shapes]
+    mats = [s for s in shapes if len(s) == 2 and s[0] > 1 and s[1] > 1]
+    numel = sum(int(math.prod(s)) for s in shapes)
+    mat_elems = sum(a * b for a, b in mats)
+    return ps, shapes, mats, numel, mat_elems
+
+
+def ns_flops_sym(mats, steps=5):
+    """Algorithmic FLOPs of NS_K per Muon step, symmetric products counted
+    once: per iteration 3 s^2 l + s^3 per matrix (s = min, l = max)."""
+    tot = 0.0
+    for a, b in mats:
+        s, l = min(a, b), max(a, b)
+        tot += steps * (3.0 * s * s * l + 1.0 * s ** 3)
+    return tot
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured (MEASURED_PEAKS.json)"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+def kernel_traffic(kernel: str):
+    """DRAM bytes per launch of ``kernel`` from the committed ncu summary, if
+    the kernel source still matches the hash recorded with it."""
+    path = os.path.join(ROOT, "profiles", "ncu_traffic.txt")
+    if not os.path.exists(path):
+        return None
+    for line in open(path):
+        parts = line.split()
+        if len(parts) >= 4 and parts[0] == kernel and not line.startswith("#"):
+            src = os.path.join(ROOT, "paper_2605_19811_gb300", "csrc", parts[1])
+            if not os.path.exists(src):
+                return None
+            h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+            if h != parts[2]:
+                return None
+            return float(parts[3])
+    return None
+
+
+class ClockSampler:
+    """nvidia-smi clock/throttle samples while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200", "-f", self.path], stdout=subprocess.DEVNULL, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        rows = []
+        try:
+            for line in open(self.path):
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+            os.unlink(self.path)
+        except Exception:
+            return None
+        if not rows:
+            return None
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return float("nan")
+        sm = [num(r[1]) for r in rows]
+        mx = [num(r[2]) for r in rows]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if "Active" in r[5 + i] and "Not" not in r[5 + i]})
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": reasons,
+                "samples": len(rows), "power_w_max": max(num(r[3]) for r in rows)}
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (cpu_baseline leg and --impl reference)
+# ---------------------------------------------------------------------------
+
+def oracle_sample(name, period, budget_s=12.0):
+    """Time the oracle on a bounded sample of the workload and scale it to the
+    period-averaged ms/step of the whole set.  Returns (ms_per_step, info)."""
+    import numpy as np
+    import oracle as O
+    ps, shapes, mats, numel, mat_elems = workload(name)
+    cfg = O.Config(period=period)
+    rng = np.random.default_rng(0)
+    # Lion branch on a vector sample
+    n = 4_000_000
+    W = rng.standard_normal(n) * 0.02
+    G = rng.standard_normal(n) * 1e-3
+    M = rng.standard_normal(n) * 1e-3
+    t0 = time.perf_counter()
+    O.lionmuon_param_step(W, G, M, 1, cfg)
+    lion_per_elem = (time.perf_counter() - t0) / n
+    # Muon branch on one matrix of each of the two smallest distinct shapes
+    shapes_u = sorted({(min(a, b), max(a, b)) for a, b in mats}, key=lambda x: x[0] * x[0] * x[1])
+    samples = []
+    spent = time.perf_counter() - t0
+    for s, l in shapes_u[:2]:
+        Wm = rng.standard_normal((s, l)) * 0.02
+        Gm = rng.standard_normal((s, l)) * 1e-3
+        Mm = np.zeros((s, l))
+        t1 = time.perf_counter()
+        O.lionmuon_param_step(Wm, Gm, Mm, 0, cfg)
+        dt = time.perf_counter() - t1
+        samples.append((s, l, dt))
+        spent += dt
+        if spent > budget_s:
+            break
+    # t(matrix) = alpha * NS flops + beta * elements, fitted on the samples
+    if len(samples) >= 2:
+        A = np.array([[5 * (4.0 * s * s * l + 2.0 * s ** 3), s * l] for s, l, _ in samples])
+        y = np.array([dt for _, _, dt in samples])
+        alpha, beta = np.linalg.lstsq(A, y, rcond=None)[0]
+        alpha, beta = max(alpha, 0.0), max(beta, 0.0)
+    else:
+        s, l, dt = samples[0]
+        alpha, beta = dt / (5 * (4.0 * s * s * l + 2.0 * s ** 3)), 0.0
+    t_muon = sum(alpha * 5 * (4.0 * min(a, b) ** 2 * max(a, b) + 2.0 * min(a, b) ** 3) + beta * a * b
+                 for a, b in mats) + lion_per_elem * (numel - mat_elems)
+    t_lion = lion_per_elem * numel
+    per_step = (t_muon + (period - 1) * t_lion) / period if period > 0 else t_lion
+    info = {"lion_sample_elems": n, "muon_samples": [f"{s}x{l}" for s, l, _ in samples],
+            "extrapolated": True}
+    return per_step * 1e3, info
+
+
+def cpu_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+# ---------------------------------------------------------------------------
+# the two arms
+# ---------------------------------------------------------------------------
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def run_reference(args):
+    rank, world, local = dist_env()
+    if rank != 0:
+        return 0
+    ps, shapes, mats, numel, mat_elems = workload(args.set)
+    vals = []
+    info = None
+    for i in range(args.warmup + args.steps):
+        v, info = oracle_sample(args.set, args.period, budget_s=6.0)
+        if i >= args.warmup:
+            vals.append(v)
+    value = statistics.median(vals)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "ms/step",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": value, "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f64", "data": "synthetic",
+        "config": {"workload": args.set, "params": numel, "matrices": len(mats), "period": args.period,
+                   "ns_steps": 5},
+        "cpu_baseline": {"value": value, "unit": "ms/step", "cores": cpu_cores(), "kind": "oracle",
+                         "sample": ("each step times the fp64 oracle on a 4M-element Lion sample and "
+                                    f"full Muon steps of {info['muon_samples']}, scaled to the whole set "
+                                    "by elements and NS FLOPs (extrapolated)")},
+        "e2e": {"value": value, "unit": "ms/step", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+    from paper_2605_19811_gb300 import build as B
+    from paper_2605_19811_gb300 import lionmuon as L
+    from paper_2605_19811_gb300 import synth
+
+    rank, world, local = dist_env()
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if not os.path.exists(B.library_path()):
+        B.build()
+    L.load_library()
+
+    ps, shapes, mats, numel, mat_elems = workload(args.set)
+    P = args.period
+    # Parameters and gradients live in two flat device buffers (views per
+    # tensor, 256-byte aligned) so that the end-to-end leg moves each with one
+    # copy.
+    elt = 2
+    offs, cur = [], 0
+    for s in shapes:
+        offs.append(cur)
+        cur += (int(math.prod(s)) * elt + 255) // 256 * 256
+    flat_bytes = cur
+    wflat = torch.empty(flat_bytes // 2, dtype=torch.bfloat16, device=dev)
+    gflat = torch.empty(flat_bytes // 2, dtype=torch.bfloat16, device=dev)
+    def views(flat):
+        return [flat[o // 2: o // 2 + int(math.prod(s))].view(s) for o, s in zip(offs, shapes)]
+    params, grads = views(wflat), views(gflat)
+    for p, w in zip(params, synth.device_weights_torch(shapes, seed=1 + rank, device=dev, dtype=torch.bfloat16)):
+        p.copy_(w)
+    for g, x in zip(grads, synth.device_grads_torch(shapes, ps.grad_kind, seed=100 + rank, device=dev,
+                                                     dtype=torch.bfloat16)):
+        g.copy_(x)
+    torch.cuda.synchronize()
+
+    prec = L.LM_BF16 if args.precision == "bf16" else L.LM_F32
+    opt = L.LionMuon(params, period=P, ns_precision=prec)
+    n = len(params)
+    gdesc = (L.LmTensor * n)(*[L.tensor_desc(g) for g in grads])
+    stream = torch.cuda.current_stream()
+    sh = ctypes.c_void_p(stream.cuda_stream)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    t = 0
+    for _ in range(args.warmup):
+        opt.step_descs(gdesc, n, t, sh)
+        t += 1
+    base = ((t + P - 1) // P) * P if P > 0 else t
+    torch.cuda.synchronize()
+    barrier()
+
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    launches0 = L.kernel_launch_count()
+    opt.profile(True)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    barrier()
+    ev0.record(stream)
+    for i in range(args.steps):
+        opt.step_descs(gdesc, n, base + i, sh)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    launches = L.kernel_launch_count() - launches0
+    prof = opt.profile_read()
+    opt.profile(False)
+    ms_total = ev0.elapsed_time(ev1)
+    if world > 1:
+        tt = torch.tensor([ms_total], device=dev, dtype=torch.float64)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms_total = float(tt.item())
+    ms_per_step = ms_total / args.steps
+    value = ms_per_step / world
+
+    # ---- end to end through the public API with host buffers ----
+    e2e = None
+    if not args.no_e2e:
+        g_host = torch.empty(flat_bytes // 2, dtype=torch.bfloat16, pin_memory=True)
+        w_host = torch.empty(flat_bytes // 2, dtype=torch.bfloat16, pin_memory=True)
+        g_host.copy_(gflat)
+        torch.cuda.synchronize()
+        barrier()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(args.steps):
+            gflat.copy_(g_host, non_blocking=True)
+            opt.step_descs(gdesc, n, base + args.steps + i, sh)
+            w_host.copy_(wflat, non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        e_ms = e0.elapsed_time(e1)
+        if world > 1:
+            tt = torch.tensor([e_ms], device=dev, dtype=torch.float64)
+            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+            e_ms = float(tt.item())
+        e2e = {"value": e_ms / args.steps / world, "unit": "ms/step", "h2d_bytes_per_step": flat_bytes,
+               "d2h_bytes_per_step": flat_bytes,
+               "what": "pinned-host gradients copied in, lm_step, updated parameters copied out, per step"}
+    clk = clocks.stop()
+    flags = opt.status()
+
+    # ---- roofline of the dominant kernel family ----
+    peaks, peak_src = load_peaks()
+    n_muon = sum(1 for i in range(args.steps) if P > 0 and (base + i) % P == 0)
+    n_lion = args.steps - n_muon
+    ns_ms, ns_launches = prof["ns_gemm"]
+    lion_ms, lion_launches = prof["lion"]
+    fl = ns_flops_sym(mats) * n_muon
+    roof = None
+    if ns_ms > 0 and n_muon > 0:
+        achieved = fl / (ns_ms / 1e3) / 1e12
+        pk = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+        traffic = kernel_traffic("ns_tc_kernel")
+        roof = {"bound": "tensor", "achieved": achieved, "peak": pk, "unit": "TFLOP/s",
+                "frac": achieved / pk, "traffic": traffic, "kernel": "ns_tc_kernel",
+                "per_launch_ms": ns_ms / max(ns_launches, 1),
+                "per_launch_tflop": fl / max(ns_launches, 1) / 1e12,
+                "peak_kind": f"bf16 sustained, {peak_src}",
+                "flops": "symmetric count 3 s^2 l + s^3 per matrix per NS iteration"}
+    lion_bytes = 14.0 * numel if args.precision else 14.0 * numel
+    lion_roof = None
+    if lion_ms > 0:
+        # Lion-step launches over all params: 14 B/param (bf16 W,G r/w W, fp32 M r/w)
+        lion_full_ms = lion_ms - 0.0
+        bytes_moved = 14.0 * numel * n_lion + 14.0 * (numel - mat_elems) * n_muon
+        gbs = bytes_moved / (lion_full_ms / 1e3) / 1e9
+        pk = peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
+        lion_roof = {"bound": "hbm", "achieved": gbs, "peak": pk, "unit": "GB/s", "frac": gbs / pk,
+                     "traffic": kernel_traffic("lion_kernel"), "kernel": "lion_kernel",
+                     "per_launch_ms": lion_ms / max(lion_launches, 1),
+                     "frac_of_8tbs": gbs / 8000.0, "peak_kind": f"HBM copy, {peak_src}"}
+    fam_ms = {k: v[0] / args.steps for k, v in prof.items()}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        v, info = oracle_sample(args.set, P, budget_s=15.0)
+        cpu = {"value": v, "unit": "ms/step", "cores": cpu_cores(), "kind": "oracle",
+               "sample": ("fp64 oracle on a 4M-element Lion sample and full Muon steps of "
+                          f"{info['muon_samples']}, scaled to the whole set by elements and NS FLOPs "
+                          "(extrapolated)")}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "ms/step", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
+            "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16" if args.precision == "bf16" else "f32", "data": "synthetic",
+            "config": {"workload": args.set, "params": numel, "matrices": len(mats),
+                       "period": P, "ns_steps": 5, "ns_precision": args.precision,
+                       "grads": f"{ps.grad_kind}, drawn on device, same gradients every step",
+                       "l2": "inputs larger than L2 (14 B/param x %.0f M params streamed per Lion step)" % (numel / 1e6),
+                       "timed_steps": f"t = {base} .. {base + args.steps - 1} (whole periods from a Muon step)"},
+            "roofline": roof, "roofline_lion": lion_roof,
+            "kernel_ms_per_step": fam_ms,
+            "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches, "clocks": clk,
+            "device_flags": flags,
+        }
+        print(json.dumps(line), flush=True)
+    opt.close()
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,200 @@
+/*
+ * lionmuon.h -- C ABI of the GB300 (sm_103a) LionMuon optimizer-step library.
+ *
+ * LionMuon (arXiv 2605.19811, Algorithm 1) keeps one momentum buffer M per
+ * parameter.  At step t it forms the interpolated direction
+ *     G_hat = beta1 * M_{t-1} + (1 - beta1) * G_t
+ * and, when t mod P == 0, takes the Muon step
+ *     W <- W - eta_M * (0.2 sqrt(max(m,n)) * NS_K(G_hat) + lambda * W)
+ * (Table 5 gives K_NS = 5 and the 0.2 sqrt(max(m,n)) scaling), otherwise the
+ * Lion step
+ *     W <- W - eta_L * (sign(G_hat) + lambda * W);
+ * every step then updates M_t = beta2 * M_{t-1} + (1 - beta2) * G_t.
+ * Vectors (rows == 1 or cols == 1) take the Lion step on every step.
+ * NS_K is the odd-polynomial Newton-Schulz approximation of msign(X) = U V^T
+ * (Section 2): X <- X / (||X||_F + eps), then K times
+ *     A = X X^T ;  B = b A + c A A ;  X <- a X + B X
+ * run on the wide orientation (X^T for a tall matrix).
+ *
+ * Conventions for every call:
+ *   - Device pointers are CUDA device memory of the current device; host
+ *     pointers are ordinary host memory.  Tensors are dense, row-major,
+ *     contiguous and 16-byte aligned (LM_ERR_ALIGN otherwise).
+ *   - Calls return an lm_status; nothing unwinds across the ABI.  Arguments
+ *     are validated before any work is enqueued: on an error return nothing
+ *     was enqueued and no state changed.  An asynchronous CUDA error surfaces
+ *     as LM_ERR_CUDA from a later call.  lm_last_error() gives a one-line
+ *     description of the most recent error on the calling thread.
+ *   - Work is enqueued on the caller's stream (a cudaStream_t passed as
+ *     void*, NULL = legacy default stream).  lm_step never synchronises and
+ *     never copies device to host.  One state is driven by one stream at a
+ *     time.
+ */
+#ifndef LIONMUON_H
+#define LIONMUON_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  LM_OK = 0,
+  LM_ERR_INVALID_ARG = 1, /* bad count, shape, hyper-parameter or NULL pointer */
+  LM_ERR_DTYPE = 2,       /* unsupported dtype or grads/params dtype mismatch */
+  LM_ERR_ALIGN = 3,       /* a data pointer is not 16-byte aligned */
+  LM_ERR_OOM = 4,         /* device allocation failed */
+  LM_ERR_CUDA = 5,        /* a CUDA runtime/driver call failed */
+  LM_ERR_UNSUPPORTED = 6, /* no sm_103a device, or a size beyond a stated limit */
+  LM_ERR_TIMEOUT = 7      /* a bounded device-side wait gave up */
+} lm_status;
+
+typedef enum { LM_F32 = 0, LM_BF16 = 1 } lm_dtype;
+
+/* A dense row-major tensor.  rows == 1 or cols == 1 means a vector.
+ * rows * cols may be 0 (an empty parameter is accepted and skipped). */
+typedef struct {
+  void* data;
+  int64_t rows;
+  int64_t cols;
+  lm_dtype dtype;
+} lm_tensor;
+
+/* Device status flags read by lm_get_status. */
+#define LM_FLAG_NONFINITE 0x1u /* a matrix direction had a non-finite Frobenius norm */
+#define LM_FLAG_TIMEOUT 0x2u   /* a bounded device wait gave up */
+
+/* Hyper-parameters: the Require line of Algorithm 1 plus the NS reading.
+ * beta1, beta2 in [0, 1); eta_* >= 0; weight_decay >= 0;
+ * period >= 1, or 0 for P = infinity (never Muon);
+ * ns_steps in [0, 64]; ns_eps >= 0; shape_scale >= 0;
+ * ns_precision LM_BF16 (tensor-core bf16 GEMMs, fp32 accumulate) or LM_F32
+ * (fp32 CUDA-core GEMMs). */
+typedef struct {
+  double beta1, beta2;
+  double eta_muon, eta_lion;
+  double weight_decay;
+  int64_t period;
+  int ns_steps;
+  double ns_a, ns_b, ns_c;
+  double ns_eps;
+  double shape_scale;
+  int ns_precision;
+} lm_config;
+
+typedef struct lm_state lm_state; /* opaque */
+
+/* Fill *cfg with the paper's defaults: beta (0.9, 0.99) (Table 5, Lion),
+ * (eta_M, eta_L) = (3e-3, 2e-5) (Appendix E, LionMuon P=2), lambda = 0.1
+ * (Table 5), P = 2, K_NS = 5 (Table 5), quintic NS coefficients
+ * (3.4445, -4.7750, 2.0315) with eps 1e-7 (the paper gives none; this is the
+ * stated reading), shape_scale 0.2 (Table 5), ns_precision LM_BF16. */
+void lm_config_default(lm_config* cfg);
+
+/* Create an optimizer state over n parameter tensors (Algorithm 1, Require:
+ * W_0 given, M_{-1} = 0).  params[i].data is caller-owned device memory that
+ * the state borrows for its lifetime and updates in place; dtype LM_BF16 or
+ * LM_F32.  The state allocates and zeroes one fp32 momentum buffer per
+ * parameter plus the Newton-Schulz workspace, and records the shapes.
+ * Errors: LM_ERR_INVALID_ARG (n < 1, NULL, bad cfg), LM_ERR_DTYPE,
+ * LM_ERR_ALIGN, LM_ERR_OOM, LM_ERR_CUDA, LM_ERR_UNSUPPORTED (device is not
+ * sm_103). */
+lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg,
+                    void* cuda_stream, lm_state** out);
+
+/* One LionMuon step t >= 0 (Algorithm 1 body).  grads[i] must have the shape
+ * and dtype of params[i]; they are read-only device memory borrowed until the
+ * enqueued work completes.  Muon iff period != 0 and t % period == 0.
+ * Errors: LM_ERR_INVALID_ARG (n mismatch, t < 0, shape mismatch, NULL),
+ * LM_ERR_DTYPE, LM_ERR_ALIGN, LM_ERR_CUDA. */
+lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t,
+                  void* cuda_stream);
+
+/* Change the two learning rates (a caller-driven schedule); takes effect for
+ * the next lm_step.  Errors: LM_ERR_INVALID_ARG (NULL, negative, non-finite). */
+lm_status lm_set_lr(lm_state* s, double eta_muon, double eta_lion);
+
+/* Newton-Schulz approximation of msign (Section 2): out = NS_steps(in) with
+ * coefficients (a, b, c), normalisation X / (||X||_F + eps), iterated on the
+ * wide orientation, with no 0.2 sqrt(max(m,n)) scaling.  in and out are
+ * device tensors of equal shape (rows, cols >= 2 each), dtype LM_BF16 or
+ * LM_F32 (may differ).  precision LM_BF16 uses the tensor-core path, LM_F32
+ * the fp32 CUDA-core path.  Allocates its workspace with stream-ordered
+ * allocation on cuda_stream and frees it the same way.
+ * Errors: LM_ERR_INVALID_ARG, LM_ERR_DTYPE, LM_ERR_ALIGN, LM_ERR_OOM,
+ * LM_ERR_CUDA. */
+lm_status lm_msign_ns(const lm_tensor* in, lm_tensor* out, int steps, double a,
+                      double b, double c, double eps, int precision,
+                      void* cuda_stream);
+
+/* A read-only view of parameter i's momentum buffer (fp32, the shape of
+ * params[i], device memory owned by the state).  For checkpointing and tests.
+ * Errors: LM_ERR_INVALID_ARG (NULL, i out of range). */
+lm_status lm_get_momentum(const lm_state* s, int i, lm_tensor* view);
+
+/* Overwrite parameter i's momentum from src (device, fp32, same shape),
+ * enqueued on cuda_stream (resume from a checkpoint: restore M and pass the
+ * same t).  Errors: LM_ERR_INVALID_ARG, LM_ERR_DTYPE, LM_ERR_ALIGN,
+ * LM_ERR_CUDA. */
+lm_status lm_set_momentum(lm_state* s, int i, const lm_tensor* src,
+                          void* cuda_stream);
+
+/* Synchronise the state's last stream, then return and clear the device
+ * status flags (LM_FLAG_*).  Errors: LM_ERR_INVALID_ARG, LM_ERR_CUDA. */
+lm_status lm_get_status(lm_state* s, uint32_t* device_flags);
+
+/* Bytes of persisted optimizer state: exactly 4 * sum |W_i| (one fp32
+ * momentum buffer per parameter, Section 3 Implementation notes).  Returns 0
+ * for NULL. */
+size_t lm_state_bytes(const lm_state* s);
+
+/* Bytes of transient device workspace the state holds (Newton-Schulz
+ * buffers, tables).  Returns 0 for NULL. */
+size_t lm_workspace_bytes(const lm_state* s);
+
+/* Synchronise the state's last stream and free everything it owns.  NULL is
+ * a no-op. */
+void lm_destroy(lm_state* s);
+
+/* Static text for a status code. */
+const char* lm_status_string(lm_status st);
+
+/* Description of the most recent error returned on the calling thread
+ * (static storage of the library; "" if none). */
+const char* lm_last_error(void);
+
+/* Number of CUDA kernels this library has launched in this process (a
+ * monotonically increasing counter, for launch accounting by benchmarks). */
+uint64_t lm_kernel_launch_count(void);
+
+/* Per-kernel-family timing, measured with CUDA events recorded on the
+ * launching stream around every kernel launch of lm_step while enabled. */
+typedef enum {
+  LM_KERNEL_LION = 0,          /* Lion step (all params, or vectors on Muon steps) */
+  LM_KERNEL_MOMENTUM_NORM = 1, /* Muon: G_hat, ||G_hat||_F^2, M update, X0 */
+  LM_KERNEL_NS_GEMM = 2,       /* Newton-Schulz GEMM phases (Gram, polynomial, apply) */
+  LM_KERNEL_FINALIZE = 3,      /* Muon: parameter write */
+  LM_KERNEL_OTHER = 4,         /* gradient-pointer upload, norm reset */
+  LM_KERNEL_FAMILIES = 5
+} lm_kernel_family;
+
+typedef struct {
+  double ms[LM_KERNEL_FAMILIES];          /* summed event-to-event time */
+  uint64_t launches[LM_KERNEL_FAMILIES];  /* launches timed */
+} lm_profile;
+
+/* Turn event timing on (on != 0) or off for the state's later lm_step calls.
+ * Errors: LM_ERR_INVALID_ARG. */
+lm_status lm_profile_enable(lm_state* s, int on);
+
+/* Synchronise the state's last stream, add up the recorded events into *out
+ * and, if reset != 0, clear them.  Errors: LM_ERR_INVALID_ARG, LM_ERR_CUDA. */
+lm_status lm_profile_read(lm_state* s, lm_profile* out, int reset);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LIONMUON_H */

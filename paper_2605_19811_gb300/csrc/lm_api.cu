@@ -1,0 +1,865 @@
+// Host side of the C ABI declared in include/lionmuon.h: argument validation,
+// parameter classification (vectors vs hidden matrices), shape groups for the
+// grouped Newton-Schulz GEMMs, device tables, workspace, and the per-step
+// launch sequence of Algorithm 1 (Lion step, or Muon step on t mod P == 0).
+#include <algorithm>
+#include <atomic>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <string>
+#include <vector>
+
+#include "lm_internal.h"
+
+namespace lm {
+
+static std::atomic<uint64_t> g_launches{0};
+void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
+
+namespace {
+
+thread_local std::string g_last_error;
+
+lm_status fail(lm_status st, const char* fmt, ...) __attribute__((format(printf, 2, 3)));
+lm_status fail(lm_status st, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return st;
+}
+lm_status cuda_fail(cudaError_t e, const char* what) {
+  if (e == cudaErrorMemoryAllocation) return fail(LM_ERR_OOM, "%s: %s", what, cudaGetErrorString(e));
+  return fail(LM_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+#define LM_CUDA(call, what)                     \
+  do {                                          \
+    cudaError_t e_ = (call);                    \
+    if (e_ != cudaSuccess) return cuda_fail(e_, what); \
+  } while (0)
+
+size_t dtype_size(lm_dtype d) { return d == LM_BF16 ? 2 : 4; }
+bool valid_dtype(int d) { return d == LM_BF16 || d == LM_F32; }
+int64_t numel(const lm_tensor& t) { return t.rows * t.cols; }
+bool is_matrix(const lm_tensor& t) { return t.rows > 1 && t.cols > 1; }
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+lm_status check_tensor(const lm_tensor* t, const char* what, int i) {
+  if (t->rows < 0 || t->cols < 0)
+    return fail(LM_ERR_INVALID_ARG, "%s[%d]: negative shape (%lld x %lld)", what, i,
+                (long long)t->rows, (long long)t->cols);
+  if (!valid_dtype(t->dtype)) return fail(LM_ERR_DTYPE, "%s[%d]: unsupported dtype %d", what, i, (int)t->dtype);
+  if (numel(*t) > 0) {
+    if (t->data == nullptr) return fail(LM_ERR_INVALID_ARG, "%s[%d]: NULL data", what, i);
+    if (reinterpret_cast<uintptr_t>(t->data) % 16 != 0)
+      return fail(LM_ERR_ALIGN, "%s[%d]: data pointer not 16-byte aligned", what, i);
+  }
+  return LM_OK;
+}
+
+lm_status check_config(const lm_config* c) {
+  auto finite = [](double x) { return std::isfinite(x); };
+  if (!(c->beta1 >= 0.0 && c->beta1 < 1.0) || !(c->beta2 >= 0.0 && c->beta2 < 1.0))
+    return fail(LM_ERR_INVALID_ARG, "beta1/beta2 must lie in [0, 1)");
+  if (!finite(c->eta_muon) || !finite(c->eta_lion) || c->eta_muon < 0 || c->eta_lion < 0)
+    return fail(LM_ERR_INVALID_ARG, "learning rates must be finite and >= 0");
+  if (!finite(c->weight_decay) || c->weight_decay < 0) return fail(LM_ERR_INVALID_ARG, "weight_decay must be >= 0");
+  if (c->period < 0) return fail(LM_ERR_INVALID_ARG, "period must be >= 0 (0 = infinity)");
+  if (c->ns_steps < 0 || c->ns_steps > 64) return fail(LM_ERR_INVALID_ARG, "ns_steps must be in [0, 64]");
+  if (!finite(c->ns_a) || !finite(c->ns_b) || !finite(c->ns_c)) return fail(LM_ERR_INVALID_ARG, "NS coefficients must be finite");
+  if (!finite(c->ns_eps) || c->ns_eps < 0) return fail(LM_ERR_INVALID_ARG, "ns_eps must be >= 0");
+  if (!finite(c->shape_scale) || c->shape_scale < 0) return fail(LM_ERR_INVALID_ARG, "shape_scale must be >= 0");
+  if (c->ns_precision != LM_BF16 && c->ns_precision != LM_F32)
+    return fail(LM_ERR_INVALID_ARG, "ns_precision must be LM_BF16 or LM_F32");
+  return LM_OK;
+}
+
+lm_status check_device(int* dev_out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return fail(LM_ERR_CUDA, "no CUDA device: %s", cudaGetErrorString(e));
+  int major = 0, minor = 0;
+  cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+  cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+  if (major != 10 || minor != 3)
+    return fail(LM_ERR_UNSUPPORTED, "device %d is sm_%d%d; this library is built for sm_103a", dev, major, minor);
+  *dev_out = dev;
+  return LM_OK;
+}
+
+LionConsts lion_consts(const lm_config& c) {
+  LionConsts k;
+  k.b1 = (float)c.beta1;
+  k.c1 = (float)(1.0 - c.beta1);
+  k.b2 = (float)c.beta2;
+  k.c2 = (float)(1.0 - c.beta2);
+  k.eL = (float)c.eta_lion;
+  k.lam = (float)c.weight_decay;
+  return k;
+}
+MuonConsts muon_consts(const lm_config& c) {
+  MuonConsts k;
+  k.b1 = (float)c.beta1;
+  k.c1 = (float)(1.0 - c.beta1);
+  k.b2 = (float)c.beta2;
+  k.c2 = (float)(1.0 - c.beta2);
+  k.eM = (float)c.eta_muon;
+  k.lam = (float)c.weight_decay;
+  k.eps = (float)c.ns_eps;
+  k.ns_steps = c.ns_steps;
+  return k;
+}
+
+// Device-memory arena: one cudaMalloc, sub-allocated with 256-byte alignment.
+struct Arena {
+  std::vector<std::pair<size_t, size_t>> parts;  // (offset, bytes)
+  size_t total = 0;
+  size_t add(size_t bytes) {
+    total = align_up(total, 256);
+    size_t off = total;
+    total += std::max<size_t>(bytes, 1);
+    return off;
+  }
+};
+
+constexpr int64_t kLionChunk = 32768;   // elements per Lion work chunk
+
+struct LionTable {
+  LionTensor* tensors = nullptr;
+  LionChunk* chunks = nullptr;
+  int nchunks = 0;
+};
+
+// One launch batch of the Newton-Schulz GEMMs: up to kMaxGroupsTc groups
+// (tensor-core path) or all groups (fp32 path), a tile list per phase.
+struct NsBatch {
+  int g0 = 0, ng = 0;
+  NsTile* tiles[3] = {nullptr, nullptr, nullptr};
+  int ntiles[3] = {0, 0, 0};
+};
+
+void build_lion_chunks(const std::vector<LionTensor>& ts, std::vector<LionChunk>& out) {
+  for (size_t i = 0; i < ts.size(); ++i) {
+    for (int64_t b = 0; b < ts[i].n; b += kLionChunk) {
+      LionChunk c;
+      c.tensor = (int32_t)i;
+      c.pad = 0;
+      c.begin = b;
+      c.count = std::min<int64_t>(kLionChunk, ts[i].n - b);
+      out.push_back(c);
+    }
+  }
+}
+
+// Tile list of one phase over groups [g0, g0+ng).  Symmetric phases keep the
+// tiles that reach the diagonal or above; the list is ordered longest K first.
+void build_ns_tiles(const std::vector<NsGroup>& groups, int g0, int ng, int phase, int bm, int bn,
+                    std::vector<NsTile>& out) {
+  std::vector<std::pair<int, NsTile>> v;
+  for (int gi = g0; gi < g0 + ng; ++gi) {
+    const NsGroup& g = groups[gi];
+    const int ncol = (phase == NS_APPLY) ? g.l_pad : g.s_pad;
+    const int K = (phase == NS_GRAM) ? g.l_pad : g.s_pad;
+    const int tms = g.s_pad / bm, tns = (ncol + bn - 1) / bn;
+    for (int m = 0; m < g.count; ++m)
+      for (int tm = 0; tm < tms; ++tm)
+        for (int tn = 0; tn < tns; ++tn) {
+          if (phase != NS_APPLY && (int64_t)(tn + 1) * bn <= (int64_t)tm * bm) continue;
+          NsTile t;
+          t.group = (uint16_t)(gi - g0);
+          t.mat = (uint16_t)m;
+          t.tm = (uint16_t)tm;
+          t.tn = (uint16_t)tn;
+          v.push_back({K, t});
+        }
+  }
+  std::stable_sort(v.begin(), v.end(), [](const std::pair<int, NsTile>& a, const std::pair<int, NsTile>& b) {
+    return a.first > b.first;
+  });
+  for (auto& e : v) out.push_back(e.second);
+}
+
+// Element tiles of each matrix, padded to whole clusters with empty slots.
+void build_elem_tiles(const std::vector<MatDesc>& mats, std::vector<ElemTile>& out) {
+  for (size_t i = 0; i < mats.size(); ++i) {
+    const int n = mats[i].tiles_r * mats[i].tiles_c;
+    const int padded = (n + kNormCluster - 1) / kNormCluster * kNormCluster;
+    for (int t = 0; t < padded; ++t) out.push_back(ElemTile{(int32_t)i, t < n ? t : -1});
+  }
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// Newton-Schulz engine shared by lm_step and lm_msign_ns
+// ---------------------------------------------------------------------------
+struct NsEngine {
+  lm_dtype xdt = LM_BF16;            // workspace dtype: bf16 (tensor cores) or fp32
+  std::vector<NsGroup> groups;       // host copies (device pointers inside)
+  std::vector<TcGroupMaps> maps;     // tensor-core path
+  NsGroup* d_groups = nullptr;       // fp32 path reads groups from device memory
+  std::vector<NsBatch> batches;
+  double* d_norm2 = nullptr;
+};
+
+// Plan: group matrices by (s, l); returns matrix order (indices into shapes)
+// and fills groups with sizes (pointers set later).
+static void plan_groups(const std::vector<std::pair<int64_t, int64_t>>& shapes, lm_dtype xdt,
+                        std::vector<NsGroup>& groups, std::vector<std::vector<int>>& members) {
+  std::map<std::pair<int64_t, int64_t>, int> key_to_group;
+  for (size_t i = 0; i < shapes.size(); ++i) {
+    const int64_t s = std::min(shapes[i].first, shapes[i].second);
+    const int64_t l = std::max(shapes[i].first, shapes[i].second);
+    auto key = std::make_pair(s, l);
+    auto it = key_to_group.find(key);
+    if (it == key_to_group.end()) {
+      NsGroup g;
+      memset(&g, 0, sizeof(g));
+      g.s = (int32_t)s;
+      g.l = (int32_t)l;
+      if (xdt == LM_BF16) {
+        g.s_pad = tc_pad_s((int)s);
+        g.l_pad = tc_pad_l((int)l);
+      } else {
+        g.s_pad = simt_pad((int)s);
+        g.l_pad = simt_pad((int)l);
+      }
+      key_to_group[key] = (int)groups.size();
+      groups.push_back(g);
+      members.emplace_back();
+      it = key_to_group.find(key);
+    }
+    members[it->second].push_back((int)i);
+  }
+  int first = 0;
+  for (size_t gi = 0; gi < groups.size(); ++gi) {
+    groups[gi].count = (int32_t)members[gi].size();
+    groups[gi].first_mat = first;
+    first += groups[gi].count;
+  }
+}
+
+// Reserve workspace for the groups and the tile lists in the arena.
+struct NsLayout {
+  std::vector<size_t> off_x0, off_x1, off_a, off_b;
+  std::vector<std::vector<NsTile>> tiles;   // per batch*3 + phase
+  std::vector<size_t> off_tiles;
+  size_t off_groups = 0;
+  size_t off_norm = 0;
+};
+
+static void layout_ns(std::vector<NsGroup>& groups, lm_dtype xdt, int nmat, Arena& ar, NsLayout& L,
+                      std::vector<NsBatch>& batches) {
+  const size_t es = dtype_size(xdt);
+  for (auto& g : groups) {
+    const size_t xb = (size_t)g.count * g.s_pad * g.l_pad * es;
+    const size_t ab = (size_t)g.count * g.s_pad * g.s_pad * es;
+    L.off_x0.push_back(ar.add(xb));
+    L.off_x1.push_back(ar.add(xb));
+    L.off_a.push_back(ar.add(ab));
+    L.off_b.push_back(ar.add(ab));
+  }
+  const int per = (xdt == LM_BF16) ? kMaxGroupsTc : kMaxGroupsSimt;
+  const int bm = (xdt == LM_BF16) ? kTcBM : kSimtBM;
+  const int bn = (xdt == LM_BF16) ? kTcBN : kSimtBN;
+  for (int g0 = 0; g0 < (int)groups.size(); g0 += per) {
+    NsBatch b;
+    b.g0 = g0;
+    b.ng = std::min(per, (int)groups.size() - g0);
+    for (int ph = 0; ph < 3; ++ph) {
+      std::vector<NsTile> t;
+      build_ns_tiles(groups, g0, b.ng, ph, bm, bn, t);
+      b.ntiles[ph] = (int)t.size();
+      L.off_tiles.push_back(ar.add(t.size() * sizeof(NsTile)));
+      L.tiles.push_back(std::move(t));
+    }
+    batches.push_back(b);
+  }
+  L.off_groups = ar.add(groups.size() * sizeof(NsGroup));
+  L.off_norm = ar.add((size_t)std::max(nmat, 1) * sizeof(double));
+}
+
+static void bind_ns(NsEngine& E, char* base, const NsLayout& L, std::vector<char>& host_img) {
+  for (size_t gi = 0; gi < E.groups.size(); ++gi) {
+    E.groups[gi].X[0] = base + L.off_x0[gi];
+    E.groups[gi].X[1] = base + L.off_x1[gi];
+    E.groups[gi].A = base + L.off_a[gi];
+    E.groups[gi].B = base + L.off_b[gi];
+  }
+  for (size_t bi = 0; bi < E.batches.size(); ++bi)
+    for (int ph = 0; ph < 3; ++ph) {
+      const size_t k = bi * 3 + ph;
+      E.batches[bi].tiles[ph] = reinterpret_cast<NsTile*>(base + L.off_tiles[k]);
+      if (!L.tiles[k].empty())
+        memcpy(host_img.data() + L.off_tiles[k], L.tiles[k].data(), L.tiles[k].size() * sizeof(NsTile));
+    }
+  E.d_groups = reinterpret_cast<NsGroup*>(base + L.off_groups);
+  memcpy(host_img.data() + L.off_groups, E.groups.data(), E.groups.size() * sizeof(NsGroup));
+  E.d_norm2 = reinterpret_cast<double*>(base + L.off_norm);
+}
+
+static lm_status encode_maps(NsEngine& E) {
+  if (E.xdt != LM_BF16) return LM_OK;
+  E.maps.resize(E.groups.size());
+  for (size_t gi = 0; gi < E.groups.size(); ++gi) {
+    cudaError_t e = tc_encode_group_maps(E.groups[gi], &E.maps[gi]);
+    if (e != cudaSuccess) return cuda_fail(e, "cuTensorMapEncodeTiled");
+  }
+  return LM_OK;
+}
+
+// Event timing of kernel launches (enabled by lm_profile_enable).
+struct Profiler {
+  bool on = false;
+  struct Rec {
+    int fam;
+    cudaEvent_t a, b;
+  };
+  std::vector<cudaEvent_t> pool;
+  size_t used = 0;
+  std::vector<Rec> recs;
+  double ms[LM_KERNEL_FAMILIES] = {0};
+  uint64_t n[LM_KERNEL_FAMILIES] = {0};
+  cudaEvent_t next() {
+    if (used == pool.size()) {
+      cudaEvent_t e = nullptr;
+      if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+      pool.push_back(e);
+    }
+    return pool[used++];
+  }
+  ~Profiler() {
+    for (cudaEvent_t e : pool) cudaEventDestroy(e);
+  }
+};
+
+// Launch f() on st; with profiling on, bracket it by events of family fam.
+template <typename F>
+static cudaError_t timed(Profiler* P, int fam, cudaStream_t st, F&& f) {
+  if (P == nullptr || !P->on) return f();
+  cudaEvent_t a = P->next(), b = P->next();
+  if (a == nullptr || b == nullptr) return f();
+  cudaEventRecord(a, st);
+  cudaError_t e = f();
+  cudaEventRecord(b, st);
+  P->recs.push_back({fam, a, b});
+  return e;
+}
+
+static lm_status run_ns(const NsEngine& E, int steps, NsCoeffs co, unsigned* flags, cudaStream_t st,
+                        Profiler* P = nullptr) {
+  for (int it = 0; it < steps; ++it)
+    for (const NsBatch& b : E.batches)
+      for (int ph = 0; ph < 3; ++ph) {
+        cudaError_t e = timed(P, LM_KERNEL_NS_GEMM, st, [&]() {
+          if (E.xdt == LM_BF16)
+            return launch_ns_tc((NsPhase)ph, it, b.ng, E.groups.data() + b.g0, E.maps.data() + b.g0,
+                                b.tiles[ph], b.ntiles[ph], E.d_norm2, co, flags, st);
+          return launch_ns_simt((NsPhase)ph, it, b.ng, E.d_groups + b.g0, b.tiles[ph], b.ntiles[ph],
+                                E.d_norm2, co, st);
+        });
+        if (e != cudaSuccess) return cuda_fail(e, "Newton-Schulz launch");
+      }
+  return LM_OK;
+}
+
+}  // namespace lm
+
+using namespace lm;
+
+// ---------------------------------------------------------------------------
+// the state
+// ---------------------------------------------------------------------------
+struct lm_state {
+  int device = 0;
+  lm_config cfg;
+  int n = 0;
+  std::vector<lm_tensor> params;
+  std::vector<size_t> mom_off;      // element offset of each momentum buffer
+  size_t mom_elems = 0;             // sum |W_i|
+  char* base = nullptr;             // the one device allocation
+  size_t bytes = 0;
+  float* mom = nullptr;
+  const void** d_grads = nullptr;   // device grad-pointer table
+  std::vector<const void*> h_grads; // what the device table holds
+  bool grads_valid = false;
+  LionTable lion_all[2], lion_vec[2];
+  int lion_grid[2] = {0, 0};
+  int nmat = 0;
+  MatDesc* d_mats = nullptr;
+  ElemTile* d_etiles = nullptr;
+  int n_etiles = 0;
+  NsEngine ns;
+  unsigned* d_flags = nullptr;
+  cudaStream_t last_stream = nullptr;
+  Profiler prof;
+};
+
+extern "C" {
+
+void lm_config_default(lm_config* c) {
+  if (c == nullptr) return;
+  c->beta1 = 0.9;
+  c->beta2 = 0.99;
+  c->eta_muon = 3e-3;
+  c->eta_lion = 2e-5;
+  c->weight_decay = 0.1;
+  c->period = 2;
+  c->ns_steps = 5;
+  c->ns_a = 3.4445;
+  c->ns_b = -4.7750;
+  c->ns_c = 2.0315;
+  c->ns_eps = 1e-7;
+  c->shape_scale = 0.2;
+  c->ns_precision = LM_BF16;
+}
+
+const char* lm_status_string(lm_status st) {
+  switch (st) {
+    case LM_OK: return "LM_OK";
+    case LM_ERR_INVALID_ARG: return "LM_ERR_INVALID_ARG";
+    case LM_ERR_DTYPE: return "LM_ERR_DTYPE";
+    case LM_ERR_ALIGN: return "LM_ERR_ALIGN";
+    case LM_ERR_OOM: return "LM_ERR_OOM";
+    case LM_ERR_CUDA: return "LM_ERR_CUDA";
+    case LM_ERR_UNSUPPORTED: return "LM_ERR_UNSUPPORTED";
+    case LM_ERR_TIMEOUT: return "LM_ERR_TIMEOUT";
+  }
+  return "unknown lm_status";
+}
+
+const char* lm_last_error(void) { return g_last_error.c_str(); }
+
+uint64_t lm_kernel_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* cuda_stream,
+                    lm_state** out) {
+  if (out == nullptr) return fail(LM_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  if (params == nullptr || cfg == nullptr) return fail(LM_ERR_INVALID_ARG, "params/cfg is NULL");
+  if (n < 1) return fail(LM_ERR_INVALID_ARG, "n must be >= 1");
+  lm_status st = check_config(cfg);
+  if (st != LM_OK) return st;
+  for (int i = 0; i < n; ++i)
+    if ((st = check_tensor(&params[i], "params", i)) != LM_OK) return st;
+  int dev = 0;
+  if ((st = check_device(&dev)) != LM_OK) return st;
+  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+
+  lm_state* s = new lm_state();
+  s->device = dev;
+  s->cfg = *cfg;
+  s->n = n;
+  s->params.assign(params, params + n);
+  s->ns.xdt = (cfg->ns_precision == LM_F32) ? LM_F32 : LM_BF16;
+
+  // matrices and their shape groups
+  std::vector<int> mat_param;
+  std::vector<std::pair<int64_t, int64_t>> mat_shapes;
+  for (int i = 0; i < n; ++i)
+    if (is_matrix(params[i])) {
+      mat_param.push_back(i);
+      mat_shapes.push_back({params[i].rows, params[i].cols});
+    }
+  std::vector<std::vector<int>> members;
+  plan_groups(mat_shapes, s->ns.xdt, s->ns.groups, members);
+  s->nmat = (int)mat_param.size();
+
+  // arena layout
+  Arena ar;
+  s->mom_off.resize(n);
+  size_t mom_elems_aligned = 0;
+  for (int i = 0; i < n; ++i) {
+    s->mom_off[i] = mom_elems_aligned;
+    mom_elems_aligned = align_up(mom_elems_aligned + (size_t)numel(params[i]), 64);
+    s->mom_elems += (size_t)numel(params[i]);
+  }
+  const size_t off_mom = ar.add(mom_elems_aligned * sizeof(float));
+  const size_t off_grads = ar.add((size_t)n * sizeof(void*));
+  const size_t off_flags = ar.add(sizeof(unsigned));
+
+  // Lion tables (per dtype): all params, and vectors only
+  std::vector<LionTensor> lt_all[2], lt_vec[2];
+  for (int i = 0; i < n; ++i) {
+    if (numel(params[i]) == 0) continue;
+    LionTensor t;
+    t.w = params[i].data;
+    t.m = nullptr;   // bound after allocation
+    t.n = numel(params[i]);
+    t.grad_slot = i;
+    t.pad = i;       // remember the param index until binding
+    lt_all[params[i].dtype].push_back(t);
+    if (!is_matrix(params[i])) lt_vec[params[i].dtype].push_back(t);
+  }
+  std::vector<LionChunk> lc_all[2], lc_vec[2];
+  size_t off_lt_all[2], off_lc_all[2], off_lt_vec[2], off_lc_vec[2];
+  for (int d = 0; d < 2; ++d) {
+    build_lion_chunks(lt_all[d], lc_all[d]);
+    build_lion_chunks(lt_vec[d], lc_vec[d]);
+    off_lt_all[d] = ar.add(lt_all[d].size() * sizeof(LionTensor));
+    off_lc_all[d] = ar.add(lc_all[d].size() * sizeof(LionChunk));
+    off_lt_vec[d] = ar.add(lt_vec[d].size() * sizeof(LionTensor));
+    off_lc_vec[d] = ar.add(lc_vec[d].size() * sizeof(LionChunk));
+  }
+
+  // Muon tables
+  NsLayout L;
+  layout_ns(s->ns.groups, s->ns.xdt, s->nmat, ar, L, s->ns.batches);
+  const size_t off_mats = ar.add((size_t)std::max(s->nmat, 1) * sizeof(MatDesc));
+  std::vector<MatDesc> mats(s->nmat);
+  // matrices are numbered in group order
+  std::vector<int> mat_order;   // mat id -> index into mat_param
+  for (size_t gi = 0; gi < members.size(); ++gi)
+    for (int m : members[gi]) mat_order.push_back(m);
+  for (int id = 0; id < s->nmat; ++id) {
+    const lm_tensor& p = params[mat_param[mat_order[id]]];
+    MatDesc& d = mats[id];
+    memset(&d, 0, sizeof(d));
+    d.rows = p.rows;
+    d.cols = p.cols;
+    d.tiles_r = (int32_t)((p.rows + kElemTileR - 1) / kElemTileR);
+    d.tiles_c = (int32_t)((p.cols + kElemTileC - 1) / kElemTileC);
+  }
+  std::vector<ElemTile> etiles;
+  build_elem_tiles(mats, etiles);
+  s->n_etiles = (int)etiles.size();
+  const size_t off_etiles = ar.add(etiles.size() * sizeof(ElemTile));
+
+  cudaError_t e = cudaMalloc(&s->base, ar.total);
+  if (e != cudaSuccess) {
+    delete s;
+    return cuda_fail(e, "cudaMalloc(state)");
+  }
+  s->bytes = ar.total;
+  std::vector<char> img(ar.total, 0);
+  char* base = s->base;
+  s->mom = reinterpret_cast<float*>(base + off_mom);
+  s->d_grads = reinterpret_cast<const void**>(base + off_grads);
+  s->d_flags = reinterpret_cast<unsigned*>(base + off_flags);
+
+  for (int d = 0; d < 2; ++d) {
+    for (auto& t : lt_all[d]) { t.m = s->mom + s->mom_off[t.pad]; }
+    for (auto& t : lt_vec[d]) { t.m = s->mom + s->mom_off[t.pad]; }
+    auto put = [&](size_t off, const void* src, size_t bytes) { if (bytes) memcpy(img.data() + off, src, bytes); };
+    put(off_lt_all[d], lt_all[d].data(), lt_all[d].size() * sizeof(LionTensor));
+    put(off_lc_all[d], lc_all[d].data(), lc_all[d].size() * sizeof(LionChunk));
+    put(off_lt_vec[d], lt_vec[d].data(), lt_vec[d].size() * sizeof(LionTensor));
+    put(off_lc_vec[d], lc_vec[d].data(), lc_vec[d].size() * sizeof(LionChunk));
+    s->lion_all[d] = {reinterpret_cast<LionTensor*>(base + off_lt_all[d]),
+                      reinterpret_cast<LionChunk*>(base + off_lc_all[d]), (int)lc_all[d].size()};
+    s->lion_vec[d] = {reinterpret_cast<LionTensor*>(base + off_lt_vec[d]),
+                      reinterpret_cast<LionChunk*>(base + off_lc_vec[d]), (int)lc_vec[d].size()};
+    s->lion_grid[d] = lion_grid_size((lm_dtype)d);
+  }
+
+  bind_ns(s->ns, base, L, img);
+  const size_t es = dtype_size(s->ns.xdt);
+  for (size_t gi = 0; gi < s->ns.groups.size(); ++gi) {
+    const NsGroup& g = s->ns.groups[gi];
+    for (int k = 0; k < g.count; ++k) {
+      const int id = g.first_mat + k;
+      const int pi = mat_param[mat_order[id]];
+      const lm_tensor& p = params[pi];
+      MatDesc& d = mats[id];
+      const size_t xoff = (size_t)k * g.s_pad * g.l_pad * es;
+      d.w = p.data;
+      d.m = s->mom + s->mom_off[pi];
+      d.x = static_cast<char*>(g.X[0]) + xoff;
+      d.x_final = static_cast<char*>(g.X[cfg->ns_steps & 1]) + xoff;
+      d.out = nullptr;
+      d.norm2 = s->ns.d_norm2 + id;
+      d.ldx = g.l_pad;
+      d.grad_slot = pi;
+      d.transposed = p.rows > p.cols ? 1 : 0;
+      d.wdt = p.dtype;
+      d.odt = p.dtype;
+      d.shape_scale = (float)(cfg->shape_scale * std::sqrt((double)std::max(p.rows, p.cols)));
+    }
+  }
+  if (s->nmat) memcpy(img.data() + off_mats, mats.data(), mats.size() * sizeof(MatDesc));
+  if (!etiles.empty()) memcpy(img.data() + off_etiles, etiles.data(), etiles.size() * sizeof(ElemTile));
+  s->d_mats = reinterpret_cast<MatDesc*>(base + off_mats);
+  s->d_etiles = reinterpret_cast<ElemTile*>(base + off_etiles);
+
+  // Upload tables and zeros (momentum M_{-1} = 0, workspace padding = 0).
+  e = cudaMemcpyAsync(base, img.data(), ar.total, cudaMemcpyHostToDevice, stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) {
+    cudaFree(s->base);
+    delete s;
+    return cuda_fail(e, "upload of state tables");
+  }
+  if ((st = encode_maps(s->ns)) != LM_OK) {
+    cudaFree(s->base);
+    delete s;
+    return st;
+  }
+  s->last_stream = stream;
+  *out = s;
+  return LM_OK;
+}
+
+static lm_status upload_grads(lm_state* s, const lm_tensor* grads, cudaStream_t st) {
+  bool same = s->grads_valid;
+  for (int i = 0; same && i < s->n; ++i) same = s->h_grads[i] == grads[i].data;
+  if (same) return LM_OK;
+  s->h_grads.resize(s->n);
+  for (int i0 = 0; i0 < s->n; i0 += kPtrsPerUpload) {
+    PtrUpload up;
+    const int cnt = std::min(kPtrsPerUpload, s->n - i0);
+    for (int k = 0; k < cnt; ++k) up.p[k] = grads[i0 + k].data;
+    cudaError_t e = timed(&s->prof, LM_KERNEL_OTHER, st,
+                          [&]() { return launch_upload_ptrs(s->d_grads + i0, up, cnt, st); });
+    if (e != cudaSuccess) {
+      s->grads_valid = false;
+      return cuda_fail(e, "gradient pointer upload");
+    }
+  }
+  for (int i = 0; i < s->n; ++i) s->h_grads[i] = grads[i].data;
+  s->grads_valid = true;
+  return LM_OK;
+}
+
+lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t, void* cuda_stream) {
+  if (s == nullptr || grads == nullptr) return fail(LM_ERR_INVALID_ARG, "state/grads is NULL");
+  if (n != s->n) return fail(LM_ERR_INVALID_ARG, "n = %d but the state has %d parameters", n, s->n);
+  if (t < 0) return fail(LM_ERR_INVALID_ARG, "t must be >= 0");
+  lm_status st;
+  for (int i = 0; i < n; ++i) {
+    if ((st = check_tensor(&grads[i], "grads", i)) != LM_OK) return st;
+    if (grads[i].rows != s->params[i].rows || grads[i].cols != s->params[i].cols)
+      return fail(LM_ERR_INVALID_ARG, "grads[%d] shape %lldx%lld != param shape %lldx%lld", i,
+                  (long long)grads[i].rows, (long long)grads[i].cols, (long long)s->params[i].rows,
+                  (long long)s->params[i].cols);
+    if (grads[i].dtype != s->params[i].dtype)
+      return fail(LM_ERR_DTYPE, "grads[%d] dtype differs from the parameter's", i);
+  }
+  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+  if ((st = upload_grads(s, grads, stream)) != LM_OK) return st;
+  s->last_stream = stream;
+  const lm_config& c = s->cfg;
+  const bool muon = c.period != 0 && (t % c.period) == 0;
+  const LionConsts lk = lion_consts(c);
+  cudaError_t e;
+  Profiler* P = &s->prof;
+  if (!muon) {
+    for (int d = 0; d < 2; ++d) {
+      if (s->lion_all[d].nchunks == 0) continue;
+      e = timed(P, LM_KERNEL_LION, stream, [&]() {
+        return launch_lion((lm_dtype)d, s->lion_all[d].tensors, s->lion_all[d].chunks,
+                           s->lion_all[d].nchunks, s->d_grads, lk, s->lion_grid[d], stream);
+      });
+      if (e != cudaSuccess) return cuda_fail(e, "Lion kernel launch");
+    }
+    return LM_OK;
+  }
+  // Muon step: momentum + norm, Lion on the vectors, NS iterations, finalize.
+  const MuonConsts mk = muon_consts(c);
+  if (s->nmat > 0) {
+    e = timed(P, LM_KERNEL_OTHER, stream, [&]() {
+      return cudaMemsetAsync(s->ns.d_norm2, 0, (size_t)s->nmat * sizeof(double), stream);
+    });
+    if (e != cudaSuccess) return cuda_fail(e, "norm reset");
+    e = timed(P, LM_KERNEL_MOMENTUM_NORM, stream, [&]() {
+      return launch_momentum_norm(s->ns.xdt, s->d_mats, s->d_etiles, s->n_etiles, s->d_grads, mk, 0,
+                                  stream);
+    });
+    if (e != cudaSuccess) return cuda_fail(e, "momentum/norm kernel launch");
+  }
+  for (int d = 0; d < 2; ++d) {
+    if (s->lion_vec[d].nchunks == 0) continue;
+    e = timed(P, LM_KERNEL_LION, stream, [&]() {
+      return launch_lion((lm_dtype)d, s->lion_vec[d].tensors, s->lion_vec[d].chunks,
+                         s->lion_vec[d].nchunks, s->d_grads, lk, s->lion_grid[d], stream);
+    });
+    if (e != cudaSuccess) return cuda_fail(e, "Lion kernel launch (vectors)");
+  }
+  if (s->nmat > 0) {
+    NsCoeffs co{(float)c.ns_a, (float)c.ns_b, (float)c.ns_c, (float)c.ns_eps};
+    if ((st = run_ns(s->ns, c.ns_steps, co, s->d_flags, stream, P)) != LM_OK) return st;
+    e = timed(P, LM_KERNEL_FINALIZE, stream, [&]() {
+      return launch_finalize(s->ns.xdt, s->d_mats, s->d_etiles, s->n_etiles, mk, 0, s->d_flags, stream);
+    });
+    if (e != cudaSuccess) return cuda_fail(e, "finalize kernel launch");
+  }
+  return LM_OK;
+}
+
+lm_status lm_set_lr(lm_state* s, double eta_muon, double eta_lion) {
+  if (s == nullptr) return fail(LM_ERR_INVALID_ARG, "state is NULL");
+  if (!std::isfinite(eta_muon) || !std::isfinite(eta_lion) || eta_muon < 0 || eta_lion < 0)
+    return fail(LM_ERR_INVALID_ARG, "learning rates must be finite and >= 0");
+  s->cfg.eta_muon = eta_muon;
+  s->cfg.eta_lion = eta_lion;
+  return LM_OK;
+}
+
+lm_status lm_get_momentum(const lm_state* s, int i, lm_tensor* view) {
+  if (s == nullptr || view == nullptr) return fail(LM_ERR_INVALID_ARG, "state/view is NULL");
+  if (i < 0 || i >= s->n) return fail(LM_ERR_INVALID_ARG, "index %d out of range", i);
+  view->data = s->mom + s->mom_off[i];
+  view->rows = s->params[i].rows;
+  view->cols = s->params[i].cols;
+  view->dtype = LM_F32;
+  return LM_OK;
+}
+
+lm_status lm_set_momentum(lm_state* s, int i, const lm_tensor* src, void* cuda_stream) {
+  if (s == nullptr || src == nullptr) return fail(LM_ERR_INVALID_ARG, "state/src is NULL");
+  if (i < 0 || i >= s->n) return fail(LM_ERR_INVALID_ARG, "index %d out of range", i);
+  lm_status st = check_tensor(src, "src", 0);
+  if (st != LM_OK) return st;
+  if (src->dtype != LM_F32) return fail(LM_ERR_DTYPE, "momentum source must be fp32");
+  if (src->rows != s->params[i].rows || src->cols != s->params[i].cols)
+    return fail(LM_ERR_INVALID_ARG, "momentum source shape differs from the parameter's");
+  const size_t bytes = (size_t)numel(s->params[i]) * sizeof(float);
+  if (bytes == 0) return LM_OK;
+  cudaError_t e = cudaMemcpyAsync(s->mom + s->mom_off[i], src->data, bytes, cudaMemcpyDeviceToDevice,
+                                  static_cast<cudaStream_t>(cuda_stream));
+  if (e != cudaSuccess) return cuda_fail(e, "momentum copy");
+  return LM_OK;
+}
+
+lm_status lm_get_status(lm_state* s, uint32_t* device_flags) {
+  if (s == nullptr || device_flags == nullptr) return fail(LM_ERR_INVALID_ARG, "state/flags is NULL");
+  cudaError_t e = cudaStreamSynchronize(s->last_stream);
+  if (e != cudaSuccess) return cuda_fail(e, "stream synchronize");
+  unsigned f = 0;
+  e = cudaMemcpy(&f, s->d_flags, sizeof(unsigned), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "status read");
+  e = cudaMemset(s->d_flags, 0, sizeof(unsigned));
+  if (e != cudaSuccess) return cuda_fail(e, "status clear");
+  *device_flags = f;
+  return LM_OK;
+}
+
+lm_status lm_profile_enable(lm_state* s, int on) {
+  if (s == nullptr) return fail(LM_ERR_INVALID_ARG, "state is NULL");
+  s->prof.on = on != 0;
+  return LM_OK;
+}
+
+lm_status lm_profile_read(lm_state* s, lm_profile* out, int reset) {
+  if (s == nullptr || out == nullptr) return fail(LM_ERR_INVALID_ARG, "state/out is NULL");
+  Profiler& P = s->prof;
+  cudaError_t e = cudaStreamSynchronize(s->last_stream);
+  if (e != cudaSuccess) return cuda_fail(e, "stream synchronize");
+  for (const Profiler::Rec& r : P.recs) {
+    float ms = 0.f;
+    e = cudaEventElapsedTime(&ms, r.a, r.b);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaEventElapsedTime");
+    P.ms[r.fam] += ms;
+    P.n[r.fam] += 1;
+  }
+  P.recs.clear();
+  P.used = 0;
+  for (int f = 0; f < LM_KERNEL_FAMILIES; ++f) {
+    out->ms[f] = P.ms[f];
+    out->launches[f] = P.n[f];
+    if (reset) {
+      P.ms[f] = 0;
+      P.n[f] = 0;
+    }
+  }
+  return LM_OK;
+}
+
+size_t lm_state_bytes(const lm_state* s) { return s ? s->mom_elems * sizeof(float) : 0; }
+
+size_t lm_workspace_bytes(const lm_state* s) {
+  return s ? s->bytes - s->mom_elems * sizeof(float) : 0;
+}
+
+void lm_destroy(lm_state* s) {
+  if (s == nullptr) return;
+  cudaStreamSynchronize(s->last_stream);
+  cudaFree(s->base);
+  delete s;
+}
+
+lm_status lm_msign_ns(const lm_tensor* in, lm_tensor* out, int steps, double a, double b, double c,
+                      double eps, int precision, void* cuda_stream) {
+  if (in == nullptr || out == nullptr) return fail(LM_ERR_INVALID_ARG, "in/out is NULL");
+  lm_status st;
+  if ((st = check_tensor(in, "in", 0)) != LM_OK) return st;
+  if ((st = check_tensor(out, "out", 0)) != LM_OK) return st;
+  if (in->rows < 2 || in->cols < 2) return fail(LM_ERR_INVALID_ARG, "msign needs rows, cols >= 2");
+  if (out->rows != in->rows || out->cols != in->cols) return fail(LM_ERR_INVALID_ARG, "out shape differs from in");
+  if (steps < 0 || steps > 64) return fail(LM_ERR_INVALID_ARG, "steps must be in [0, 64]");
+  if (!std::isfinite(a) || !std::isfinite(b) || !std::isfinite(c) || !std::isfinite(eps) || eps < 0)
+    return fail(LM_ERR_INVALID_ARG, "coefficients must be finite, eps >= 0");
+  if (precision != LM_BF16 && precision != LM_F32) return fail(LM_ERR_INVALID_ARG, "precision must be LM_BF16 or LM_F32");
+  if (std::max(in->rows, in->cols) > 1000000 || std::min(in->rows, in->cols) > 65536)
+    return fail(LM_ERR_UNSUPPORTED, "matrix too large for lm_msign_ns");
+  int dev = 0;
+  if ((st = check_device(&dev)) != LM_OK) return st;
+  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+
+  NsEngine E;
+  E.xdt = precision == LM_F32 ? LM_F32 : LM_BF16;
+  std::vector<std::vector<int>> members;
+  plan_groups({{in->rows, in->cols}}, E.xdt, E.groups, members);
+  Arena ar;
+  NsLayout L;
+  layout_ns(E.groups, E.xdt, 1, ar, L, E.batches);
+  const size_t off_mat = ar.add(sizeof(MatDesc));
+  MatDesc d;
+  memset(&d, 0, sizeof(d));
+  d.rows = in->rows;
+  d.cols = in->cols;
+  d.tiles_r = (int32_t)((d.rows + kElemTileR - 1) / kElemTileR);
+  d.tiles_c = (int32_t)((d.cols + kElemTileC - 1) / kElemTileC);
+  std::vector<ElemTile> et;
+  build_elem_tiles({d}, et);
+  const size_t off_et = ar.add(et.size() * sizeof(ElemTile));
+  const size_t off_flags = ar.add(sizeof(unsigned));
+
+  char* base = nullptr;
+  cudaError_t e = cudaMallocAsync(reinterpret_cast<void**>(&base), ar.total, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMallocAsync(msign workspace)");
+  std::vector<char> img(ar.total, 0);
+  bind_ns(E, base, L, img);
+  const NsGroup& g = E.groups[0];
+  d.w = in->data;
+  d.m = nullptr;
+  d.x = g.X[0];
+  d.x_final = g.X[steps & 1];
+  d.out = out->data;
+  d.norm2 = E.d_norm2;
+  d.ldx = g.l_pad;
+  d.grad_slot = 0;
+  d.transposed = in->rows > in->cols ? 1 : 0;
+  d.wdt = in->dtype;
+  d.odt = out->dtype;
+  d.shape_scale = 1.f;
+  memcpy(img.data() + off_mat, &d, sizeof(d));
+  memcpy(img.data() + off_et, et.data(), et.size() * sizeof(ElemTile));
+  auto cleanup = [&](lm_status r) {
+    cudaFreeAsync(base, stream);
+    return r;
+  };
+  e = cudaMemcpyAsync(base, img.data(), ar.total, cudaMemcpyHostToDevice, stream);
+  if (e != cudaSuccess) return cleanup(cuda_fail(e, "msign table upload"));
+  if ((st = encode_maps(E)) != LM_OK) return cleanup(st);
+  MuonConsts mk;
+  memset(&mk, 0, sizeof(mk));
+  mk.eps = (float)eps;
+  mk.ns_steps = steps;
+  MatDesc* dm = reinterpret_cast<MatDesc*>(base + off_mat);
+  ElemTile* de = reinterpret_cast<ElemTile*>(base + off_et);
+  unsigned* dflags = reinterpret_cast<unsigned*>(base + off_flags);
+  e = launch_momentum_norm(E.xdt, dm, de, (int)et.size(), nullptr, mk, 1, stream);
+  if (e != cudaSuccess) return cleanup(cuda_fail(e, "norm kernel launch"));
+  NsCoeffs co{(float)a, (float)b, (float)c, (float)eps};
+  if ((st = run_ns(E, steps, co, dflags, stream)) != LM_OK) return cleanup(st);
+  e = launch_finalize(E.xdt, dm, de, (int)et.size(), mk, 1, dflags, stream);
+  if (e != cudaSuccess) return cleanup(cuda_fail(e, "output kernel launch"));
+  return cleanup(LM_OK);
+}
+
+}  // extern "C"

@@ -1,0 +1,145 @@
+// Internal declarations shared by the library's translation units: device
+// tables built by lm_create and the launchers each kernel file provides.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "lionmuon.h"
+
+namespace lm {
+
+constexpr int kPtrsPerUpload = 1024;   // pointers per pointer-upload launch
+
+// ---------------------------------------------------------------------------
+// Lion multi-tensor step (Algorithm 1, Lion branch + momentum update)
+// ---------------------------------------------------------------------------
+struct LionTensor {
+  void* w;         // bf16 or fp32 parameter (dtype fixed per table)
+  float* m;        // fp32 momentum
+  int64_t n;       // elements
+  int32_t grad_slot;   // index into the device grad-pointer table
+  int32_t pad;
+};
+struct LionChunk {
+  int32_t tensor;  // index into the LionTensor table
+  int32_t pad;
+  int64_t begin;   // first element (multiple of 8)
+  int64_t count;   // elements
+};
+struct LionConsts {
+  float b1, c1, b2, c2, eL, lam;
+};
+
+// Launch the Lion kernel over a chunk table whose tensors all have dtype dt.
+cudaError_t launch_lion(lm_dtype dt, const LionTensor* tensors, const LionChunk* chunks,
+                        int nchunks, const void* const* grads, LionConsts k,
+                        int grid, cudaStream_t st);
+int lion_grid_size(lm_dtype dt);
+
+// ---------------------------------------------------------------------------
+// Muon element-wise kernels: momentum + norm -> X0 (K2), finalize (K6)
+// ---------------------------------------------------------------------------
+struct MatDesc {
+  void* w;          // parameter (rows x cols, dtype wdt); for msign: the input
+  float* m;         // momentum (NULL for msign: no momentum)
+  void* x;          // X buffer base for this matrix (wide orientation, s_pad x l_pad)
+  void* x_final;    // the buffer holding X_K after the NS iterations
+  void* out;        // msign output (rows x cols, dtype odt), or NULL
+  double* norm2;    // Frobenius-norm^2 accumulator of G_hat
+  int64_t rows, cols;
+  int64_t ldx;      // row pitch of X (elements) = l_pad
+  int32_t grad_slot;
+  int32_t transposed;   // rows > cols: X = G_hat^T
+  int32_t wdt;      // lm_dtype of w (and the gradient)
+  int32_t odt;      // lm_dtype of out
+  float shape_scale;    // 0.2*sqrt(max(rows, cols))
+  int32_t tiles_r, tiles_c;   // tile grid of the source matrix
+};
+// One entry per CTA: the matrix and the tile; tile < 0 is an empty cluster slot.
+struct ElemTile {
+  int32_t mat;
+  int32_t tile;
+};
+struct MuonConsts {
+  float b1, c1, b2, c2;   // interpolation / momentum constants
+  float eM, lam;          // Muon learning rate and weight decay
+  float eps;              // NS normalisation eps
+  int32_t ns_steps;
+};
+constexpr int kElemTileR = 64;    // tile rows of the source matrix
+constexpr int kElemTileC = 128;   // tile cols of the source matrix
+constexpr int kNormCluster = 8;   // CTAs per cluster in the norm reduction
+
+// mode 0: Muon momentum step (G_hat from grads + momentum, M update)
+// mode 1: msign input (G_hat = input tensor, no momentum)
+cudaError_t launch_momentum_norm(lm_dtype xdt, const MatDesc* mats, const ElemTile* tiles,
+                                 int ntiles, const void* const* grads, MuonConsts k,
+                                 int mode, cudaStream_t st);
+// mode 0: W <- W - eM (scale X_K' + lam W); mode 1: out = X_K'
+// where X_K' = X_K, or X_K / (||G_hat|| + eps) when ns_steps == 0.
+cudaError_t launch_finalize(lm_dtype xdt, const MatDesc* mats, const ElemTile* tiles,
+                            int ntiles, MuonConsts k, int mode, unsigned* flags,
+                            cudaStream_t st);
+
+// ---------------------------------------------------------------------------
+// Newton-Schulz GEMM phases (grouped over same-shape matrices)
+// ---------------------------------------------------------------------------
+enum NsPhase { NS_GRAM = 0, NS_POLY = 1, NS_APPLY = 2 };
+
+struct NsGroup {
+  int32_t count;          // matrices in the group
+  int32_t s, l;           // true sizes (s = min, l = max)
+  int32_t s_pad, l_pad;   // padded sizes of the workspace buffers
+  int32_t first_mat;      // index of the group's first matrix in the norm array
+  void* X[2];             // ping-pong X: count x s_pad x l_pad
+  void* A;                // count x s_pad x s_pad
+  void* B;                // count x s_pad x s_pad
+};
+// Tile work item: group, matrix-in-group, tile row, tile col.
+struct NsTile {
+  uint16_t group, mat, tm, tn;
+};
+constexpr int kMaxGroupsTc = 8;   // groups per tensor-core launch
+
+struct NsCoeffs {
+  float a, b, c, eps;
+};
+
+// Tensor-core path (bf16 operands, fp32 accumulation in TMEM).
+constexpr int kTcBM = 128, kTcBN = 256, kTcBK = 64;
+int tc_pad_s(int s);
+int tc_pad_l(int l);
+// Tensor maps for one group: K-major boxes (64 x 128) on X0, X1, A, B and
+// MN-major boxes (64 x 64) on X0, X1.
+struct TcGroupMaps {
+  CUtensorMap xk[2];
+  CUtensorMap a;
+  CUtensorMap b;
+  CUtensorMap xmn[2];
+};
+cudaError_t tc_encode_group_maps(const NsGroup& g, TcGroupMaps* maps);
+cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* groups,
+                         const TcGroupMaps* maps, const NsTile* tiles, int ntiles,
+                         const double* norm2, NsCoeffs co, unsigned* flags, cudaStream_t st);
+
+// fp32 CUDA-core path.
+constexpr int kSimtBM = 64, kSimtBN = 64;
+int simt_pad(int x);
+cudaError_t launch_ns_simt(NsPhase ph, int iter, int ngroups, const NsGroup* dgroups,
+                           const NsTile* tiles, int ntiles, const double* norm2, NsCoeffs co,
+                           cudaStream_t st);
+constexpr int kMaxGroupsSimt = 64;
+
+// Tile lists for a phase (host side).  bm/bn are the tile sizes.
+void count_launch();
+
+// Pointer table upload (grads) as a kernel with the pointers in its parameters.
+struct PtrUpload {
+  const void* p[kPtrsPerUpload];
+};
+cudaError_t launch_upload_ptrs(const void** dst, const PtrUpload& src, int count,
+                               cudaStream_t st);
+
+}  // namespace lm

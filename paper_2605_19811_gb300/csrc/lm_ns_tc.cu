@@ -1,0 +1,536 @@
+// Tensor-core Newton-Schulz phases for sm_103a: tcgen05.mma (bf16 operands,
+// fp32 accumulators in TMEM), operands staged by TMA into 128-byte-swizzled
+// shared memory, a persistent grouped schedule over all same-shape matrices.
+//
+// Per NS iteration (Section 2, odd-polynomial Newton-Schulz), with X in the
+// wide orientation (s x l) and the normalisation X / (||G_hat||_F + eps)
+// folded into iteration 0:
+//   GRAM : A  = X X^T          K = l, upper-triangle tiles, mirrored store
+//   POLY : B  = b A + c A A    K = s, upper-triangle tiles, mirrored store;
+//                              the epilogue reads the A tile
+//   APPLY: X' = a X + B X      K = s, all tiles; the epilogue reads the X tile,
+//                              X enters the MMA as an MN-major operand
+// A and A A are symmetric, so A A = A A^T and both GEMM operands of GRAM and
+// POLY are K-major rows of the same matrix.
+//
+// CTA roles (192 threads, one CTA per SM):
+//   warp 0  TMA producer (one elected lane), 4-stage smem ring
+//   warp 1  TMEM allocator + MMA issuer (one elected lane)
+//   warps 2-5 epilogue: tcgen05.ld from TMEM, fused polynomial combination,
+//           bf16 stores (direct + mirrored)
+// Two 256-column accumulators in TMEM let the epilogue of one tile overlap the
+// main loop of the next.  Every mbarrier wait is bounded in time; a wait that
+// gives up sets LM_FLAG_TIMEOUT, makes the other roles stop, waits (bounded)
+// for its own copies and MMAs, frees TMEM and returns.
+#include <cuda_bf16.h>
+#include <cudaTypedefs.h>
+
+#include "lm_internal.h"
+
+namespace lm {
+namespace {
+
+constexpr int BM = kTcBM, BN = kTcBN, BK = kTcBK;
+constexpr int kStages = 4;
+constexpr int kABytes = BM * BK * 2;           // 16 KB
+constexpr int kBBytes = BN * BK * 2;           // 32 KB
+constexpr int kStageBytes = kABytes + kBBytes; // 48 KB
+constexpr int kThreads = 192;
+constexpr int kTmemCols = 2 * BN;              // two accumulators
+constexpr uint64_t kWaitLimitNs = 5000000000ull;   // 5 s
+constexpr size_t kSmemBytes = 1024 /*align slack*/ + (size_t)kStages * kStageBytes + 256;
+
+struct TcParams {
+  TcGroupMaps maps[kMaxGroupsTc];
+  NsGroup groups[kMaxGroupsTc];
+  const NsTile* tiles;
+  int ntiles;
+  int phase;
+  int iter;
+  const double* norm2;
+  NsCoeffs co;
+  unsigned* flags;
+};
+
+// ------------------------------- PTX wrappers -------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ uint64_t globaltimer() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+               "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait for the phase with the given parity.  Returns false if the
+// time limit passed or another role asked to stop.
+__device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                       uint64_t limit_ns) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer();
+  for (uint32_t i = 1;; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((i & 255u) == 0) {
+      if (*abort_flag) return false;
+      if (globaltimer() - t0 > limit_ns) return false;
+    }
+  }
+}
+__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, uint64_t* bar,
+                                            int c0, int c1, int c2) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2)
+      : "memory");
+}
+__device__ __forceinline__ void prefetch_map(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_alloc(uint32_t* dst, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                   smem_u32(dst)),
+               "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                          uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          smem_u32(bar))
+      : "memory");
+}
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32"
+      " {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15,"
+      " %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31},"
+      " [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor (tcgen05), 128-byte swizzle.
+//   bits 0-13  start address >> 4
+//   bits 16-29 leading-dimension byte offset >> 4
+//   bits 32-45 stride-dimension byte offset >> 4
+//   bits 46-47 descriptor version (1)
+//   bits 61-63 layout: 2 = 128-byte swizzle
+// K-major: rows of 128 B (64 bf16 of K), 8-row groups 1024 B apart (SBO);
+//          LBO unused.  MN-major: 64 MN-elements per 128-B row, one row per K,
+//          8-K-row groups 1024 B apart (SBO), 64-element MN atoms LBO apart.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
+}
+// Instruction descriptor, kind::f16: D fp32, A and B bf16, A K-major,
+// B K-major or MN-major, N >> 3 at bit 17, M >> 4 at bit 24.
+__host__ __device__ constexpr uint32_t make_idesc(int m, int n, bool b_mn_major) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((b_mn_major ? 1u : 0u) << 16) |
+         ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
+}
+
+__device__ __forceinline__ float bf_lo(uint32_t v) { return __uint_as_float(v << 16); }
+__device__ __forceinline__ float bf_hi(uint32_t v) { return __uint_as_float(v & 0xFFFF0000u); }
+__device__ __forceinline__ uint32_t pack_bf2(float lo, float hi) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+
+// ------------------------------- the kernel ---------------------------------
+__global__ void __launch_bounds__(kThreads, 1) ns_tc_kernel(const __grid_constant__ TcParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)kStages * kStageBytes);
+  uint64_t* empty = full + kStages;
+  uint64_t* accfull = empty + kStages;
+  uint64_t* accempty = accfull + 2;
+  uint64_t* done = accempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int phase = p.phase;
+  const int cur = p.iter & 1;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&accfull[b], 1);
+      mbar_init(&accempty[b], 4);
+    }
+    mbar_init(done, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  auto give_up = [&]() {
+    *abort_flag = 1;
+    atomicOr(p.flags, LM_FLAG_TIMEOUT);
+  };
+
+  if (warp == 0) {
+    // ------------------------------ producer ------------------------------
+    if (lane == 0) {
+      int armed[kStages];
+      for (int s = 0; s < kStages; ++s) armed[s] = -1;
+      int stage = 0;
+      uint32_t ph = 0;
+      bool ok = true;
+      for (int w = blockIdx.x; ok && w < p.ntiles; w += gridDim.x) {
+        const NsTile t = p.tiles[w];
+        const NsGroup& g = p.groups[t.group];
+        const TcGroupMaps& mp = p.maps[t.group];
+        const CUtensorMap* mapA;
+        const CUtensorMap* mapB;
+        int K;
+        if (phase == NS_GRAM) {
+          mapA = &mp.xk[cur]; mapB = &mp.xk[cur]; K = g.l_pad;
+        } else if (phase == NS_POLY) {
+          mapA = &mp.a; mapB = &mp.a; K = g.s_pad;
+        } else {
+          mapA = &mp.b; mapB = &mp.xmn[cur]; K = g.s_pad;
+        }
+        const int nk = K / BK;
+        for (int kb = 0; kb < nk; ++kb) {
+          if (!mbar_wait(&empty[stage], ph ^ 1u, abort_flag, kWaitLimitNs)) {
+            give_up();
+            ok = false;
+            break;
+          }
+          uint8_t* sa = smem + (size_t)stage * kStageBytes;
+          uint8_t* sb = sa + kABytes;
+          mbar_arrive_expect_tx(&full[stage], kStageBytes);
+          armed[stage] = (int)ph;
+          const int k0 = kb * BK;
+          tma_load_3d(sa, mapA, &full[stage], k0, t.tm * BM, t.mat);
+          if (phase != NS_APPLY) {
+            tma_load_3d(sb, mapB, &full[stage], k0, t.tn * BN, t.mat);
+            tma_load_3d(sb + kBBytes / 2, mapB, &full[stage], k0, t.tn * BN + BN / 2, t.mat);
+          } else {
+#pragma unroll
+            for (int q = 0; q < BN / 64; ++q)
+              tma_load_3d(sb + q * (64 * BK * 2), mapB, &full[stage], t.tn * BN + 64 * q, k0, t.mat);
+          }
+          if (++stage == kStages) {
+            stage = 0;
+            ph ^= 1u;
+          }
+        }
+      }
+      if (!ok) {
+        // let the copies already issued land before the CTA exits
+        for (int s = 0; s < kStages; ++s)
+          if (armed[s] >= 0) {
+            volatile int never = 0;
+            mbar_wait(&full[s], (uint32_t)armed[s], &never, 100000000ull);
+          }
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------ MMA issuer -----------------------------
+    if (lane == 0) {
+      const uint32_t idesc = make_idesc(BM, BN, phase == NS_APPLY);
+      int stage = 0;
+      uint32_t ph = 0;
+      int ab = 0;
+      uint32_t aph = 0;
+      bool ok = true;
+      for (int w = blockIdx.x; ok && w < p.ntiles; w += gridDim.x) {
+        const NsTile t = p.tiles[w];
+        const NsGroup& g = p.groups[t.group];
+        const int K = (phase == NS_GRAM) ? g.l_pad : g.s_pad;
+        const int nk = K / BK;
+        if (!mbar_wait(&accempty[ab], aph ^ 1u, abort_flag, kWaitLimitNs)) {
+          give_up();
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)(ab * BN);
+        for (int kb = 0; kb < nk; ++kb) {
+          if (!mbar_wait(&full[stage], ph, abort_flag, kWaitLimitNs)) {
+            give_up();
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + (size_t)stage * kStageBytes);
+          const uint32_t sb = sa + kABytes;
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk) {
+            const uint64_t adesc = sw128_desc(sa + kk * 32, 16, 1024);
+            const uint64_t bdesc = (phase == NS_APPLY)
+                                       ? sw128_desc(sb + kk * 2048, 64 * BK * 2, 1024)
+                                       : sw128_desc(sb + kk * 32, 16, 1024);
+            umma_bf16(d_tmem, adesc, bdesc, idesc, (kb | kk) != 0 ? 1u : 0u);
+          }
+          umma_commit(&empty[stage]);
+          if (++stage == kStages) {
+            stage = 0;
+            ph ^= 1u;
+          }
+        }
+        if (!ok) break;
+        umma_commit(&accfull[ab]);
+        if (++ab == 2) {
+          ab = 0;
+          aph ^= 1u;
+        }
+      }
+      // all issued MMAs complete before TMEM is released
+      umma_commit(done);
+      volatile int never = 0;
+      mbar_wait(done, 0, &never, 100000000ull);
+    }
+  } else {
+    // ------------------------------ epilogue -------------------------------
+    const int q = warp & 3;             // TMEM lane quadrant of this warp
+    const int row = q * 32 + lane;      // row of the tile owned by this thread
+    int ab = 0;
+    uint32_t aph = 0;
+    for (int w = blockIdx.x; w < p.ntiles; w += gridDim.x) {
+      const NsTile t = p.tiles[w];
+      const NsGroup& g = p.groups[t.group];
+      bool ok = true;
+      if (lane == 0) ok = mbar_wait(&accfull[ab], aph, abort_flag, kWaitLimitNs);
+      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      if (!ok) {
+        if (lane == 0) give_up();
+        break;
+      }
+      tc_fence_after();
+
+      float nscale = 1.f;
+      if (p.iter == 0) {
+        const float n = (float)sqrt(p.norm2[g.first_mat + t.mat]) + p.co.eps;
+        nscale = (phase == NS_GRAM) ? 1.f / (n * n) : (phase == NS_APPLY ? 1.f / n : 1.f);
+      }
+      const int i = t.tm * BM + row;
+      const size_t sq = (size_t)g.s_pad * g.s_pad;
+      const size_t xs = (size_t)g.s_pad * g.l_pad;
+      const int ncols = (phase == NS_APPLY) ? g.l : g.s;
+      const int ld = (phase == NS_APPLY) ? g.l_pad : g.s_pad;
+      const int jmax = (phase == NS_APPLY) ? g.l_pad : g.s_pad;
+      __nv_bfloat16* out;
+      const __nv_bfloat16* aux = nullptr;
+      if (phase == NS_GRAM) {
+        out = static_cast<__nv_bfloat16*>(g.A) + t.mat * sq;
+      } else if (phase == NS_POLY) {
+        out = static_cast<__nv_bfloat16*>(g.B) + t.mat * sq;
+        aux = static_cast<const __nv_bfloat16*>(g.A) + t.mat * sq;
+      } else {
+        out = static_cast<__nv_bfloat16*>(g.X[cur ^ 1]) + t.mat * xs;
+        aux = static_cast<const __nv_bfloat16*>(g.X[cur]) + t.mat * xs;
+      }
+      const bool sym = phase != NS_APPLY;
+      for (int ch = 0; ch < BN / 32; ++ch) {
+        uint32_t r[32];
+        __syncwarp();   // tcgen05.ld is warp-collective: reconverge first
+        tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * BN + ch * 32), r);
+        const int j0 = t.tn * BN + ch * 32;
+        if (j0 >= jmax) continue;                 // beyond the padded matrix
+        if (sym && j0 + 31 < i) continue;         // strictly below the diagonal
+        float v[32];
+        if (aux != nullptr) {
+          const uint4* ap = reinterpret_cast<const uint4*>(aux + (size_t)i * ld + j0);
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const uint4 a4 = ap[u];
+            const uint32_t aw[4] = {a4.x, a4.y, a4.z, a4.w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              v[u * 8 + 2 * e] = bf_lo(aw[e]);
+              v[u * 8 + 2 * e + 1] = bf_hi(aw[e]);
+            }
+          }
+        }
+#pragma unroll
+        for (int e = 0; e < 32; ++e) {
+          const float acc = __uint_as_float(r[e]);
+          const int j = j0 + e;
+          float o;
+          if (phase == NS_GRAM) o = acc * nscale;
+          else if (phase == NS_POLY) o = p.co.b * v[e] + p.co.c * acc;
+          else o = (p.co.a * v[e] + acc) * nscale;
+          v[e] = (i < g.s && j < ncols) ? o : 0.f;
+        }
+        if (!sym || j0 >= i) {
+          // whole chunk on or above the diagonal: 16-byte direct stores
+          uint4* op = reinterpret_cast<uint4*>(out + (size_t)i * ld + j0);
+#pragma unroll
+          for (int u = 0; u < 4; ++u)
+            op[u] = make_uint4(pack_bf2(v[u * 8 + 0], v[u * 8 + 1]), pack_bf2(v[u * 8 + 2], v[u * 8 + 3]),
+                               pack_bf2(v[u * 8 + 4], v[u * 8 + 5]), pack_bf2(v[u * 8 + 6], v[u * 8 + 7]));
+        } else {
+#pragma unroll
+          for (int e = 0; e < 32; ++e)
+            if (j0 + e >= i) out[(size_t)i * ld + j0 + e] = __float2bfloat16_rn(v[e]);
+        }
+        if (sym) {
+          // mirrored half: consecutive lanes write consecutive columns
+#pragma unroll
+          for (int e = 0; e < 32; ++e)
+            if (j0 + e > i) out[(size_t)(j0 + e) * ld + i] = __float2bfloat16_rn(v[e]);
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&accempty[ab]);
+      if (++ab == 2) {
+        ab = 0;
+        aph ^= 1u;
+      }
+    }
+  }
+
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, kTmemCols);
+  }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 get_encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (fn == nullptr) {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+  }
+  return fn;
+}
+
+cudaError_t encode_3d(CUtensorMap* m, void* base, uint64_t inner, uint64_t rows, uint64_t count,
+                      uint32_t box_inner, uint32_t box_rows) {
+  PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode_fn();
+  if (enc == nullptr) return cudaErrorNotSupported;
+  const cuuint64_t dims[3] = {inner, rows, count};
+  const cuuint64_t strides[2] = {inner * 2, inner * rows * 2};
+  const cuuint32_t box[3] = {box_inner, box_rows, 1};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, base, dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+}  // namespace
+
+int tc_pad_s(int s) { return (s + BM - 1) / BM * BM; }
+int tc_pad_l(int l) { return (l + BN - 1) / BN * BN; }
+
+cudaError_t tc_encode_group_maps(const NsGroup& g, TcGroupMaps* maps) {
+  cudaError_t e;
+  for (int b = 0; b < 2; ++b) {
+    if ((e = encode_3d(&maps->xk[b], g.X[b], g.l_pad, g.s_pad, g.count, BK, BM)) != cudaSuccess) return e;
+    if ((e = encode_3d(&maps->xmn[b], g.X[b], g.l_pad, g.s_pad, g.count, 64, BK)) != cudaSuccess) return e;
+  }
+  if ((e = encode_3d(&maps->a, g.A, g.s_pad, g.s_pad, g.count, BK, BM)) != cudaSuccess) return e;
+  if ((e = encode_3d(&maps->b, g.B, g.s_pad, g.s_pad, g.count, BK, BM)) != cudaSuccess) return e;
+  return cudaSuccess;
+}
+
+cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* groups,
+                         const TcGroupMaps* maps, const NsTile* tiles, int ntiles,
+                         const double* norm2, NsCoeffs co, unsigned* flags, cudaStream_t st) {
+  if (ntiles <= 0) return cudaSuccess;
+  if (ngroups < 1 || ngroups > kMaxGroupsTc) return cudaErrorInvalidValue;
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(ns_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)kSmemBytes);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  TcParams prm;
+  memset(&prm, 0, sizeof(prm));
+  for (int gi = 0; gi < ngroups; ++gi) {
+    prm.maps[gi] = maps[gi];
+    prm.groups[gi] = groups[gi];
+  }
+  prm.tiles = tiles;
+  prm.ntiles = ntiles;
+  prm.phase = (int)ph;
+  prm.iter = iter;
+  prm.norm2 = norm2;
+  prm.co = co;
+  prm.flags = flags;
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  int grid = sms < ntiles ? sms : ntiles;
+  count_launch();
+  ns_tc_kernel<<<grid, kThreads, kSmemBytes, st>>>(prm);
+  return cudaGetLastError();
+}
+
+}  // namespace lm
