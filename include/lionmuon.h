@@ -129,6 +129,27 @@ lm_status lm_msign_ns(const lm_tensor* in, lm_tensor* out, int steps, double a,
                       double b, double c, double eps, int precision,
                       void* cuda_stream);
 
+/* The same computation as lm_msign_ns, for callers that cannot allocate
+ * device memory while they run: for example a program whose device memory is
+ * fully budgeted up front by its own allocator, or a latency-critical loop in
+ * which cudaMalloc/cudaFree (cudaFree synchronises the device) are not
+ * acceptable.  This entry point allocates nothing.  Its workspace is a fixed
+ * 64 MiB area inside the library (a static device array that every GPU which
+ * loads the library holds until the process exits); a matrix whose workspace
+ * does not fit is rejected with LM_ERR_UNSUPPORTED and a message giving the
+ * bytes needed.  Roughly: bf16 precision fits up to 1280 x 5120, fp32
+ * precision up to 1024 x 4096.  The caller still provides in and out.
+ * The first call on a device looks up the area's device address on that
+ * device (cudaGetSymbolAddress); make that first call before any stream
+ * capture.  All calls share the one area, which keeps the last call's data:
+ * each call clears what must start at zero, and calls whose GPU work may
+ * overlap (unordered streams or threads) race on the area and must be
+ * serialised by the caller.  Arguments and errors as for lm_msign_ns.
+ * The paper has no counterpart of this call; it is a deployment variant. */
+lm_status lm_msign_ns_noalloc(const lm_tensor* in, lm_tensor* out, int steps,
+                              double a, double b, double c, double eps,
+                              int precision, void* cuda_stream);
+
 /* A read-only view of parameter i's momentum buffer (fp32, the shape of
  * params[i], device memory owned by the state).  For checkpointing and tests.
  * Errors: LM_ERR_INVALID_ARG (NULL, i out of range). */

@@ -195,6 +195,8 @@ void build_elem_tiles(const std::vector<MatDesc>& mats, std::vector<ElemTile>& o
 
 }  // namespace
 
+lm_status set_error(lm_status st, const char* msg) { return fail(st, "%s", msg); }
+
 // ---------------------------------------------------------------------------
 // Newton-Schulz engine shared by lm_step and lm_msign_ns
 // ---------------------------------------------------------------------------

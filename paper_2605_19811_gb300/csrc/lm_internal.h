@@ -132,8 +132,9 @@ cudaError_t launch_ns_simt(NsPhase ph, int iter, int ngroups, const NsGroup* dgr
                            cudaStream_t st);
 constexpr int kMaxGroupsSimt = 64;
 
-// Tile lists for a phase (host side).  bm/bn are the tile sizes.
+// Launch accounting (lm_kernel_launch_count) and the thread's last-error text.
 void count_launch();
+lm_status set_error(lm_status st, const char* msg);
 
 // Pointer table upload (grads) as a kernel with the pointers in its parameters.
 struct PtrUpload {

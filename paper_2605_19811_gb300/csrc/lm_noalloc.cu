@@ -1,0 +1,259 @@
+// lm_msign_ns_noalloc: the Newton-Schulz msign approximation of lm_msign_ns,
+// run in a fixed scratch area that is part of the library image instead of
+// memory allocated per call.
+//
+// The scratch is a file-scope __device__ array of kNoAllocScratchBytes.  Every
+// GPU that loads this library holds it until the process exits.  Host code
+// cannot use the array's name as a device address (on the host it names a
+// stand-in object), so the device address is looked up once per device with
+// cudaGetSymbolAddress, with that device current, on the first call made on
+// that device, and cached.
+//
+// All calls share the array and it keeps what the last call left there: the
+// parts that must start at zero (the padded X0 buffer, the norm accumulator,
+// the status word) are cleared on every call, and calls whose GPU work
+// overlaps (different streams, or different host threads, without ordering
+// between them) race on it.
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+
+#include "lm_internal.h"
+
+namespace lm {
+namespace {
+
+constexpr size_t kNoAllocScratchBytes = (size_t)64 << 20;   // 64 MiB
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_scratch_mu;
+char* g_scratch_addr[kMaxDevices] = {nullptr};
+
+cudaError_t scratch_address(int dev, char** out) {
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (g_scratch_addr[dev] == nullptr) {
+    void* p = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess) return e;
+    g_scratch_addr[dev] = static_cast<char*>(p);
+  }
+  *out = g_scratch_addr[dev];
+  return cudaSuccess;
+}
+
+size_t align256(size_t x) { return (x + 255) / 256 * 256; }
+
+// Number of tiles of one Newton-Schulz phase for a single matrix, and the
+// (tm, tn) of tile k in the same order the allocating path builds them
+// (row-major; symmetric phases keep tiles that reach the diagonal).
+__host__ __device__ inline int phase_tiles(int phase, int s_pad, int l_pad, int bm, int bn) {
+  const int tms = s_pad / bm;
+  const int ncol = phase == NS_APPLY ? l_pad : s_pad;
+  const int tns = (ncol + bn - 1) / bn;
+  if (phase == NS_APPLY) return tms * tns;
+  int n = 0;
+  for (int tm = 0; tm < tms; ++tm)
+    for (int tn = 0; tn < tns; ++tn)
+      if ((int64_t)(tn + 1) * bn > (int64_t)tm * bm) ++n;
+  return n;
+}
+
+struct BuildArgs {
+  MatDesc mat;
+  NsGroup group;
+  MatDesc* d_mat;
+  NsGroup* d_group;
+  ElemTile* d_etiles;
+  int n_etiles;
+  int n_real_etiles;
+  NsTile* d_tiles[3];
+  int bm, bn;
+  double* d_norm2;
+  unsigned* d_flags;
+};
+
+// Writes the descriptor tables of one msign call into the scratch area.
+__global__ void build_tables_kernel(BuildArgs a) {
+  if (blockIdx.x != 0) return;
+  if (threadIdx.x == 0) {
+    *a.d_mat = a.mat;
+    *a.d_group = a.group;
+    *a.d_norm2 = 0.0;
+    *a.d_flags = 0u;
+  }
+  for (int i = threadIdx.x; i < a.n_etiles; i += blockDim.x)
+    a.d_etiles[i] = ElemTile{0, i < a.n_real_etiles ? i : -1};
+  if (threadIdx.x < 3) {
+    const int ph = threadIdx.x;
+    const NsGroup& g = a.group;
+    const int tms = g.s_pad / a.bm;
+    const int ncol = ph == NS_APPLY ? g.l_pad : g.s_pad;
+    const int tns = (ncol + a.bn - 1) / a.bn;
+    int k = 0;
+    for (int tm = 0; tm < tms; ++tm)
+      for (int tn = 0; tn < tns; ++tn) {
+        if (ph != NS_APPLY && (int64_t)(tn + 1) * a.bn <= (int64_t)tm * a.bm) continue;
+        a.d_tiles[ph][k++] = NsTile{0, 0, (uint16_t)tm, (uint16_t)tn};
+      }
+  }
+}
+
+}  // namespace
+}  // namespace lm
+
+using namespace lm;
+
+extern "C" lm_status lm_msign_ns_noalloc(const lm_tensor* in, lm_tensor* out, int steps, double a,
+                                         double b, double c, double eps, int precision,
+                                         void* cuda_stream) {
+  if (in == nullptr || out == nullptr) return set_error(LM_ERR_INVALID_ARG, "in/out is NULL");
+  for (const lm_tensor* t : {in, static_cast<const lm_tensor*>(out)}) {
+    if (t->dtype != LM_BF16 && t->dtype != LM_F32) return set_error(LM_ERR_DTYPE, "unsupported dtype");
+    if (t->rows < 2 || t->cols < 2) return set_error(LM_ERR_INVALID_ARG, "msign needs rows, cols >= 2");
+    if (t->data == nullptr) return set_error(LM_ERR_INVALID_ARG, "NULL data");
+    if (reinterpret_cast<uintptr_t>(t->data) % 16 != 0)
+      return set_error(LM_ERR_ALIGN, "data pointer not 16-byte aligned");
+  }
+  if (out->rows != in->rows || out->cols != in->cols)
+    return set_error(LM_ERR_INVALID_ARG, "out shape differs from in");
+  if (steps < 0 || steps > 64) return set_error(LM_ERR_INVALID_ARG, "steps must be in [0, 64]");
+  if (!std::isfinite(a) || !std::isfinite(b) || !std::isfinite(c) || !std::isfinite(eps) || eps < 0)
+    return set_error(LM_ERR_INVALID_ARG, "coefficients must be finite, eps >= 0");
+  if (precision != LM_BF16 && precision != LM_F32)
+    return set_error(LM_ERR_INVALID_ARG, "precision must be LM_BF16 or LM_F32");
+  if (in->rows > 65536 || in->cols > 65536)
+    return set_error(LM_ERR_UNSUPPORTED, "lm_msign_ns_noalloc: matrix dimension above 65536");
+
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return set_error(LM_ERR_CUDA, "no CUDA device");
+  int major = 0, minor = 0;
+  cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+  cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+  if (major != 10 || minor != 3) return set_error(LM_ERR_UNSUPPORTED, "device is not sm_103");
+  if (dev >= kMaxDevices) return set_error(LM_ERR_UNSUPPORTED, "device ordinal above 63");
+
+  // Layout of this call inside the scratch area.
+  const lm_dtype xdt = precision == LM_F32 ? LM_F32 : LM_BF16;
+  const int s = (int)std::min(in->rows, in->cols), l = (int)std::max(in->rows, in->cols);
+  const int s_pad = xdt == LM_BF16 ? tc_pad_s(s) : simt_pad(s);
+  const int l_pad = xdt == LM_BF16 ? tc_pad_l(l) : simt_pad(l);
+  const int bm = xdt == LM_BF16 ? kTcBM : kSimtBM, bn = xdt == LM_BF16 ? kTcBN : kSimtBN;
+  const size_t es = xdt == LM_BF16 ? 2 : 4;
+  const int tiles_r = (int)((in->rows + kElemTileR - 1) / kElemTileR);
+  const int tiles_c = (int)((in->cols + kElemTileC - 1) / kElemTileC);
+  const int n_real_et = tiles_r * tiles_c;
+  const int n_et = (n_real_et + kNormCluster - 1) / kNormCluster * kNormCluster;
+  int ntiles[3];
+  for (int ph = 0; ph < 3; ++ph) ntiles[ph] = phase_tiles(ph, s_pad, l_pad, bm, bn);
+
+  size_t off = 0;
+  const size_t off_flags = off;   off = align256(off + sizeof(unsigned));
+  const size_t off_norm = off;    off = align256(off + sizeof(double));
+  const size_t off_mat = off;     off = align256(off + sizeof(MatDesc));
+  const size_t off_group = off;   off = align256(off + sizeof(NsGroup));
+  const size_t off_et = off;      off = align256(off + (size_t)n_et * sizeof(ElemTile));
+  size_t off_tiles[3];
+  for (int ph = 0; ph < 3; ++ph) {
+    off_tiles[ph] = off;
+    off = align256(off + (size_t)ntiles[ph] * sizeof(NsTile));
+  }
+  const size_t xbytes = (size_t)s_pad * l_pad * es, abytes = (size_t)s_pad * s_pad * es;
+  const size_t off_x0 = off;  off = align256(off + xbytes);
+  const size_t off_x1 = off;  off = align256(off + xbytes);
+  const size_t off_a = off;   off = align256(off + abytes);
+  const size_t off_b = off;   off = align256(off + abytes);
+  if (off > kNoAllocScratchBytes) {
+    char msg[256];
+    snprintf(msg, sizeof(msg),
+             "lm_msign_ns_noalloc: a %lldx%lld matrix needs %zu bytes of scratch; the limit is %zu "
+             "(64 MiB)", (long long)in->rows, (long long)in->cols, off, kNoAllocScratchBytes);
+    return set_error(LM_ERR_UNSUPPORTED, msg);
+  }
+
+  char* base = nullptr;
+  cudaError_t e = scratch_address(dev, &base);
+  if (e != cudaSuccess) return set_error(LM_ERR_CUDA, cudaGetErrorString(e));
+  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+
+  NsGroup g;
+  memset(&g, 0, sizeof(g));
+  g.count = 1;
+  g.s = s;
+  g.l = l;
+  g.s_pad = s_pad;
+  g.l_pad = l_pad;
+  g.first_mat = 0;
+  g.X[0] = base + off_x0;
+  g.X[1] = base + off_x1;
+  g.A = base + off_a;
+  g.B = base + off_b;
+
+  BuildArgs ba;
+  memset(&ba, 0, sizeof(ba));
+  MatDesc& d = ba.mat;
+  d.w = in->data;
+  d.m = nullptr;
+  d.x = g.X[0];
+  d.x_final = g.X[steps & 1];
+  d.out = out->data;
+  d.norm2 = reinterpret_cast<double*>(base + off_norm);
+  d.rows = in->rows;
+  d.cols = in->cols;
+  d.ldx = l_pad;
+  d.grad_slot = 0;
+  d.transposed = in->rows > in->cols ? 1 : 0;
+  d.wdt = in->dtype;
+  d.odt = out->dtype;
+  d.shape_scale = 1.f;
+  d.tiles_r = tiles_r;
+  d.tiles_c = tiles_c;
+  ba.group = g;
+  ba.d_mat = reinterpret_cast<MatDesc*>(base + off_mat);
+  ba.d_group = reinterpret_cast<NsGroup*>(base + off_group);
+  ba.d_etiles = reinterpret_cast<ElemTile*>(base + off_et);
+  ba.n_etiles = n_et;
+  ba.n_real_etiles = n_real_et;
+  for (int ph = 0; ph < 3; ++ph) ba.d_tiles[ph] = reinterpret_cast<NsTile*>(base + off_tiles[ph]);
+  ba.bm = bm;
+  ba.bn = bn;
+  ba.d_norm2 = d.norm2;
+  ba.d_flags = reinterpret_cast<unsigned*>(base + off_flags);
+
+  TcGroupMaps maps;
+  if (xdt == LM_BF16) {
+    e = tc_encode_group_maps(g, &maps);
+    if (e != cudaSuccess) return set_error(LM_ERR_CUDA, "cuTensorMapEncodeTiled failed");
+  }
+
+  // X0's padding must read as zero; the other buffers are fully written
+  // before they are read.
+  e = cudaMemsetAsync(g.X[0], 0, xbytes, stream);
+  if (e != cudaSuccess) return set_error(LM_ERR_CUDA, cudaGetErrorString(e));
+  count_launch();
+  build_tables_kernel<<<1, 256, 0, stream>>>(ba);
+  if ((e = cudaGetLastError()) != cudaSuccess) return set_error(LM_ERR_CUDA, cudaGetErrorString(e));
+
+  MuonConsts mk;
+  memset(&mk, 0, sizeof(mk));
+  mk.eps = (float)eps;
+  mk.ns_steps = steps;
+  e = launch_momentum_norm(xdt, ba.d_mat, ba.d_etiles, n_et, nullptr, mk, 1, stream);
+  if (e != cudaSuccess) return set_error(LM_ERR_CUDA, cudaGetErrorString(e));
+  const NsCoeffs co{(float)a, (float)b, (float)c, (float)eps};
+  for (int it = 0; it < steps; ++it)
+    for (int ph = 0; ph < 3; ++ph) {
+      if (xdt == LM_BF16)
+        e = launch_ns_tc((NsPhase)ph, it, 1, &g, &maps, ba.d_tiles[ph], ntiles[ph], d.norm2, co,
+                         ba.d_flags, stream);
+      else
+        e = launch_ns_simt((NsPhase)ph, it, 1, ba.d_group, ba.d_tiles[ph], ntiles[ph], d.norm2, co,
+                           stream);
+      if (e != cudaSuccess) return set_error(LM_ERR_CUDA, cudaGetErrorString(e));
+    }
+  e = launch_finalize(xdt, ba.d_mat, ba.d_etiles, n_et, mk, 1, ba.d_flags, stream);
+  if (e != cudaSuccess) return set_error(LM_ERR_CUDA, cudaGetErrorString(e));
+  return LM_OK;
+}

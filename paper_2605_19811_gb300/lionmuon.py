@@ -26,7 +26,8 @@ STATUS_NAMES = {0: "LM_OK", 1: "LM_ERR_INVALID_ARG", 2: "LM_ERR_DTYPE", 3: "LM_E
 EXPORTED = ("lm_config_default", "lm_create", "lm_step", "lm_set_lr", "lm_msign_ns",
             "lm_get_momentum", "lm_set_momentum", "lm_get_status", "lm_state_bytes",
             "lm_workspace_bytes", "lm_destroy", "lm_status_string", "lm_last_error",
-            "lm_kernel_launch_count", "lm_profile_enable", "lm_profile_read")
+            "lm_kernel_launch_count", "lm_profile_enable", "lm_profile_read",
+            "lm_msign_ns_noalloc")
 
 KERNEL_FAMILIES = ("lion", "momentum_norm", "ns_gemm", "finalize", "other")
 
@@ -81,6 +82,9 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib.lm_msign_ns.argtypes = [P(LmTensor), P(LmTensor), c_int, c_double, c_double, c_double,
                                 c_double, c_int, c_void_p]
     lib.lm_msign_ns.restype = c_int
+    lib.lm_msign_ns_noalloc.argtypes = [P(LmTensor), P(LmTensor), c_int, c_double, c_double, c_double,
+                                        c_double, c_int, c_void_p]
+    lib.lm_msign_ns_noalloc.restype = c_int
     lib.lm_get_momentum.argtypes = [c_void_p, c_int, P(LmTensor)]
     lib.lm_get_momentum.restype = c_int
     lib.lm_set_momentum.argtypes = [c_void_p, c_int, P(LmTensor), c_void_p]
@@ -243,4 +247,15 @@ def msign_ns(x, out, steps: int = 5, a: float = 3.4445, b: float = -4.7750, c: f
     di, do = tensor_desc(x), tensor_desc(out)
     _check(lib, lib.lm_msign_ns(ctypes.byref(di), ctypes.byref(do), steps, a, b, c, eps, precision,
                                 _stream_handle(stream)), "lm_msign_ns")
+    return out
+
+
+def msign_ns_noalloc(x, out, steps: int = 5, a: float = 3.4445, b: float = -4.7750, c: float = 2.0315,
+                     eps: float = 1e-7, precision: int = LM_BF16, stream=None):
+    """out <- NS_steps(x) via lm_msign_ns_noalloc (fixed in-library workspace,
+    no device allocation; calls must not overlap on the GPU)."""
+    lib = load_library()
+    di, do = tensor_desc(x), tensor_desc(out)
+    _check(lib, lib.lm_msign_ns_noalloc(ctypes.byref(di), ctypes.byref(do), steps, a, b, c, eps,
+                                        precision, _stream_handle(stream)), "lm_msign_ns_noalloc")
     return out
