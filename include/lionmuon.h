@@ -195,10 +195,12 @@ uint64_t lm_kernel_launch_count(void);
 typedef enum {
   LM_KERNEL_LION = 0,          /* Lion step (all params, or vectors on Muon steps) */
   LM_KERNEL_MOMENTUM_NORM = 1, /* Muon: G_hat, ||G_hat||_F^2, M update, X0 */
-  LM_KERNEL_NS_GEMM = 2,       /* Newton-Schulz GEMM phases (Gram, polynomial, apply) */
-  LM_KERNEL_FINALIZE = 3,      /* Muon: parameter write */
-  LM_KERNEL_OTHER = 4,         /* gradient-pointer upload, norm reset */
-  LM_KERNEL_FAMILIES = 5
+  LM_KERNEL_NS_GRAM = 2,       /* Newton-Schulz: A = X X^T */
+  LM_KERNEL_NS_POLY = 3,       /* Newton-Schulz: B = b A + c A A */
+  LM_KERNEL_NS_APPLY = 4,      /* Newton-Schulz: X <- a X + B X */
+  LM_KERNEL_FINALIZE = 5,      /* Muon: parameter write */
+  LM_KERNEL_OTHER = 6,         /* gradient-pointer upload, norm reset */
+  LM_KERNEL_FAMILIES = 7
 } lm_kernel_family;
 
 typedef struct {

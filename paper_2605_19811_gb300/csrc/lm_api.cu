@@ -141,6 +141,8 @@ struct NsBatch {
   int g0 = 0, ng = 0;
   NsTile* tiles[3] = {nullptr, nullptr, nullptr};
   int ntiles[3] = {0, 0, 0};
+  int* offsets[3] = {nullptr, nullptr, nullptr};   // per-pair tile ranges (tensor-core path)
+  int npairs[3] = {0, 0, 0};
 };
 
 void build_lion_chunks(const std::vector<LionTensor>& ts, std::vector<LionChunk>& out) {
@@ -158,6 +160,30 @@ void build_lion_chunks(const std::vector<LionTensor>& ts, std::vector<LionChunk>
 
 // Tile list of one phase over groups [g0, g0+ng).  Symmetric phases keep the
 // tiles that reach the diagonal or above; the list is ordered longest K first.
+// Greedy longest-first assignment of tiles (sorted by decreasing cost) to
+// workers: each tile goes to the least-loaded worker.  Output: tiles grouped
+// by worker and the npairs + 1 range starts.
+void balance_tiles(const std::vector<std::pair<int, NsTile>>& sorted, int workers,
+                   std::vector<NsTile>& out, std::vector<int>& offsets) {
+  std::vector<std::vector<NsTile>> per(workers);
+  std::vector<std::pair<int64_t, int>> heap;   // (load, worker), min-heap
+  for (int k = 0; k < workers; ++k) heap.push_back({0, k});
+  auto cmp = [](const std::pair<int64_t, int>& a, const std::pair<int64_t, int>& b) { return a > b; };
+  std::make_heap(heap.begin(), heap.end(), cmp);
+  for (const auto& e : sorted) {
+    std::pop_heap(heap.begin(), heap.end(), cmp);
+    auto& top = heap.back();
+    per[top.second].push_back(e.second);
+    top.first += e.first;
+    std::push_heap(heap.begin(), heap.end(), cmp);
+  }
+  offsets.assign(1, 0);
+  for (int k = 0; k < workers; ++k) {
+    out.insert(out.end(), per[k].begin(), per[k].end());
+    offsets.push_back((int)out.size());
+  }
+}
+
 void build_ns_tiles(const std::vector<NsGroup>& groups, int g0, int ng, int phase, int bm, int bn,
                     std::vector<NsTile>& out) {
   std::vector<std::pair<int, NsTile>> v;
@@ -165,7 +191,7 @@ void build_ns_tiles(const std::vector<NsGroup>& groups, int g0, int ng, int phas
     const NsGroup& g = groups[gi];
     const int ncol = (phase == NS_APPLY) ? g.l_pad : g.s_pad;
     const int K = (phase == NS_GRAM) ? g.l_pad : g.s_pad;
-    const int tms = g.s_pad / bm, tns = (ncol + bn - 1) / bn;
+    const int tms = (g.s_pad + bm - 1) / bm, tns = (ncol + bn - 1) / bn;
     for (int m = 0; m < g.count; ++m)
       for (int tm = 0; tm < tms; ++tm)
         for (int tn = 0; tn < tns; ++tn) {
@@ -251,6 +277,8 @@ struct NsLayout {
   std::vector<size_t> off_x0, off_x1, off_a, off_b;
   std::vector<std::vector<NsTile>> tiles;   // per batch*3 + phase
   std::vector<size_t> off_tiles;
+  std::vector<std::vector<int>> offsets;    // per batch*3 + phase (tensor-core path)
+  std::vector<size_t> off_offsets;
   size_t off_groups = 0;
   size_t off_norm = 0;
 };
@@ -276,9 +304,29 @@ static void layout_ns(std::vector<NsGroup>& groups, lm_dtype xdt, int nmat, Aren
     for (int ph = 0; ph < 3; ++ph) {
       std::vector<NsTile> t;
       build_ns_tiles(groups, g0, b.ng, ph, bm, bn, t);
+      std::vector<int> offs;
+      if (xdt == LM_BF16 && !t.empty()) {
+        // cost of a tile: its K blocks plus an allowance for the epilogue
+        std::vector<std::pair<int, NsTile>> sorted;
+        for (const NsTile& x : t) {
+          const NsGroup& g = groups[g0 + x.group];
+          const int nk = ((ph == NS_GRAM) ? g.l_pad : g.s_pad) / kTcBK;
+          sorted.push_back({nk + 6, x});
+        }
+        std::stable_sort(sorted.begin(), sorted.end(),
+                         [](const std::pair<int, NsTile>& a, const std::pair<int, NsTile>& c) {
+                           return a.first > c.first;
+                         });
+        const int workers = std::min<int>(tc_max_pairs(), (int)t.size());
+        t.clear();
+        balance_tiles(sorted, workers, t, offs);
+        b.npairs[ph] = workers;
+      }
       b.ntiles[ph] = (int)t.size();
       L.off_tiles.push_back(ar.add(t.size() * sizeof(NsTile)));
       L.tiles.push_back(std::move(t));
+      L.off_offsets.push_back(ar.add(offs.size() * sizeof(int)));
+      L.offsets.push_back(std::move(offs));
     }
     batches.push_back(b);
   }
@@ -299,6 +347,10 @@ static void bind_ns(NsEngine& E, char* base, const NsLayout& L, std::vector<char
       E.batches[bi].tiles[ph] = reinterpret_cast<NsTile*>(base + L.off_tiles[k]);
       if (!L.tiles[k].empty())
         memcpy(host_img.data() + L.off_tiles[k], L.tiles[k].data(), L.tiles[k].size() * sizeof(NsTile));
+      if (!L.offsets[k].empty()) {
+        E.batches[bi].offsets[ph] = reinterpret_cast<int*>(base + L.off_offsets[k]);
+        memcpy(host_img.data() + L.off_offsets[k], L.offsets[k].data(), L.offsets[k].size() * sizeof(int));
+      }
     }
   E.d_groups = reinterpret_cast<NsGroup*>(base + L.off_groups);
   memcpy(host_img.data() + L.off_groups, E.groups.data(), E.groups.size() * sizeof(NsGroup));
@@ -358,10 +410,11 @@ static lm_status run_ns(const NsEngine& E, int steps, NsCoeffs co, unsigned* fla
   for (int it = 0; it < steps; ++it)
     for (const NsBatch& b : E.batches)
       for (int ph = 0; ph < 3; ++ph) {
-        cudaError_t e = timed(P, LM_KERNEL_NS_GEMM, st, [&]() {
+        cudaError_t e = timed(P, LM_KERNEL_NS_GRAM + ph, st, [&]() {
           if (E.xdt == LM_BF16)
             return launch_ns_tc((NsPhase)ph, it, b.ng, E.groups.data() + b.g0, E.maps.data() + b.g0,
-                                b.tiles[ph], b.ntiles[ph], E.d_norm2, co, flags, st);
+                                b.tiles[ph], b.ntiles[ph], b.offsets[ph], b.npairs[ph], E.d_norm2, co,
+                                flags, st);
           return launch_ns_simt((NsPhase)ph, it, b.ng, E.d_groups + b.g0, b.tiles[ph], b.ntiles[ph],
                                 E.d_norm2, co, st);
         });

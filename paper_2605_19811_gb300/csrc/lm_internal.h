@@ -107,22 +107,27 @@ struct NsCoeffs {
   float a, b, c, eps;
 };
 
-// Tensor-core path (bf16 operands, fp32 accumulation in TMEM).
-constexpr int kTcBM = 128, kTcBN = 256, kTcBK = 64;
+// Tensor-core path (bf16 operands, fp32 accumulation in TMEM): one
+// kTcBM x kTcBN output tile per CTA pair; s is padded to 128, l to kTcBN.
+constexpr int kTcBM = 256, kTcBN = 256, kTcBK = 64;
 int tc_pad_s(int s);
 int tc_pad_l(int l);
 // Tensor maps for one group: K-major boxes (64 x 128) on X0, X1, A, B and
-// MN-major boxes (64 x 64) on X0, X1.
+// MN-major boxes (64 x 64) on X0, X1.  Padded sizes are whole boxes.
 struct TcGroupMaps {
-  CUtensorMap xk[2];
+  CUtensorMap xk[2];    // K-major operand / aux loads: box 64 x 128
   CUtensorMap a;
   CUtensorMap b;
-  CUtensorMap xmn[2];
+  CUtensorMap xmn[2];   // MN-major operand loads: box 64 x 64
+  CUtensorMap xst[2];   // X' stores: box 64 x 32
 };
 cudaError_t tc_encode_group_maps(const NsGroup& g, TcGroupMaps* maps);
+int tc_max_pairs();   // CTA pairs that fit the device (one CTA per SM)
+// offsets: NULL (round robin over tiles) or npairs + 1 range starts.
 cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* groups,
                          const TcGroupMaps* maps, const NsTile* tiles, int ntiles,
-                         const double* norm2, NsCoeffs co, unsigned* flags, cudaStream_t st);
+                         const int* offsets, int npairs, const double* norm2, NsCoeffs co,
+                         unsigned* flags, cudaStream_t st);
 
 // fp32 CUDA-core path.
 constexpr int kSimtBM = 64, kSimtBN = 64;

@@ -50,7 +50,7 @@ size_t align256(size_t x) { return (x + 255) / 256 * 256; }
 // (tm, tn) of tile k in the same order the allocating path builds them
 // (row-major; symmetric phases keep tiles that reach the diagonal).
 __host__ __device__ inline int phase_tiles(int phase, int s_pad, int l_pad, int bm, int bn) {
-  const int tms = s_pad / bm;
+  const int tms = (s_pad + bm - 1) / bm;
   const int ncol = phase == NS_APPLY ? l_pad : s_pad;
   const int tns = (ncol + bn - 1) / bn;
   if (phase == NS_APPLY) return tms * tns;
@@ -89,7 +89,7 @@ __global__ void build_tables_kernel(BuildArgs a) {
   if (threadIdx.x < 3) {
     const int ph = threadIdx.x;
     const NsGroup& g = a.group;
-    const int tms = g.s_pad / a.bm;
+    const int tms = (g.s_pad + a.bm - 1) / a.bm;
     const int ncol = ph == NS_APPLY ? g.l_pad : g.s_pad;
     const int tns = (ncol + a.bn - 1) / a.bn;
     int k = 0;
@@ -246,8 +246,8 @@ extern "C" lm_status lm_msign_ns_noalloc(const lm_tensor* in, lm_tensor* out, in
   for (int it = 0; it < steps; ++it)
     for (int ph = 0; ph < 3; ++ph) {
       if (xdt == LM_BF16)
-        e = launch_ns_tc((NsPhase)ph, it, 1, &g, &maps, ba.d_tiles[ph], ntiles[ph], d.norm2, co,
-                         ba.d_flags, stream);
+        e = launch_ns_tc((NsPhase)ph, it, 1, &g, &maps, ba.d_tiles[ph], ntiles[ph], nullptr, 0,
+                         d.norm2, co, ba.d_flags, stream);
       else
         e = launch_ns_simt((NsPhase)ph, it, 1, ba.d_group, ba.d_tiles[ph], ntiles[ph], d.norm2, co,
                            stream);

@@ -1,6 +1,7 @@
 // Tensor-core Newton-Schulz phases for sm_103a: tcgen05.mma (bf16 operands,
-// fp32 accumulators in TMEM), operands staged by TMA into 128-byte-swizzled
-// shared memory, a persistent grouped schedule over all same-shape matrices.
+// fp32 accumulators in TMEM) on CTA pairs (cta_group::2, one 256 x 256 tile
+// per pair), operands staged by TMA into 128-byte-swizzled shared memory, a
+// persistent grouped schedule over all same-shape matrices.
 //
 // Per NS iteration (Section 2, odd-polynomial Newton-Schulz), with X in the
 // wide orientation (s x l) and the normalisation X / (||G_hat||_F + eps)
@@ -13,13 +14,27 @@
 // A and A A are symmetric, so A A = A A^T and both GEMM operands of GRAM and
 // POLY are K-major rows of the same matrix.
 //
-// CTA roles (192 threads, one CTA per SM):
-//   warp 0  TMA producer (one elected lane), 4-stage smem ring
-//   warp 1  TMEM allocator + MMA issuer (one elected lane)
-//   warps 2-5 epilogue: tcgen05.ld from TMEM, fused polynomial combination,
-//           bf16 stores (direct + mirrored)
-// Two 256-column accumulators in TMEM let the epilogue of one tile overlap the
-// main loop of the next.  Every mbarrier wait is bounded in time; a wait that
+// A cluster of two CTAs computes one 256 x 256 tile: CTA r holds rows
+// [128 r, 128 r + 128) of the A operand and N-rows [128 r, 128 r + 128) of the
+// B operand, the pair's MMA (issued by CTA 0) leaves rows 128 r .. of the
+// tile in CTA r's TMEM.  Each SM thus stages and reads half of B, which halves
+// the shared-memory traffic per FLOP of a one-CTA 128 x 256 tile.
+//
+// CTA roles (352 threads, one CTA per SM):
+//   warp 0    TMA producer (one elected lane), 5-stage smem ring; both CTAs'
+//             copies signal CTA 0's full barrier
+//   warp 1    TMEM allocator (both CTAs) + MMA issuer (CTA 0, one lane)
+//   warps 2-9 epilogue: tcgen05.ld from TMEM, fused polynomial combination;
+//             GRAM/POLY store bf16 directly (direct + mirrored half), APPLY
+//             writes X' over its aux tile in shared memory and TMA-stores it;
+//             each TMEM lane quadrant is served by two warps, one per half of
+//             the tile's columns
+//   warp 10   aux loader: TMA of the tile the POLY/APPLY epilogue combines
+//             with the accumulator (A or X), issued while the main loop runs
+// Tiles are assigned to pairs on the host by a longest-first greedy balance
+// of their K lengths (a contiguous range per pair).
+// kAccBufs 256-column accumulators in TMEM (two let the epilogue of one tile
+// overlap the main loop of the next).  Every mbarrier wait is bounded in time; a wait that
 // gives up sets LM_FLAG_TIMEOUT, makes the other roles stop, waits (bounded)
 // for its own copies and MMAs, frees TMEM and returns.
 #include <cuda_bf16.h>
@@ -30,20 +45,28 @@
 namespace lm {
 namespace {
 
-constexpr int BM = kTcBM, BN = kTcBN, BK = kTcBK;
-constexpr int kStages = 4;
-constexpr int kABytes = BM * BK * 2;           // 16 KB
-constexpr int kBBytes = BN * BK * 2;           // 32 KB
-constexpr int kStageBytes = kABytes + kBBytes; // 48 KB
-constexpr int kThreads = 192;
-constexpr int kTmemCols = 2 * BN;              // two accumulators
-constexpr uint64_t kWaitLimitNs = 5000000000ull;   // 5 s
-constexpr size_t kSmemBytes = 1024 /*align slack*/ + (size_t)kStages * kStageBytes + 256;
+constexpr int BM = kTcBM, BN = kTcBN, BK = kTcBK;   // pair tile 256 x 256, K step 64
+constexpr int kHalf = 128;                           // A rows / B N-rows per CTA
+constexpr int kStages = 5;
+constexpr int kABytes = kHalf * BK * 2;              // 16 KB
+constexpr int kBBytes = kHalf * BK * 2;              // 16 KB
+constexpr int kStageBytes = kABytes + kBBytes;       // 32 KB per CTA
+constexpr int kEpiWarps = 8;
+constexpr int kAuxWarp = 2 + kEpiWarps;              // warp that loads the epilogue's aux tile
+constexpr int kThreads = 32 * (3 + kEpiWarps);
+constexpr int kAccBufs = 2;                          // accumulators in TMEM
+constexpr int kTmemCols = kAccBufs * BN;
+constexpr uint64_t kWaitLimitNs = 5000000000ull;     // 5 s
+constexpr int kAuxBoxBytes = kHalf * 64 * 2;         // one 64-column box of the CTA's rows: 16 KB
+constexpr size_t kAuxOffset = (size_t)kStages * kStageBytes;
+constexpr size_t kBarOffset = kAuxOffset + 4 * kAuxBoxBytes;
+constexpr size_t kSmemBytes = 1024 /*align slack*/ + kBarOffset + 256;
 
 struct TcParams {
   TcGroupMaps maps[kMaxGroupsTc];
   NsGroup groups[kMaxGroupsTc];
   const NsTile* tiles;
+  const int* offsets;   // tiles of pair k: [offsets[k], offsets[k+1]); NULL: round robin
   int ntiles;
   int phase;
   int iter;
@@ -97,16 +120,61 @@ __device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile 
     }
   }
 }
-__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, uint64_t* bar,
+// 3-D tiled TMA load into this CTA's shared memory; completion is signalled
+// on the mbarrier at shared::cluster address bar_cluster (either CTA of the pair).
+__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, uint32_t bar_cluster,
                                             int c0, int c1, int c2) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(c0), "r"(c1), "r"(c2)
+      : "memory");
+}
+// 3-D tiled TMA load signalling this CTA's own mbarrier.
+__device__ __forceinline__ void tma_load_3d_local(void* dst, const CUtensorMap* map, uint64_t* bar,
+                                                  int c0, int c1, int c2) {
   asm volatile(
       "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
       " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(smem_u32(dst)),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2)
       : "memory");
 }
-__device__ __forceinline__ void prefetch_map(const CUtensorMap* map) {
-  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+// 3-D tiled TMA store from this CTA's shared memory (bulk-group completion).
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, const void* src, int c0, int c1,
+                                             int c2) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
+          reinterpret_cast<uint64_t>(map)),
+      "r"(smem_u32(src)), "r"(c0), "r"(c1), "r"(c2)
+      : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read() {
+  asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+// Make this thread's generic-proxy shared-memory writes visible to the TMA.
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// shared::cluster address of the same shared variable in CTA `rank`
+__device__ __forceinline__ uint32_t peer_addr(const void* p, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_u32(p)), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar_cluster) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster)
+               : "memory");
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
+                   : "memory");
 }
 __device__ __forceinline__ void tc_fence_before() {
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -115,16 +183,16 @@ __device__ __forceinline__ void tc_fence_after() {
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 }
 __device__ __forceinline__ void tmem_alloc(uint32_t* dst, uint32_t ncols) {
-  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                    smem_u32(dst)),
                "r"(ncols)
                : "memory");
 }
 __device__ __forceinline__ void tmem_relinquish() {
-  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
 }
 __device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
-  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
                : "memory");
 }
 __device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
@@ -132,13 +200,21 @@ __device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc, uint6
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
       "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
       "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
-__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+// Arrive on the barrier at the same shared-memory offset in both CTAs of the
+// pair once all previously issued MMAs of this thread have completed.
+__device__ __forceinline__ void umma_commit_pair(uint64_t* bar) {
   asm volatile(
-      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+      " [%0], %1;" ::"r"(smem_u32(bar)), "h"((uint16_t)0x3)
+      : "memory");
+}
+__device__ __forceinline__ void umma_commit_local(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
           smem_u32(bar))
       : "memory");
 }
@@ -176,7 +252,8 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr, uint32_t lbo, uin
   return d;
 }
 // Instruction descriptor, kind::f16: D fp32, A and B bf16, A K-major,
-// B K-major or MN-major, N >> 3 at bit 17, M >> 4 at bit 24.
+// B K-major or MN-major, N >> 3 at bit 17, M >> 4 at bit 24 (M = 256 for a
+// CTA pair).
 __host__ __device__ constexpr uint32_t make_idesc(int m, int n, bool b_mn_major) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((b_mn_major ? 1u : 0u) << 16) |
          ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
@@ -190,31 +267,44 @@ __device__ __forceinline__ uint32_t pack_bf2(float lo, float hi) {
 }
 
 // ------------------------------- the kernel ---------------------------------
-__global__ void __launch_bounds__(kThreads, 1) ns_tc_kernel(const __grid_constant__ TcParams p) {
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+    ns_tc_kernel(const __grid_constant__ TcParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)kStages * kStageBytes);
+  uint8_t* auxbuf = smem + kAuxOffset;   // 4 x (128 rows x 64 cols) bf16, 128-byte swizzled
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kBarOffset);
   uint64_t* empty = full + kStages;
   uint64_t* accfull = empty + kStages;
   uint64_t* accempty = accfull + 2;
-  uint64_t* done = accempty + 2;
+  uint64_t* aux_full = accempty + 2;
+  uint64_t* aux_empty = aux_full + 1;
+  uint64_t* done = aux_empty + 1;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int phase = p.phase;
   const int cur = p.iter & 1;
+  const uint32_t rank = cluster_rank();          // 0: MMA issuer of the pair
+  const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
+  const bool aux_phase = phase != NS_GRAM;       // epilogue reads the A (POLY) or X (APPLY) tile
+  // this pair's tiles: a host-balanced range, or round robin
+  const int w_begin = p.offsets ? p.offsets[pair] : pair;
+  const int w_end = p.offsets ? p.offsets[pair + 1] : p.ntiles;
+  const int w_step = p.offsets ? 1 : npairs;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
-    for (int b = 0; b < 2; ++b) {
+    for (int b = 0; b < kAccBufs; ++b) {
       mbar_init(&accfull[b], 1);
-      mbar_init(&accempty[b], 4);
+      mbar_init(&accempty[b], 2 * kEpiWarps);
     }
+    mbar_init(aux_full, 1);
+    mbar_init(aux_empty, kEpiWarps);
     mbar_init(done, 1);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -224,7 +314,7 @@ __global__ void __launch_bounds__(kThreads, 1) ns_tc_kernel(const __grid_constan
     tmem_relinquish();
   }
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();     // barriers of both CTAs initialised before any remote use
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
@@ -241,7 +331,7 @@ __global__ void __launch_bounds__(kThreads, 1) ns_tc_kernel(const __grid_constan
       int stage = 0;
       uint32_t ph = 0;
       bool ok = true;
-      for (int w = blockIdx.x; ok && w < p.ntiles; w += gridDim.x) {
+      for (int w = w_begin; ok && w < w_end; w += w_step) {
         const NsTile t = p.tiles[w];
         const NsGroup& g = p.groups[t.group];
         const TcGroupMaps& mp = p.maps[t.group];
@@ -256,6 +346,8 @@ __global__ void __launch_bounds__(kThreads, 1) ns_tc_kernel(const __grid_constan
           mapA = &mp.b; mapB = &mp.xmn[cur]; K = g.s_pad;
         }
         const int nk = K / BK;
+        const int row_a = t.tm * BM + (int)rank * kHalf;
+        const int col_b = t.tn * BN + (int)rank * kHalf;
         for (int kb = 0; kb < nk; ++kb) {
           if (!mbar_wait(&empty[stage], ph ^ 1u, abort_flag, kWaitLimitNs)) {
             give_up();
@@ -264,17 +356,17 @@ __global__ void __launch_bounds__(kThreads, 1) ns_tc_kernel(const __grid_constan
           }
           uint8_t* sa = smem + (size_t)stage * kStageBytes;
           uint8_t* sb = sa + kABytes;
-          mbar_arrive_expect_tx(&full[stage], kStageBytes);
+          const uint32_t fb = peer_addr(&full[stage], 0);
+          if (rank == 0) mbar_arrive_expect_tx(&full[stage], 2 * kStageBytes);
           armed[stage] = (int)ph;
           const int k0 = kb * BK;
-          tma_load_3d(sa, mapA, &full[stage], k0, t.tm * BM, t.mat);
+          tma_load_3d(sa, mapA, fb, k0, row_a, t.mat);
           if (phase != NS_APPLY) {
-            tma_load_3d(sb, mapB, &full[stage], k0, t.tn * BN, t.mat);
-            tma_load_3d(sb + kBBytes / 2, mapB, &full[stage], k0, t.tn * BN + BN / 2, t.mat);
+            tma_load_3d(sb, mapB, fb, k0, col_b, t.mat);
           } else {
 #pragma unroll
-            for (int q = 0; q < BN / 64; ++q)
-              tma_load_3d(sb + q * (64 * BK * 2), mapB, &full[stage], t.tn * BN + 64 * q, k0, t.mat);
+            for (int q = 0; q < kHalf / 64; ++q)
+              tma_load_3d(sb + q * (64 * BK * 2), mapB, fb, col_b + 64 * q, k0, t.mat);
           }
           if (++stage == kStages) {
             stage = 0;
@@ -282,7 +374,7 @@ __global__ void __launch_bounds__(kThreads, 1) ns_tc_kernel(const __grid_constan
           }
         }
       }
-      if (!ok) {
+      if (!ok && rank == 0) {
         // let the copies already issued land before the CTA exits
         for (int s = 0; s < kStages; ++s)
           if (armed[s] >= 0) {
@@ -293,14 +385,14 @@ __global__ void __launch_bounds__(kThreads, 1) ns_tc_kernel(const __grid_constan
     }
   } else if (warp == 1) {
     // ------------------------------ MMA issuer -----------------------------
-    if (lane == 0) {
+    if (lane == 0 && rank == 0) {
       const uint32_t idesc = make_idesc(BM, BN, phase == NS_APPLY);
       int stage = 0;
       uint32_t ph = 0;
       int ab = 0;
       uint32_t aph = 0;
       bool ok = true;
-      for (int w = blockIdx.x; ok && w < p.ntiles; w += gridDim.x) {
+      for (int w = w_begin; ok && w < w_end; w += w_step) {
         const NsTile t = p.tiles[w];
         const NsGroup& g = p.groups[t.group];
         const int K = (phase == NS_GRAM) ? g.l_pad : g.s_pad;
@@ -328,35 +420,73 @@ __global__ void __launch_bounds__(kThreads, 1) ns_tc_kernel(const __grid_constan
                                        : sw128_desc(sb + kk * 32, 16, 1024);
             umma_bf16(d_tmem, adesc, bdesc, idesc, (kb | kk) != 0 ? 1u : 0u);
           }
-          umma_commit(&empty[stage]);
+          umma_commit_pair(&empty[stage]);
           if (++stage == kStages) {
             stage = 0;
             ph ^= 1u;
           }
         }
         if (!ok) break;
-        umma_commit(&accfull[ab]);
-        if (++ab == 2) {
+        umma_commit_pair(&accfull[ab]);
+        if (++ab == kAccBufs) {
           ab = 0;
           aph ^= 1u;
         }
       }
       // all issued MMAs complete before TMEM is released
-      umma_commit(done);
+      umma_commit_local(done);
       volatile int never = 0;
       mbar_wait(done, 0, &never, 100000000ull);
     }
+  } else if (warp == kAuxWarp) {
+    // --------------------------- aux tile loader ---------------------------
+    // The epilogue of POLY needs the A tile, that of APPLY the X tile; both
+    // are loaded by TMA into auxbuf while the tile's main loop runs.
+    if (lane == 0 && aux_phase) {
+      uint32_t xph = 0;
+      int armed = -1;
+      bool ok = true;
+      for (int w = w_begin; ok && w < w_end; w += w_step) {
+        const NsTile t = p.tiles[w];
+        const TcGroupMaps& mp = p.maps[t.group];
+        const CUtensorMap* map = (phase == NS_POLY) ? &mp.a : &mp.xk[cur];
+        if (!mbar_wait(aux_empty, xph ^ 1u, abort_flag, kWaitLimitNs)) {
+          give_up();
+          ok = false;
+          break;
+        }
+        mbar_arrive_expect_tx(aux_full, 4 * kAuxBoxBytes);
+        armed = (int)xph;
+        const int row0 = t.tm * BM + (int)rank * kHalf;
+#pragma unroll
+        for (int b = 0; b < 4; ++b)
+          tma_load_3d_local(auxbuf + b * kAuxBoxBytes, map, aux_full, t.tn * BN + 64 * b, row0, t.mat);
+        xph ^= 1u;
+      }
+      if (!ok && armed >= 0) {
+        volatile int never = 0;
+        mbar_wait(aux_full, (uint32_t)armed, &never, 100000000ull);
+      }
+    }
   } else {
     // ------------------------------ epilogue -------------------------------
-    const int q = warp & 3;             // TMEM lane quadrant of this warp
-    const int row = q * 32 + lane;      // row of the tile owned by this thread
+    // Thread (quadrant q, lane) owns one row of this CTA's half tile and the
+    // 128 columns [half*128, half*128 + 128) of it, in four 32-column chunks.
+    const int q = warp & 3;                   // TMEM lane quadrant of this warp
+    const int half = (warp - 2) >> 2;         // which 128 columns of the tile
+    const int row = q * 32 + lane;            // row of this CTA's half tile
+    const uint32_t acc_empty0 = peer_addr(&accempty[0], 0);
+    const uint32_t acc_empty1 = peer_addr(&accempty[kAccBufs - 1], 0);
     int ab = 0;
-    uint32_t aph = 0;
-    for (int w = blockIdx.x; w < p.ntiles; w += gridDim.x) {
+    uint32_t aph = 0, xph = 0;
+    for (int w = w_begin; w < w_end; w += w_step) {
       const NsTile t = p.tiles[w];
       const NsGroup& g = p.groups[t.group];
       bool ok = true;
-      if (lane == 0) ok = mbar_wait(&accfull[ab], aph, abort_flag, kWaitLimitNs);
+      if (lane == 0) {
+        ok = mbar_wait(&accfull[ab], aph, abort_flag, kWaitLimitNs);
+        if (ok && aux_phase) ok = mbar_wait(aux_full, xph, abort_flag, kWaitLimitNs);
+      }
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
       if (!ok) {
         if (lane == 0) give_up();
@@ -369,37 +499,40 @@ __global__ void __launch_bounds__(kThreads, 1) ns_tc_kernel(const __grid_constan
         const float n = (float)sqrt(p.norm2[g.first_mat + t.mat]) + p.co.eps;
         nscale = (phase == NS_GRAM) ? 1.f / (n * n) : (phase == NS_APPLY ? 1.f / n : 1.f);
       }
-      const int i = t.tm * BM + row;
+      const int i = t.tm * BM + (int)rank * kHalf + row;
       const size_t sq = (size_t)g.s_pad * g.s_pad;
       const size_t xs = (size_t)g.s_pad * g.l_pad;
       const int ncols = (phase == NS_APPLY) ? g.l : g.s;
       const int ld = (phase == NS_APPLY) ? g.l_pad : g.s_pad;
       const int jmax = (phase == NS_APPLY) ? g.l_pad : g.s_pad;
+      const bool row_in = i < g.s_pad;        // rows past the padded matrix are skipped
       __nv_bfloat16* out;
-      const __nv_bfloat16* aux = nullptr;
       if (phase == NS_GRAM) {
         out = static_cast<__nv_bfloat16*>(g.A) + t.mat * sq;
       } else if (phase == NS_POLY) {
         out = static_cast<__nv_bfloat16*>(g.B) + t.mat * sq;
-        aux = static_cast<const __nv_bfloat16*>(g.A) + t.mat * sq;
       } else {
-        out = static_cast<__nv_bfloat16*>(g.X[cur ^ 1]) + t.mat * xs;
-        aux = static_cast<const __nv_bfloat16*>(g.X[cur]) + t.mat * xs;
+        out = nullptr;   // APPLY results leave through auxbuf and TMA stores
       }
+      (void)xs;
       const bool sym = phase != NS_APPLY;
-      for (int ch = 0; ch < BN / 32; ++ch) {
+      for (int c4 = 0; c4 < 4; ++c4) {
+        const int ch = half * 4 + c4;
         uint32_t r[32];
         __syncwarp();   // tcgen05.ld is warp-collective: reconverge first
         tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * BN + ch * 32), r);
         const int j0 = t.tn * BN + ch * 32;
-        if (j0 >= jmax) continue;                 // beyond the padded matrix
+        if (j0 >= jmax || !row_in) continue;      // beyond the padded matrix
         if (sym && j0 + 31 < i) continue;         // strictly below the diagonal
         float v[32];
-        if (aux != nullptr) {
-          const uint4* ap = reinterpret_cast<const uint4*>(aux + (size_t)i * ld + j0);
+        // this row's 32 aux values in the swizzled box: 16-byte chunk c of
+        // row r sits at chunk position c ^ (r mod 8)
+        uint4* abox = reinterpret_cast<uint4*>(auxbuf + (ch >> 1) * kAuxBoxBytes + row * 128);
+        const int csub = (ch & 1) * 4;
+        if (aux_phase) {
 #pragma unroll
           for (int u = 0; u < 4; ++u) {
-            const uint4 a4 = ap[u];
+            const uint4 a4 = abox[(csub + u) ^ (row & 7)];
             const uint32_t aw[4] = {a4.x, a4.y, a4.z, a4.w};
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
@@ -418,7 +551,14 @@ __global__ void __launch_bounds__(kThreads, 1) ns_tc_kernel(const __grid_constan
           else o = (p.co.a * v[e] + acc) * nscale;
           v[e] = (i < g.s && j < ncols) ? o : 0.f;
         }
-        if (!sym || j0 >= i) {
+        if (!sym) {
+          // APPLY: results replace the aux values, stored by TMA below
+#pragma unroll
+          for (int u = 0; u < 4; ++u)
+            abox[(csub + u) ^ (row & 7)] =
+                make_uint4(pack_bf2(v[u * 8 + 0], v[u * 8 + 1]), pack_bf2(v[u * 8 + 2], v[u * 8 + 3]),
+                           pack_bf2(v[u * 8 + 4], v[u * 8 + 5]), pack_bf2(v[u * 8 + 6], v[u * 8 + 7]));
+        } else if (j0 >= i) {
           // whole chunk on or above the diagonal: 16-byte direct stores
           uint4* op = reinterpret_cast<uint4*>(out + (size_t)i * ld + j0);
 #pragma unroll
@@ -439,17 +579,37 @@ __global__ void __launch_bounds__(kThreads, 1) ns_tc_kernel(const __grid_constan
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&accempty[ab]);
-      if (++ab == 2) {
+      if (lane == 0) mbar_arrive_cluster(ab == 0 ? acc_empty0 : acc_empty1);
+      if (++ab == kAccBufs) {
         ab = 0;
         aph ^= 1u;
       }
+      if (phase == NS_APPLY) {
+        // this warp's 32 rows x 128 columns of X' leave by two TMA stores
+        fence_proxy_async_smem();
+        __syncwarp();
+        const int r0 = t.tm * BM + (int)rank * kHalf + q * 32;
+        if (lane == 0 && r0 < g.s_pad) {
+#pragma unroll
+          for (int b = 2 * half; b < 2 * half + 2; ++b)
+            tma_store_3d(&p.maps[t.group].xst[cur ^ 1], auxbuf + b * kAuxBoxBytes + q * 32 * 128,
+                         t.tn * BN + 64 * b, r0, t.mat);
+          bulk_commit();
+          bulk_wait_read();   // auxbuf may be refilled once the stores have read it
+        }
+      }
+      if (aux_phase) {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(aux_empty);
+        xph ^= 1u;
+      }
     }
+    if (lane == 0) bulk_wait_all();
   }
 
   __syncwarp();
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();     // neither CTA leaves while its peer may still signal it
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem_base, kTmemCols);
@@ -485,23 +645,32 @@ cudaError_t encode_3d(CUtensorMap* m, void* base, uint64_t inner, uint64_t rows,
 
 }  // namespace
 
-int tc_pad_s(int s) { return (s + BM - 1) / BM * BM; }
+int tc_pad_s(int s) { return (s + kHalf - 1) / kHalf * kHalf; }
 int tc_pad_l(int l) { return (l + BN - 1) / BN * BN; }
 
 cudaError_t tc_encode_group_maps(const NsGroup& g, TcGroupMaps* maps) {
   cudaError_t e;
   for (int b = 0; b < 2; ++b) {
-    if ((e = encode_3d(&maps->xk[b], g.X[b], g.l_pad, g.s_pad, g.count, BK, BM)) != cudaSuccess) return e;
+    if ((e = encode_3d(&maps->xk[b], g.X[b], g.l_pad, g.s_pad, g.count, BK, kHalf)) != cudaSuccess) return e;
+    if ((e = encode_3d(&maps->xst[b], g.X[b], g.l_pad, g.s_pad, g.count, 64, 32)) != cudaSuccess) return e;
     if ((e = encode_3d(&maps->xmn[b], g.X[b], g.l_pad, g.s_pad, g.count, 64, BK)) != cudaSuccess) return e;
   }
-  if ((e = encode_3d(&maps->a, g.A, g.s_pad, g.s_pad, g.count, BK, BM)) != cudaSuccess) return e;
-  if ((e = encode_3d(&maps->b, g.B, g.s_pad, g.s_pad, g.count, BK, BM)) != cudaSuccess) return e;
+  if ((e = encode_3d(&maps->a, g.A, g.s_pad, g.s_pad, g.count, BK, kHalf)) != cudaSuccess) return e;
+  if ((e = encode_3d(&maps->b, g.B, g.s_pad, g.s_pad, g.count, BK, kHalf)) != cudaSuccess) return e;
   return cudaSuccess;
+}
+
+int tc_max_pairs() {
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  return sms / 2 > 0 ? sms / 2 : 1;
 }
 
 cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* groups,
                          const TcGroupMaps* maps, const NsTile* tiles, int ntiles,
-                         const double* norm2, NsCoeffs co, unsigned* flags, cudaStream_t st) {
+                         const int* offsets, int npairs, const double* norm2, NsCoeffs co,
+                         unsigned* flags, cudaStream_t st) {
   if (ntiles <= 0) return cudaSuccess;
   if (ngroups < 1 || ngroups > kMaxGroupsTc) return cudaErrorInvalidValue;
   static bool attr_set = false;
@@ -518,16 +687,19 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
     prm.groups[gi] = groups[gi];
   }
   prm.tiles = tiles;
+  prm.offsets = offsets;
   prm.ntiles = ntiles;
   prm.phase = (int)ph;
   prm.iter = iter;
   prm.norm2 = norm2;
   prm.co = co;
   prm.flags = flags;
-  int dev = 0, sms = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  int grid = sms < ntiles ? sms : ntiles;
+  int pairs = npairs;
+  if (offsets == nullptr) {
+    pairs = tc_max_pairs();
+    if (pairs > ntiles) pairs = ntiles;
+  }
+  const int grid = 2 * (pairs > 0 ? pairs : 1);
   count_launch();
   ns_tc_kernel<<<grid, kThreads, kSmemBytes, st>>>(prm);
   return cudaGetLastError();

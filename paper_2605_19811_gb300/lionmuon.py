@@ -29,7 +29,7 @@ EXPORTED = ("lm_config_default", "lm_create", "lm_step", "lm_set_lr", "lm_msign_
             "lm_kernel_launch_count", "lm_profile_enable", "lm_profile_read",
             "lm_msign_ns_noalloc")
 
-KERNEL_FAMILIES = ("lion", "momentum_norm", "ns_gemm", "finalize", "other")
+KERNEL_FAMILIES = ("lion", "momentum_norm", "ns_gram", "ns_poly", "ns_apply", "finalize", "other")
 
 
 class LmTensor(ctypes.Structure):
@@ -47,7 +47,7 @@ class LmConfig(ctypes.Structure):
 
 
 class LmProfile(ctypes.Structure):
-    _fields_ = [("ms", ctypes.c_double * 5), ("launches", ctypes.c_uint64 * 5)]
+    _fields_ = [("ms", ctypes.c_double * 7), ("launches", ctypes.c_uint64 * 7)]
 
 
 class LionMuonError(RuntimeError):
@@ -216,11 +216,15 @@ class LionMuon:
         _check(self._lib, self._lib.lm_profile_enable(self._h, 1 if on else 0), "lm_profile_enable")
 
     def profile_read(self, reset: bool = True) -> dict:
-        """{family: (total ms, launches)} of the timed launches (synchronises)."""
+        """{family: (total ms, launches)} of the timed launches (synchronises);
+        "ns_gemm" sums the three Newton-Schulz phases."""
         p = LmProfile()
         _check(self._lib, self._lib.lm_profile_read(self._h, ctypes.byref(p), 1 if reset else 0),
                "lm_profile_read")
-        return {name: (p.ms[i], int(p.launches[i])) for i, name in enumerate(KERNEL_FAMILIES)}
+        out = {name: (p.ms[i], int(p.launches[i])) for i, name in enumerate(KERNEL_FAMILIES)}
+        out["ns_gemm"] = (sum(out[k][0] for k in ("ns_gram", "ns_poly", "ns_apply")),
+                          sum(out[k][1] for k in ("ns_gram", "ns_poly", "ns_apply")))
+        return out
 
     def state_bytes(self) -> int:
         return int(self._lib.lm_state_bytes(self._h))

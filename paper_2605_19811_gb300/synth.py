@@ -62,6 +62,13 @@ def _stress() -> ParamSet:
     return ParamSet("stress_7b", tuple(shapes), "bf16", "outlier")
 
 
+def _layers_only(name: str, layers: int, d: int) -> ParamSet:
+    shapes: List[Tuple[int, ...]] = []
+    for _ in range(layers):
+        shapes += [(d, 3 * d), (d, d), (d, 4 * d), (4 * d, d)]
+    return ParamSet(name, tuple(shapes), "bf16", "student_t")
+
+
 PARAM_SETS = {
     "tiny": ParamSet("tiny", ((256, 256), (256, 1024), (1024, 256), (256, 256), (256,)),
                      "f32", "normal"),
@@ -69,6 +76,9 @@ PARAM_SETS = {
     "gpt_355m": _gpt("gpt_355m", 24, 1024),
     "gpt_720m": _gpt("gpt_720m", 36, 1280),
     "stress_7b": _stress(),
+    # four hidden layers of the 720M-shaped set (no embedding, no vectors):
+    # a small case with the same matrix shapes, for profiling captures
+    "gpt_720m_4layers": _layers_only("gpt_720m_4layers", 4, 1280),
 }
 
 
