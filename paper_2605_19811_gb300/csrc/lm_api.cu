@@ -189,9 +189,11 @@ void build_ns_tiles(const std::vector<NsGroup>& groups, int g0, int ng, int phas
   std::vector<std::pair<int, NsTile>> v;
   for (int gi = g0; gi < g0 + ng; ++gi) {
     const NsGroup& g = groups[gi];
-    const int ncol = (phase == NS_APPLY) ? g.l_pad : g.s_pad;
+    // output rows x cols: s x s (GRAM, POLY), s x l (APPLY wide), l x s (APPLY tall)
+    const int nrow = (phase == NS_APPLY && g.tall) ? g.l_pad : g.s_pad;
+    const int ncol = (phase == NS_APPLY) ? (g.tall ? g.s_pad : g.l_pad) : g.s_pad;
     const int K = (phase == NS_GRAM) ? g.l_pad : g.s_pad;
-    const int tms = (g.s_pad + bm - 1) / bm, tns = (ncol + bn - 1) / bn;
+    const int tms = (nrow + bm - 1) / bm, tns = (ncol + bn - 1) / bn;
     for (int m = 0; m < g.count; ++m)
       for (int tm = 0; tm < tms; ++tm)
         for (int tn = 0; tn < tns; ++tn) {
@@ -210,12 +212,12 @@ void build_ns_tiles(const std::vector<NsGroup>& groups, int g0, int ng, int phas
   for (auto& e : v) out.push_back(e.second);
 }
 
-// Element tiles of each matrix, padded to whole clusters with empty slots.
-void build_elem_tiles(const std::vector<MatDesc>& mats, std::vector<ElemTile>& out) {
+// Element chunks of each matrix (kElemChunk elements, the last one ragged).
+void build_elem_chunks(const std::vector<MatDesc>& mats, std::vector<ElemChunk>& out) {
   for (size_t i = 0; i < mats.size(); ++i) {
-    const int n = mats[i].tiles_r * mats[i].tiles_c;
-    const int padded = (n + kNormCluster - 1) / kNormCluster * kNormCluster;
-    for (int t = 0; t < padded; ++t) out.push_back(ElemTile{(int32_t)i, t < n ? t : -1});
+    const int64_t n = mats[i].rows * mats[i].cols;
+    for (int64_t b = 0; b < n; b += kElemChunk)
+      out.push_back(ElemChunk{(int32_t)i, 0, b, std::min<int64_t>(kElemChunk, n - b)});
   }
 }
 
@@ -239,17 +241,20 @@ struct NsEngine {
 // and fills groups with sizes (pointers set later).
 static void plan_groups(const std::vector<std::pair<int64_t, int64_t>>& shapes, lm_dtype xdt,
                         std::vector<NsGroup>& groups, std::vector<std::vector<int>>& members) {
+  // one group per (rows, cols): same (s, l) but opposite orientation are
+  // different groups, since X keeps the parameter's orientation
   std::map<std::pair<int64_t, int64_t>, int> key_to_group;
   for (size_t i = 0; i < shapes.size(); ++i) {
     const int64_t s = std::min(shapes[i].first, shapes[i].second);
     const int64_t l = std::max(shapes[i].first, shapes[i].second);
-    auto key = std::make_pair(s, l);
+    auto key = shapes[i];
     auto it = key_to_group.find(key);
     if (it == key_to_group.end()) {
       NsGroup g;
       memset(&g, 0, sizeof(g));
       g.s = (int32_t)s;
       g.l = (int32_t)l;
+      g.tall = shapes[i].first > shapes[i].second ? 1 : 0;
       if (xdt == LM_BF16) {
         g.s_pad = tc_pad_s((int)s);
         g.l_pad = tc_pad_l((int)l);
@@ -447,8 +452,8 @@ struct lm_state {
   int lion_grid[2] = {0, 0};
   int nmat = 0;
   MatDesc* d_mats = nullptr;
-  ElemTile* d_etiles = nullptr;
-  int n_etiles = 0;
+  ElemChunk* d_echunks = nullptr;
+  int n_echunks = 0;
   NsEngine ns;
   unsigned* d_flags = nullptr;
   cudaStream_t last_stream = nullptr;
@@ -577,13 +582,11 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
     memset(&d, 0, sizeof(d));
     d.rows = p.rows;
     d.cols = p.cols;
-    d.tiles_r = (int32_t)((p.rows + kElemTileR - 1) / kElemTileR);
-    d.tiles_c = (int32_t)((p.cols + kElemTileC - 1) / kElemTileC);
   }
-  std::vector<ElemTile> etiles;
-  build_elem_tiles(mats, etiles);
-  s->n_etiles = (int)etiles.size();
-  const size_t off_etiles = ar.add(etiles.size() * sizeof(ElemTile));
+  std::vector<ElemChunk> echunks;
+  build_elem_chunks(mats, echunks);
+  s->n_echunks = (int)echunks.size();
+  const size_t off_echunks = ar.add(echunks.size() * sizeof(ElemChunk));
 
   cudaError_t e = cudaMalloc(&s->base, ar.total);
   if (e != cudaSuccess) {
@@ -628,18 +631,17 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
       d.x_final = static_cast<char*>(g.X[cfg->ns_steps & 1]) + xoff;
       d.out = nullptr;
       d.norm2 = s->ns.d_norm2 + id;
-      d.ldx = g.l_pad;
+      d.ldx = g.tall ? g.s_pad : g.l_pad;
       d.grad_slot = pi;
-      d.transposed = p.rows > p.cols ? 1 : 0;
       d.wdt = p.dtype;
       d.odt = p.dtype;
       d.shape_scale = (float)(cfg->shape_scale * std::sqrt((double)std::max(p.rows, p.cols)));
     }
   }
   if (s->nmat) memcpy(img.data() + off_mats, mats.data(), mats.size() * sizeof(MatDesc));
-  if (!etiles.empty()) memcpy(img.data() + off_etiles, etiles.data(), etiles.size() * sizeof(ElemTile));
+  if (!echunks.empty()) memcpy(img.data() + off_echunks, echunks.data(), echunks.size() * sizeof(ElemChunk));
   s->d_mats = reinterpret_cast<MatDesc*>(base + off_mats);
-  s->d_etiles = reinterpret_cast<ElemTile*>(base + off_etiles);
+  s->d_echunks = reinterpret_cast<ElemChunk*>(base + off_echunks);
 
   // Upload tables and zeros (momentum M_{-1} = 0, workspace padding = 0).
   e = cudaMemcpyAsync(base, img.data(), ar.total, cudaMemcpyHostToDevice, stream);
@@ -721,7 +723,7 @@ lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t, void* c
     });
     if (e != cudaSuccess) return cuda_fail(e, "norm reset");
     e = timed(P, LM_KERNEL_MOMENTUM_NORM, stream, [&]() {
-      return launch_momentum_norm(s->ns.xdt, s->d_mats, s->d_etiles, s->n_etiles, s->d_grads, mk, 0,
+      return launch_momentum_norm(s->ns.xdt, s->d_mats, s->d_echunks, s->n_echunks, s->d_grads, mk, 0,
                                   stream);
     });
     if (e != cudaSuccess) return cuda_fail(e, "momentum/norm kernel launch");
@@ -738,7 +740,7 @@ lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t, void* c
     NsCoeffs co{(float)c.ns_a, (float)c.ns_b, (float)c.ns_c, (float)c.ns_eps};
     if ((st = run_ns(s->ns, c.ns_steps, co, s->d_flags, stream, P)) != LM_OK) return st;
     e = timed(P, LM_KERNEL_FINALIZE, stream, [&]() {
-      return launch_finalize(s->ns.xdt, s->d_mats, s->d_etiles, s->n_etiles, mk, 0, s->d_flags, stream);
+      return launch_finalize(s->ns.xdt, s->d_mats, s->d_echunks, s->n_echunks, mk, 0, s->d_flags, stream);
     });
     if (e != cudaSuccess) return cuda_fail(e, "finalize kernel launch");
   }
@@ -867,11 +869,9 @@ lm_status lm_msign_ns(const lm_tensor* in, lm_tensor* out, int steps, double a, 
   memset(&d, 0, sizeof(d));
   d.rows = in->rows;
   d.cols = in->cols;
-  d.tiles_r = (int32_t)((d.rows + kElemTileR - 1) / kElemTileR);
-  d.tiles_c = (int32_t)((d.cols + kElemTileC - 1) / kElemTileC);
-  std::vector<ElemTile> et;
-  build_elem_tiles({d}, et);
-  const size_t off_et = ar.add(et.size() * sizeof(ElemTile));
+  std::vector<ElemChunk> et;
+  build_elem_chunks({d}, et);
+  const size_t off_et = ar.add(et.size() * sizeof(ElemChunk));
   const size_t off_flags = ar.add(sizeof(unsigned));
 
   char* base = nullptr;
@@ -886,14 +886,13 @@ lm_status lm_msign_ns(const lm_tensor* in, lm_tensor* out, int steps, double a, 
   d.x_final = g.X[steps & 1];
   d.out = out->data;
   d.norm2 = E.d_norm2;
-  d.ldx = g.l_pad;
+  d.ldx = g.tall ? g.s_pad : g.l_pad;
   d.grad_slot = 0;
-  d.transposed = in->rows > in->cols ? 1 : 0;
   d.wdt = in->dtype;
   d.odt = out->dtype;
   d.shape_scale = 1.f;
   memcpy(img.data() + off_mat, &d, sizeof(d));
-  memcpy(img.data() + off_et, et.data(), et.size() * sizeof(ElemTile));
+  memcpy(img.data() + off_et, et.data(), et.size() * sizeof(ElemChunk));
   auto cleanup = [&](lm_status r) {
     cudaFreeAsync(base, stream);
     return r;
@@ -906,7 +905,7 @@ lm_status lm_msign_ns(const lm_tensor* in, lm_tensor* out, int steps, double a, 
   mk.eps = (float)eps;
   mk.ns_steps = steps;
   MatDesc* dm = reinterpret_cast<MatDesc*>(base + off_mat);
-  ElemTile* de = reinterpret_cast<ElemTile*>(base + off_et);
+  ElemChunk* de = reinterpret_cast<ElemChunk*>(base + off_et);
   unsigned* dflags = reinterpret_cast<unsigned*>(base + off_flags);
   e = launch_momentum_norm(E.xdt, dm, de, (int)et.size(), nullptr, mk, 1, stream);
   if (e != cudaSuccess) return cleanup(cuda_fail(e, "norm kernel launch"));

@@ -1,22 +1,18 @@
 // Element-wise kernels of the LionMuon step (arXiv 2605.19811, Algorithm 1):
 //   * lion_kernel           : Lion branch + momentum update, multi-tensor,
 //                             one pass over W, G, M with 16-byte vector I/O.
-//   * momentum_norm_kernel  : Muon steps, first half: G_hat, ||G_hat||_F^2
-//                             (warp shuffle -> CTA -> cluster DSMEM -> one
-//                             fp64 atomic per cluster), M update, and
-//                             X0 = G_hat in the wide orientation.
+//   * momentum_norm_kernel  : Muon steps, first part: G_hat, ||G_hat||_F^2
+//                             (warp shuffle, one fp64 atomic per warp and
+//                             32K-element chunk), M update, X0 = G_hat.
 //   * finalize_kernel       : Muon steps, last part: W <- W - eta_M (0.2
 //                             sqrt(max(m,n)) X_K + lambda W) (Table 5 scaling),
 //                             or the plain msign output.
 // All arithmetic is fp32 with each product and sum rounded separately
 // (__fmul_rn / __fadd_rn / __fsub_rn): no contraction into FMA, so the Lion
 // step is reproducible bit for bit by a same-order float32 evaluation.
-#include <cooperative_groups.h>
 #include <cuda_bf16.h>
 
 #include "lm_internal.h"
-
-namespace cg = cooperative_groups;
 
 namespace lm {
 namespace {
@@ -124,205 +120,153 @@ __global__ void __launch_bounds__(kLionThreads)
 }
 
 // ---------------------------------------------------------------------------
-// Muon: momentum + Frobenius norm + X0
+// Muon: momentum + Frobenius norm + X0, and finalize.  X keeps the
+// parameter's orientation (row pitch ldx), so both kernels stream element
+// ranges of a matrix: element e = r * cols + c of W, G, M is element
+// r * ldx + c of X.
 // ---------------------------------------------------------------------------
 constexpr int kElemThreads = 256;
-constexpr int kSmPitch = kElemTileR + 1;   // transposing tile [kElemTileC][kElemTileR + 1]
-static_assert(kElemTileR * kElemTileC == 32 * kElemThreads, "4 vectors of 8 per thread");
 
+__device__ __forceinline__ int64_t x_index(const MatDesc& d, int64_t e) {
+  const int64_t r = e / d.cols;
+  return r * d.ldx + (e - r * d.cols);
+}
+
+// One vector of 8 elements of the Muon direction: G_hat = b1 M + c1 G (fp32,
+// same operation order as the Lion step), M <- b2 M + c2 G, X0 = G_hat.
 template <typename XT, typename GT>
-__device__ float momentum_norm_tile(const MatDesc& d, int tile, const GT* g, const MuonConsts& k,
-                                    int mode, float* sm) {
-  const int tr = tile / d.tiles_c, tcol = tile - tr * d.tiles_c;
-  const int64_t r0 = (int64_t)tr * kElemTileR, c0 = (int64_t)tcol * kElemTileC;
-  XT* x = static_cast<XT*>(d.x);
-  const bool vec = (d.cols & 7) == 0;
+__device__ __forceinline__ float momentum_vec(const MatDesc& d, int64_t e, const GT* g,
+                                              const MuonConsts& k, int mode) {
+  float gv[8], mv[8], gh[8];
+  load8(g + e, gv);
+  if (mode == 0) load8(d.m + e, mv);
   float acc = 0.f;
 #pragma unroll
-  for (int it = 0; it < 4; ++it) {
-    const int slot = threadIdx.x + it * kElemThreads;
-    const int rr = slot >> 4, vv = slot & 15;
-    const int64_t r = r0 + rr, c = c0 + vv * 8;
-    if (r >= d.rows || c >= d.cols) continue;
-    const int cnt = (int)min((int64_t)8, d.cols - c);
-    const int64_t off = r * d.cols + c;
-    float gv[8], mv[8], gh[8];
-    if (vec) {
-      load8(g + off, gv);
-      if (mode == 0) load8(d.m + off, mv);
-    } else {
-#pragma unroll
-      for (int e = 0; e < 8; ++e) {
-        gv[e] = e < cnt ? to_f(g[off + e]) : 0.f;
-        mv[e] = (e < cnt && mode == 0) ? d.m[off + e] : 0.f;
-      }
-    }
-#pragma unroll
-    for (int e = 0; e < 8; ++e) {
-      if (mode == 0) {
-        gh[e] = __fadd_rn(__fmul_rn(k.b1, mv[e]), __fmul_rn(k.c1, gv[e]));
-        mv[e] = __fadd_rn(__fmul_rn(k.b2, mv[e]), __fmul_rn(k.c2, gv[e]));
-      } else {
-        gh[e] = gv[e];
-      }
-      if (e < cnt) acc = fmaf(gh[e], gh[e], acc);
-    }
+  for (int j = 0; j < 8; ++j) {
     if (mode == 0) {
-      if (vec) {
-        store8(d.m + off, mv);
-      } else {
-        for (int e = 0; e < cnt; ++e) d.m[off + e] = mv[e];
-      }
-    }
-    if (!d.transposed) {
-      XT* xp = x + r * d.ldx + c;
-      if (vec) {
-        store8(xp, gh);
-      } else {
-        for (int e = 0; e < cnt; ++e) xp[e] = from_f<XT>(gh[e]);
-      }
+      gh[j] = __fadd_rn(__fmul_rn(k.b1, mv[j]), __fmul_rn(k.c1, gv[j]));
+      mv[j] = __fadd_rn(__fmul_rn(k.b2, mv[j]), __fmul_rn(k.c2, gv[j]));
     } else {
-#pragma unroll
-      for (int e = 0; e < 8; ++e) sm[(vv * 8 + e) * kSmPitch + rr] = gh[e];
+      gh[j] = gv[j];
     }
+    acc = fmaf(gh[j], gh[j], acc);
   }
-  if (d.transposed) {
-    __syncthreads();
-    // X0[c][r] = G_hat[r][c]: consecutive threads write consecutive r.
-    for (int it = 0; it < (kElemTileR * kElemTileC) / kElemThreads; ++it) {
-      const int slot = threadIdx.x + it * kElemThreads;
-      const int cc = slot / kElemTileR, rr = slot % kElemTileR;
-      const int64_t r = r0 + rr, c = c0 + cc;
-      if (r < d.rows && c < d.cols) x[c * d.ldx + r] = from_f<XT>(sm[cc * kSmPitch + rr]);
+  if (mode == 0) store8(d.m + e, mv);
+  store8(static_cast<XT*>(d.x) + x_index(d, e), gh);
+  return acc;
+}
+
+template <typename XT, typename GT>
+__device__ float momentum_chunk(const MatDesc& d, int64_t begin, int64_t count, const GT* g,
+                                const MuonConsts& k, int mode) {
+  float acc = 0.f;
+  if ((d.cols & 7) == 0) {
+    // rows hold whole vectors; count is a multiple of 8
+    const int64_t nvec = count >> 3;
+    int64_t v = threadIdx.x;
+    for (; v + kElemThreads < nvec; v += 2 * kElemThreads) {
+      acc += momentum_vec<XT>(d, begin + v * 8, g, k, mode);
+      acc += momentum_vec<XT>(d, begin + (v + kElemThreads) * 8, g, k, mode);
+    }
+    if (v < nvec) acc += momentum_vec<XT>(d, begin + v * 8, g, k, mode);
+  } else {
+    XT* x = static_cast<XT*>(d.x);
+    for (int64_t e = begin + threadIdx.x; e < begin + count; e += kElemThreads) {
+      const float gv = to_f(g[e]);
+      float gh = gv;
+      if (mode == 0) {
+        const float mv = d.m[e];
+        gh = __fadd_rn(__fmul_rn(k.b1, mv), __fmul_rn(k.c1, gv));
+        d.m[e] = __fadd_rn(__fmul_rn(k.b2, mv), __fmul_rn(k.c2, gv));
+      }
+      acc = fmaf(gh, gh, acc);
+      x[x_index(d, e)] = from_f<XT>(gh);
     }
   }
   return acc;
 }
 
 template <typename XT>
-__global__ void __cluster_dims__(kNormCluster, 1, 1) __launch_bounds__(kElemThreads)
-    momentum_norm_kernel(const MatDesc* __restrict__ mats, const ElemTile* __restrict__ tiles,
-                         const void* const* __restrict__ grads, MuonConsts k, int mode) {
-  __shared__ float sm[kElemTileC * kSmPitch];
-  __shared__ float red[kElemThreads / 32];
-  __shared__ float cta_sum;
-  const ElemTile et = tiles[blockIdx.x];
-  float acc = 0.f;
-  if (et.tile >= 0) {
-    const MatDesc& d = mats[et.mat];
+__global__ void __launch_bounds__(kElemThreads)
+    momentum_norm_kernel(const MatDesc* __restrict__ mats, const ElemChunk* __restrict__ chunks,
+                         int nchunks, const void* const* __restrict__ grads, MuonConsts k, int mode) {
+  for (int c = blockIdx.x; c < nchunks; c += gridDim.x) {
+    const ElemChunk ch = chunks[c];
+    const MatDesc& d = mats[ch.mat];
     const void* src = mode == 0 ? grads[d.grad_slot] : d.w;
+    float acc;
     if (d.wdt == LM_BF16)
-      acc = momentum_norm_tile<XT>(d, et.tile, static_cast<const __nv_bfloat16*>(src), k, mode, sm);
+      acc = momentum_chunk<XT>(d, ch.begin, ch.count, static_cast<const __nv_bfloat16*>(src), k, mode);
     else
-      acc = momentum_norm_tile<XT>(d, et.tile, static_cast<const float*>(src), k, mode, sm);
-  }
+      acc = momentum_chunk<XT>(d, ch.begin, ch.count, static_cast<const float*>(src), k, mode);
+    // ||G_hat||_F^2: warp shuffle, then one fp64 atomic per warp and chunk
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    float s = 0.f;
-#pragma unroll
-    for (int i = 0; i < kElemThreads / 32; ++i) s += red[i];
-    cta_sum = s;
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if ((threadIdx.x & 31) == 0) atomicAdd(d.norm2, (double)acc);
   }
-  // Every CTA of a cluster works on the same matrix: reduce the cluster's
-  // partial sums through distributed shared memory, one atomic per cluster.
-  cg::cluster_group cluster = cg::this_cluster();
-  cluster.sync();
-  if (cluster.block_rank() == 0 && threadIdx.x == 0) {
-    double s = 0.0;
-    for (unsigned r = 0; r < cluster.num_blocks(); ++r) s += (double)*cluster.map_shared_rank(&cta_sum, r);
-    atomicAdd(mats[et.mat].norm2, s);
-  }
-  cluster.sync();
 }
 
-// ---------------------------------------------------------------------------
-// Muon: finalize (parameter write) / msign output
-// ---------------------------------------------------------------------------
+// W <- W - eta_M (s X_K + lambda W), or out = X_K (msign); X_K is scaled by
+// 1/(||G_hat|| + eps) when no NS iteration ran.
 template <typename XT, typename PT>
-__device__ void finalize_tile(const MatDesc& d, int tile, const MuonConsts& k, int mode, float xs,
-                              bool scale_x, float* sm) {
-  const int tr = tile / d.tiles_c, tcol = tile - tr * d.tiles_c;
-  const int64_t r0 = (int64_t)tr * kElemTileR, c0 = (int64_t)tcol * kElemTileC;
-  const XT* x = static_cast<const XT*>(d.x_final);
-  if (d.transposed) {
-    // stage X_K[c][r] (r contiguous in memory) into sm[cc][rr]
-    for (int it = 0; it < (kElemTileR * kElemTileC) / kElemThreads; ++it) {
-      const int slot = threadIdx.x + it * kElemThreads;
-      const int cc = slot / kElemTileR, rr = slot % kElemTileR;
-      const int64_t r = r0 + rr, c = c0 + cc;
-      sm[cc * kSmPitch + rr] = (r < d.rows && c < d.cols) ? to_f(x[c * d.ldx + r]) : 0.f;
-    }
-    __syncthreads();
+__device__ __forceinline__ void finalize_vec(const MatDesc& d, int64_t e, PT* p, const MuonConsts& k,
+                                             int mode, float xs, bool scale_x) {
+  float xv[8], pv[8];
+  load8(static_cast<const XT*>(d.x_final) + x_index(d, e), xv);
+  if (mode == 0) load8(p + e, pv);
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    if (scale_x) xv[j] = __fmul_rn(xv[j], xs);
+    pv[j] = mode == 0 ? __fsub_rn(pv[j], __fmul_rn(k.eM, __fadd_rn(__fmul_rn(d.shape_scale, xv[j]),
+                                                                   __fmul_rn(k.lam, pv[j]))))
+                      : xv[j];
   }
+  store8(p + e, pv);
+}
+
+template <typename XT, typename PT>
+__device__ void finalize_chunk(const MatDesc& d, int64_t begin, int64_t count, const MuonConsts& k,
+                               int mode, float xs, bool scale_x) {
   PT* p = static_cast<PT*>(mode == 0 ? d.w : d.out);
-  const bool vec = (d.cols & 7) == 0;
-#pragma unroll
-  for (int it = 0; it < 4; ++it) {
-    const int slot = threadIdx.x + it * kElemThreads;
-    const int rr = slot >> 4, vv = slot & 15;
-    const int64_t r = r0 + rr, c = c0 + vv * 8;
-    if (r >= d.rows || c >= d.cols) continue;
-    const int cnt = (int)min((int64_t)8, d.cols - c);
-    const int64_t off = r * d.cols + c;
-    float xv[8];
-    if (d.transposed) {
-#pragma unroll
-      for (int e = 0; e < 8; ++e) xv[e] = sm[(vv * 8 + e) * kSmPitch + rr];
-    } else if (vec) {
-      load8(x + r * d.ldx + c, xv);
-    } else {
-#pragma unroll
-      for (int e = 0; e < 8; ++e) xv[e] = e < cnt ? to_f(x[r * d.ldx + c + e]) : 0.f;
+  if ((d.cols & 7) == 0) {
+    const int64_t nvec = count >> 3;
+    int64_t v = threadIdx.x;
+    for (; v + kElemThreads < nvec; v += 2 * kElemThreads) {
+      finalize_vec<XT>(d, begin + v * 8, p, k, mode, xs, scale_x);
+      finalize_vec<XT>(d, begin + (v + kElemThreads) * 8, p, k, mode, xs, scale_x);
     }
-    if (scale_x) {
-#pragma unroll
-      for (int e = 0; e < 8; ++e) xv[e] = __fmul_rn(xv[e], xs);
-    }
-    float pv[8];
-    if (mode == 0) {
-      if (vec) {
-        load8(p + off, pv);
-      } else {
-#pragma unroll
-        for (int e = 0; e < 8; ++e) pv[e] = e < cnt ? to_f(p[off + e]) : 0.f;
-      }
-#pragma unroll
-      for (int e = 0; e < 8; ++e)
-        pv[e] = __fsub_rn(pv[e], __fmul_rn(k.eM, __fadd_rn(__fmul_rn(d.shape_scale, xv[e]),
-                                                           __fmul_rn(k.lam, pv[e]))));
-    } else {
-#pragma unroll
-      for (int e = 0; e < 8; ++e) pv[e] = xv[e];
-    }
-    if (vec) {
-      store8(p + off, pv);
-    } else {
-      for (int e = 0; e < cnt; ++e) p[off + e] = from_f<PT>(pv[e]);
+    if (v < nvec) finalize_vec<XT>(d, begin + v * 8, p, k, mode, xs, scale_x);
+  } else {
+    const XT* x = static_cast<const XT*>(d.x_final);
+    for (int64_t e = begin + threadIdx.x; e < begin + count; e += kElemThreads) {
+      float xv = to_f(x[x_index(d, e)]);
+      if (scale_x) xv = __fmul_rn(xv, xs);
+      float pv = mode == 0 ? to_f(p[e]) : 0.f;
+      pv = mode == 0 ? __fsub_rn(pv, __fmul_rn(k.eM, __fadd_rn(__fmul_rn(d.shape_scale, xv),
+                                                              __fmul_rn(k.lam, pv))))
+                     : xv;
+      p[e] = from_f<PT>(pv);
     }
   }
 }
 
 template <typename XT>
 __global__ void __launch_bounds__(kElemThreads)
-    finalize_kernel(const MatDesc* __restrict__ mats, const ElemTile* __restrict__ tiles,
+    finalize_kernel(const MatDesc* __restrict__ mats, const ElemChunk* __restrict__ chunks, int nchunks,
                     MuonConsts k, int mode, unsigned* flags) {
-  __shared__ float sm[kElemTileC * kSmPitch];
-  const ElemTile et = tiles[blockIdx.x];
-  if (et.tile < 0) return;
-  const MatDesc& d = mats[et.mat];
-  const double n2 = *d.norm2;
-  const float nrm = (float)sqrt(n2);
-  if (threadIdx.x == 0 && et.tile == 0 && !isfinite(nrm)) atomicOr(flags, LM_FLAG_NONFINITE);
-  const bool scale_x = k.ns_steps == 0;
-  const float xs = scale_x ? 1.f / __fadd_rn(nrm, k.eps) : 1.f;
-  const int pdt = mode == 0 ? d.wdt : d.odt;
-  if (pdt == LM_BF16)
-    finalize_tile<XT, __nv_bfloat16>(d, et.tile, k, mode, xs, scale_x, sm);
-  else
-    finalize_tile<XT, float>(d, et.tile, k, mode, xs, scale_x, sm);
+  for (int c = blockIdx.x; c < nchunks; c += gridDim.x) {
+    const ElemChunk ch = chunks[c];
+    const MatDesc& d = mats[ch.mat];
+    const float nrm = (float)sqrt(*d.norm2);
+    if (threadIdx.x == 0 && ch.begin == 0 && !isfinite(nrm)) atomicOr(flags, LM_FLAG_NONFINITE);
+    const bool scale_x = k.ns_steps == 0;
+    const float xs = scale_x ? 1.f / __fadd_rn(nrm, k.eps) : 1.f;
+    const int pdt = mode == 0 ? d.wdt : d.odt;
+    if (pdt == LM_BF16)
+      finalize_chunk<XT, __nv_bfloat16>(d, ch.begin, ch.count, k, mode, xs, scale_x);
+    else
+      finalize_chunk<XT, float>(d, ch.begin, ch.count, k, mode, xs, scale_x);
+  }
 }
 
 __global__ void upload_ptrs_kernel(const void** dst, const __grid_constant__ PtrUpload src,
@@ -362,27 +306,42 @@ cudaError_t launch_lion(lm_dtype dt, const LionTensor* tensors, const LionChunk*
   return cudaGetLastError();
 }
 
-cudaError_t launch_momentum_norm(lm_dtype xdt, const MatDesc* mats, const ElemTile* tiles,
-                                 int ntiles, const void* const* grads, MuonConsts k, int mode,
+int elem_grid_size() {
+  int dev = 0, sms = 0, per_sm = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, finalize_kernel<__nv_bfloat16>, kElemThreads, 0);
+  if (per_sm < 1) per_sm = 1;
+  if (sms < 1) sms = 1;
+  return sms * per_sm;
+}
+
+cudaError_t launch_momentum_norm(lm_dtype xdt, const MatDesc* mats, const ElemChunk* chunks,
+                                 int nchunks, const void* const* grads, MuonConsts k, int mode,
                                  cudaStream_t st) {
-  if (ntiles <= 0) return cudaSuccess;
-  if (ntiles % kNormCluster != 0) return cudaErrorInvalidValue;
+  if (nchunks <= 0) return cudaSuccess;
+  static int grid_cap = 0;
+  if (grid_cap == 0) grid_cap = elem_grid_size();
+  const int grid = nchunks < grid_cap ? nchunks : grid_cap;
   count_launch();
   if (xdt == LM_BF16)
-    momentum_norm_kernel<__nv_bfloat16><<<ntiles, kElemThreads, 0, st>>>(mats, tiles, grads, k, mode);
+    momentum_norm_kernel<__nv_bfloat16><<<grid, kElemThreads, 0, st>>>(mats, chunks, nchunks, grads, k, mode);
   else
-    momentum_norm_kernel<float><<<ntiles, kElemThreads, 0, st>>>(mats, tiles, grads, k, mode);
+    momentum_norm_kernel<float><<<grid, kElemThreads, 0, st>>>(mats, chunks, nchunks, grads, k, mode);
   return cudaGetLastError();
 }
 
-cudaError_t launch_finalize(lm_dtype xdt, const MatDesc* mats, const ElemTile* tiles, int ntiles,
+cudaError_t launch_finalize(lm_dtype xdt, const MatDesc* mats, const ElemChunk* chunks, int nchunks,
                             MuonConsts k, int mode, unsigned* flags, cudaStream_t st) {
-  if (ntiles <= 0) return cudaSuccess;
+  if (nchunks <= 0) return cudaSuccess;
+  static int grid_cap = 0;
+  if (grid_cap == 0) grid_cap = elem_grid_size();
+  const int grid = nchunks < grid_cap ? nchunks : grid_cap;
   count_launch();
   if (xdt == LM_BF16)
-    finalize_kernel<__nv_bfloat16><<<ntiles, kElemThreads, 0, st>>>(mats, tiles, k, mode, flags);
+    finalize_kernel<__nv_bfloat16><<<grid, kElemThreads, 0, st>>>(mats, chunks, nchunks, k, mode, flags);
   else
-    finalize_kernel<float><<<ntiles, kElemThreads, 0, st>>>(mats, tiles, k, mode, flags);
+    finalize_kernel<float><<<grid, kElemThreads, 0, st>>>(mats, chunks, nchunks, k, mode, flags);
   return cudaGetLastError();
 }
 

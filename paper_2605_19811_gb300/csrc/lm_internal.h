@@ -44,43 +44,42 @@ int lion_grid_size(lm_dtype dt);
 struct MatDesc {
   void* w;          // parameter (rows x cols, dtype wdt); for msign: the input
   float* m;         // momentum (NULL for msign: no momentum)
-  void* x;          // X buffer base for this matrix (wide orientation, s_pad x l_pad)
+  void* x;          // X buffer base for this matrix (the parameter's orientation, padded)
   void* x_final;    // the buffer holding X_K after the NS iterations
   void* out;        // msign output (rows x cols, dtype odt), or NULL
   double* norm2;    // Frobenius-norm^2 accumulator of G_hat
   int64_t rows, cols;
-  int64_t ldx;      // row pitch of X (elements) = l_pad
+  int64_t ldx;      // row pitch of X (elements): l_pad (wide) or s_pad (tall)
   int32_t grad_slot;
-  int32_t transposed;   // rows > cols: X = G_hat^T
+  int32_t pad_;
   int32_t wdt;      // lm_dtype of w (and the gradient)
   int32_t odt;      // lm_dtype of out
   float shape_scale;    // 0.2*sqrt(max(rows, cols))
-  int32_t tiles_r, tiles_c;   // tile grid of the source matrix
 };
-// One entry per CTA: the matrix and the tile; tile < 0 is an empty cluster slot.
-struct ElemTile {
+// A range of elements of one matrix (row-major over rows x cols); begin is a
+// multiple of 8.
+struct ElemChunk {
   int32_t mat;
-  int32_t tile;
+  int32_t pad_;
+  int64_t begin;
+  int64_t count;
 };
+constexpr int64_t kElemChunk = 32768;   // elements per chunk
 struct MuonConsts {
   float b1, c1, b2, c2;   // interpolation / momentum constants
   float eM, lam;          // Muon learning rate and weight decay
   float eps;              // NS normalisation eps
   int32_t ns_steps;
 };
-constexpr int kElemTileR = 64;    // tile rows of the source matrix
-constexpr int kElemTileC = 128;   // tile cols of the source matrix
-constexpr int kNormCluster = 8;   // CTAs per cluster in the norm reduction
-
 // mode 0: Muon momentum step (G_hat from grads + momentum, M update)
 // mode 1: msign input (G_hat = input tensor, no momentum)
-cudaError_t launch_momentum_norm(lm_dtype xdt, const MatDesc* mats, const ElemTile* tiles,
-                                 int ntiles, const void* const* grads, MuonConsts k,
+cudaError_t launch_momentum_norm(lm_dtype xdt, const MatDesc* mats, const ElemChunk* chunks,
+                                 int nchunks, const void* const* grads, MuonConsts k,
                                  int mode, cudaStream_t st);
 // mode 0: W <- W - eM (scale X_K' + lam W); mode 1: out = X_K'
 // where X_K' = X_K, or X_K / (||G_hat|| + eps) when ns_steps == 0.
-cudaError_t launch_finalize(lm_dtype xdt, const MatDesc* mats, const ElemTile* tiles,
-                            int ntiles, MuonConsts k, int mode, unsigned* flags,
+cudaError_t launch_finalize(lm_dtype xdt, const MatDesc* mats, const ElemChunk* chunks,
+                            int nchunks, MuonConsts k, int mode, unsigned* flags,
                             cudaStream_t st);
 
 // ---------------------------------------------------------------------------
@@ -93,7 +92,9 @@ struct NsGroup {
   int32_t s, l;           // true sizes (s = min, l = max)
   int32_t s_pad, l_pad;   // padded sizes of the workspace buffers
   int32_t first_mat;      // index of the group's first matrix in the norm array
-  void* X[2];             // ping-pong X: count x s_pad x l_pad
+  int32_t tall;           // 1: X kept as l x s (rows > cols), 0: as s x l
+  int32_t pad_;
+  void* X[2];             // ping-pong X: count x (s_pad x l_pad, or l_pad x s_pad if tall)
   void* A;                // count x s_pad x s_pad
   void* B;                // count x s_pad x s_pad
 };

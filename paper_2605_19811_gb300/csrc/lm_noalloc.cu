@@ -49,9 +49,10 @@ size_t align256(size_t x) { return (x + 255) / 256 * 256; }
 // Number of tiles of one Newton-Schulz phase for a single matrix, and the
 // (tm, tn) of tile k in the same order the allocating path builds them
 // (row-major; symmetric phases keep tiles that reach the diagonal).
-__host__ __device__ inline int phase_tiles(int phase, int s_pad, int l_pad, int bm, int bn) {
-  const int tms = (s_pad + bm - 1) / bm;
-  const int ncol = phase == NS_APPLY ? l_pad : s_pad;
+__host__ __device__ inline int phase_tiles(int phase, int s_pad, int l_pad, int tall, int bm, int bn) {
+  const int nrow = (phase == NS_APPLY && tall) ? l_pad : s_pad;
+  const int ncol = phase == NS_APPLY ? (tall ? s_pad : l_pad) : s_pad;
+  const int tms = (nrow + bm - 1) / bm;
   const int tns = (ncol + bn - 1) / bn;
   if (phase == NS_APPLY) return tms * tns;
   int n = 0;
@@ -66,9 +67,8 @@ struct BuildArgs {
   NsGroup group;
   MatDesc* d_mat;
   NsGroup* d_group;
-  ElemTile* d_etiles;
-  int n_etiles;
-  int n_real_etiles;
+  ElemChunk* d_chunks;
+  int n_chunks;
   NsTile* d_tiles[3];
   int bm, bn;
   double* d_norm2;
@@ -84,13 +84,17 @@ __global__ void build_tables_kernel(BuildArgs a) {
     *a.d_norm2 = 0.0;
     *a.d_flags = 0u;
   }
-  for (int i = threadIdx.x; i < a.n_etiles; i += blockDim.x)
-    a.d_etiles[i] = ElemTile{0, i < a.n_real_etiles ? i : -1};
+  const int64_t numel = a.mat.rows * a.mat.cols;
+  for (int i = threadIdx.x; i < a.n_chunks; i += blockDim.x) {
+    const int64_t b = (int64_t)i * kElemChunk;
+    a.d_chunks[i] = ElemChunk{0, 0, b, numel - b < kElemChunk ? numel - b : kElemChunk};
+  }
   if (threadIdx.x < 3) {
     const int ph = threadIdx.x;
     const NsGroup& g = a.group;
-    const int tms = (g.s_pad + a.bm - 1) / a.bm;
-    const int ncol = ph == NS_APPLY ? g.l_pad : g.s_pad;
+    const int nrow = (ph == NS_APPLY && g.tall) ? g.l_pad : g.s_pad;
+    const int ncol = ph == NS_APPLY ? (g.tall ? g.s_pad : g.l_pad) : g.s_pad;
+    const int tms = (nrow + a.bm - 1) / a.bm;
     const int tns = (ncol + a.bn - 1) / a.bn;
     int k = 0;
     for (int tm = 0; tm < tms; ++tm)
@@ -142,19 +146,18 @@ extern "C" lm_status lm_msign_ns_noalloc(const lm_tensor* in, lm_tensor* out, in
   const int l_pad = xdt == LM_BF16 ? tc_pad_l(l) : simt_pad(l);
   const int bm = xdt == LM_BF16 ? kTcBM : kSimtBM, bn = xdt == LM_BF16 ? kTcBN : kSimtBN;
   const size_t es = xdt == LM_BF16 ? 2 : 4;
-  const int tiles_r = (int)((in->rows + kElemTileR - 1) / kElemTileR);
-  const int tiles_c = (int)((in->cols + kElemTileC - 1) / kElemTileC);
-  const int n_real_et = tiles_r * tiles_c;
-  const int n_et = (n_real_et + kNormCluster - 1) / kNormCluster * kNormCluster;
+  const int tall = in->rows > in->cols ? 1 : 0;
+  const int64_t numel = in->rows * in->cols;
+  const int n_et = (int)((numel + kElemChunk - 1) / kElemChunk);
   int ntiles[3];
-  for (int ph = 0; ph < 3; ++ph) ntiles[ph] = phase_tiles(ph, s_pad, l_pad, bm, bn);
+  for (int ph = 0; ph < 3; ++ph) ntiles[ph] = phase_tiles(ph, s_pad, l_pad, tall, bm, bn);
 
   size_t off = 0;
   const size_t off_flags = off;   off = align256(off + sizeof(unsigned));
   const size_t off_norm = off;    off = align256(off + sizeof(double));
   const size_t off_mat = off;     off = align256(off + sizeof(MatDesc));
   const size_t off_group = off;   off = align256(off + sizeof(NsGroup));
-  const size_t off_et = off;      off = align256(off + (size_t)n_et * sizeof(ElemTile));
+  const size_t off_et = off;      off = align256(off + (size_t)n_et * sizeof(ElemChunk));
   size_t off_tiles[3];
   for (int ph = 0; ph < 3; ++ph) {
     off_tiles[ph] = off;
@@ -186,6 +189,7 @@ extern "C" lm_status lm_msign_ns_noalloc(const lm_tensor* in, lm_tensor* out, in
   g.s_pad = s_pad;
   g.l_pad = l_pad;
   g.first_mat = 0;
+  g.tall = tall;
   g.X[0] = base + off_x0;
   g.X[1] = base + off_x1;
   g.A = base + off_a;
@@ -202,20 +206,16 @@ extern "C" lm_status lm_msign_ns_noalloc(const lm_tensor* in, lm_tensor* out, in
   d.norm2 = reinterpret_cast<double*>(base + off_norm);
   d.rows = in->rows;
   d.cols = in->cols;
-  d.ldx = l_pad;
+  d.ldx = tall ? s_pad : l_pad;
   d.grad_slot = 0;
-  d.transposed = in->rows > in->cols ? 1 : 0;
   d.wdt = in->dtype;
   d.odt = out->dtype;
   d.shape_scale = 1.f;
-  d.tiles_r = tiles_r;
-  d.tiles_c = tiles_c;
   ba.group = g;
   ba.d_mat = reinterpret_cast<MatDesc*>(base + off_mat);
   ba.d_group = reinterpret_cast<NsGroup*>(base + off_group);
-  ba.d_etiles = reinterpret_cast<ElemTile*>(base + off_et);
-  ba.n_etiles = n_et;
-  ba.n_real_etiles = n_real_et;
+  ba.d_chunks = reinterpret_cast<ElemChunk*>(base + off_et);
+  ba.n_chunks = n_et;
   for (int ph = 0; ph < 3; ++ph) ba.d_tiles[ph] = reinterpret_cast<NsTile*>(base + off_tiles[ph]);
   ba.bm = bm;
   ba.bn = bn;
@@ -240,7 +240,7 @@ extern "C" lm_status lm_msign_ns_noalloc(const lm_tensor* in, lm_tensor* out, in
   memset(&mk, 0, sizeof(mk));
   mk.eps = (float)eps;
   mk.ns_steps = steps;
-  e = launch_momentum_norm(xdt, ba.d_mat, ba.d_etiles, n_et, nullptr, mk, 1, stream);
+  e = launch_momentum_norm(xdt, ba.d_mat, ba.d_chunks, n_et, nullptr, mk, 1, stream);
   if (e != cudaSuccess) return set_error(LM_ERR_CUDA, cudaGetErrorString(e));
   const NsCoeffs co{(float)a, (float)b, (float)c, (float)eps};
   for (int it = 0; it < steps; ++it)
@@ -253,7 +253,7 @@ extern "C" lm_status lm_msign_ns_noalloc(const lm_tensor* in, lm_tensor* out, in
                            stream);
       if (e != cudaSuccess) return set_error(LM_ERR_CUDA, cudaGetErrorString(e));
     }
-  e = launch_finalize(xdt, ba.d_mat, ba.d_etiles, n_et, mk, 1, ba.d_flags, stream);
+  e = launch_finalize(xdt, ba.d_mat, ba.d_chunks, n_et, mk, 1, ba.d_flags, stream);
   if (e != cudaSuccess) return set_error(LM_ERR_CUDA, cudaGetErrorString(e));
   return LM_OK;
 }

@@ -3,16 +3,17 @@
 // per pair), operands staged by TMA into 128-byte-swizzled shared memory, a
 // persistent grouped schedule over all same-shape matrices.
 //
-// Per NS iteration (Section 2, odd-polynomial Newton-Schulz), with X in the
-// wide orientation (s x l) and the normalisation X / (||G_hat||_F + eps)
-// folded into iteration 0:
+// Per NS iteration (Section 2, odd-polynomial Newton-Schulz), with the
+// normalisation X / (||G_hat||_F + eps) folded into iteration 0.  A wide
+// matrix (s x l, s <= l) iterates as
 //   GRAM : A  = X X^T          K = l, upper-triangle tiles, mirrored store
 //   POLY : B  = b A + c A A    K = s, upper-triangle tiles, mirrored store;
 //                              the epilogue reads the A tile
-//   APPLY: X' = a X + B X      K = s, all tiles; the epilogue reads the X tile,
-//                              X enters the MMA as an MN-major operand
-// A and A A are symmetric, so A A = A A^T and both GEMM operands of GRAM and
-// POLY are K-major rows of the same matrix.
+//   APPLY: X' = a X + B X      K = s, all tiles; the epilogue reads the X tile
+// and a tall one (l x s, kept in its own orientation) as A = X^T X and
+// X' = a X + X B, which is the same function (p(X X^T) X = X p(X^T X)).
+// A and A A are symmetric, so A A = A A^T and X B = X B^T: every operand is
+// either K-major rows or MN-major columns of a stored matrix.
 //
 // A cluster of two CTAs computes one 256 x 256 tile: CTA r holds rows
 // [128 r, 128 r + 128) of the A operand and N-rows [128 r, 128 r + 128) of the
@@ -107,10 +108,10 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 // Bounded wait for the phase with the given parity.  Returns false if the
-// time limit passed or another role asked to stop.
-__device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                       uint64_t limit_ns) {
-  if (mbar_try_wait(bar, parity)) return true;
+// time limit passed or another role asked to stop.  The first probe is
+// inlined; the slow path is a call.
+__device__ __noinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                            uint64_t limit_ns) {
   const uint64_t t0 = globaltimer();
   for (uint32_t i = 1;; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
@@ -119,6 +120,11 @@ __device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile 
       if (globaltimer() - t0 > limit_ns) return false;
     }
   }
+}
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                          uint64_t limit_ns) {
+  if (mbar_try_wait(bar, parity)) return true;
+  return mbar_wait_slow(bar, parity, abort_flag, limit_ns);
 }
 // 3-D tiled TMA load into this CTA's shared memory; completion is signalled
 // on the mbarrier at shared::cluster address bar_cluster (either CTA of the pair).
@@ -254,9 +260,49 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr, uint32_t lbo, uin
 // Instruction descriptor, kind::f16: D fp32, A and B bf16, A K-major,
 // B K-major or MN-major, N >> 3 at bit 17, M >> 4 at bit 24 (M = 256 for a
 // CTA pair).
-__host__ __device__ constexpr uint32_t make_idesc(int m, int n, bool b_mn_major) {
-  return (1u << 4) | (1u << 7) | (1u << 10) | ((b_mn_major ? 1u : 0u) << 16) |
-         ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
+__host__ __device__ constexpr uint32_t make_idesc(int m, int n, bool a_mn_major, bool b_mn_major) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((a_mn_major ? 1u : 0u) << 15) |
+         ((b_mn_major ? 1u : 0u) << 16) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
+}
+
+// Operands of one tile.  Wide groups hold X as s x l, tall groups as l x s
+// (the parameter's own orientation):
+//   GRAM  wide: A = X X^T, both operands K-major rows of X (K = l)
+//         tall: A = X^T X, both operands MN-major columns of X (K = l)
+//   POLY      : B = b A + c A A, both operands K-major rows of A (K = s)
+//   APPLY wide: X' = a X + B X, B rows K-major, X MN-major (K = s)
+//         tall: X' = a X + X B, X rows K-major, B rows K-major (B symmetric)
+struct TileOps {
+  const CUtensorMap* map_a;
+  const CUtensorMap* map_b;
+  bool a_mn, b_mn;
+  int K;
+};
+__device__ __forceinline__ TileOps tile_ops(int phase, const NsGroup& g, const TcGroupMaps& mp, int cur) {
+  TileOps o;
+  if (phase == NS_GRAM) {
+    const bool mn = g.tall != 0;
+    o.map_a = mn ? &mp.xmn[cur] : &mp.xk[cur];
+    o.map_b = o.map_a;
+    o.a_mn = o.b_mn = mn;
+    o.K = g.l_pad;
+  } else if (phase == NS_POLY) {
+    o.map_a = o.map_b = &mp.a;
+    o.a_mn = o.b_mn = false;
+    o.K = g.s_pad;
+  } else if (g.tall) {
+    o.map_a = &mp.xk[cur];
+    o.map_b = &mp.b;
+    o.a_mn = o.b_mn = false;
+    o.K = g.s_pad;
+  } else {
+    o.map_a = &mp.b;
+    o.map_b = &mp.xmn[cur];
+    o.a_mn = false;
+    o.b_mn = true;
+    o.K = g.s_pad;
+  }
+  return o;
 }
 
 __device__ __forceinline__ float bf_lo(uint32_t v) { return __uint_as_float(v << 16); }
@@ -264,6 +310,48 @@ __device__ __forceinline__ float bf_hi(uint32_t v) { return __uint_as_float(v & 
 __device__ __forceinline__ uint32_t pack_bf2(float lo, float hi) {
   __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&h);
+}
+
+// Producer k-loop of one tile, specialised on the operand layouts (a loop
+// with per-block layout branches measured ~12% slower end to end).
+// K-major operand half: one 64 (K) x 128 box; MN-major: two 64 (MN) x 64 (K)
+// boxes.  Returns false if a wait gave up.
+struct ProducerRing {
+  int stage;
+  uint32_t ph;
+  int armed[kStages];
+};
+template <bool AMN, bool BMN>
+__device__ __forceinline__ bool produce_tile(ProducerRing& R, uint8_t* smem, uint64_t* full, uint64_t* empty,
+                                             volatile int* abort_flag, uint32_t rank, int nk,
+                                             const CUtensorMap* map_a, const CUtensorMap* map_b,
+                                             int row_a, int col_b, int mat) {
+  for (int kb = 0; kb < nk; ++kb) {
+    if (!mbar_wait(&empty[R.stage], R.ph ^ 1u, abort_flag, kWaitLimitNs)) return false;
+    uint8_t* sa = smem + (size_t)R.stage * kStageBytes;
+    uint8_t* sb = sa + kABytes;
+    const uint32_t fb = peer_addr(&full[R.stage], 0);
+    if (rank == 0) mbar_arrive_expect_tx(&full[R.stage], 2 * kStageBytes);
+    R.armed[R.stage] = (int)R.ph;
+    const int k0 = kb * BK;
+    if (!AMN) {
+      tma_load_3d(sa, map_a, fb, k0, row_a, mat);
+    } else {
+      tma_load_3d(sa, map_a, fb, row_a, k0, mat);
+      tma_load_3d(sa + 64 * BK * 2, map_a, fb, row_a + 64, k0, mat);
+    }
+    if (!BMN) {
+      tma_load_3d(sb, map_b, fb, k0, col_b, mat);
+    } else {
+      tma_load_3d(sb, map_b, fb, col_b, k0, mat);
+      tma_load_3d(sb + 64 * BK * 2, map_b, fb, col_b + 64, k0, mat);
+    }
+    if (++R.stage == kStages) {
+      R.stage = 0;
+      R.ph ^= 1u;
+    }
+  }
+  return true;
 }
 
 // ------------------------------- the kernel ---------------------------------
@@ -326,67 +414,41 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     // ------------------------------ producer ------------------------------
     if (lane == 0) {
-      int armed[kStages];
-      for (int s = 0; s < kStages; ++s) armed[s] = -1;
-      int stage = 0;
-      uint32_t ph = 0;
+      ProducerRing R;
+      R.stage = 0;
+      R.ph = 0;
+      for (int s = 0; s < kStages; ++s) R.armed[s] = -1;
       bool ok = true;
       for (int w = w_begin; ok && w < w_end; w += w_step) {
         const NsTile t = p.tiles[w];
         const NsGroup& g = p.groups[t.group];
-        const TcGroupMaps& mp = p.maps[t.group];
-        const CUtensorMap* mapA;
-        const CUtensorMap* mapB;
-        int K;
-        if (phase == NS_GRAM) {
-          mapA = &mp.xk[cur]; mapB = &mp.xk[cur]; K = g.l_pad;
-        } else if (phase == NS_POLY) {
-          mapA = &mp.a; mapB = &mp.a; K = g.s_pad;
-        } else {
-          mapA = &mp.b; mapB = &mp.xmn[cur]; K = g.s_pad;
-        }
-        const int nk = K / BK;
+        const TileOps ops = tile_ops(phase, g, p.maps[t.group], cur);
+        const int nk = ops.K / BK;
         const int row_a = t.tm * BM + (int)rank * kHalf;
         const int col_b = t.tn * BN + (int)rank * kHalf;
-        for (int kb = 0; kb < nk; ++kb) {
-          if (!mbar_wait(&empty[stage], ph ^ 1u, abort_flag, kWaitLimitNs)) {
-            give_up();
-            ok = false;
-            break;
-          }
-          uint8_t* sa = smem + (size_t)stage * kStageBytes;
-          uint8_t* sb = sa + kABytes;
-          const uint32_t fb = peer_addr(&full[stage], 0);
-          if (rank == 0) mbar_arrive_expect_tx(&full[stage], 2 * kStageBytes);
-          armed[stage] = (int)ph;
-          const int k0 = kb * BK;
-          tma_load_3d(sa, mapA, fb, k0, row_a, t.mat);
-          if (phase != NS_APPLY) {
-            tma_load_3d(sb, mapB, fb, k0, col_b, t.mat);
-          } else {
-#pragma unroll
-            for (int q = 0; q < kHalf / 64; ++q)
-              tma_load_3d(sb + q * (64 * BK * 2), mapB, fb, col_b + 64 * q, k0, t.mat);
-          }
-          if (++stage == kStages) {
-            stage = 0;
-            ph ^= 1u;
-          }
-        }
+        if (!ops.a_mn && !ops.b_mn)
+          ok = produce_tile<false, false>(R, smem, full, empty, abort_flag, rank, nk, ops.map_a, ops.map_b,
+                                          row_a, col_b, t.mat);
+        else if (!ops.a_mn)
+          ok = produce_tile<false, true>(R, smem, full, empty, abort_flag, rank, nk, ops.map_a, ops.map_b,
+                                         row_a, col_b, t.mat);
+        else
+          ok = produce_tile<true, true>(R, smem, full, empty, abort_flag, rank, nk, ops.map_a, ops.map_b,
+                                        row_a, col_b, t.mat);
+        if (!ok) give_up();
       }
       if (!ok && rank == 0) {
         // let the copies already issued land before the CTA exits
         for (int s = 0; s < kStages; ++s)
-          if (armed[s] >= 0) {
+          if (R.armed[s] >= 0) {
             volatile int never = 0;
-            mbar_wait(&full[s], (uint32_t)armed[s], &never, 100000000ull);
+            mbar_wait(&full[s], (uint32_t)R.armed[s], &never, 100000000ull);
           }
       }
     }
   } else if (warp == 1) {
     // ------------------------------ MMA issuer -----------------------------
     if (lane == 0 && rank == 0) {
-      const uint32_t idesc = make_idesc(BM, BN, phase == NS_APPLY);
       int stage = 0;
       uint32_t ph = 0;
       int ab = 0;
@@ -395,8 +457,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       for (int w = w_begin; ok && w < w_end; w += w_step) {
         const NsTile t = p.tiles[w];
         const NsGroup& g = p.groups[t.group];
-        const int K = (phase == NS_GRAM) ? g.l_pad : g.s_pad;
-        const int nk = K / BK;
+        const TileOps ops = tile_ops(phase, g, p.maps[t.group], cur);
+        const int nk = ops.K / BK;
+        const uint32_t idesc = make_idesc(BM, BN, ops.a_mn, ops.b_mn);
         if (!mbar_wait(&accempty[ab], aph ^ 1u, abort_flag, kWaitLimitNs)) {
           give_up();
           break;
@@ -414,10 +477,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           const uint32_t sb = sa + kABytes;
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk) {
-            const uint64_t adesc = sw128_desc(sa + kk * 32, 16, 1024);
-            const uint64_t bdesc = (phase == NS_APPLY)
-                                       ? sw128_desc(sb + kk * 2048, 64 * BK * 2, 1024)
-                                       : sw128_desc(sb + kk * 32, 16, 1024);
+            const uint64_t adesc = ops.a_mn ? sw128_desc(sa + kk * 2048, 64 * BK * 2, 1024)
+                                            : sw128_desc(sa + kk * 32, 16, 1024);
+            const uint64_t bdesc = ops.b_mn ? sw128_desc(sb + kk * 2048, 64 * BK * 2, 1024)
+                                            : sw128_desc(sb + kk * 32, 16, 1024);
             umma_bf16(d_tmem, adesc, bdesc, idesc, (kb | kk) != 0 ? 1u : 0u);
           }
           umma_commit_pair(&empty[stage]);
@@ -502,10 +565,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const int i = t.tm * BM + (int)rank * kHalf + row;
       const size_t sq = (size_t)g.s_pad * g.s_pad;
       const size_t xs = (size_t)g.s_pad * g.l_pad;
-      const int ncols = (phase == NS_APPLY) ? g.l : g.s;
-      const int ld = (phase == NS_APPLY) ? g.l_pad : g.s_pad;
-      const int jmax = (phase == NS_APPLY) ? g.l_pad : g.s_pad;
-      const bool row_in = i < g.s_pad;        // rows past the padded matrix are skipped
+      // output extents: s x s (GRAM, POLY); s x l (APPLY, wide); l x s (APPLY, tall)
+      const bool apply_tall = phase == NS_APPLY && g.tall;
+      const int nrows = apply_tall ? g.l : g.s;
+      const int row_lim = apply_tall ? g.l_pad : g.s_pad;
+      const int ncols = (phase == NS_APPLY) ? (g.tall ? g.s : g.l) : g.s;
+      const int ld = (phase == NS_APPLY) ? (g.tall ? g.s_pad : g.l_pad) : g.s_pad;
+      const int jmax = ld;
+      const bool row_in = i < row_lim;        // rows past the padded matrix are skipped
       __nv_bfloat16* out;
       if (phase == NS_GRAM) {
         out = static_cast<__nv_bfloat16*>(g.A) + t.mat * sq;
@@ -549,7 +616,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           if (phase == NS_GRAM) o = acc * nscale;
           else if (phase == NS_POLY) o = p.co.b * v[e] + p.co.c * acc;
           else o = (p.co.a * v[e] + acc) * nscale;
-          v[e] = (i < g.s && j < ncols) ? o : 0.f;
+          v[e] = (i < nrows && j < ncols) ? o : 0.f;
         }
         if (!sym) {
           // APPLY: results replace the aux values, stored by TMA below
@@ -589,11 +656,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         fence_proxy_async_smem();
         __syncwarp();
         const int r0 = t.tm * BM + (int)rank * kHalf + q * 32;
-        if (lane == 0 && r0 < g.s_pad) {
+        if (lane == 0 && r0 < row_lim) {
 #pragma unroll
           for (int b = 2 * half; b < 2 * half + 2; ++b)
-            tma_store_3d(&p.maps[t.group].xst[cur ^ 1], auxbuf + b * kAuxBoxBytes + q * 32 * 128,
-                         t.tn * BN + 64 * b, r0, t.mat);
+            if (t.tn * BN + 64 * b < jmax)   // boxes past the padded columns hold nothing
+              tma_store_3d(&p.maps[t.group].xst[cur ^ 1], auxbuf + b * kAuxBoxBytes + q * 32 * 128,
+                           t.tn * BN + 64 * b, r0, t.mat);
           bulk_commit();
           bulk_wait_read();   // auxbuf may be refilled once the stores have read it
         }
@@ -650,10 +718,12 @@ int tc_pad_l(int l) { return (l + BN - 1) / BN * BN; }
 
 cudaError_t tc_encode_group_maps(const NsGroup& g, TcGroupMaps* maps) {
   cudaError_t e;
+  // X buffers: s_pad x l_pad (wide) or l_pad x s_pad (tall), row-major
+  const uint64_t inner = g.tall ? g.s_pad : g.l_pad, rows = g.tall ? g.l_pad : g.s_pad;
   for (int b = 0; b < 2; ++b) {
-    if ((e = encode_3d(&maps->xk[b], g.X[b], g.l_pad, g.s_pad, g.count, BK, kHalf)) != cudaSuccess) return e;
-    if ((e = encode_3d(&maps->xst[b], g.X[b], g.l_pad, g.s_pad, g.count, 64, 32)) != cudaSuccess) return e;
-    if ((e = encode_3d(&maps->xmn[b], g.X[b], g.l_pad, g.s_pad, g.count, 64, BK)) != cudaSuccess) return e;
+    if ((e = encode_3d(&maps->xk[b], g.X[b], inner, rows, g.count, BK, kHalf)) != cudaSuccess) return e;
+    if ((e = encode_3d(&maps->xst[b], g.X[b], inner, rows, g.count, 64, 32)) != cudaSuccess) return e;
+    if ((e = encode_3d(&maps->xmn[b], g.X[b], inner, rows, g.count, 64, BK)) != cudaSuccess) return e;
   }
   if ((e = encode_3d(&maps->a, g.A, g.s_pad, g.s_pad, g.count, BK, kHalf)) != cudaSuccess) return e;
   if ((e = encode_3d(&maps->b, g.B, g.s_pad, g.s_pad, g.count, BK, kHalf)) != cudaSuccess) return e;
