@@ -452,8 +452,8 @@ struct lm_state {
   int lion_grid[2] = {0, 0};
   int nmat = 0;
   MatDesc* d_mats = nullptr;
-  ElemChunk* d_echunks = nullptr;
-  int n_echunks = 0;
+  ElemChunk* d_echunks[2] = {nullptr, nullptr};   // chunks of bf16 / fp32 matrices
+  int n_echunks[2] = {0, 0};
   NsEngine ns;
   unsigned* d_flags = nullptr;
   cudaStream_t last_stream = nullptr;
@@ -583,10 +583,10 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
     d.rows = p.rows;
     d.cols = p.cols;
   }
-  std::vector<ElemChunk> echunks;
-  build_elem_chunks(mats, echunks);
-  s->n_echunks = (int)echunks.size();
-  const size_t off_echunks = ar.add(echunks.size() * sizeof(ElemChunk));
+  // element chunks, split by the parameter dtype (filled once dtypes are bound)
+  std::vector<ElemChunk> echunks_all;
+  build_elem_chunks(mats, echunks_all);
+  const size_t off_echunks = ar.add(echunks_all.size() * sizeof(ElemChunk));
 
   cudaError_t e = cudaMalloc(&s->base, ar.total);
   if (e != cudaSuccess) {
@@ -639,9 +639,18 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
     }
   }
   if (s->nmat) memcpy(img.data() + off_mats, mats.data(), mats.size() * sizeof(MatDesc));
-  if (!echunks.empty()) memcpy(img.data() + off_echunks, echunks.data(), echunks.size() * sizeof(ElemChunk));
+  {
+    std::vector<ElemChunk> sorted;
+    for (int dt = 0; dt < 2; ++dt) {
+      for (const ElemChunk& c : echunks_all)
+        if (mats[c.mat].wdt == dt) sorted.push_back(c);
+      s->n_echunks[dt] = (int)sorted.size() - (dt == 1 ? s->n_echunks[0] : 0);
+    }
+    if (!sorted.empty()) memcpy(img.data() + off_echunks, sorted.data(), sorted.size() * sizeof(ElemChunk));
+  }
   s->d_mats = reinterpret_cast<MatDesc*>(base + off_mats);
-  s->d_echunks = reinterpret_cast<ElemChunk*>(base + off_echunks);
+  s->d_echunks[0] = reinterpret_cast<ElemChunk*>(base + off_echunks);
+  s->d_echunks[1] = s->d_echunks[0] + s->n_echunks[0];
 
   // Upload tables and zeros (momentum M_{-1} = 0, workspace padding = 0).
   e = cudaMemcpyAsync(base, img.data(), ar.total, cudaMemcpyHostToDevice, stream);
@@ -722,11 +731,14 @@ lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t, void* c
       return cudaMemsetAsync(s->ns.d_norm2, 0, (size_t)s->nmat * sizeof(double), stream);
     });
     if (e != cudaSuccess) return cuda_fail(e, "norm reset");
-    e = timed(P, LM_KERNEL_MOMENTUM_NORM, stream, [&]() {
-      return launch_momentum_norm(s->ns.xdt, s->d_mats, s->d_echunks, s->n_echunks, s->d_grads, mk, 0,
-                                  stream);
-    });
-    if (e != cudaSuccess) return cuda_fail(e, "momentum/norm kernel launch");
+    for (int dt = 0; dt < 2; ++dt) {
+      if (s->n_echunks[dt] == 0) continue;
+      e = timed(P, LM_KERNEL_MOMENTUM_NORM, stream, [&]() {
+        return launch_momentum_norm(s->ns.xdt, (lm_dtype)dt, s->d_mats, s->d_echunks[dt], s->n_echunks[dt],
+                                    s->d_grads, mk, 0, stream);
+      });
+      if (e != cudaSuccess) return cuda_fail(e, "momentum/norm kernel launch");
+    }
   }
   for (int d = 0; d < 2; ++d) {
     if (s->lion_vec[d].nchunks == 0) continue;
@@ -739,10 +751,14 @@ lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t, void* c
   if (s->nmat > 0) {
     NsCoeffs co{(float)c.ns_a, (float)c.ns_b, (float)c.ns_c, (float)c.ns_eps};
     if ((st = run_ns(s->ns, c.ns_steps, co, s->d_flags, stream, P)) != LM_OK) return st;
-    e = timed(P, LM_KERNEL_FINALIZE, stream, [&]() {
-      return launch_finalize(s->ns.xdt, s->d_mats, s->d_echunks, s->n_echunks, mk, 0, s->d_flags, stream);
-    });
-    if (e != cudaSuccess) return cuda_fail(e, "finalize kernel launch");
+    for (int dt = 0; dt < 2; ++dt) {
+      if (s->n_echunks[dt] == 0) continue;
+      e = timed(P, LM_KERNEL_FINALIZE, stream, [&]() {
+        return launch_finalize(s->ns.xdt, (lm_dtype)dt, s->d_mats, s->d_echunks[dt], s->n_echunks[dt], mk, 0,
+                               s->d_flags, stream);
+      });
+      if (e != cudaSuccess) return cuda_fail(e, "finalize kernel launch");
+    }
   }
   return LM_OK;
 }
@@ -907,11 +923,11 @@ lm_status lm_msign_ns(const lm_tensor* in, lm_tensor* out, int steps, double a, 
   MatDesc* dm = reinterpret_cast<MatDesc*>(base + off_mat);
   ElemChunk* de = reinterpret_cast<ElemChunk*>(base + off_et);
   unsigned* dflags = reinterpret_cast<unsigned*>(base + off_flags);
-  e = launch_momentum_norm(E.xdt, dm, de, (int)et.size(), nullptr, mk, 1, stream);
+  e = launch_momentum_norm(E.xdt, in->dtype, dm, de, (int)et.size(), nullptr, mk, 1, stream);
   if (e != cudaSuccess) return cleanup(cuda_fail(e, "norm kernel launch"));
   NsCoeffs co{(float)a, (float)b, (float)c, (float)eps};
   if ((st = run_ns(E, steps, co, dflags, stream)) != LM_OK) return cleanup(st);
-  e = launch_finalize(E.xdt, dm, de, (int)et.size(), mk, 1, dflags, stream);
+  e = launch_finalize(E.xdt, out->dtype, dm, de, (int)et.size(), mk, 1, dflags, stream);
   if (e != cudaSuccess) return cleanup(cuda_fail(e, "output kernel launch"));
   return cleanup(LM_OK);
 }

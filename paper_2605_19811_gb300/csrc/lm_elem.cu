@@ -128,18 +128,20 @@ __global__ void __launch_bounds__(kLionThreads)
 constexpr int kElemThreads = 256;
 
 __device__ __forceinline__ int64_t x_index(const MatDesc& d, int64_t e) {
+  // matrices in a state have fewer than 2^32 elements per row-block here;
+  // 32-bit division when the element index fits
+  if (e < 0xFFFFFFFFll && d.cols < 0xFFFFFFFFll) {
+    const uint32_t r = (uint32_t)e / (uint32_t)d.cols;
+    return (int64_t)r * d.ldx + (e - (int64_t)r * d.cols);
+  }
   const int64_t r = e / d.cols;
   return r * d.ldx + (e - r * d.cols);
 }
 
-// One vector of 8 elements of the Muon direction: G_hat = b1 M + c1 G (fp32,
-// same operation order as the Lion step), M <- b2 M + c2 G, X0 = G_hat.
-template <typename XT, typename GT>
-__device__ __forceinline__ float momentum_vec(const MatDesc& d, int64_t e, const GT* g,
-                                              const MuonConsts& k, int mode) {
-  float gv[8], mv[8], gh[8];
-  load8(g + e, gv);
-  if (mode == 0) load8(d.m + e, mv);
+// Muon direction for 8 elements: G_hat = b1 M + c1 G (fp32, same operation
+// order as the Lion step), M <- b2 M + c2 G; returns sum G_hat^2.
+__device__ __forceinline__ float momentum_math(float (&gv)[8], float (&mv)[8], float (&gh)[8],
+                                               const MuonConsts& k, int mode) {
   float acc = 0.f;
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
@@ -151,8 +153,6 @@ __device__ __forceinline__ float momentum_vec(const MatDesc& d, int64_t e, const
     }
     acc = fmaf(gh[j], gh[j], acc);
   }
-  if (mode == 0) store8(d.m + e, mv);
-  store8(static_cast<XT*>(d.x) + x_index(d, e), gh);
   return acc;
 }
 
@@ -160,17 +160,40 @@ template <typename XT, typename GT>
 __device__ float momentum_chunk(const MatDesc& d, int64_t begin, int64_t count, const GT* g,
                                 const MuonConsts& k, int mode) {
   float acc = 0.f;
+  XT* x = static_cast<XT*>(d.x);
   if ((d.cols & 7) == 0) {
-    // rows hold whole vectors; count is a multiple of 8
+    // rows hold whole vectors; count is a multiple of 8.  Two vectors per
+    // trip, both loaded before anything is stored.
     const int64_t nvec = count >> 3;
     int64_t v = threadIdx.x;
     for (; v + kElemThreads < nvec; v += 2 * kElemThreads) {
-      acc += momentum_vec<XT>(d, begin + v * 8, g, k, mode);
-      acc += momentum_vec<XT>(d, begin + (v + kElemThreads) * 8, g, k, mode);
+      const int64_t ea = begin + v * 8, eb = ea + kElemThreads * 8;
+      float ga[8], ma[8], gb[8], mb[8], ha[8], hb[8];
+      load8(g + ea, ga);
+      load8(g + eb, gb);
+      if (mode == 0) {
+        load8(d.m + ea, ma);
+        load8(d.m + eb, mb);
+      }
+      acc += momentum_math(ga, ma, ha, k, mode);
+      acc += momentum_math(gb, mb, hb, k, mode);
+      if (mode == 0) {
+        store8(d.m + ea, ma);
+        store8(d.m + eb, mb);
+      }
+      store8(x + x_index(d, ea), ha);
+      store8(x + x_index(d, eb), hb);
     }
-    if (v < nvec) acc += momentum_vec<XT>(d, begin + v * 8, g, k, mode);
+    if (v < nvec) {
+      const int64_t ea = begin + v * 8;
+      float ga[8], ma[8], ha[8];
+      load8(g + ea, ga);
+      if (mode == 0) load8(d.m + ea, ma);
+      acc += momentum_math(ga, ma, ha, k, mode);
+      if (mode == 0) store8(d.m + ea, ma);
+      store8(x + x_index(d, ea), ha);
+    }
   } else {
-    XT* x = static_cast<XT*>(d.x);
     for (int64_t e = begin + threadIdx.x; e < begin + count; e += kElemThreads) {
       const float gv = to_f(g[e]);
       float gh = gv;
@@ -186,19 +209,15 @@ __device__ float momentum_chunk(const MatDesc& d, int64_t begin, int64_t count, 
   return acc;
 }
 
-template <typename XT>
-__global__ void __launch_bounds__(kElemThreads)
+template <typename XT, typename GT, int MODE>
+__global__ void __launch_bounds__(kElemThreads, 3)
     momentum_norm_kernel(const MatDesc* __restrict__ mats, const ElemChunk* __restrict__ chunks,
-                         int nchunks, const void* const* __restrict__ grads, MuonConsts k, int mode) {
+                         int nchunks, const void* const* __restrict__ grads, MuonConsts k) {
   for (int c = blockIdx.x; c < nchunks; c += gridDim.x) {
     const ElemChunk ch = chunks[c];
     const MatDesc& d = mats[ch.mat];
-    const void* src = mode == 0 ? grads[d.grad_slot] : d.w;
-    float acc;
-    if (d.wdt == LM_BF16)
-      acc = momentum_chunk<XT>(d, ch.begin, ch.count, static_cast<const __nv_bfloat16*>(src), k, mode);
-    else
-      acc = momentum_chunk<XT>(d, ch.begin, ch.count, static_cast<const float*>(src), k, mode);
+    const GT* src = static_cast<const GT*>(MODE == 0 ? grads[d.grad_slot] : d.w);
+    float acc = momentum_chunk<XT>(d, ch.begin, ch.count, src, k, MODE);
     // ||G_hat||_F^2: warp shuffle, then one fp64 atomic per warp and chunk
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
@@ -208,36 +227,48 @@ __global__ void __launch_bounds__(kElemThreads)
 
 // W <- W - eta_M (s X_K + lambda W), or out = X_K (msign); X_K is scaled by
 // 1/(||G_hat|| + eps) when no NS iteration ran.
-template <typename XT, typename PT>
-__device__ __forceinline__ void finalize_vec(const MatDesc& d, int64_t e, PT* p, const MuonConsts& k,
-                                             int mode, float xs, bool scale_x) {
-  float xv[8], pv[8];
-  load8(static_cast<const XT*>(d.x_final) + x_index(d, e), xv);
-  if (mode == 0) load8(p + e, pv);
+__device__ __forceinline__ void finalize_math(float (&xv)[8], float (&pv)[8], float shape_scale,
+                                              const MuonConsts& k, int mode, float xs, bool scale_x) {
 #pragma unroll
   for (int j = 0; j < 8; ++j) {
     if (scale_x) xv[j] = __fmul_rn(xv[j], xs);
-    pv[j] = mode == 0 ? __fsub_rn(pv[j], __fmul_rn(k.eM, __fadd_rn(__fmul_rn(d.shape_scale, xv[j]),
+    pv[j] = mode == 0 ? __fsub_rn(pv[j], __fmul_rn(k.eM, __fadd_rn(__fmul_rn(shape_scale, xv[j]),
                                                                    __fmul_rn(k.lam, pv[j]))))
                       : xv[j];
   }
-  store8(p + e, pv);
 }
 
 template <typename XT, typename PT>
 __device__ void finalize_chunk(const MatDesc& d, int64_t begin, int64_t count, const MuonConsts& k,
                                int mode, float xs, bool scale_x) {
   PT* p = static_cast<PT*>(mode == 0 ? d.w : d.out);
+  const XT* x = static_cast<const XT*>(d.x_final);
   if ((d.cols & 7) == 0) {
     const int64_t nvec = count >> 3;
     int64_t v = threadIdx.x;
     for (; v + kElemThreads < nvec; v += 2 * kElemThreads) {
-      finalize_vec<XT>(d, begin + v * 8, p, k, mode, xs, scale_x);
-      finalize_vec<XT>(d, begin + (v + kElemThreads) * 8, p, k, mode, xs, scale_x);
+      const int64_t ea = begin + v * 8, eb = ea + kElemThreads * 8;
+      float xa[8], pa[8], xb[8], pb[8];
+      load8(x + x_index(d, ea), xa);
+      load8(x + x_index(d, eb), xb);
+      if (mode == 0) {
+        load8(p + ea, pa);
+        load8(p + eb, pb);
+      }
+      finalize_math(xa, pa, d.shape_scale, k, mode, xs, scale_x);
+      finalize_math(xb, pb, d.shape_scale, k, mode, xs, scale_x);
+      store8(p + ea, pa);
+      store8(p + eb, pb);
     }
-    if (v < nvec) finalize_vec<XT>(d, begin + v * 8, p, k, mode, xs, scale_x);
+    if (v < nvec) {
+      const int64_t ea = begin + v * 8;
+      float xa[8], pa[8];
+      load8(x + x_index(d, ea), xa);
+      if (mode == 0) load8(p + ea, pa);
+      finalize_math(xa, pa, d.shape_scale, k, mode, xs, scale_x);
+      store8(p + ea, pa);
+    }
   } else {
-    const XT* x = static_cast<const XT*>(d.x_final);
     for (int64_t e = begin + threadIdx.x; e < begin + count; e += kElemThreads) {
       float xv = to_f(x[x_index(d, e)]);
       if (scale_x) xv = __fmul_rn(xv, xs);
@@ -250,10 +281,10 @@ __device__ void finalize_chunk(const MatDesc& d, int64_t begin, int64_t count, c
   }
 }
 
-template <typename XT>
-__global__ void __launch_bounds__(kElemThreads)
+template <typename XT, typename PT, int MODE>
+__global__ void __launch_bounds__(kElemThreads, 3)
     finalize_kernel(const MatDesc* __restrict__ mats, const ElemChunk* __restrict__ chunks, int nchunks,
-                    MuonConsts k, int mode, unsigned* flags) {
+                    MuonConsts k, unsigned* flags) {
   for (int c = blockIdx.x; c < nchunks; c += gridDim.x) {
     const ElemChunk ch = chunks[c];
     const MatDesc& d = mats[ch.mat];
@@ -261,11 +292,7 @@ __global__ void __launch_bounds__(kElemThreads)
     if (threadIdx.x == 0 && ch.begin == 0 && !isfinite(nrm)) atomicOr(flags, LM_FLAG_NONFINITE);
     const bool scale_x = k.ns_steps == 0;
     const float xs = scale_x ? 1.f / __fadd_rn(nrm, k.eps) : 1.f;
-    const int pdt = mode == 0 ? d.wdt : d.odt;
-    if (pdt == LM_BF16)
-      finalize_chunk<XT, __nv_bfloat16>(d, ch.begin, ch.count, k, mode, xs, scale_x);
-    else
-      finalize_chunk<XT, float>(d, ch.begin, ch.count, k, mode, xs, scale_x);
+    finalize_chunk<XT, PT>(d, ch.begin, ch.count, k, MODE, xs, scale_x);
   }
 }
 
@@ -310,13 +337,33 @@ int elem_grid_size() {
   int dev = 0, sms = 0, per_sm = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, finalize_kernel<__nv_bfloat16>, kElemThreads, 0);
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, finalize_kernel<__nv_bfloat16, __nv_bfloat16, 0>,
+                                                kElemThreads, 0);
   if (per_sm < 1) per_sm = 1;
   if (sms < 1) sms = 1;
   return sms * per_sm;
 }
 
-cudaError_t launch_momentum_norm(lm_dtype xdt, const MatDesc* mats, const ElemChunk* chunks,
+namespace {
+template <typename XT, typename GT>
+void mn_launch(int grid, cudaStream_t st, const MatDesc* mats, const ElemChunk* chunks, int nchunks,
+               const void* const* grads, MuonConsts k, int mode) {
+  if (mode == 0)
+    momentum_norm_kernel<XT, GT, 0><<<grid, kElemThreads, 0, st>>>(mats, chunks, nchunks, grads, k);
+  else
+    momentum_norm_kernel<XT, GT, 1><<<grid, kElemThreads, 0, st>>>(mats, chunks, nchunks, grads, k);
+}
+template <typename XT, typename PT>
+void fin_launch(int grid, cudaStream_t st, const MatDesc* mats, const ElemChunk* chunks, int nchunks,
+                MuonConsts k, int mode, unsigned* flags) {
+  if (mode == 0)
+    finalize_kernel<XT, PT, 0><<<grid, kElemThreads, 0, st>>>(mats, chunks, nchunks, k, flags);
+  else
+    finalize_kernel<XT, PT, 1><<<grid, kElemThreads, 0, st>>>(mats, chunks, nchunks, k, flags);
+}
+}  // namespace
+
+cudaError_t launch_momentum_norm(lm_dtype xdt, lm_dtype gdt, const MatDesc* mats, const ElemChunk* chunks,
                                  int nchunks, const void* const* grads, MuonConsts k, int mode,
                                  cudaStream_t st) {
   if (nchunks <= 0) return cudaSuccess;
@@ -324,24 +371,30 @@ cudaError_t launch_momentum_norm(lm_dtype xdt, const MatDesc* mats, const ElemCh
   if (grid_cap == 0) grid_cap = elem_grid_size();
   const int grid = nchunks < grid_cap ? nchunks : grid_cap;
   count_launch();
-  if (xdt == LM_BF16)
-    momentum_norm_kernel<__nv_bfloat16><<<grid, kElemThreads, 0, st>>>(mats, chunks, nchunks, grads, k, mode);
-  else
-    momentum_norm_kernel<float><<<grid, kElemThreads, 0, st>>>(mats, chunks, nchunks, grads, k, mode);
+  if (xdt == LM_BF16) {
+    if (gdt == LM_BF16) mn_launch<__nv_bfloat16, __nv_bfloat16>(grid, st, mats, chunks, nchunks, grads, k, mode);
+    else mn_launch<__nv_bfloat16, float>(grid, st, mats, chunks, nchunks, grads, k, mode);
+  } else {
+    if (gdt == LM_BF16) mn_launch<float, __nv_bfloat16>(grid, st, mats, chunks, nchunks, grads, k, mode);
+    else mn_launch<float, float>(grid, st, mats, chunks, nchunks, grads, k, mode);
+  }
   return cudaGetLastError();
 }
 
-cudaError_t launch_finalize(lm_dtype xdt, const MatDesc* mats, const ElemChunk* chunks, int nchunks,
-                            MuonConsts k, int mode, unsigned* flags, cudaStream_t st) {
+cudaError_t launch_finalize(lm_dtype xdt, lm_dtype pdt, const MatDesc* mats, const ElemChunk* chunks,
+                            int nchunks, MuonConsts k, int mode, unsigned* flags, cudaStream_t st) {
   if (nchunks <= 0) return cudaSuccess;
   static int grid_cap = 0;
   if (grid_cap == 0) grid_cap = elem_grid_size();
   const int grid = nchunks < grid_cap ? nchunks : grid_cap;
   count_launch();
-  if (xdt == LM_BF16)
-    finalize_kernel<__nv_bfloat16><<<grid, kElemThreads, 0, st>>>(mats, chunks, nchunks, k, mode, flags);
-  else
-    finalize_kernel<float><<<grid, kElemThreads, 0, st>>>(mats, chunks, nchunks, k, mode, flags);
+  if (xdt == LM_BF16) {
+    if (pdt == LM_BF16) fin_launch<__nv_bfloat16, __nv_bfloat16>(grid, st, mats, chunks, nchunks, k, mode, flags);
+    else fin_launch<__nv_bfloat16, float>(grid, st, mats, chunks, nchunks, k, mode, flags);
+  } else {
+    if (pdt == LM_BF16) fin_launch<float, __nv_bfloat16>(grid, st, mats, chunks, nchunks, k, mode, flags);
+    else fin_launch<float, float>(grid, st, mats, chunks, nchunks, k, mode, flags);
+  }
   return cudaGetLastError();
 }
 

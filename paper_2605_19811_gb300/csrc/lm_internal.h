@@ -73,12 +73,14 @@ struct MuonConsts {
 };
 // mode 0: Muon momentum step (G_hat from grads + momentum, M update)
 // mode 1: msign input (G_hat = input tensor, no momentum)
-cudaError_t launch_momentum_norm(lm_dtype xdt, const MatDesc* mats, const ElemChunk* chunks,
+// gdt: dtype of every chunk's gradient (mode 0) or input (mode 1).
+cudaError_t launch_momentum_norm(lm_dtype xdt, lm_dtype gdt, const MatDesc* mats, const ElemChunk* chunks,
                                  int nchunks, const void* const* grads, MuonConsts k,
                                  int mode, cudaStream_t st);
 // mode 0: W <- W - eM (scale X_K' + lam W); mode 1: out = X_K'
 // where X_K' = X_K, or X_K / (||G_hat|| + eps) when ns_steps == 0.
-cudaError_t launch_finalize(lm_dtype xdt, const MatDesc* mats, const ElemChunk* chunks,
+// pdt: dtype of every chunk's parameter (mode 0) or output (mode 1).
+cudaError_t launch_finalize(lm_dtype xdt, lm_dtype pdt, const MatDesc* mats, const ElemChunk* chunks,
                             int nchunks, MuonConsts k, int mode, unsigned* flags,
                             cudaStream_t st);
 

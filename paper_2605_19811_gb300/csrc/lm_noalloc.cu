@@ -240,7 +240,7 @@ extern "C" lm_status lm_msign_ns_noalloc(const lm_tensor* in, lm_tensor* out, in
   memset(&mk, 0, sizeof(mk));
   mk.eps = (float)eps;
   mk.ns_steps = steps;
-  e = launch_momentum_norm(xdt, ba.d_mat, ba.d_chunks, n_et, nullptr, mk, 1, stream);
+  e = launch_momentum_norm(xdt, in->dtype, ba.d_mat, ba.d_chunks, n_et, nullptr, mk, 1, stream);
   if (e != cudaSuccess) return set_error(LM_ERR_CUDA, cudaGetErrorString(e));
   const NsCoeffs co{(float)a, (float)b, (float)c, (float)eps};
   for (int it = 0; it < steps; ++it)
@@ -253,7 +253,7 @@ extern "C" lm_status lm_msign_ns_noalloc(const lm_tensor* in, lm_tensor* out, in
                            stream);
       if (e != cudaSuccess) return set_error(LM_ERR_CUDA, cudaGetErrorString(e));
     }
-  e = launch_finalize(xdt, ba.d_mat, ba.d_chunks, n_et, mk, 1, ba.d_flags, stream);
+  e = launch_finalize(xdt, out->dtype, ba.d_mat, ba.d_chunks, n_et, mk, 1, ba.d_flags, stream);
   if (e != cudaSuccess) return set_error(LM_ERR_CUDA, cudaGetErrorString(e));
   return LM_OK;
 }
