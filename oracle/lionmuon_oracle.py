@@ -166,8 +166,9 @@ def ns_scalar_map(x: np.ndarray, steps: int, a: float, b: float, c: float) -> np
 # ---------------------------------------------------------------------------
 
 def lion_update(W, G_hat, eta_lion, weight_decay):
-    """Lion branch of Algorithm 1: W <- W - eta_L (sign(G_hat) + lambda W)."""
-    return W - eta_lion * (sign(G_hat) + weight_decay * W)
+    """Lion branch of Algorithm 1: W <- W - eta_L (sign(G_hat) + lambda W)
+    (in fp64 whatever the precision G_hat was formed in)."""
+    return W - eta_lion * (sign(G_hat).astype(np.float64) + weight_decay * W)
 
 
 def muon_update(W, G_hat, cfg: Config):
@@ -203,7 +204,7 @@ def lionmuon_param_step(W, G, M_prev, t: int, cfg: Config, sign_in_f32: bool = F
         if sign_in_f32:
             b1, c1 = np.float32(cfg.beta1), np.float32(1.0 - cfg.beta1)
             direction = (b1 * M_prev.astype(np.float32)) + (c1 * G.astype(np.float32))
-        W_new = W - cfg.eta_lion * (sign(direction).astype(np.float64) + cfg.weight_decay * W)
+        W_new = lion_update(W, direction, cfg.eta_lion, cfg.weight_decay)
     M_new = momentum_update(M_prev, G, cfg.beta2)
     return W_new, M_new
 
