@@ -222,6 +222,17 @@ def cpu_cores():
 # the two arms
 # ---------------------------------------------------------------------------
 
+def max_over_ranks(value: float, world: int, device) -> float:
+    """Max of a per-rank scalar over all ranks (the timing rule for N > 1)."""
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 def dist_env():
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -333,11 +344,7 @@ def run_ours(args):
     launches = L.kernel_launch_count() - launches0
     prof = opt.profile_read()
     opt.profile(False)
-    ms_total = ev0.elapsed_time(ev1)
-    if world > 1:
-        tt = torch.tensor([ms_total], device=dev, dtype=torch.float64)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms_total = float(tt.item())
+    ms_total = max_over_ranks(ev0.elapsed_time(ev1), world, dev)
     ms_per_step = ms_total / args.steps
     value = ms_per_step / world
 
@@ -358,11 +365,7 @@ def run_ours(args):
         e1.record(stream)
         torch.cuda.synchronize()
         barrier()
-        e_ms = e0.elapsed_time(e1)
-        if world > 1:
-            tt = torch.tensor([e_ms], device=dev, dtype=torch.float64)
-            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-            e_ms = float(tt.item())
+        e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
         e2e = {"value": e_ms / args.steps / world, "unit": "ms/step", "h2d_bytes_per_step": flat_bytes,
                "d2h_bytes_per_step": flat_bytes,
                "what": "pinned-host gradients copied in, lm_step, updated parameters copied out, per step"}
@@ -387,7 +390,6 @@ def run_ours(args):
                 "per_launch_tflop": fl / max(ns_launches, 1) / 1e12,
                 "peak_kind": f"bf16 sustained, {peak_src}",
                 "flops": "symmetric count 3 s^2 l + s^3 per matrix per NS iteration"}
-    lion_bytes = 14.0 * numel if args.precision else 14.0 * numel
     lion_roof = None
     if lion_ms > 0:
         # Lion-step launches over all params: 14 B/param (bf16 W,G r/w W, fp32 M r/w)

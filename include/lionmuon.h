@@ -190,6 +190,17 @@ const char* lm_last_error(void);
  * monotonically increasing counter, for launch accounting by benchmarks). */
 uint64_t lm_kernel_launch_count(void);
 
+/* Failure-detection probe: launches one thread that waits, with the bounded
+ * wait every device-side wait of this library uses, on a barrier that nothing
+ * signals.  When limit_ns passes the kernel records LM_FLAG_TIMEOUT and
+ * returns normally, leaving the context usable.  Synchronises cuda_stream and
+ * stores the flags in *device_flags.  Returns LM_ERR_TIMEOUT when the wait gave
+ * up (the expected outcome), LM_OK otherwise.  The paper has no counterpart;
+ * it tests the library's own error path.  Errors: LM_ERR_INVALID_ARG (NULL,
+ * limit_ns outside (0, 1e10]), LM_ERR_UNSUPPORTED, LM_ERR_CUDA. */
+lm_status lm_probe_bounded_wait(uint64_t limit_ns, uint32_t* device_flags,
+                                void* cuda_stream);
+
 /* Per-kernel-family timing, measured with CUDA events recorded on the
  * launching stream around every kernel launch of lm_step while enabled. */
 typedef enum {

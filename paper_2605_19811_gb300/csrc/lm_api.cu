@@ -842,6 +842,29 @@ lm_status lm_profile_read(lm_state* s, lm_profile* out, int reset) {
   return LM_OK;
 }
 
+lm_status lm_probe_bounded_wait(uint64_t limit_ns, uint32_t* device_flags, void* cuda_stream) {
+  if (device_flags == nullptr) return fail(LM_ERR_INVALID_ARG, "device_flags is NULL");
+  if (limit_ns == 0 || limit_ns > 10000000000ull) return fail(LM_ERR_INVALID_ARG, "limit_ns must be in (0, 1e10]");
+  lm_status st;
+  int dev = 0;
+  if ((st = check_device(&dev)) != LM_OK) return st;
+  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+  unsigned* d = nullptr;
+  cudaError_t e = cudaMallocAsync(reinterpret_cast<void**>(&d), sizeof(unsigned), stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMallocAsync(probe flag)");
+  unsigned h = 0;
+  e = cudaMemsetAsync(d, 0, sizeof(unsigned), stream);
+  if (e == cudaSuccess) e = launch_bounded_wait_probe(limit_ns, d, stream);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(&h, d, sizeof(unsigned), cudaMemcpyDeviceToHost, stream);
+  cudaFreeAsync(d, stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return cuda_fail(e, "bounded-wait probe");
+  *device_flags = h;
+  return (h & LM_FLAG_TIMEOUT) ? fail(LM_ERR_TIMEOUT, "bounded wait gave up after %llu ns",
+                                      (unsigned long long)limit_ns)
+                               : LM_OK;
+}
+
 size_t lm_state_bytes(const lm_state* s) { return s ? s->mom_elems * sizeof(float) : 0; }
 
 size_t lm_workspace_bytes(const lm_state* s) {

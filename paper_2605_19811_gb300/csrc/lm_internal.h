@@ -126,6 +126,8 @@ struct TcGroupMaps {
 };
 cudaError_t tc_encode_group_maps(const NsGroup& g, TcGroupMaps* maps);
 int tc_max_pairs();   // CTA pairs that fit the device (one CTA per SM)
+// One bounded wait on a barrier that is never signalled (failure-detection probe).
+cudaError_t launch_bounded_wait_probe(uint64_t limit_ns, unsigned* flags, cudaStream_t st);
 // offsets: NULL (round robin over tiles) or npairs + 1 range starts.
 cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* groups,
                          const TcGroupMaps* maps, const NsTile* tiles, int ntiles,

@@ -684,6 +684,20 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   }
 }
 
+// Diagnostic: one thread waits, with the same bounded wait as the NS kernel,
+// on an mbarrier nobody arrives on; when the limit passes it records
+// LM_FLAG_TIMEOUT and returns normally.
+__global__ void bounded_wait_probe_kernel(uint64_t limit_ns, unsigned* flags) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    if (!mbar_wait(&bar, 0, &abort_flag, limit_ns)) atomicOr(flags, LM_FLAG_TIMEOUT);
+  }
+}
+
 PFN_cuTensorMapEncodeTiled_v12000 get_encode_fn() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
   if (fn == nullptr) {
@@ -712,6 +726,12 @@ cudaError_t encode_3d(CUtensorMap* m, void* base, uint64_t inner, uint64_t rows,
 }
 
 }  // namespace
+
+cudaError_t launch_bounded_wait_probe(uint64_t limit_ns, unsigned* flags, cudaStream_t st) {
+  count_launch();
+  bounded_wait_probe_kernel<<<1, 32, 0, st>>>(limit_ns, flags);
+  return cudaGetLastError();
+}
 
 int tc_pad_s(int s) { return (s + kHalf - 1) / kHalf * kHalf; }
 int tc_pad_l(int l) { return (l + BN - 1) / BN * BN; }

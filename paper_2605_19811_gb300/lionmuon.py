@@ -27,7 +27,7 @@ EXPORTED = ("lm_config_default", "lm_create", "lm_step", "lm_set_lr", "lm_msign_
             "lm_get_momentum", "lm_set_momentum", "lm_get_status", "lm_state_bytes",
             "lm_workspace_bytes", "lm_destroy", "lm_status_string", "lm_last_error",
             "lm_kernel_launch_count", "lm_profile_enable", "lm_profile_read",
-            "lm_msign_ns_noalloc")
+            "lm_msign_ns_noalloc", "lm_probe_bounded_wait")
 
 KERNEL_FAMILIES = ("lion", "momentum_norm", "ns_gram", "ns_poly", "ns_apply", "finalize", "other")
 
@@ -103,6 +103,8 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib.lm_last_error.restype = ctypes.c_char_p
     lib.lm_kernel_launch_count.argtypes = []
     lib.lm_kernel_launch_count.restype = ctypes.c_uint64
+    lib.lm_probe_bounded_wait.argtypes = [ctypes.c_uint64, P(ctypes.c_uint32), c_void_p]
+    lib.lm_probe_bounded_wait.restype = c_int
     lib.lm_profile_enable.argtypes = [c_void_p, c_int]
     lib.lm_profile_enable.restype = c_int
     lib.lm_profile_read.argtypes = [c_void_p, P(LmProfile), c_int]
@@ -252,6 +254,14 @@ def msign_ns(x, out, steps: int = 5, a: float = 3.4445, b: float = -4.7750, c: f
     _check(lib, lib.lm_msign_ns(ctypes.byref(di), ctypes.byref(do), steps, a, b, c, eps, precision,
                                 _stream_handle(stream)), "lm_msign_ns")
     return out
+
+
+def probe_bounded_wait(limit_ns: int, stream=None):
+    """Run the bounded-wait probe; returns (status, device flags)."""
+    lib = load_library()
+    f = ctypes.c_uint32()
+    st = lib.lm_probe_bounded_wait(limit_ns, ctypes.byref(f), _stream_handle(stream))
+    return st, int(f.value)
 
 
 def msign_ns_noalloc(x, out, steps: int = 5, a: float = 3.4445, b: float = -4.7750, c: float = 2.0315,

@@ -1,0 +1,119 @@
+"""Plant plausible mistakes in the oracle (on the CPU) and check that the pins
+in test_oracle_pins.py catch each of them: the pins are only worth something
+if a dropped term, a wrong sign, a transposed operand, the post-update buffer
+or a wrong branch makes at least one of them fail."""
+
+import math
+
+import numpy as np
+import pytest
+
+import oracle
+import oracle.lionmuon_oracle as OM
+from tests import test_oracle_pins as pins
+
+# every pin, with representative arguments for the parametrised ones
+PIN_CALLS = [
+    (pins.test_ns_closed_form_on_known_svd, (16, 64, False, oracle.NS_QUINTIC, 5)),
+    (pins.test_ns_closed_form_on_known_svd, (16, 64, True, oracle.NS_CUBIC, 7)),
+    (pins.test_ns_closed_form_on_known_svd, (16, 16, False, (2.0, -1.3, 0.4), 3)),
+    (pins.test_ns_rank_one, ()),
+    (pins.test_ns_transpose_identity, ()),
+    (pins.test_ns_orthogonal_equivariance, ()),
+    (pins.test_ns_scale_invariance, ()),
+    (pins.test_ns_zero_steps_is_normalisation, ()),
+    (pins.test_cubic_ns_converges_to_svd_msign, ()),
+    (pins.test_msign_svd_brute_force_2x2_and_rank_deficient, ()),
+    (pins.test_msign_svd_is_polar_factor, ()),
+    (pins.test_dispatch_rule, ()),
+    (pins.test_direction_uses_pre_update_buffer, ()),
+    (pins.test_lion_step_magnitude_invariant, ()),
+    (pins.test_momentum_closed_form_constant_gradient, ()),
+    (pins.test_muon_step_closed_form_on_known_svd, ()),
+    (pins.test_vectors_take_lion_step_on_muon_steps, ()),
+    (pins.test_reduction_P_infinity_beta_equal_is_signum, ()),
+    (pins.test_reduction_P_infinity_is_lion, ()),
+    (pins.test_reduction_P1_beta_equal_is_muon, ()),
+    (pins.test_period_alternation_pattern, ()),
+    (pins.test_heavy_ball_equals_ema_signmuon, ()),
+    (pins.test_decay_frank_wolfe_rewrite, ()),
+    (pins.test_bf16_round_known_values, ()),
+    (pins.test_lion_f32_matches_fp64_within_rounding, ()),
+]
+
+
+def _ns_factory(variant):
+    def ns(G, steps, a, b, c, eps=1e-7):
+        X = np.array(G, dtype=np.float64)
+        tr = X.shape[0] > X.shape[1]
+        if tr:
+            X = X.T.copy()
+        if variant != "no_normalisation":
+            X = X / (np.linalg.norm(X) + eps)
+        n = steps + 1 if variant == "extra_iteration" else steps
+        for _ in range(n):
+            A = X.T @ X if variant == "transposed_gram" and X.shape[0] == X.shape[1] else X @ X.T
+            if variant == "dropped_c":
+                B = b * A
+            elif variant == "wrong_sign_c":
+                B = b * A - c * (A @ A)
+            else:
+                B = b * A + c * (A @ A)
+            X = a * X + (X @ B if variant == "right_multiply" else B @ X)
+        return X.T.copy() if tr else X
+    return ns
+
+
+def _patch(monkeypatch, name, fn):
+    monkeypatch.setattr(OM, name, fn)
+    monkeypatch.setattr(oracle, name, fn)
+
+
+def _mutations():
+    muts = {}
+    for v in ("no_normalisation", "extra_iteration", "transposed_gram", "dropped_c", "wrong_sign_c",
+              "right_multiply"):
+        muts["ns_" + v] = [("ns_polynomial", _ns_factory(v))]
+    muts["post_update_buffer"] = [("lionmuon_param_step", _post_update_step)]
+    muts["lion_missing_decay"] = [("lion_update", lambda W, Gh, eta, lam: W - eta * OM.sign(Gh))]
+    muts["lion_wrong_sign"] = [("lion_update", lambda W, Gh, eta, lam: W + eta * (OM.sign(Gh) - lam * W))]
+    muts["momentum_uses_beta1"] = [("momentum_update", lambda M, G, b2: 0.9 * M + 0.1 * G)]
+    muts["dispatch_off_by_one"] = [("is_muon_step", lambda t, P: P != 0 and t % P == 1 % max(P, 1))]
+    muts["scale_uses_min"] = [("muon_update", _muon_min_scale)]
+    muts["bf16_truncates"] = [("bf16_round", _bf16_truncate)]
+    return muts
+
+
+def _post_update_step(W, G, M_prev, t, cfg, sign_in_f32=False):
+    W = np.asarray(W, dtype=np.float64)
+    G = np.asarray(G, dtype=np.float64)
+    M_new = OM.momentum_update(np.asarray(M_prev, dtype=np.float64), G, cfg.beta2)
+    G_hat = OM.interpolated_direction(M_new, G, cfg.beta1)
+    if OM.is_matrix(W.shape) and OM.is_muon_step(t, cfg.period):
+        return OM.muon_update(W, G_hat, cfg), M_new
+    return OM.lion_update(W, G_hat, cfg.eta_lion, cfg.weight_decay), M_new
+
+
+def _muon_min_scale(W, G_hat, cfg):
+    O = OM.ns_polynomial(G_hat, cfg.ns_steps, cfg.ns_a, cfg.ns_b, cfg.ns_c, cfg.ns_eps)
+    return W - cfg.eta_muon * (cfg.shape_scale * math.sqrt(min(W.shape)) * O + cfg.weight_decay * W)
+
+
+def _bf16_truncate(x):
+    f = np.ascontiguousarray(np.asarray(x, dtype=np.float32))
+    u = f.view(np.uint32) & np.uint32(0xFFFF0000)
+    return u.view(np.float32).copy()
+
+
+@pytest.mark.filterwarnings("ignore::RuntimeWarning")
+@pytest.mark.parametrize("name", sorted(_mutations()))
+def test_each_planted_mistake_is_caught(name, monkeypatch):
+    for fn_name, fn in _mutations()[name]:
+        _patch(monkeypatch, fn_name, fn)
+    caught = []
+    for pin, args in PIN_CALLS:
+        try:
+            pin(*args)
+        except (AssertionError, ValueError):
+            caught.append(pin.__name__)
+    assert caught, f"no pin detects the mutation {name}"
