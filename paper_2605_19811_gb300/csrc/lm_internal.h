@@ -115,14 +115,19 @@ struct NsCoeffs {
 constexpr int kTcBM = 256, kTcBN = 256, kTcBK = 64;
 int tc_pad_s(int s);
 int tc_pad_l(int l);
-// Tensor maps for one group: K-major boxes (64 x 128) on X0, X1, A, B and
-// MN-major boxes (64 x 64) on X0, X1.  Padded sizes are whole boxes.
+// Tensor maps for one group: K-major boxes (64 x 128), MN-major boxes
+// (64 x 64) and store boxes (64 x 32) on X0, X1, A, B.  A and B hold only
+// their 256 x 256 tiles on or above the diagonal.
 struct TcGroupMaps {
   CUtensorMap xk[2];    // K-major operand / aux loads: box 64 x 128
   CUtensorMap a;
   CUtensorMap b;
   CUtensorMap xmn[2];   // MN-major operand loads: box 64 x 64
-  CUtensorMap xst[2];   // X' stores: box 64 x 32
+  CUtensorMap amn;      // transposed reads of stored A / B tiles: box 64 x 64
+  CUtensorMap bmn;
+  CUtensorMap xst[2];   // result stores: box 64 x 32
+  CUtensorMap ast;
+  CUtensorMap bst;
 };
 cudaError_t tc_encode_group_maps(const NsGroup& g, TcGroupMaps* maps);
 int tc_max_pairs();   // CTA pairs that fit the device (one CTA per SM)

@@ -6,8 +6,8 @@
 // Per NS iteration (Section 2, odd-polynomial Newton-Schulz), with the
 // normalisation X / (||G_hat||_F + eps) folded into iteration 0.  A wide
 // matrix (s x l, s <= l) iterates as
-//   GRAM : A  = X X^T          K = l, upper-triangle tiles, mirrored store
-//   POLY : B  = b A + c A A    K = s, upper-triangle tiles, mirrored store;
+//   GRAM : A  = X X^T          K = l, only tiles on or above the diagonal
+//   POLY : B  = b A + c A A    K = s, only tiles on or above the diagonal;
 //                              the epilogue reads the A tile
 //   APPLY: X' = a X + B X      K = s, all tiles; the epilogue reads the X tile
 // and a tall one (l x s, kept in its own orientation) as A = X^T X and
@@ -25,11 +25,10 @@
 //   warp 0    TMA producer (one elected lane), 5-stage smem ring; both CTAs'
 //             copies signal CTA 0's full barrier
 //   warp 1    TMEM allocator (both CTAs) + MMA issuer (CTA 0, one lane)
-//   warps 2-9 epilogue: tcgen05.ld from TMEM, fused polynomial combination;
-//             GRAM/POLY store bf16 directly (direct + mirrored half), APPLY
-//             writes X' over its aux tile in shared memory and TMA-stores it;
-//             each TMEM lane quadrant is served by two warps, one per half of
-//             the tile's columns
+//   warps 2-9 epilogue: tcgen05.ld from TMEM, fused polynomial combination,
+//             results written into shared memory (over the aux tile) and
+//             stored by TMA; each TMEM lane quadrant is served by two warps,
+//             one per half of the tile's columns
 //   warp 10   aux loader: TMA of the tile the POLY/APPLY epilogue combines
 //             with the accumulator (A or X), issued while the main loop runs
 // Tiles are assigned to pairs on the host by a longest-first greedy balance
@@ -269,40 +268,56 @@ __host__ __device__ constexpr uint32_t make_idesc(int m, int n, bool a_mn_major,
 // (the parameter's own orientation):
 //   GRAM  wide: A = X X^T, both operands K-major rows of X (K = l)
 //         tall: A = X^T X, both operands MN-major columns of X (K = l)
-//   POLY      : B = b A + c A A, both operands K-major rows of A (K = s)
-//   APPLY wide: X' = a X + B X, B rows K-major, X MN-major (K = s)
-//         tall: X' = a X + X B, X rows K-major, B rows K-major (B symmetric)
-struct TileOps {
+//   POLY      : B = b A + c A A, operands rows of A (K = s)
+//   APPLY wide: X' = a X + B X, rows of B and MN-major X (K = s)
+//         tall: X' = a X + X B, K-major rows of X and rows of B (K = s)
+// A and B are symmetric and only their 256 x 256 tiles on or above the
+// diagonal are stored.  A row block r of A (or B) therefore reads K blocks
+// k >= 256 r K-major from the stored tiles, and K blocks below 256 r as the
+// transposed stored tile, i.e. MN-major.  The split falls on a 256 boundary,
+// so both CTAs of a pair use the same layout for every K block.
+struct OpSeg {
+  int kb_end;                    // K blocks [previous end, kb_end)
+  bool a_mn, b_mn;
   const CUtensorMap* map_a;
   const CUtensorMap* map_b;
-  bool a_mn, b_mn;
-  int K;
 };
-__device__ __forceinline__ TileOps tile_ops(int phase, const NsGroup& g, const TcGroupMaps& mp, int cur) {
-  TileOps o;
+struct TilePlan {
+  int nseg;
+  int nk;
+  OpSeg seg[3];
+};
+__device__ __forceinline__ void plan_push(TilePlan& P, int kb_end, bool a_mn, bool b_mn,
+                                          const CUtensorMap* ma, const CUtensorMap* mb) {
+  const int prev = P.nseg ? P.seg[P.nseg - 1].kb_end : 0;
+  if (kb_end <= prev) return;    // empty range
+  P.seg[P.nseg++] = OpSeg{kb_end, a_mn, b_mn, ma, mb};
+}
+__device__ __forceinline__ TilePlan tile_plan(int phase, const NsGroup& g, const TcGroupMaps& mp, int cur,
+                                              const NsTile& t) {
+  TilePlan P;
+  P.nseg = 0;
   if (phase == NS_GRAM) {
-    const bool mn = g.tall != 0;
-    o.map_a = mn ? &mp.xmn[cur] : &mp.xk[cur];
-    o.map_b = o.map_a;
-    o.a_mn = o.b_mn = mn;
-    o.K = g.l_pad;
-  } else if (phase == NS_POLY) {
-    o.map_a = o.map_b = &mp.a;
-    o.a_mn = o.b_mn = false;
-    o.K = g.s_pad;
-  } else if (g.tall) {
-    o.map_a = &mp.xk[cur];
-    o.map_b = &mp.b;
-    o.a_mn = o.b_mn = false;
-    o.K = g.s_pad;
-  } else {
-    o.map_a = &mp.b;
-    o.map_b = &mp.xmn[cur];
-    o.a_mn = false;
-    o.b_mn = true;
-    o.K = g.s_pad;
+    P.nk = g.l_pad / BK;
+    if (g.tall) plan_push(P, P.nk, true, true, &mp.xmn[cur], &mp.xmn[cur]);
+    else plan_push(P, P.nk, false, false, &mp.xk[cur], &mp.xk[cur]);
+    return P;
   }
-  return o;
+  P.nk = g.s_pad / BK;
+  const int ka = min(t.tm * (BM / BK), P.nk);   // first K block on or above row block tm
+  const int kn = min(t.tn * (BN / BK), P.nk);   // the same for column block tn
+  if (phase == NS_POLY) {            // A-operand rows tm, B-operand rows tn (tn >= tm)
+    plan_push(P, ka, true, true, &mp.amn, &mp.amn);
+    plan_push(P, kn, false, true, &mp.a, &mp.amn);
+    plan_push(P, P.nk, false, false, &mp.a, &mp.a);
+  } else if (!g.tall) {              // rows tm of B, X MN-major
+    plan_push(P, ka, true, true, &mp.bmn, &mp.xmn[cur]);
+    plan_push(P, P.nk, false, true, &mp.b, &mp.xmn[cur]);
+  } else {                           // rows of X K-major, rows tn of B
+    plan_push(P, kn, false, true, &mp.xk[cur], &mp.bmn);
+    plan_push(P, P.nk, false, false, &mp.xk[cur], &mp.b);
+  }
+  return P;
 }
 
 __device__ __forceinline__ float bf_lo(uint32_t v) { return __uint_as_float(v << 16); }
@@ -322,11 +337,11 @@ struct ProducerRing {
   int armed[kStages];
 };
 template <bool AMN, bool BMN>
-__device__ __forceinline__ bool produce_tile(ProducerRing& R, uint8_t* smem, uint64_t* full, uint64_t* empty,
-                                             volatile int* abort_flag, uint32_t rank, int nk,
-                                             const CUtensorMap* map_a, const CUtensorMap* map_b,
-                                             int row_a, int col_b, int mat) {
-  for (int kb = 0; kb < nk; ++kb) {
+__device__ __forceinline__ bool produce_range(ProducerRing& R, uint8_t* smem, uint64_t* full, uint64_t* empty,
+                                              volatile int* abort_flag, uint32_t rank, int kb0, int kb1,
+                                              const CUtensorMap* map_a, const CUtensorMap* map_b,
+                                              int row_a, int col_b, int mat) {
+  for (int kb = kb0; kb < kb1; ++kb) {
     if (!mbar_wait(&empty[R.stage], R.ph ^ 1u, abort_flag, kWaitLimitNs)) return false;
     uint8_t* sa = smem + (size_t)R.stage * kStageBytes;
     uint8_t* sb = sa + kABytes;
@@ -349,6 +364,32 @@ __device__ __forceinline__ bool produce_tile(ProducerRing& R, uint8_t* smem, uin
     if (++R.stage == kStages) {
       R.stage = 0;
       R.ph ^= 1u;
+    }
+  }
+  return true;
+}
+
+// MMA issue for K blocks [kb0, kb1) of one tile with fixed operand layouts.
+template <bool AMN, bool BMN>
+__device__ __forceinline__ bool mma_range(int& stage, uint32_t& ph, uint8_t* smem, uint64_t* full,
+                                          uint64_t* empty, volatile int* abort_flag, int kb0, int kb1,
+                                          uint32_t d_tmem) {
+  const uint32_t idesc = make_idesc(BM, BN, AMN, BMN);
+  for (int kb = kb0; kb < kb1; ++kb) {
+    if (!mbar_wait(&full[stage], ph, abort_flag, kWaitLimitNs)) return false;
+    tc_fence_after();
+    const uint32_t sa = smem_u32(smem + (size_t)stage * kStageBytes);
+    const uint32_t sb = sa + kABytes;
+#pragma unroll
+    for (int kk = 0; kk < BK / 16; ++kk) {
+      const uint64_t adesc = AMN ? sw128_desc(sa + kk * 2048, 64 * BK * 2, 1024) : sw128_desc(sa + kk * 32, 16, 1024);
+      const uint64_t bdesc = BMN ? sw128_desc(sb + kk * 2048, 64 * BK * 2, 1024) : sw128_desc(sb + kk * 32, 16, 1024);
+      umma_bf16(d_tmem, adesc, bdesc, idesc, (kb | kk) != 0 ? 1u : 0u);
+    }
+    umma_commit_pair(&empty[stage]);
+    if (++stage == kStages) {
+      stage = 0;
+      ph ^= 1u;
     }
   }
   return true;
@@ -422,19 +463,23 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       for (int w = w_begin; ok && w < w_end; w += w_step) {
         const NsTile t = p.tiles[w];
         const NsGroup& g = p.groups[t.group];
-        const TileOps ops = tile_ops(phase, g, p.maps[t.group], cur);
-        const int nk = ops.K / BK;
+        const TilePlan P = tile_plan(phase, g, p.maps[t.group], cur, t);
         const int row_a = t.tm * BM + (int)rank * kHalf;
         const int col_b = t.tn * BN + (int)rank * kHalf;
-        if (!ops.a_mn && !ops.b_mn)
-          ok = produce_tile<false, false>(R, smem, full, empty, abort_flag, rank, nk, ops.map_a, ops.map_b,
-                                          row_a, col_b, t.mat);
-        else if (!ops.a_mn)
-          ok = produce_tile<false, true>(R, smem, full, empty, abort_flag, rank, nk, ops.map_a, ops.map_b,
-                                         row_a, col_b, t.mat);
-        else
-          ok = produce_tile<true, true>(R, smem, full, empty, abort_flag, rank, nk, ops.map_a, ops.map_b,
-                                        row_a, col_b, t.mat);
+        int kb0 = 0;
+        for (int sg = 0; ok && sg < P.nseg; ++sg) {
+          const OpSeg& S = P.seg[sg];
+          if (!S.a_mn && !S.b_mn)
+            ok = produce_range<false, false>(R, smem, full, empty, abort_flag, rank, kb0, S.kb_end, S.map_a,
+                                             S.map_b, row_a, col_b, t.mat);
+          else if (!S.a_mn)
+            ok = produce_range<false, true>(R, smem, full, empty, abort_flag, rank, kb0, S.kb_end, S.map_a,
+                                            S.map_b, row_a, col_b, t.mat);
+          else
+            ok = produce_range<true, true>(R, smem, full, empty, abort_flag, rank, kb0, S.kb_end, S.map_a,
+                                           S.map_b, row_a, col_b, t.mat);
+          kb0 = S.kb_end;
+        }
         if (!ok) give_up();
       }
       if (!ok && rank == 0) {
@@ -457,38 +502,25 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       for (int w = w_begin; ok && w < w_end; w += w_step) {
         const NsTile t = p.tiles[w];
         const NsGroup& g = p.groups[t.group];
-        const TileOps ops = tile_ops(phase, g, p.maps[t.group], cur);
-        const int nk = ops.K / BK;
-        const uint32_t idesc = make_idesc(BM, BN, ops.a_mn, ops.b_mn);
+        const TilePlan P = tile_plan(phase, g, p.maps[t.group], cur, t);
         if (!mbar_wait(&accempty[ab], aph ^ 1u, abort_flag, kWaitLimitNs)) {
           give_up();
           break;
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(ab * BN);
-        for (int kb = 0; kb < nk; ++kb) {
-          if (!mbar_wait(&full[stage], ph, abort_flag, kWaitLimitNs)) {
-            give_up();
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const uint32_t sa = smem_u32(smem + (size_t)stage * kStageBytes);
-          const uint32_t sb = sa + kABytes;
-#pragma unroll
-          for (int kk = 0; kk < BK / 16; ++kk) {
-            const uint64_t adesc = ops.a_mn ? sw128_desc(sa + kk * 2048, 64 * BK * 2, 1024)
-                                            : sw128_desc(sa + kk * 32, 16, 1024);
-            const uint64_t bdesc = ops.b_mn ? sw128_desc(sb + kk * 2048, 64 * BK * 2, 1024)
-                                            : sw128_desc(sb + kk * 32, 16, 1024);
-            umma_bf16(d_tmem, adesc, bdesc, idesc, (kb | kk) != 0 ? 1u : 0u);
-          }
-          umma_commit_pair(&empty[stage]);
-          if (++stage == kStages) {
-            stage = 0;
-            ph ^= 1u;
-          }
+        int kb0 = 0;
+        for (int sg = 0; ok && sg < P.nseg; ++sg) {
+          const OpSeg& S = P.seg[sg];
+          if (!S.a_mn && !S.b_mn)
+            ok = mma_range<false, false>(stage, ph, smem, full, empty, abort_flag, kb0, S.kb_end, d_tmem);
+          else if (!S.a_mn)
+            ok = mma_range<false, true>(stage, ph, smem, full, empty, abort_flag, kb0, S.kb_end, d_tmem);
+          else
+            ok = mma_range<true, true>(stage, ph, smem, full, empty, abort_flag, kb0, S.kb_end, d_tmem);
+          kb0 = S.kb_end;
         }
+        if (!ok) give_up();
         if (!ok) break;
         umma_commit_pair(&accfull[ab]);
         if (++ab == kAccBufs) {
@@ -535,6 +567,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     // ------------------------------ epilogue -------------------------------
     // Thread (quadrant q, lane) owns one row of this CTA's half tile and the
     // 128 columns [half*128, half*128 + 128) of it, in four 32-column chunks.
+    // Results go into auxbuf (over the aux values, if any) in the 128-byte
+    // swizzled box layout and leave by TMA stores, 32 rows x 64 columns each.
     const int q = warp & 3;                   // TMEM lane quadrant of this warp
     const int half = (warp - 2) >> 2;         // which 128 columns of the tile
     const int row = q * 32 + lane;            // row of this CTA's half tile
@@ -562,40 +596,26 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         const float n = (float)sqrt(p.norm2[g.first_mat + t.mat]) + p.co.eps;
         nscale = (phase == NS_GRAM) ? 1.f / (n * n) : (phase == NS_APPLY ? 1.f / n : 1.f);
       }
-      const int i = t.tm * BM + (int)rank * kHalf + row;
-      const size_t sq = (size_t)g.s_pad * g.s_pad;
-      const size_t xs = (size_t)g.s_pad * g.l_pad;
-      // output extents: s x s (GRAM, POLY); s x l (APPLY, wide); l x s (APPLY, tall)
+      // output extents: s x s (GRAM, POLY), s x l (APPLY wide), l x s (APPLY tall)
       const bool apply_tall = phase == NS_APPLY && g.tall;
       const int nrows = apply_tall ? g.l : g.s;
       const int row_lim = apply_tall ? g.l_pad : g.s_pad;
       const int ncols = (phase == NS_APPLY) ? (g.tall ? g.s : g.l) : g.s;
-      const int ld = (phase == NS_APPLY) ? (g.tall ? g.s_pad : g.l_pad) : g.s_pad;
-      const int jmax = ld;
-      const bool row_in = i < row_lim;        // rows past the padded matrix are skipped
-      __nv_bfloat16* out;
-      if (phase == NS_GRAM) {
-        out = static_cast<__nv_bfloat16*>(g.A) + t.mat * sq;
-      } else if (phase == NS_POLY) {
-        out = static_cast<__nv_bfloat16*>(g.B) + t.mat * sq;
-      } else {
-        out = nullptr;   // APPLY results leave through auxbuf and TMA stores
-      }
-      (void)xs;
-      const bool sym = phase != NS_APPLY;
+      const int jmax = (phase == NS_APPLY) ? (g.tall ? g.s_pad : g.l_pad) : g.s_pad;
+      const int r0 = t.tm * BM + (int)rank * kHalf + q * 32;   // first row of this warp
+      const int i = r0 + lane;
+      const bool warp_in = r0 < row_lim;        // rows past the padded matrix are skipped
       for (int c4 = 0; c4 < 4; ++c4) {
         const int ch = half * 4 + c4;
         uint32_t r[32];
         __syncwarp();   // tcgen05.ld is warp-collective: reconverge first
         tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * BN + ch * 32), r);
         const int j0 = t.tn * BN + ch * 32;
-        if (j0 >= jmax || !row_in) continue;      // beyond the padded matrix
-        if (sym && j0 + 31 < i) continue;         // strictly below the diagonal
-        float v[32];
-        // this row's 32 aux values in the swizzled box: 16-byte chunk c of
-        // row r sits at chunk position c ^ (r mod 8)
+        if (!warp_in || j0 >= jmax) continue;   // beyond the padded matrix
+        // 16-byte chunk c of row r of a box sits at chunk position c ^ (r mod 8)
         uint4* abox = reinterpret_cast<uint4*>(auxbuf + (ch >> 1) * kAuxBoxBytes + row * 128);
         const int csub = (ch & 1) * 4;
+        float v[32];
         if (aux_phase) {
 #pragma unroll
           for (int u = 0; u < 4; ++u) {
@@ -618,31 +638,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           else o = (p.co.a * v[e] + acc) * nscale;
           v[e] = (i < nrows && j < ncols) ? o : 0.f;
         }
-        if (!sym) {
-          // APPLY: results replace the aux values, stored by TMA below
 #pragma unroll
-          for (int u = 0; u < 4; ++u)
-            abox[(csub + u) ^ (row & 7)] =
-                make_uint4(pack_bf2(v[u * 8 + 0], v[u * 8 + 1]), pack_bf2(v[u * 8 + 2], v[u * 8 + 3]),
-                           pack_bf2(v[u * 8 + 4], v[u * 8 + 5]), pack_bf2(v[u * 8 + 6], v[u * 8 + 7]));
-        } else if (j0 >= i) {
-          // whole chunk on or above the diagonal: 16-byte direct stores
-          uint4* op = reinterpret_cast<uint4*>(out + (size_t)i * ld + j0);
-#pragma unroll
-          for (int u = 0; u < 4; ++u)
-            op[u] = make_uint4(pack_bf2(v[u * 8 + 0], v[u * 8 + 1]), pack_bf2(v[u * 8 + 2], v[u * 8 + 3]),
-                               pack_bf2(v[u * 8 + 4], v[u * 8 + 5]), pack_bf2(v[u * 8 + 6], v[u * 8 + 7]));
-        } else {
-#pragma unroll
-          for (int e = 0; e < 32; ++e)
-            if (j0 + e >= i) out[(size_t)i * ld + j0 + e] = __float2bfloat16_rn(v[e]);
-        }
-        if (sym) {
-          // mirrored half: consecutive lanes write consecutive columns
-#pragma unroll
-          for (int e = 0; e < 32; ++e)
-            if (j0 + e > i) out[(size_t)(j0 + e) * ld + i] = __float2bfloat16_rn(v[e]);
-        }
+        for (int u = 0; u < 4; ++u)
+          abox[(csub + u) ^ (row & 7)] =
+              make_uint4(pack_bf2(v[u * 8 + 0], v[u * 8 + 1]), pack_bf2(v[u * 8 + 2], v[u * 8 + 3]),
+                         pack_bf2(v[u * 8 + 4], v[u * 8 + 5]), pack_bf2(v[u * 8 + 6], v[u * 8 + 7]));
       }
       tc_fence_before();
       __syncwarp();
@@ -651,23 +651,21 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         ab = 0;
         aph ^= 1u;
       }
-      if (phase == NS_APPLY) {
-        // this warp's 32 rows x 128 columns of X' leave by two TMA stores
-        fence_proxy_async_smem();
-        __syncwarp();
-        const int r0 = t.tm * BM + (int)rank * kHalf + q * 32;
-        if (lane == 0 && r0 < row_lim) {
+      // this warp's 32 rows x 128 columns leave by two TMA stores
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0 && warp_in) {
+        const TcGroupMaps& mp = p.maps[t.group];
+        const CUtensorMap* dst = (phase == NS_GRAM) ? &mp.ast : (phase == NS_POLY ? &mp.bst : &mp.xst[cur ^ 1]);
 #pragma unroll
-          for (int b = 2 * half; b < 2 * half + 2; ++b)
-            if (t.tn * BN + 64 * b < jmax)   // boxes past the padded columns hold nothing
-              tma_store_3d(&p.maps[t.group].xst[cur ^ 1], auxbuf + b * kAuxBoxBytes + q * 32 * 128,
-                           t.tn * BN + 64 * b, r0, t.mat);
-          bulk_commit();
-          bulk_wait_read();   // auxbuf may be refilled once the stores have read it
-        }
+        for (int b = 2 * half; b < 2 * half + 2; ++b)
+          if (t.tn * BN + 64 * b < jmax)   // boxes past the padded columns hold nothing
+            tma_store_3d(dst, auxbuf + b * kAuxBoxBytes + q * 32 * 128, t.tn * BN + 64 * b, r0, t.mat);
+        bulk_commit();
+        bulk_wait_read();   // auxbuf may be rewritten once the stores have read it
       }
+      __syncwarp();
       if (aux_phase) {
-        __syncwarp();
         if (lane == 0) mbar_arrive(aux_empty);
         xph ^= 1u;
       }
@@ -747,6 +745,10 @@ cudaError_t tc_encode_group_maps(const NsGroup& g, TcGroupMaps* maps) {
   }
   if ((e = encode_3d(&maps->a, g.A, g.s_pad, g.s_pad, g.count, BK, kHalf)) != cudaSuccess) return e;
   if ((e = encode_3d(&maps->b, g.B, g.s_pad, g.s_pad, g.count, BK, kHalf)) != cudaSuccess) return e;
+  if ((e = encode_3d(&maps->amn, g.A, g.s_pad, g.s_pad, g.count, 64, BK)) != cudaSuccess) return e;
+  if ((e = encode_3d(&maps->bmn, g.B, g.s_pad, g.s_pad, g.count, 64, BK)) != cudaSuccess) return e;
+  if ((e = encode_3d(&maps->ast, g.A, g.s_pad, g.s_pad, g.count, 64, 32)) != cudaSuccess) return e;
+  if ((e = encode_3d(&maps->bst, g.B, g.s_pad, g.s_pad, g.count, 64, 32)) != cudaSuccess) return e;
   return cudaSuccess;
 }
 
