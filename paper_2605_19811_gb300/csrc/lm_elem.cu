@@ -95,7 +95,28 @@ __global__ void __launch_bounds__(kLionThreads)
     float* m = t.m + ch.begin;
     const int64_t nvec = ch.count >> 3;
     int64_t v = threadIdx.x;
-    // two independent vectors per trip keep more loads in flight
+    // four independent vectors per trip keep enough loads in flight to run
+    // at the copy bandwidth; then pairs and a single vector for the tail
+    for (; v + 3 * kLionThreads < nvec; v += 4 * kLionThreads) {
+      float w0[8], g0[8], m0[8], w1[8], g1[8], m1[8], w2[8], g2[8], m2[8], w3[8], g3[8], m3[8];
+      const int64_t i0 = v * 8, i1 = i0 + kLionThreads * 8, i2 = i1 + kLionThreads * 8,
+                    i3 = i2 + kLionThreads * 8;
+      load8(w + i0, w0); load8(g + i0, g0); load8(m + i0, m0);
+      load8(w + i1, w1); load8(g + i1, g1); load8(m + i1, m1);
+      load8(w + i2, w2); load8(g + i2, g2); load8(m + i2, m2);
+      load8(w + i3, w3); load8(g + i3, g3); load8(m + i3, m3);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        lion_elem(w0[e], m0[e], g0[e], k);
+        lion_elem(w1[e], m1[e], g1[e], k);
+        lion_elem(w2[e], m2[e], g2[e], k);
+        lion_elem(w3[e], m3[e], g3[e], k);
+      }
+      store8(w + i0, w0); store8(m + i0, m0);
+      store8(w + i1, w1); store8(m + i1, m1);
+      store8(w + i2, w2); store8(m + i2, m2);
+      store8(w + i3, w3); store8(m + i3, m3);
+    }
     for (; v + kLionThreads < nvec; v += 2 * kLionThreads) {
       float wa[8], ga[8], ma[8], wb[8], gb[8], mb[8];
       const int64_t ia = v * 8, ib = (v + kLionThreads) * 8;
@@ -156,35 +177,39 @@ __device__ __forceinline__ float momentum_math(float (&gv)[8], float (&mv)[8], f
   return acc;
 }
 
+// 8-element vectors in flight per thread and trip, and CTAs per SM, as
+// measured best on the 720M-shaped set (momentum 3 / 2, finalize 2 / 3)
+constexpr int kMomVec = 3, kMomCtas = 2;
+constexpr int kFinVec = 2, kFinCtas = 3;
+
 template <typename XT, typename GT>
 __device__ float momentum_chunk(const MatDesc& d, int64_t begin, int64_t count, const GT* g,
                                 const MuonConsts& k, int mode) {
   float acc = 0.f;
   XT* x = static_cast<XT*>(d.x);
   if ((d.cols & 7) == 0) {
-    // rows hold whole vectors; count is a multiple of 8.  Two vectors per
-    // trip, both loaded before anything is stored.
+    // rows hold whole vectors; count is a multiple of 8.  kMomVec vectors
+    // per trip, all loaded before anything is stored.
     const int64_t nvec = count >> 3;
     int64_t v = threadIdx.x;
-    for (; v + kElemThreads < nvec; v += 2 * kElemThreads) {
-      const int64_t ea = begin + v * 8, eb = ea + kElemThreads * 8;
-      float ga[8], ma[8], gb[8], mb[8], ha[8], hb[8];
-      load8(g + ea, ga);
-      load8(g + eb, gb);
-      if (mode == 0) {
-        load8(d.m + ea, ma);
-        load8(d.m + eb, mb);
+    for (; v + (kMomVec - 1) * kElemThreads < nvec; v += kMomVec * kElemThreads) {
+      float gv[kMomVec][8], mv[kMomVec][8], hv[kMomVec][8];
+#pragma unroll
+      for (int u = 0; u < kMomVec; ++u) {
+        const int64_t e = begin + (v + u * kElemThreads) * 8;
+        load8(g + e, gv[u]);
+        if (mode == 0) load8(d.m + e, mv[u]);
       }
-      acc += momentum_math(ga, ma, ha, k, mode);
-      acc += momentum_math(gb, mb, hb, k, mode);
-      if (mode == 0) {
-        store8(d.m + ea, ma);
-        store8(d.m + eb, mb);
+#pragma unroll
+      for (int u = 0; u < kMomVec; ++u) acc += momentum_math(gv[u], mv[u], hv[u], k, mode);
+#pragma unroll
+      for (int u = 0; u < kMomVec; ++u) {
+        const int64_t e = begin + (v + u * kElemThreads) * 8;
+        if (mode == 0) store8(d.m + e, mv[u]);
+        store8(x + x_index(d, e), hv[u]);
       }
-      store8(x + x_index(d, ea), ha);
-      store8(x + x_index(d, eb), hb);
     }
-    if (v < nvec) {
+    for (; v < nvec; v += kElemThreads) {
       const int64_t ea = begin + v * 8;
       float ga[8], ma[8], ha[8];
       load8(g + ea, ga);
@@ -210,7 +235,7 @@ __device__ float momentum_chunk(const MatDesc& d, int64_t begin, int64_t count, 
 }
 
 template <typename XT, typename GT, int MODE>
-__global__ void __launch_bounds__(kElemThreads, 3)
+__global__ void __launch_bounds__(kElemThreads, kMomCtas)
     momentum_norm_kernel(const MatDesc* __restrict__ mats, const ElemChunk* __restrict__ chunks,
                          int nchunks, const void* const* __restrict__ grads, MuonConsts k) {
   for (int c = blockIdx.x; c < nchunks; c += gridDim.x) {
@@ -246,21 +271,20 @@ __device__ void finalize_chunk(const MatDesc& d, int64_t begin, int64_t count, c
   if ((d.cols & 7) == 0) {
     const int64_t nvec = count >> 3;
     int64_t v = threadIdx.x;
-    for (; v + kElemThreads < nvec; v += 2 * kElemThreads) {
-      const int64_t ea = begin + v * 8, eb = ea + kElemThreads * 8;
-      float xa[8], pa[8], xb[8], pb[8];
-      load8(x + x_index(d, ea), xa);
-      load8(x + x_index(d, eb), xb);
-      if (mode == 0) {
-        load8(p + ea, pa);
-        load8(p + eb, pb);
+    for (; v + (kFinVec - 1) * kElemThreads < nvec; v += kFinVec * kElemThreads) {
+      float xv[kFinVec][8], pv[kFinVec][8];
+#pragma unroll
+      for (int u = 0; u < kFinVec; ++u) {
+        const int64_t e = begin + (v + u * kElemThreads) * 8;
+        load8(x + x_index(d, e), xv[u]);
+        if (mode == 0) load8(p + e, pv[u]);
       }
-      finalize_math(xa, pa, d.shape_scale, k, mode, xs, scale_x);
-      finalize_math(xb, pb, d.shape_scale, k, mode, xs, scale_x);
-      store8(p + ea, pa);
-      store8(p + eb, pb);
+#pragma unroll
+      for (int u = 0; u < kFinVec; ++u) finalize_math(xv[u], pv[u], d.shape_scale, k, mode, xs, scale_x);
+#pragma unroll
+      for (int u = 0; u < kFinVec; ++u) store8(p + begin + (v + u * kElemThreads) * 8, pv[u]);
     }
-    if (v < nvec) {
+    for (; v < nvec; v += kElemThreads) {
       const int64_t ea = begin + v * 8;
       float xa[8], pa[8];
       load8(x + x_index(d, ea), xa);
@@ -282,7 +306,7 @@ __device__ void finalize_chunk(const MatDesc& d, int64_t begin, int64_t count, c
 }
 
 template <typename XT, typename PT, int MODE>
-__global__ void __launch_bounds__(kElemThreads, 3)
+__global__ void __launch_bounds__(kElemThreads, kFinCtas)
     finalize_kernel(const MatDesc* __restrict__ mats, const ElemChunk* __restrict__ chunks, int nchunks,
                     MuonConsts k, unsigned* flags) {
   for (int c = blockIdx.x; c < nchunks; c += gridDim.x) {
@@ -333,12 +357,12 @@ cudaError_t launch_lion(lm_dtype dt, const LionTensor* tensors, const LionChunk*
   return cudaGetLastError();
 }
 
-int elem_grid_size() {
+template <typename K>
+int elem_grid_size(K kernel) {
   int dev = 0, sms = 0, per_sm = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, finalize_kernel<__nv_bfloat16, __nv_bfloat16, 0>,
-                                                kElemThreads, 0);
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, kElemThreads, 0);
   if (per_sm < 1) per_sm = 1;
   if (sms < 1) sms = 1;
   return sms * per_sm;
@@ -368,7 +392,7 @@ cudaError_t launch_momentum_norm(lm_dtype xdt, lm_dtype gdt, const MatDesc* mats
                                  cudaStream_t st) {
   if (nchunks <= 0) return cudaSuccess;
   static int grid_cap = 0;
-  if (grid_cap == 0) grid_cap = elem_grid_size();
+  if (grid_cap == 0) grid_cap = elem_grid_size(momentum_norm_kernel<__nv_bfloat16, __nv_bfloat16, 0>);
   const int grid = nchunks < grid_cap ? nchunks : grid_cap;
   count_launch();
   if (xdt == LM_BF16) {
@@ -385,7 +409,7 @@ cudaError_t launch_finalize(lm_dtype xdt, lm_dtype pdt, const MatDesc* mats, con
                             int nchunks, MuonConsts k, int mode, unsigned* flags, cudaStream_t st) {
   if (nchunks <= 0) return cudaSuccess;
   static int grid_cap = 0;
-  if (grid_cap == 0) grid_cap = elem_grid_size();
+  if (grid_cap == 0) grid_cap = elem_grid_size(finalize_kernel<__nv_bfloat16, __nv_bfloat16, 0>);
   const int grid = nchunks < grid_cap ? nchunks : grid_cap;
   count_launch();
   if (xdt == LM_BF16) {
