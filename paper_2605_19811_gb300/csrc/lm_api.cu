@@ -411,7 +411,7 @@ static cudaError_t timed(Profiler* P, int fam, cudaStream_t st, F&& f) {
 }
 
 static lm_status run_ns(const NsEngine& E, int steps, NsCoeffs co, unsigned* flags, cudaStream_t st,
-                        Profiler* P = nullptr) {
+                        Profiler* P = nullptr, const FuseFinal* fuse = nullptr) {
   for (int it = 0; it < steps; ++it)
     for (const NsBatch& b : E.batches)
       for (int ph = 0; ph < 3; ++ph) {
@@ -419,7 +419,7 @@ static lm_status run_ns(const NsEngine& E, int steps, NsCoeffs co, unsigned* fla
           if (E.xdt == LM_BF16)
             return launch_ns_tc((NsPhase)ph, it, b.ng, E.groups.data() + b.g0, E.maps.data() + b.g0,
                                 b.tiles[ph], b.ntiles[ph], b.offsets[ph], b.npairs[ph], E.d_norm2, co,
-                                flags, st);
+                                flags, it == steps - 1 ? fuse : nullptr, st);
           return launch_ns_simt((NsPhase)ph, it, b.ng, E.d_groups + b.g0, b.tiles[ph], b.ntiles[ph],
                                 E.d_norm2, co, st);
         });
@@ -452,6 +452,7 @@ struct lm_state {
   int lion_grid[2] = {0, 0};
   int nmat = 0;
   MatDesc* d_mats = nullptr;
+  bool fuse_final = false;   // parameter write in the last APPLY epilogue
   ElemChunk* d_echunks[2] = {nullptr, nullptr};   // chunks of bf16 / fp32 matrices
   int n_echunks[2] = {0, 0};
   NsEngine ns;
@@ -649,6 +650,12 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
     if (!sorted.empty()) memcpy(img.data() + off_echunks, sorted.data(), sorted.size() * sizeof(ElemChunk));
   }
   s->d_mats = reinterpret_cast<MatDesc*>(base + off_mats);
+  // The last APPLY can write the parameters when they are all bf16 with
+  // 16-byte-aligned rows (the epilogue's vector accesses) and NS runs on the
+  // tensor cores with at least one iteration.
+  s->fuse_final = s->ns.xdt == LM_BF16 && cfg->ns_steps > 0 && s->nmat > 0;
+  for (const MatDesc& d : mats)
+    if (d.wdt != LM_BF16 || (d.cols & 7) != 0) s->fuse_final = false;
   s->d_echunks[0] = reinterpret_cast<ElemChunk*>(base + off_echunks);
   s->d_echunks[1] = s->d_echunks[0] + s->n_echunks[0];
 
@@ -750,8 +757,10 @@ lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t, void* c
   }
   if (s->nmat > 0) {
     NsCoeffs co{(float)c.ns_a, (float)c.ns_b, (float)c.ns_c, (float)c.ns_eps};
-    if ((st = run_ns(s->ns, c.ns_steps, co, s->d_flags, stream, P)) != LM_OK) return st;
-    for (int dt = 0; dt < 2; ++dt) {
+    const FuseFinal ff{s->d_mats, mk.eM, mk.lam};
+    if ((st = run_ns(s->ns, c.ns_steps, co, s->d_flags, stream, P, s->fuse_final ? &ff : nullptr)) != LM_OK)
+      return st;
+    for (int dt = 0; dt < 2 && !s->fuse_final; ++dt) {
       if (s->n_echunks[dt] == 0) continue;
       e = timed(P, LM_KERNEL_FINALIZE, stream, [&]() {
         return launch_finalize(s->ns.xdt, (lm_dtype)dt, s->d_mats, s->d_echunks[dt], s->n_echunks[dt], mk, 0,

@@ -133,11 +133,19 @@ cudaError_t tc_encode_group_maps(const NsGroup& g, TcGroupMaps* maps);
 int tc_max_pairs();   // CTA pairs that fit the device (one CTA per SM)
 // One bounded wait on a barrier that is never signalled (failure-detection probe).
 cudaError_t launch_bounded_wait_probe(uint64_t limit_ns, unsigned* flags, cudaStream_t st);
-// offsets: NULL (round robin over tiles) or npairs + 1 range starts.
+// The Muon parameter write fused into the epilogue of the last APPLY phase:
+// W <- W - eM (shape_scale X_K + lam W) for the bf16 parameters of mats
+// (indexed by group first_mat + matrix), X_K itself is not stored.
+struct FuseFinal {
+  const MatDesc* mats;
+  float eM, lam;
+};
+// offsets: NULL (round robin over tiles) or npairs + 1 range starts;
+// fuse: NULL, or the parameter write of the last APPLY phase.
 cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* groups,
                          const TcGroupMaps* maps, const NsTile* tiles, int ntiles,
                          const int* offsets, int npairs, const double* norm2, NsCoeffs co,
-                         unsigned* flags, cudaStream_t st);
+                         unsigned* flags, const FuseFinal* fuse, cudaStream_t st);
 
 // fp32 CUDA-core path.
 constexpr int kSimtBM = 64, kSimtBN = 64;

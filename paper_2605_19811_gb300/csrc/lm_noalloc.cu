@@ -247,7 +247,7 @@ extern "C" lm_status lm_msign_ns_noalloc(const lm_tensor* in, lm_tensor* out, in
     for (int ph = 0; ph < 3; ++ph) {
       if (xdt == LM_BF16)
         e = launch_ns_tc((NsPhase)ph, it, 1, &g, &maps, ba.d_tiles[ph], ntiles[ph], nullptr, 0,
-                         d.norm2, co, ba.d_flags, stream);
+                         d.norm2, co, ba.d_flags, nullptr, stream);
       else
         e = launch_ns_simt((NsPhase)ph, it, 1, ba.d_group, ba.d_tiles[ph], ntiles[ph], d.norm2, co,
                            stream);

@@ -31,6 +31,11 @@
 //             one per half of the tile's columns
 //   warp 10   aux loader: TMA of the tile the POLY/APPLY epilogue combines
 //             with the accumulator (A or X), issued while the main loop runs
+// The last APPLY of a Muon step can also apply the parameter update
+// W <- W - eta_M (s X_K + lambda W) (Algorithm 1, Muon branch) in its
+// epilogue: X_K goes to shared memory as bf16 as usual, then each warp reads
+// its 32 rows of W with coalesced 16-byte loads, updates and writes them, and
+// X_K itself is never stored.
 // Tiles are assigned to pairs on the host by a longest-first greedy balance
 // of their K lengths (a contiguous range per pair).
 // kAccBufs 256-column accumulators in TMEM (two let the epilogue of one tile
@@ -55,6 +60,7 @@ constexpr int kEpiWarps = 8;
 constexpr int kAuxWarp = 2 + kEpiWarps;              // warp that loads the epilogue's aux tile
 constexpr int kThreads = 32 * (3 + kEpiWarps);
 constexpr int kAccBufs = 2;                          // accumulators in TMEM
+constexpr int kFuseBatch = 4;   // W loads in flight per thread in the fused parameter write
 constexpr int kTmemCols = kAccBufs * BN;
 constexpr uint64_t kWaitLimitNs = 5000000000ull;     // 5 s
 constexpr int kAuxBoxBytes = kHalf * 64 * 2;         // one 64-column box of the CTA's rows: 16 KB
@@ -73,6 +79,7 @@ struct TcParams {
   const double* norm2;
   NsCoeffs co;
   unsigned* flags;
+  FuseFinal fuse;       // fuse.mats != NULL: this APPLY writes the parameters
 };
 
 // ------------------------------- PTX wrappers -------------------------------
@@ -579,6 +586,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     for (int w = w_begin; w < w_end; w += w_step) {
       const NsTile t = p.tiles[w];
       const NsGroup& g = p.groups[t.group];
+      const bool fused = phase == NS_APPLY && p.fuse.mats != nullptr;
+      const MatDesc* fd = fused ? &p.fuse.mats[g.first_mat + t.mat] : nullptr;
       bool ok = true;
       if (lane == 0) {
         ok = mbar_wait(&accfull[ab], aph, abort_flag, kWaitLimitNs);
@@ -605,6 +614,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const int r0 = t.tm * BM + (int)rank * kHalf + q * 32;   // first row of this warp
       const int i = r0 + lane;
       const bool warp_in = r0 < row_lim;        // rows past the padded matrix are skipped
+      if (fused && lane == 0 && q == 0 && half == 0 && rank == 0 && t.tm == 0 && t.tn == 0 &&
+          !isfinite((float)sqrt(p.norm2[g.first_mat + t.mat])))
+        atomicOr(p.flags, LM_FLAG_NONFINITE);
       for (int c4 = 0; c4 < 4; ++c4) {
         const int ch = half * 4 + c4;
         uint32_t r[32];
@@ -654,7 +666,47 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       // this warp's 32 rows x 128 columns leave by two TMA stores
       fence_proxy_async_smem();
       __syncwarp();
-      if (lane == 0 && warp_in) {
+      if (fused) {
+        // Last APPLY: W <- W - eta_M (s X_K + lambda W), with X_K the bf16
+        // values just written to auxbuf.  Half-warp h covers row 2k + h of the
+        // warp's 32 rows, 16 lanes x 8 columns = 256 contiguous bytes of W.
+        if (warp_in) {
+          const int cc = lane & 15;
+          const int jc = t.tn * BN + half * 128 + cc * 8;
+          const unsigned char* box = auxbuf + (2 * half + (cc >> 3)) * kAuxBoxBytes;
+          const int ibase = t.tm * BM + (int)rank * kHalf + q * 32 + (lane >> 4);
+          __nv_bfloat16* wcol = static_cast<__nv_bfloat16*>(fd->w) + jc;
+          for (int k0 = 0; k0 < 16; k0 += kFuseBatch) {
+            uint4 wv[kFuseBatch], xv[kFuseBatch];
+#pragma unroll
+            for (int u = 0; u < kFuseBatch; ++u) {   // all loads of the batch first
+              const int rr = q * 32 + 2 * (k0 + u) + (lane >> 4);
+              const int ii = ibase + 2 * (k0 + u);
+              xv[u] = *reinterpret_cast<const uint4*>(box + rr * 128 + (((cc & 7) ^ (rr & 7)) << 4));
+              wv[u] = (ii < nrows && jc < ncols)
+                          ? *reinterpret_cast<const uint4*>(wcol + (int64_t)ii * fd->cols)
+                          : make_uint4(0u, 0u, 0u, 0u);
+            }
+#pragma unroll
+            for (int u = 0; u < kFuseBatch; ++u) {
+              const int ii = ibase + 2 * (k0 + u);
+              if (ii >= nrows || jc >= ncols) continue;
+              const uint32_t xw[4] = {xv[u].x, xv[u].y, xv[u].z, xv[u].w};
+              uint32_t ww[4] = {wv[u].x, wv[u].y, wv[u].z, wv[u].w};
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const float w0 = bf_lo(ww[e]), w1 = bf_hi(ww[e]);
+                const float n0 = __fsub_rn(w0, __fmul_rn(p.fuse.eM, __fadd_rn(__fmul_rn(fd->shape_scale, bf_lo(xw[e])),
+                                                                             __fmul_rn(p.fuse.lam, w0))));
+                const float n1 = __fsub_rn(w1, __fmul_rn(p.fuse.eM, __fadd_rn(__fmul_rn(fd->shape_scale, bf_hi(xw[e])),
+                                                                             __fmul_rn(p.fuse.lam, w1))));
+                ww[e] = pack_bf2(n0, n1);
+              }
+              *reinterpret_cast<uint4*>(wcol + (int64_t)ii * fd->cols) = make_uint4(ww[0], ww[1], ww[2], ww[3]);
+            }
+          }
+        }
+      } else if (lane == 0 && warp_in) {
         const TcGroupMaps& mp = p.maps[t.group];
         const CUtensorMap* dst = (phase == NS_GRAM) ? &mp.ast : (phase == NS_POLY ? &mp.bst : &mp.xst[cur ^ 1]);
 #pragma unroll
@@ -762,7 +814,7 @@ int tc_max_pairs() {
 cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* groups,
                          const TcGroupMaps* maps, const NsTile* tiles, int ntiles,
                          const int* offsets, int npairs, const double* norm2, NsCoeffs co,
-                         unsigned* flags, cudaStream_t st) {
+                         unsigned* flags, const FuseFinal* fuse, cudaStream_t st) {
   if (ntiles <= 0) return cudaSuccess;
   if (ngroups < 1 || ngroups > kMaxGroupsTc) return cudaErrorInvalidValue;
   static bool attr_set = false;
@@ -786,6 +838,7 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
   prm.norm2 = norm2;
   prm.co = co;
   prm.flags = flags;
+  if (fuse != nullptr && ph == NS_APPLY) prm.fuse = *fuse;
   int pairs = npairs;
   if (offsets == nullptr) {
     pairs = tc_max_pairs();

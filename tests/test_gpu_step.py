@@ -242,3 +242,27 @@ def test_set_lr_and_checkpoint_resume():
     a, b = run(-1), run(2)
     for x, y in zip(a, b):
         np.testing.assert_array_equal(bits(x), bits(y))
+
+
+def test_fused_parameter_write_matches_finalize_kernel_bit_exact():
+    """The Muon parameter write W <- W - eta_M (s X_K + lambda W) runs in the
+    last Newton-Schulz epilogue when every matrix is bf16 with a column count
+    divisible by 8, and in a separate kernel otherwise; both evaluate the same
+    float32 expression on the same bf16 X_K, so the weights agree bit for bit.
+    A 40 x 36 matrix added to the set switches the fusion off."""
+    import torch
+    from paper_2605_19811_gb300 import lionmuon as L
+    shapes = [(256, 384), (384, 256), (320, 320), (128,)]
+    W0, grads = make_problem(shapes + [(40, 36)], "student_t", 2)
+    out = []
+    for n in (len(shapes), len(shapes) + 1):
+        params = [host_tensor(w, "bf16").cuda() for w in W0[:n]]
+        opt = L.LionMuon(params, period=2, eta_muon=0.02, weight_decay=0.1)
+        for t in range(2):
+            opt.step([host_tensor(g, "bf16").cuda() for g in grads[t][:n]], t)
+        torch.cuda.synchronize()
+        assert opt.status() == 0
+        out.append([bits(p) for p in params[:len(shapes)]])
+        opt.close()
+    for a, b in zip(*out):
+        np.testing.assert_array_equal(a, b)
