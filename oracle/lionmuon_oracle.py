@@ -33,6 +33,11 @@ Readings taken where the paper is silent (each listed in the design doc):
 * sign(0) = 0 and sign(NaN) = NaN.
 * 1-D parameters (vectors) take the Lion step on every step.
 * P = infinity is encoded as ``period = 0``.
+* Iteration-dependent NS coefficients (the minimax / Chebyshev-type msign
+  iterations of Section 2) keep the Frobenius normalisation, so the first
+  interval of singular values is [l_0, 1] with l_0 a parameter; the minimax
+  table is the per-interval best odd polynomial with the interval mapped
+  forward, optionally divided by a safety factor.
 
 Parity status: the fp64 update rules are pinned by closed forms and
 invariants in tests/test_oracle_pins.py.  The end-to-end trajectory values are
@@ -73,6 +78,9 @@ class Config:
     ns_c: float = NS_QUINTIC[2]
     ns_eps: float = 1e-7
     shape_scale: float = 0.2   # NS scaling 0.2*sqrt(max(m,n)) (Table 5)
+    # Optional per-iteration coefficients ((a_0, b_0, c_0), ...): when set they
+    # replace (ns_a, ns_b, ns_c) and their count replaces ns_steps.
+    ns_coeffs: Optional[Tuple[Tuple[float, float, float], ...]] = None
 
 
 # ---------------------------------------------------------------------------
@@ -140,6 +148,91 @@ def ns_polynomial(G: np.ndarray, steps: int, a: float, b: float, c: float,
     return X.T.copy() if transposed else X
 
 
+def ns_polynomial_schedule(G: np.ndarray, coeffs, eps: float = 1e-7) -> np.ndarray:
+    """NS with an odd polynomial that changes from iteration to iteration:
+    iteration k (k = 0, 1, ...) uses coeffs[k] = (a_k, b_k, c_k), i.e.
+        A = X X^T,  B = b_k A + c_k A A,  X <- a_k X + B X,
+    mapping each singular value s to a_k s + b_k s^3 + c_k s^5.  This is the
+    shape of the minimax-optimised (Polar Express) and Chebyshev-type msign
+    iterations that Section 2 names next to classical Newton-Schulz; they
+    differ from it only in the coefficient table.  Normalisation and the
+    tall-matrix orientation are as in ns_polynomial."""
+    X = np.array(G, dtype=np.float64)
+    if X.ndim != 2:
+        raise ValueError("NS needs a 2-D matrix")
+    transposed = X.shape[0] > X.shape[1]
+    if transposed:
+        X = X.T.copy()
+    X = X / (np.linalg.norm(X) + eps)
+    for a_k, b_k, c_k in coeffs:
+        A = X @ X.T
+        B = b_k * A + c_k * (A @ A)
+        X = a_k * X + B @ X
+    return X.T.copy() if transposed else X
+
+
+def ns_scalar_map_schedule(x: np.ndarray, coeffs) -> np.ndarray:
+    """phi_K o ... o phi_1 (x) with phi_k(x) = a_k x + b_k x^3 + c_k x^5,
+    applied in iteration order."""
+    x = np.array(x, dtype=np.float64)
+    for a_k, b_k, c_k in coeffs:
+        x = a_k * x + b_k * x ** 3 + c_k * x ** 5
+    return x
+
+
+def odd_poly_eval(q, x):
+    """p(x) = sum_j q_j x^(2j+1)."""
+    x = np.asarray(x, dtype=np.float64)
+    return sum(qj * x ** (2 * j + 1) for j, qj in enumerate(q))
+
+
+def minimax_odd_polynomial(lo: float, hi: float, degree: int, grid: int = 20001):
+    """The odd polynomial p of the given degree (3 or 5) that minimises
+    max_{x in [lo, hi]} |1 - p(x)|: the per-iteration polynomial of the
+    minimax ("Polar Express") msign iteration and, at degree 3, of the
+    Chebyshev-type iteration (Section 2 names both).  Solved as written, as a
+    linear program over a dense grid (Chebyshev-spaced, endpoints included):
+        minimise E  subject to  -E <= 1 - p(x_i) <= E  for every grid point.
+    scipy's LP solver (HiGHS) is the library primitive.  Returns (q, E) with
+    q the coefficients of x, x^3[, x^5]."""
+    from scipy.optimize import linprog
+    if degree not in (3, 5) or not (0 < lo < hi):
+        raise ValueError("degree 3 or 5 on 0 < lo < hi")
+    d = (degree + 1) // 2
+    t = np.cos(np.pi * np.arange(grid) / (grid - 1))
+    x = np.sort(0.5 * (lo + hi) + 0.5 * (hi - lo) * t)
+    V = np.stack([x ** (2 * j + 1) for j in range(d)], axis=1)
+    ones = np.ones((grid, 1))
+    # variables (q_0 .. q_{d-1}, E); constraints  p - E <= 1  and  -p - E <= -1
+    A_ub = np.vstack([np.hstack([V, -ones]), np.hstack([-V, -ones])])
+    b_ub = np.concatenate([np.ones(grid), -np.ones(grid)])
+    cost = np.zeros(d + 1)
+    cost[-1] = 1.0
+    res = linprog(cost, A_ub=A_ub, b_ub=b_ub, bounds=[(None, None)] * (d + 1), method="highs")
+    if not res.success:
+        raise RuntimeError("minimax LP failed: " + res.message)
+    return res.x[:d].copy(), float(res.x[d])
+
+
+def minimax_schedule(steps: int, lo: float, degree: int = 5, safety: float = 1.0):
+    """Coefficient table of the minimax msign iteration after the
+    Frobenius normalisation (singular values in [lo, 1]): iteration k uses the
+    minimax odd polynomial on the current interval [l_k, u_k], divided by
+    ``safety`` (>= 1), and the next interval is that polynomial's image,
+    l_{k+1} = p_k(l_k) and u_{k+1} = max of p_k on [l_k, u_k] (taken on the
+    LP grid).  Degree 5 is the Polar Express construction, degree 3 the
+    Chebyshev-type one.  Returns ((a_k, b_k, c_k), ...)."""
+    out = []
+    l, u = float(lo), 1.0
+    for _ in range(steps):
+        q, _E = minimax_odd_polynomial(l, u, degree)
+        q = q / safety
+        grid = np.linspace(l, u, 20001)
+        l, u = float(odd_poly_eval(q, l)), float(odd_poly_eval(q, grid).max())
+        out.append((float(q[0]), float(q[1]), float(q[2]) if len(q) > 2 else 0.0))
+    return tuple(out)
+
+
 def msign_svd(G: np.ndarray) -> np.ndarray:
     """Exact msign(G) = U V^T from the thin SVD G = U S V^T (Section 2,
     "msign(X) = U V^T"; Section 2.1, LMO of the spectral norm).  Zero singular
@@ -174,7 +267,10 @@ def lion_update(W, G_hat, eta_lion, weight_decay):
 def muon_update(W, G_hat, cfg: Config):
     """Muon branch of Algorithm 1 with Table 5's NS scaling:
     W <- W - eta_M (0.2 sqrt(max(m,n)) NS_K(G_hat) + lambda W)."""
-    O = ns_polynomial(G_hat, cfg.ns_steps, cfg.ns_a, cfg.ns_b, cfg.ns_c, cfg.ns_eps)
+    if cfg.ns_coeffs is not None:
+        O = ns_polynomial_schedule(G_hat, cfg.ns_coeffs, cfg.ns_eps)
+    else:
+        O = ns_polynomial(G_hat, cfg.ns_steps, cfg.ns_a, cfg.ns_b, cfg.ns_c, cfg.ns_eps)
     scale = cfg.shape_scale * math.sqrt(max(W.shape))
     return W - cfg.eta_muon * (scale * O + cfg.weight_decay * W)
 

@@ -11,6 +11,7 @@ import pytest
 import oracle
 import oracle.lionmuon_oracle as OM
 from tests import test_oracle_pins as pins
+from tests import test_oracle_pins_msign_variants as vpins
 
 # every pin, with representative arguments for the parametrised ones
 PIN_CALLS = [
@@ -39,6 +40,11 @@ PIN_CALLS = [
     (pins.test_decay_frank_wolfe_rewrite, ()),
     (pins.test_bf16_round_known_values, ()),
     (pins.test_lion_f32_matches_fp64_within_rounding, ()),
+    (vpins.test_minimax_cubic_matches_closed_form, (0.2, 1.0)),
+    (vpins.test_minimax_quintic_equioscillates, (0.1, 1.0)),
+    (vpins.test_ns_schedule_closed_form_on_known_svd, ()),
+    (vpins.test_ns_schedule_constant_table_is_classical_ns, ()),
+    (vpins.test_minimax_schedule_maps_interval_forward, (5, 5)),
 ]
 
 
@@ -81,7 +87,57 @@ def _mutations():
     muts["dispatch_off_by_one"] = [("is_muon_step", lambda t, P: P != 0 and t % P == 1 % max(P, 1))]
     muts["scale_uses_min"] = [("muon_update", _muon_min_scale)]
     muts["bf16_truncates"] = [("bf16_round", _bf16_truncate)]
+    muts["schedule_reversed"] = [("ns_polynomial_schedule", _schedule_factory(reverse=True)),
+                                 ("ns_scalar_map_schedule", _scalar_schedule_factory(reverse=True))]
+    muts["schedule_first_only"] = [("ns_polynomial_schedule", _schedule_factory(first_only=True)),
+                                   ("ns_scalar_map_schedule", _scalar_schedule_factory(first_only=True))]
+    muts["minimax_least_squares"] = [("minimax_odd_polynomial", _least_squares_poly)]
+    muts["minimax_no_interval_update"] = [("minimax_schedule", _schedule_fixed_interval)]
     return muts
+
+
+def _order(coeffs, reverse, first_only):
+    coeffs = list(coeffs)
+    if first_only:
+        return [coeffs[0]] * len(coeffs)
+    return coeffs[::-1] if reverse else coeffs
+
+
+def _schedule_factory(reverse=False, first_only=False):
+    def f(G, coeffs, eps=1e-7):
+        X = np.array(G, dtype=np.float64)
+        tr = X.shape[0] > X.shape[1]
+        if tr:
+            X = X.T.copy()
+        X = X / (np.linalg.norm(X) + eps)
+        for a, b, c in _order(coeffs, reverse, first_only):
+            A = X @ X.T
+            X = a * X + (b * A + c * (A @ A)) @ X
+        return X.T.copy() if tr else X
+    return f
+
+
+def _scalar_schedule_factory(reverse=False, first_only=False):
+    def f(x, coeffs):
+        x = np.array(x, dtype=np.float64)
+        for a, b, c in _order(coeffs, reverse, first_only):
+            x = a * x + b * x ** 3 + c * x ** 5
+        return x
+    return f
+
+
+def _least_squares_poly(lo, hi, degree, grid=20001):
+    x = np.linspace(lo, hi, grid)
+    d = (degree + 1) // 2
+    V = np.stack([x ** (2 * j + 1) for j in range(d)], axis=1)
+    q = np.linalg.lstsq(V, np.ones(grid), rcond=None)[0]
+    return q, float(np.abs(1 - V @ q).max())
+
+
+def _schedule_fixed_interval(steps, lo, degree=5, safety=1.0):
+    q, _ = OM.minimax_odd_polynomial(lo, 1.0, degree)
+    tr = (float(q[0]), float(q[1]), float(q[2]) if len(q) > 2 else 0.0)
+    return (tr,) * steps
 
 
 def _post_update_step(W, G, M_prev, t, cfg, sign_in_f32=False):
