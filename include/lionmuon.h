@@ -71,7 +71,13 @@ typedef struct {
  * period >= 1, or 0 for P = infinity (never Muon);
  * ns_steps in [0, 64]; ns_eps >= 0; shape_scale >= 0;
  * ns_precision LM_BF16 (tensor-core bf16 GEMMs, fp32 accumulate) or LM_F32
- * (fp32 CUDA-core GEMMs). */
+ * (fp32 CUDA-core GEMMs).
+ * ns_coeffs: NULL for the same (ns_a, ns_b, ns_c) in every NS iteration, or
+ * 3 * ns_steps finite values (a_k, b_k, c_k), k = 0 .. ns_steps - 1, for
+ * iteration-dependent odd polynomials X <- a_k X + (b_k A + c_k A^2) X, the
+ * form of the minimax (Polar Express) and Chebyshev-type msign iterations
+ * Section 2 names.  The table is caller memory read only by lm_create, which
+ * copies it; ns_a/ns_b/ns_c are then ignored. */
 typedef struct {
   double beta1, beta2;
   double eta_muon, eta_lion;
@@ -82,6 +88,7 @@ typedef struct {
   double ns_eps;
   double shape_scale;
   int ns_precision;
+  const double* ns_coeffs;
 } lm_config;
 
 typedef struct lm_state lm_state; /* opaque */
@@ -128,6 +135,14 @@ lm_status lm_set_lr(lm_state* s, double eta_muon, double eta_lion);
 lm_status lm_msign_ns(const lm_tensor* in, lm_tensor* out, int steps, double a,
                       double b, double c, double eps, int precision,
                       void* cuda_stream);
+
+/* lm_msign_ns with iteration-dependent coefficients: iteration k uses
+ * (coeffs[3k], coeffs[3k+1], coeffs[3k+2]); coeffs holds 3 * steps finite
+ * host values, read before the call returns (NULL is allowed only for
+ * steps == 0).  Everything else as lm_msign_ns. */
+lm_status lm_msign_ns_coeffs(const lm_tensor* in, lm_tensor* out, int steps,
+                             const double* coeffs, double eps, int precision,
+                             void* cuda_stream);
 
 /* The same computation as lm_msign_ns, for callers that cannot allocate
  * device memory while they run: for example a program whose device memory is

@@ -171,6 +171,39 @@ def ns_polynomial_schedule(G: np.ndarray, coeffs, eps: float = 1e-7) -> np.ndarr
     return X.T.copy() if transposed else X
 
 
+def ns_polynomial_schedule_storage(G: np.ndarray, coeffs, eps: float = 1e-7,
+                                   storage: str = "bf16") -> np.ndarray:
+    """The NS recurrence with every stored intermediate rounded to the
+    storage type ("bf16" or "f32"), as an implementation that keeps them in
+    that type does (the precision reading "bf16 operands, fp32 accumulation",
+    or the fp32 mode): X_0 = rd(G); per iteration A = rd(X X^T),
+    B = rd(b_k A + c_k A A), X <- rd(a_k X + B X), products and sums in fp64;
+    the normalisation 1/(||G||_F + eps) (of the unrounded G) is applied to A
+    (squared) and to X in iteration 0.  It measures how far the storage
+    precision alone moves a given coefficient table from the exact
+    recurrence."""
+    def rd(v):
+        if storage == "bf16":
+            return bf16_round(v).astype(np.float64)
+        if storage == "f32":
+            return np.asarray(v, dtype=np.float32).astype(np.float64)
+        raise ValueError("storage must be 'bf16' or 'f32'")
+    G = np.array(G, dtype=np.float64)
+    transposed = G.shape[0] > G.shape[1]
+    if transposed:
+        G = G.T.copy()
+    inv = 1.0 / (np.linalg.norm(G) + eps)
+    X = rd(G)
+    for k, (a_k, b_k, c_k) in enumerate(coeffs):
+        s_a, s_x = (inv * inv, inv) if k == 0 else (1.0, 1.0)
+        A = rd(s_a * (X @ X.T))
+        B = rd(b_k * A + c_k * (A @ A))
+        X = rd(s_x * (a_k * X + B @ X))
+    if len(coeffs) == 0:
+        X = X * inv
+    return X.T.copy() if transposed else X
+
+
 def ns_scalar_map_schedule(x: np.ndarray, coeffs) -> np.ndarray:
     """phi_K o ... o phi_1 (x) with phi_k(x) = a_k x + b_k x^3 + c_k x^5,
     applied in iteration order."""

@@ -72,6 +72,9 @@ lm_status check_config(const lm_config* c) {
   if (c->period < 0) return fail(LM_ERR_INVALID_ARG, "period must be >= 0 (0 = infinity)");
   if (c->ns_steps < 0 || c->ns_steps > 64) return fail(LM_ERR_INVALID_ARG, "ns_steps must be in [0, 64]");
   if (!finite(c->ns_a) || !finite(c->ns_b) || !finite(c->ns_c)) return fail(LM_ERR_INVALID_ARG, "NS coefficients must be finite");
+  if (c->ns_coeffs != nullptr)
+    for (int k = 0; k < 3 * c->ns_steps; ++k)
+      if (!finite(c->ns_coeffs[k])) return fail(LM_ERR_INVALID_ARG, "ns_coeffs[%d] is not finite", k);
   if (!finite(c->ns_eps) || c->ns_eps < 0) return fail(LM_ERR_INVALID_ARG, "ns_eps must be >= 0");
   if (!finite(c->shape_scale) || c->shape_scale < 0) return fail(LM_ERR_INVALID_ARG, "shape_scale must be >= 0");
   if (c->ns_precision != LM_BF16 && c->ns_precision != LM_F32)
@@ -410,11 +413,24 @@ static cudaError_t timed(Profiler* P, int fam, cudaStream_t st, F&& f) {
   return e;
 }
 
-static lm_status run_ns(const NsEngine& E, int steps, NsCoeffs co, unsigned* flags, cudaStream_t st,
+// Per-iteration coefficients: (a_k, b_k, c_k) from a 3 * steps table, or the
+// constant (a, b, c) when the table is NULL; eps goes with every iteration.
+static std::vector<NsCoeffs> ns_schedule(int steps, const double* table, double a, double b, double c,
+                                         double eps) {
+  std::vector<NsCoeffs> co((size_t)std::max(steps, 0));
+  for (int k = 0; k < steps; ++k) {
+    const double* t = table ? table + 3 * k : nullptr;
+    co[k] = NsCoeffs{(float)(t ? t[0] : a), (float)(t ? t[1] : b), (float)(t ? t[2] : c), (float)eps};
+  }
+  return co;
+}
+
+static lm_status run_ns(const NsEngine& E, int steps, const NsCoeffs* coeffs, unsigned* flags, cudaStream_t st,
                         Profiler* P = nullptr, const FuseFinal* fuse = nullptr) {
   for (int it = 0; it < steps; ++it)
     for (const NsBatch& b : E.batches)
       for (int ph = 0; ph < 3; ++ph) {
+        const NsCoeffs co = coeffs[it];
         cudaError_t e = timed(P, LM_KERNEL_NS_GRAM + ph, st, [&]() {
           if (E.xdt == LM_BF16)
             return launch_ns_tc((NsPhase)ph, it, b.ng, E.groups.data() + b.g0, E.maps.data() + b.g0,
@@ -456,6 +472,7 @@ struct lm_state {
   ElemChunk* d_echunks[2] = {nullptr, nullptr};   // chunks of bf16 / fp32 matrices
   int n_echunks[2] = {0, 0};
   NsEngine ns;
+  std::vector<NsCoeffs> ns_co;      // coefficients of each NS iteration
   unsigned* d_flags = nullptr;
   cudaStream_t last_stream = nullptr;
   Profiler prof;
@@ -478,6 +495,7 @@ void lm_config_default(lm_config* c) {
   c->ns_eps = 1e-7;
   c->shape_scale = 0.2;
   c->ns_precision = LM_BF16;
+  c->ns_coeffs = nullptr;
 }
 
 const char* lm_status_string(lm_status st) {
@@ -515,6 +533,8 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
   lm_state* s = new lm_state();
   s->device = dev;
   s->cfg = *cfg;
+  s->ns_co = ns_schedule(cfg->ns_steps, cfg->ns_coeffs, cfg->ns_a, cfg->ns_b, cfg->ns_c, cfg->ns_eps);
+  s->cfg.ns_coeffs = nullptr;   // the caller's table is not kept
   s->n = n;
   s->params.assign(params, params + n);
   s->ns.xdt = (cfg->ns_precision == LM_F32) ? LM_F32 : LM_BF16;
@@ -756,9 +776,9 @@ lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t, void* c
     if (e != cudaSuccess) return cuda_fail(e, "Lion kernel launch (vectors)");
   }
   if (s->nmat > 0) {
-    NsCoeffs co{(float)c.ns_a, (float)c.ns_b, (float)c.ns_c, (float)c.ns_eps};
     const FuseFinal ff{s->d_mats, mk.eM, mk.lam};
-    if ((st = run_ns(s->ns, c.ns_steps, co, s->d_flags, stream, P, s->fuse_final ? &ff : nullptr)) != LM_OK)
+    if ((st = run_ns(s->ns, c.ns_steps, s->ns_co.data(), s->d_flags, stream, P, s->fuse_final ? &ff : nullptr)) !=
+        LM_OK)
       return st;
     for (int dt = 0; dt < 2 && !s->fuse_final; ++dt) {
       if (s->n_echunks[dt] == 0) continue;
@@ -887,18 +907,18 @@ void lm_destroy(lm_state* s) {
   delete s;
 }
 
-lm_status lm_msign_ns(const lm_tensor* in, lm_tensor* out, int steps, double a, double b, double c,
-                      double eps, int precision, void* cuda_stream) {
-  if (in == nullptr || out == nullptr) return fail(LM_ERR_INVALID_ARG, "in/out is NULL");
+}  // extern "C"
+
+// The msign entry points: norm kernel, NS iterations with per-iteration
+// coefficients co[0 .. steps-1], output kernel; arguments already checked
+// except the tensors and the size limits.
+static lm_status msign_impl(const lm_tensor* in, lm_tensor* out, int steps, const std::vector<NsCoeffs>& co,
+                            double eps, int precision, void* cuda_stream) {
   lm_status st;
   if ((st = check_tensor(in, "in", 0)) != LM_OK) return st;
   if ((st = check_tensor(out, "out", 0)) != LM_OK) return st;
   if (in->rows < 2 || in->cols < 2) return fail(LM_ERR_INVALID_ARG, "msign needs rows, cols >= 2");
   if (out->rows != in->rows || out->cols != in->cols) return fail(LM_ERR_INVALID_ARG, "out shape differs from in");
-  if (steps < 0 || steps > 64) return fail(LM_ERR_INVALID_ARG, "steps must be in [0, 64]");
-  if (!std::isfinite(a) || !std::isfinite(b) || !std::isfinite(c) || !std::isfinite(eps) || eps < 0)
-    return fail(LM_ERR_INVALID_ARG, "coefficients must be finite, eps >= 0");
-  if (precision != LM_BF16 && precision != LM_F32) return fail(LM_ERR_INVALID_ARG, "precision must be LM_BF16 or LM_F32");
   if (std::max(in->rows, in->cols) > 1000000 || std::min(in->rows, in->cols) > 65536)
     return fail(LM_ERR_UNSUPPORTED, "matrix too large for lm_msign_ns");
   int dev = 0;
@@ -957,11 +977,34 @@ lm_status lm_msign_ns(const lm_tensor* in, lm_tensor* out, int steps, double a, 
   unsigned* dflags = reinterpret_cast<unsigned*>(base + off_flags);
   e = launch_momentum_norm(E.xdt, in->dtype, dm, de, (int)et.size(), nullptr, mk, 1, stream);
   if (e != cudaSuccess) return cleanup(cuda_fail(e, "norm kernel launch"));
-  NsCoeffs co{(float)a, (float)b, (float)c, (float)eps};
-  if ((st = run_ns(E, steps, co, dflags, stream)) != LM_OK) return cleanup(st);
+  if ((st = run_ns(E, steps, co.data(), dflags, stream)) != LM_OK) return cleanup(st);
   e = launch_finalize(E.xdt, out->dtype, dm, de, (int)et.size(), mk, 1, dflags, stream);
   if (e != cudaSuccess) return cleanup(cuda_fail(e, "output kernel launch"));
   return cleanup(LM_OK);
+}
+
+extern "C" {
+
+lm_status lm_msign_ns(const lm_tensor* in, lm_tensor* out, int steps, double a, double b, double c,
+                      double eps, int precision, void* cuda_stream) {
+  if (in == nullptr || out == nullptr) return fail(LM_ERR_INVALID_ARG, "in/out is NULL");
+  if (steps < 0 || steps > 64) return fail(LM_ERR_INVALID_ARG, "steps must be in [0, 64]");
+  if (!std::isfinite(a) || !std::isfinite(b) || !std::isfinite(c) || !std::isfinite(eps) || eps < 0)
+    return fail(LM_ERR_INVALID_ARG, "coefficients must be finite, eps >= 0");
+  if (precision != LM_BF16 && precision != LM_F32) return fail(LM_ERR_INVALID_ARG, "precision must be LM_BF16 or LM_F32");
+  return msign_impl(in, out, steps, ns_schedule(steps, nullptr, a, b, c, eps), eps, precision, cuda_stream);
+}
+
+lm_status lm_msign_ns_coeffs(const lm_tensor* in, lm_tensor* out, int steps, const double* coeffs, double eps,
+                             int precision, void* cuda_stream) {
+  if (in == nullptr || out == nullptr) return fail(LM_ERR_INVALID_ARG, "in/out is NULL");
+  if (steps < 0 || steps > 64) return fail(LM_ERR_INVALID_ARG, "steps must be in [0, 64]");
+  if (steps > 0 && coeffs == nullptr) return fail(LM_ERR_INVALID_ARG, "coeffs is NULL");
+  for (int k = 0; k < 3 * steps; ++k)
+    if (!std::isfinite(coeffs[k])) return fail(LM_ERR_INVALID_ARG, "coeffs[%d] is not finite", k);
+  if (!std::isfinite(eps) || eps < 0) return fail(LM_ERR_INVALID_ARG, "eps must be finite and >= 0");
+  if (precision != LM_BF16 && precision != LM_F32) return fail(LM_ERR_INVALID_ARG, "precision must be LM_BF16 or LM_F32");
+  return msign_impl(in, out, steps, ns_schedule(steps, coeffs, 0, 0, 0, eps), eps, precision, cuda_stream);
 }
 
 }  // extern "C"

@@ -27,7 +27,7 @@ EXPORTED = ("lm_config_default", "lm_create", "lm_step", "lm_set_lr", "lm_msign_
             "lm_get_momentum", "lm_set_momentum", "lm_get_status", "lm_state_bytes",
             "lm_workspace_bytes", "lm_destroy", "lm_status_string", "lm_last_error",
             "lm_kernel_launch_count", "lm_profile_enable", "lm_profile_read",
-            "lm_msign_ns_noalloc", "lm_probe_bounded_wait")
+            "lm_msign_ns_noalloc", "lm_probe_bounded_wait", "lm_msign_ns_coeffs")
 
 KERNEL_FAMILIES = ("lion", "momentum_norm", "ns_gram", "ns_poly", "ns_apply", "finalize", "other")
 
@@ -43,7 +43,8 @@ class LmConfig(ctypes.Structure):
                 ("weight_decay", ctypes.c_double), ("period", ctypes.c_int64),
                 ("ns_steps", ctypes.c_int), ("ns_a", ctypes.c_double), ("ns_b", ctypes.c_double),
                 ("ns_c", ctypes.c_double), ("ns_eps", ctypes.c_double),
-                ("shape_scale", ctypes.c_double), ("ns_precision", ctypes.c_int)]
+                ("shape_scale", ctypes.c_double), ("ns_precision", ctypes.c_int),
+                ("ns_coeffs", ctypes.POINTER(ctypes.c_double))]
 
 
 class LmProfile(ctypes.Structure):
@@ -82,6 +83,9 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib.lm_msign_ns.argtypes = [P(LmTensor), P(LmTensor), c_int, c_double, c_double, c_double,
                                 c_double, c_int, c_void_p]
     lib.lm_msign_ns.restype = c_int
+    lib.lm_msign_ns_coeffs.argtypes = [P(LmTensor), P(LmTensor), c_int, P(c_double), c_double, c_int,
+                                       c_void_p]
+    lib.lm_msign_ns_coeffs.restype = c_int
     lib.lm_msign_ns_noalloc.argtypes = [P(LmTensor), P(LmTensor), c_int, c_double, c_double, c_double,
                                         c_double, c_int, c_void_p]
     lib.lm_msign_ns_noalloc.restype = c_int
@@ -169,19 +173,28 @@ class LionMuon:
     """Optimizer state over a list of torch parameters (the ``lm_state``)."""
 
     def __init__(self, params: Sequence, stream=None, **cfg):
+        """cfg: lm_config fields by name; ns_coeffs may be a sequence of
+        (a_k, b_k, c_k) triples, one per NS iteration (ns_steps follows it)."""
         self._lib = load_library()
         self.params = list(params)
         c = default_config()
+        table = cfg.pop("ns_coeffs", None)
         for k, v in cfg.items():
             if not hasattr(c, k):
                 raise TypeError(f"unknown config field {k!r}")
             setattr(c, k, v)
+        keep = None
+        if table is not None:
+            keep = _coeff_array(table)
+            c.ns_steps = len(keep) // 3
+            c.ns_coeffs = keep
         self.config = c
         descs = (LmTensor * len(self.params))(*[tensor_desc(p) for p in self.params])
         h = ctypes.c_void_p()
         _check(self._lib, self._lib.lm_create(descs, len(self.params), ctypes.byref(c),
                                               _stream_handle(stream), ctypes.byref(h)), "lm_create")
         self._h = h
+        c.ns_coeffs = None   # lm_create copied the table
 
     def step(self, grads: Sequence, t: int, stream=None) -> None:
         descs = (LmTensor * len(grads))(*[tensor_desc(g) for g in grads])
@@ -253,6 +266,25 @@ def msign_ns(x, out, steps: int = 5, a: float = 3.4445, b: float = -4.7750, c: f
     di, do = tensor_desc(x), tensor_desc(out)
     _check(lib, lib.lm_msign_ns(ctypes.byref(di), ctypes.byref(do), steps, a, b, c, eps, precision,
                                 _stream_handle(stream)), "lm_msign_ns")
+    return out
+
+
+def _coeff_array(table):
+    """Flatten (a_k, b_k, c_k) triples into a ctypes double array."""
+    flat = [float(x) for tr in table for x in tr]
+    if any(len(tr) != 3 for tr in table):
+        raise ValueError("every NS coefficient entry must be an (a, b, c) triple")
+    return (ctypes.c_double * max(len(flat), 1))(*flat) if flat else None
+
+
+def msign_ns_coeffs(x, out, coeffs, eps: float = 1e-7, precision: int = LM_BF16, stream=None):
+    """out <- NS(x) with iteration-dependent coefficients: coeffs is a
+    sequence of (a_k, b_k, c_k) triples, one per iteration (lm_msign_ns_coeffs)."""
+    lib = load_library()
+    di, do = tensor_desc(x), tensor_desc(out)
+    arr = _coeff_array(coeffs)
+    _check(lib, lib.lm_msign_ns_coeffs(ctypes.byref(di), ctypes.byref(do), len(coeffs), arr, eps, precision,
+                                       _stream_handle(stream)), "lm_msign_ns_coeffs")
     return out
 
 

@@ -94,3 +94,56 @@ def test_msign_repeat_calls_identical():
     a = _msign(xh, "bf16")
     b = _msign(xh, "bf16")
     np.testing.assert_array_equal(a, b)
+
+
+MIXED_TABLE = ((3.0, -3.2, 1.2), (2.0, -1.5, 0.45), (1.875, -1.25, 0.375))
+
+
+def table_tolerance(x, table, precision):
+    """NS tolerance for a coefficient table: the stated one (2e-2 bf16,
+    1e-5 fp32), or 1.5 times the distance that storing the intermediates in
+    the path's precision alone puts between the oracle's storage-modelled
+    recurrence and its exact one, whichever is larger.  Aggressive first
+    polynomials (the minimax tables start near 8.5 x) amplify rounding of
+    small singular values; the storage-modelled oracle measures by how much
+    for this input, independently of the GPU."""
+    storage = "bf16" if precision == "bf16" else "f32"
+    d = rel_fro(O.ns_polynomial_schedule_storage(x, table, 1e-7, storage), O.ns_polynomial_schedule(x, table, 1e-7))
+    return max(TOL[precision], 1.5 * d)
+
+
+def _table(name):
+    from paper_2605_19811_gb300 import ns_coeffs as C
+    return {"polar_express": C.polar_express(5, 1e-3), "chebyshev_cubic": C.chebyshev_cubic(6, 1e-3),
+            "mixed": MIXED_TABLE}[name]
+
+
+@pytest.mark.parametrize("precision", ["bf16", "f32"])
+@pytest.mark.parametrize("name", ["polar_express", "chebyshev_cubic", "mixed"])
+@pytest.mark.parametrize("shape", [(256, 768), (768, 256), (300, 130), (64, 64)])
+def test_msign_coefficient_table_parity(precision, name, shape):
+    """Iteration-dependent coefficients (lm_msign_ns_coeffs) against the
+    oracle's NS recurrence with the same table."""
+    import torch
+    from paper_2605_19811_gb300 import lionmuon as L
+    table = _table(name)
+    in_dtype = "bf16" if precision == "bf16" else "f32"
+    xh = host_tensor(synth.draw_matrix(shape, seed=11 + sum(shape)), in_dtype)
+    x = xh.cuda()
+    out = torch.empty(x.shape, dtype=torch.float32, device="cuda")
+    L.msign_ns_coeffs(x, out, table, precision=L.LM_BF16 if precision == "bf16" else L.LM_F32)
+    torch.cuda.synchronize()
+    want = O.ns_polynomial_schedule(stored_values(xh), table, 1e-7)
+    assert rel_fro(stored_values(out), want) <= table_tolerance(stored_values(xh), table, precision)
+
+
+def test_msign_coefficient_table_argument_errors():
+    import torch
+    from paper_2605_19811_gb300 import lionmuon as L
+    x = torch.zeros((32, 48), device="cuda")
+    out = torch.empty_like(x)
+    with pytest.raises(L.LionMuonError) as e:
+        L.msign_ns_coeffs(x, out, [(1.0, float("nan"), 0.0)])
+    assert e.value.status == 1
+    with pytest.raises(L.LionMuonError):
+        L.msign_ns_coeffs(x, out, [(1.0, 0.0, 0.0)] * 65)

@@ -62,8 +62,15 @@ def _bf16_ns_bounds(W0, grads, dtype, cfg: O.Config, steps, Wo):
         for i, (p, g, m) in enumerate(zip(P, G, M)):
             if O.is_matrix(p.shape) and O.is_muon_step(t, cfg.period):
                 gh = O.interpolated_direction(m, g, cfg.beta1)
-                o = O.ns_polynomial(gh, cfg.ns_steps, cfg.ns_a, cfg.ns_b, cfg.ns_c, cfg.ns_eps)
-                acc[i] += cfg.eta_muon * cfg.shape_scale * np.sqrt(max(p.shape)) * NS_TOL_BF16 * np.linalg.norm(o)
+                tau = NS_TOL_BF16
+                if cfg.ns_coeffs is not None:
+                    o = O.ns_polynomial_schedule(gh, cfg.ns_coeffs, cfg.ns_eps)
+                    # the table's own sensitivity to bf16 storage (see test_gpu_msign.table_tolerance)
+                    d = rel_fro(O.ns_polynomial_schedule_storage(gh, cfg.ns_coeffs, cfg.ns_eps, "bf16"), o)
+                    tau = max(tau, 1.5 * d)
+                else:
+                    o = O.ns_polynomial(gh, cfg.ns_steps, cfg.ns_a, cfg.ns_b, cfg.ns_c, cfg.ns_eps)
+                acc[i] += cfg.eta_muon * cfg.shape_scale * np.sqrt(max(p.shape)) * tau * np.linalg.norm(o)
             M[i] = O.momentum_update(m, g, cfg.beta2)
     out = []
     for a, w in zip(acc, Wo):
@@ -266,3 +273,33 @@ def test_fused_parameter_write_matches_finalize_kernel_bit_exact():
         opt.close()
     for a, b in zip(*out):
         np.testing.assert_array_equal(a, b)
+
+
+@pytest.mark.parametrize("precision", [1, 0])
+def test_small_gpt_8_steps_polar_express_table(precision):
+    """Whole steps with an iteration-dependent NS table (the degree-5 minimax
+    schedule from l_0 = 1e-3): weights after 8 steps against the
+    storage-modelled oracle run with the same table."""
+    from paper_2605_19811_gb300 import ns_coeffs as C
+    table = C.polar_express(5, 1e-3)
+    steps = 8
+    shapes = SMALL_GPT.shapes
+    W0, grads = make_problem(shapes, "student_t", steps)
+    gcfg, ocfg = _cfg_pair(eta_muon=3e-3, eta_lion=2e-5, weight_decay=0.1, period=2,
+                           ns_precision=precision, ns_coeffs=table)
+    Wg, Mg, flags = run_trajectory_gpu(W0, grads, "bf16", gcfg, steps)
+    Wo, _ = run_trajectory_oracle(W0, grads, "bf16", ocfg, steps)
+    Mo = _momentum_same_order([[stored_values(host_tensor(g, "bf16")).astype(np.float32) for g in gs]
+                               for gs in grads], shapes, 0.99, steps)
+    tol = 1e-3 if precision == 0 else _bf16_ns_bounds(W0, grads, "bf16", ocfg, steps, Wo)
+    _check(Wg, Wo, Mg, Mo, tol)
+    assert flags == 0
+
+
+def test_coefficient_table_rejected_when_not_finite():
+    import torch
+    from paper_2605_19811_gb300 import lionmuon as L
+    p = [torch.zeros((32, 48), dtype=torch.bfloat16, device="cuda")]
+    with pytest.raises(L.LionMuonError) as e:
+        L.LionMuon(p, ns_coeffs=[(1.0, 0.0, 0.0), (float("inf"), 0.0, 0.0)])
+    assert e.value.status == 1

@@ -45,6 +45,7 @@ PIN_CALLS = [
     (vpins.test_ns_schedule_closed_form_on_known_svd, ()),
     (vpins.test_ns_schedule_constant_table_is_classical_ns, ()),
     (vpins.test_minimax_schedule_maps_interval_forward, (5, 5)),
+    (vpins.test_bf16_storage_ns_on_hadamard_follows_hand_rounded_scalars, ()),
 ]
 
 
@@ -93,6 +94,7 @@ def _mutations():
                                    ("ns_scalar_map_schedule", _scalar_schedule_factory(first_only=True))]
     muts["minimax_least_squares"] = [("minimax_odd_polynomial", _least_squares_poly)]
     muts["minimax_no_interval_update"] = [("minimax_schedule", _schedule_fixed_interval)]
+    muts["storage_ns_unrounded_B"] = [("ns_polynomial_schedule_storage", _storage_ns_unrounded_B)]
     return muts
 
 
@@ -161,6 +163,22 @@ def _bf16_truncate(x):
     return u.view(np.float32).copy()
 
 
+def _storage_ns_unrounded_B(G, coeffs, eps=1e-7, storage="bf16"):
+    rd = lambda v: OM.bf16_round(v).astype(np.float64)
+    G = np.array(G, dtype=np.float64)
+    tr = G.shape[0] > G.shape[1]
+    if tr:
+        G = G.T.copy()
+    inv = 1.0 / (np.linalg.norm(G) + eps)
+    X = rd(G)
+    for k, (a, b, c) in enumerate(coeffs):
+        sa, sx = (inv * inv, inv) if k == 0 else (1.0, 1.0)
+        A = rd(sa * (X @ X.T))
+        B = b * A + c * (A @ A)
+        X = rd(sx * (a * X + B @ X))
+    return X.T.copy() if tr else X
+
+
 @pytest.mark.filterwarnings("ignore::RuntimeWarning")
 @pytest.mark.parametrize("name", sorted(_mutations()))
 def test_each_planted_mistake_is_caught(name, monkeypatch):
@@ -173,3 +191,4 @@ def test_each_planted_mistake_is_caught(name, monkeypatch):
         except (AssertionError, ValueError):
             caught.append(pin.__name__)
     assert caught, f"no pin detects the mutation {name}"
+

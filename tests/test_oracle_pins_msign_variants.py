@@ -131,3 +131,47 @@ def test_polar_express_beats_constant_quintic_on_spread_spectrum():
     err_pe = np.abs(O.ns_scalar_map_schedule(x, table) - 1.0).max()
     err_q = np.abs(O.ns_scalar_map(x, 5, *O.NS_QUINTIC) - 1.0).max()
     assert err_pe < err_q
+
+
+def test_bf16_storage_ns_on_hadamard_follows_hand_rounded_scalars():
+    """For G = c H (H a 16 x 16 orthogonal Hadamard matrix, entries +-1/4)
+    every intermediate is a scalar multiple of I or H, so the stored values
+    follow a scalar recurrence whose roundings can be done by hand with
+    torch's bf16 conversion: with eps = 0 the normalised singular value is
+    x = 1/4 (||H||_F = 4), A = bf16(x^2) I, B = bf16(b A + c A^2) I and
+    X <- bf16(a X + B X) entrywise."""
+    import torch
+    from tests.test_oracle_pins import hadamard
+
+    def r(v):
+        return float(torch.tensor(v, dtype=torch.float64).to(torch.bfloat16).to(torch.float64))
+
+    H = hadamard(16)
+    assert np.allclose(H @ H.T, np.eye(16))
+    table = ((3.4445, -4.7750, 2.0315), (8.47, -25.1, 18.63), (2.0, -1.5, 0.45))
+    got = O.ns_polynomial_schedule_storage(3.0 * H, table, 0.0, "bf16")
+    # entries of X are +-h with h = x / 4 (x the singular value of X)
+    h = r(3.0 * 0.25)              # X_0 = bf16(G): entries 3/4
+    inv = 1.0 / 12.0               # ||3 H||_F = 12
+    for k, (a, b, c) in enumerate(table):
+        sa, sx = (inv * inv, inv) if k == 0 else (1.0, 1.0)
+        A = r(sa * 16 * h * h)     # X X^T = 16 h^2 I
+        B = r(b * A + c * A * A)
+        h = r(sx * (a * h + B * h))
+    want = h * (H * 4.0)           # H * 4 has entries +-1
+    np.testing.assert_array_equal(got, want)
+
+
+def test_bf16_storage_ns_tracks_exact_recurrence():
+    """bf16 storage perturbs the constant quintic by about the bf16 spacing
+    amplified a little, not by orders of magnitude, and not at all in the
+    limit of no rounding (checked through the Hadamard case above)."""
+    r = np.random.default_rng(4)
+    G = r.normal(size=(64, 160))
+    ex = O.ns_polynomial_schedule(G, (O.NS_QUINTIC,) * 5, 1e-7)
+    em = O.ns_polynomial_schedule_storage(G, (O.NS_QUINTIC,) * 5, 1e-7, "bf16")
+    e = np.linalg.norm(em - ex) / np.linalg.norm(ex)
+    assert 2.0 ** -10 < e < 5e-2
+    ef = O.ns_polynomial_schedule_storage(G, (O.NS_QUINTIC,) * 5, 1e-7, "f32")
+    e32 = np.linalg.norm(ef - ex) / np.linalg.norm(ex)
+    assert 2.0 ** -26 < e32 < 1e-5
