@@ -31,7 +31,10 @@ Readings taken where the paper is silent (each listed in the design doc):
 * The 0.2*sqrt(max(m,n)) factor multiplies the NS output inside the eta_M
   bracket; the decay term is not scaled.
 * sign(0) = 0 and sign(NaN) = NaN.
-* 1-D parameters (vectors) take the Lion step on every step.
+* 1-D parameters (vectors) take the Lion step on every step by default; the
+  AdamW fallback of Section 3 is the ``vector_rule="adamw"`` option, with
+  Table 5's 1-D learning rate 1e-3 and AdamW betas (0.8, 0.999), weight decay
+  0.1 (Table 5's), eps 1e-8, bias correction with the update count t + 1.
 * P = infinity is encoded as ``period = 0``.
 * Iteration-dependent NS coefficients (the minimax / Chebyshev-type msign
   iterations of Section 2) keep the Frobenius normalisation, so the first
@@ -81,6 +84,15 @@ class Config:
     # Optional per-iteration coefficients ((a_0, b_0, c_0), ...): when set they
     # replace (ns_a, ns_b, ns_c) and their count replaces ns_steps.
     ns_coeffs: Optional[Tuple[Tuple[float, float, float], ...]] = None
+    # 1-D parameters: "lion" (the Lion step of Algorithm 1 every step) or
+    # "adamw" (Section 3's fallback for biases and norm gains, with Table 5's
+    # 1-D learning rate 1e-3 and AdamW betas (0.8, 0.999)).
+    vector_rule: str = "lion"
+    adamw_lr: float = 1e-3
+    adamw_beta1: float = 0.8
+    adamw_beta2: float = 0.999
+    adamw_eps: float = 1e-8
+    adamw_weight_decay: float = 0.1
 
 
 # ---------------------------------------------------------------------------
@@ -308,6 +320,26 @@ def muon_update(W, G_hat, cfg: Config):
     return W - cfg.eta_muon * (scale * O + cfg.weight_decay * W)
 
 
+def adamw_update(W, G, m_prev, v_prev, step: int, lr, beta1, beta2, eps, weight_decay):
+    """AdamW with decoupled weight decay (Loshchilov and Hutter), the update
+    Section 3 gives 1-D parameters (biases, norm gains) in the LionMuon hybrid;
+    ``step`` counts this parameter's AdamW updates, 1 for the first:
+        m = beta1 m + (1 - beta1) G,   v = beta2 v + (1 - beta2) G^2
+        m_hat = m / (1 - beta1^step),  v_hat = v / (1 - beta2^step)
+        W <- W - lr lambda W - lr m_hat / (sqrt(v_hat) + eps)
+    Returns (W_new, m, v), fp64."""
+    if step < 1:
+        raise ValueError("step counts updates from 1")
+    W = np.asarray(W, dtype=np.float64)
+    G = np.asarray(G, dtype=np.float64)
+    m = beta1 * np.asarray(m_prev, dtype=np.float64) + (1.0 - beta1) * G
+    v = beta2 * np.asarray(v_prev, dtype=np.float64) + (1.0 - beta2) * G * G
+    m_hat = m / (1.0 - beta1 ** step)
+    v_hat = v / (1.0 - beta2 ** step)
+    W_new = W - lr * weight_decay * W - lr * m_hat / (np.sqrt(v_hat) + eps)
+    return W_new, m, v
+
+
 def is_matrix(shape: Sequence[int]) -> bool:
     """A parameter is a hidden matrix (takes Muon steps) unless it is a vector
     (one of its two dimensions is 1)."""
@@ -369,26 +401,45 @@ def round_to_storage(x: np.ndarray, dtype: str) -> np.ndarray:
 
 def lionmuon_step(params: List[np.ndarray], grads: List[np.ndarray],
                   moms: List[np.ndarray], t: int, cfg: Config,
-                  param_dtypes: Optional[List[str]] = None):
+                  param_dtypes: Optional[List[str]] = None,
+                  seconds: Optional[List[np.ndarray]] = None):
     """One LionMuon step over a list of parameters (Algorithm 1 applied to
-    each parameter; vectors take the Lion step every step).
+    each matrix; vectors take the Lion step every step, or AdamW when
+    ``cfg.vector_rule == "adamw"``, with M as AdamW's first moment, the
+    second moments in ``seconds`` and the update count t + 1).
 
     With ``param_dtypes`` given, the new weights are rounded to their storage
-    dtype, the momentum to float32, and Lion signs are decided on the float32
-    G_hat (storage-modelled mode); otherwise the state stays in fp64 (exact
-    mode).  Returns (new_params, new_moms)."""
+    dtype, the momentum (and second moments) to float32, and Lion signs are
+    decided on the float32 G_hat (storage-modelled mode); otherwise the state
+    stays in fp64 (exact mode).  Returns (new_params, new_moms), plus
+    new_seconds when ``seconds`` is given."""
     if not (len(params) == len(grads) == len(moms)):
         raise ValueError("params, grads and moms must have equal length")
-    new_p, new_m = [], []
+    adamw = cfg.vector_rule == "adamw"
+    if cfg.vector_rule not in ("lion", "adamw"):
+        raise ValueError("vector_rule must be 'lion' or 'adamw'")
+    if adamw and seconds is None:
+        raise ValueError("the AdamW rule needs the second moments")
+    new_p, new_m, new_v = [], [], []
     for i, (W, G, M) in enumerate(zip(params, grads, moms)):
         if np.shape(W) != np.shape(G) or np.shape(W) != np.shape(M):
             raise ValueError(f"shape mismatch at parameter {i}")
-        W1, M1 = lionmuon_param_step(W, G, M, t, cfg, sign_in_f32=param_dtypes is not None)
+        V1 = None if seconds is None else seconds[i]
+        if adamw and not is_matrix(np.shape(W)):
+            W1, M1, V1 = adamw_update(W, G, M, seconds[i], t + 1, cfg.adamw_lr, cfg.adamw_beta1,
+                                      cfg.adamw_beta2, cfg.adamw_eps, cfg.adamw_weight_decay)
+        else:
+            W1, M1 = lionmuon_param_step(W, G, M, t, cfg, sign_in_f32=param_dtypes is not None)
         if param_dtypes is not None:
             W1 = round_to_storage(W1, param_dtypes[i])
             M1 = round_to_storage(M1, "f32")
+            if V1 is not None:
+                V1 = round_to_storage(V1, "f32")
         new_p.append(W1)
         new_m.append(M1)
+        new_v.append(V1)
+    if seconds is not None:
+        return new_p, new_m, new_v
     return new_p, new_m
 
 
@@ -430,6 +481,41 @@ def lion_step_f32(w: np.ndarray, g: np.ndarray, m: np.ndarray, beta1, beta2,
     elif w_dtype != "f32":
         raise ValueError(f"unknown w dtype {w_dtype!r}")
     return w_new.astype(np.float32), m_new.astype(np.float32)
+
+
+def adamw_constants_f32(step: int, lr, beta1, beta2, eps, weight_decay):
+    """The float32 constants of one AdamW step, each rounded once from its
+    double value: b1, 1 - b1, b2, 1 - b2, lr / (1 - beta1^step),
+    1 / sqrt(1 - beta2^step), lr * lambda, eps (powers and roots in double,
+    by the C library's pow and sqrt)."""
+    f = np.float32
+    bc1 = 1.0 - math.pow(beta1, step)
+    bc2 = 1.0 - math.pow(beta2, step)
+    return (f(beta1), f(1.0 - beta1), f(beta2), f(1.0 - beta2), f(lr / bc1), f(1.0 / math.sqrt(bc2)),
+            f(lr * weight_decay), f(eps))
+
+
+def adamw_step_f32(w, g, m, v, step: int, lr, beta1, beta2, eps, weight_decay, w_dtype: str = "bf16"):
+    """AdamW step in float32 with a fixed operation order, every operation
+    rounded once (no fused multiply-add; sqrt and division correctly
+    rounded):
+        m = b1*m + c1*g ;  v = b2*v + c2*(g*g)
+        w = w - lrwd*w ;   den = sqrt(v)*rbc2 + eps ;  w = w - step_size*(m/den)
+    then bf16 round-to-nearest-even of w for bf16 parameters.  Returns
+    (w, m, v) as float32 arrays."""
+    b1, c1, b2, c2, st, rbc2, lrwd, e = adamw_constants_f32(step, lr, beta1, beta2, eps, weight_decay)
+    w = np.asarray(w, dtype=np.float32)
+    g = np.asarray(g, dtype=np.float32)
+    m = (b1 * np.asarray(m, dtype=np.float32)) + (c1 * g)
+    v = (b2 * np.asarray(v, dtype=np.float32)) + (c2 * (g * g))
+    w = w - lrwd * w
+    den = (np.sqrt(v) * rbc2) + e
+    w = w - st * (m / den)
+    if w_dtype == "bf16":
+        w = bf16_round(w)
+    elif w_dtype != "f32":
+        raise ValueError(f"unknown w dtype {w_dtype!r}")
+    return w.astype(np.float32), m.astype(np.float32), v.astype(np.float32)
 
 
 # ---------------------------------------------------------------------------

@@ -12,6 +12,7 @@ import oracle
 import oracle.lionmuon_oracle as OM
 from tests import test_oracle_pins as pins
 from tests import test_oracle_pins_msign_variants as vpins
+from tests import test_oracle_pins_adamw as apins
 
 # every pin, with representative arguments for the parametrised ones
 PIN_CALLS = [
@@ -46,6 +47,10 @@ PIN_CALLS = [
     (vpins.test_ns_schedule_constant_table_is_classical_ns, ()),
     (vpins.test_minimax_schedule_maps_interval_forward, (5, 5)),
     (vpins.test_bf16_storage_ns_on_hadamard_follows_hand_rounded_scalars, ()),
+    (apins.test_adamw_matches_torch_adamw_float64, (0.1,)),
+    (apins.test_adamw_constant_gradient_closed_form, ()),
+    (apins.test_adamw_zero_gradient_is_pure_decay, ()),
+    (apins.test_adamw_first_step_is_sign_like, ()),
 ]
 
 
@@ -95,6 +100,10 @@ def _mutations():
     muts["minimax_least_squares"] = [("minimax_odd_polynomial", _least_squares_poly)]
     muts["minimax_no_interval_update"] = [("minimax_schedule", _schedule_fixed_interval)]
     muts["storage_ns_unrounded_B"] = [("ns_polynomial_schedule_storage", _storage_ns_unrounded_B)]
+    muts["adamw_no_bias_correction"] = [("adamw_update", _adamw_variant("no_bias"))]
+    muts["adamw_coupled_decay"] = [("adamw_update", _adamw_variant("coupled"))]
+    muts["adamw_eps_inside_sqrt"] = [("adamw_update", _adamw_variant("eps_in_sqrt"))]
+    muts["adamw_beta_swap"] = [("adamw_update", _adamw_variant("swap"))]
     return muts
 
 
@@ -161,6 +170,22 @@ def _bf16_truncate(x):
     f = np.ascontiguousarray(np.asarray(x, dtype=np.float32))
     u = f.view(np.uint32) & np.uint32(0xFFFF0000)
     return u.view(np.float32).copy()
+
+
+def _adamw_variant(kind):
+    def f(W, G, m_prev, v_prev, step, lr, beta1, beta2, eps, weight_decay):
+        W = np.asarray(W, dtype=np.float64)
+        G = np.asarray(G, dtype=np.float64)
+        if kind == "swap":
+            beta1, beta2 = beta2, beta1
+        g_eff = G + weight_decay * W if kind == "coupled" else G
+        m = beta1 * m_prev + (1 - beta1) * g_eff
+        v = beta2 * v_prev + (1 - beta2) * g_eff * g_eff
+        bc1, bc2 = (1.0, 1.0) if kind == "no_bias" else (1 - beta1 ** step, 1 - beta2 ** step)
+        den = np.sqrt(v / bc2 + eps) if kind == "eps_in_sqrt" else np.sqrt(v / bc2) + eps
+        decay = 0.0 if kind == "coupled" else lr * weight_decay * W
+        return W - decay - lr * (m / bc1) / den, m, v
+    return f
 
 
 def _storage_ns_unrounded_B(G, coeffs, eps=1e-7, storage="bf16"):
