@@ -89,7 +89,21 @@ typedef struct {
   double shape_scale;
   int ns_precision;
   const double* ns_coeffs;
+  /* Update rule of 1-D parameters (rows == 1 or cols == 1): LM_VECTOR_LION
+   * (Algorithm 1's Lion step on every step, the default) or LM_VECTOR_ADAMW,
+   * the AdamW fallback Section 3 uses for biases and norm gains:
+   *   m = b1 m + (1-b1) g;  v = b2 v + (1-b2) g^2;  w -= lr wd w;
+   *   w -= lr / (1 - b1^(t+1)) * m / (sqrt(v) / sqrt(1 - b2^(t+1)) + eps)
+   * with the momentum buffer as m, one more fp32 buffer v per 1-D parameter,
+   * and t the step index passed to lm_step (t + 1 updates so far).
+   * adamw_lr >= 0 (Table 5: 1e-3), adamw_beta1/2 in [0, 1) (Table 5:
+   * 0.8, 0.999), adamw_eps > 0 (1e-8), adamw_weight_decay >= 0 (0.1). */
+  int vector_rule;
+  double adamw_lr, adamw_beta1, adamw_beta2, adamw_eps, adamw_weight_decay;
 } lm_config;
+
+#define LM_VECTOR_LION 0
+#define LM_VECTOR_ADAMW 1
 
 typedef struct lm_state lm_state; /* opaque */
 
@@ -122,6 +136,21 @@ lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t,
 /* Change the two learning rates (a caller-driven schedule); takes effect for
  * the next lm_step.  Errors: LM_ERR_INVALID_ARG (NULL, negative, non-finite). */
 lm_status lm_set_lr(lm_state* s, double eta_muon, double eta_lion);
+
+/* Change the AdamW learning rate of 1-D parameters (LM_VECTOR_ADAMW); takes
+ * effect for the next lm_step.  Errors: LM_ERR_INVALID_ARG (NULL, negative,
+ * non-finite). */
+lm_status lm_set_adamw_lr(lm_state* s, double lr);
+
+/* AdamW second moment v of 1-D parameter i (LM_VECTOR_ADAMW only): a
+ * read-only fp32 device view of the parameter's shape, owned by the state;
+ * lm_set_second_moment copies src (fp32 device memory of that shape) into it
+ * on cuda_stream, for checkpoint / resume together with lm_set_momentum.
+ * Errors: LM_ERR_INVALID_ARG (NULL, index out of range, parameter i has no
+ * second moment, shape mismatch), LM_ERR_DTYPE, LM_ERR_ALIGN, LM_ERR_CUDA. */
+lm_status lm_get_second_moment(const lm_state* s, int i, lm_tensor* view);
+lm_status lm_set_second_moment(lm_state* s, int i, const lm_tensor* src,
+                               void* cuda_stream);
 
 /* Newton-Schulz approximation of msign (Section 2): out = NS_steps(in) with
  * coefficients (a, b, c), normalisation X / (||X||_F + eps), iterated on the
@@ -182,8 +211,9 @@ lm_status lm_set_momentum(lm_state* s, int i, const lm_tensor* src,
 lm_status lm_get_status(lm_state* s, uint32_t* device_flags);
 
 /* Bytes of persisted optimizer state: exactly 4 * sum |W_i| (one fp32
- * momentum buffer per parameter, Section 3 Implementation notes).  Returns 0
- * for NULL. */
+ * momentum buffer per parameter, Section 3 Implementation notes), plus
+ * 4 * sum |w| over 1-D parameters with LM_VECTOR_ADAMW (their second
+ * moments).  Returns 0 for NULL. */
 size_t lm_state_bytes(const lm_state* s);
 
 /* Bytes of transient device workspace the state holds (Newton-Schulz
@@ -226,7 +256,8 @@ typedef enum {
   LM_KERNEL_NS_APPLY = 4,      /* Newton-Schulz: X <- a X + B X */
   LM_KERNEL_FINALIZE = 5,      /* Muon: parameter write */
   LM_KERNEL_OTHER = 6,         /* gradient-pointer upload, norm reset */
-  LM_KERNEL_FAMILIES = 7
+  LM_KERNEL_ADAMW = 7,         /* AdamW on 1-D parameters (LM_VECTOR_ADAMW) */
+  LM_KERNEL_FAMILIES = 8
 } lm_kernel_family;
 
 typedef struct {

@@ -79,6 +79,16 @@ lm_status check_config(const lm_config* c) {
   if (!finite(c->shape_scale) || c->shape_scale < 0) return fail(LM_ERR_INVALID_ARG, "shape_scale must be >= 0");
   if (c->ns_precision != LM_BF16 && c->ns_precision != LM_F32)
     return fail(LM_ERR_INVALID_ARG, "ns_precision must be LM_BF16 or LM_F32");
+  if (c->vector_rule != LM_VECTOR_LION && c->vector_rule != LM_VECTOR_ADAMW)
+    return fail(LM_ERR_INVALID_ARG, "vector_rule must be LM_VECTOR_LION or LM_VECTOR_ADAMW");
+  if (c->vector_rule == LM_VECTOR_ADAMW) {
+    if (!finite(c->adamw_lr) || c->adamw_lr < 0) return fail(LM_ERR_INVALID_ARG, "adamw_lr must be finite and >= 0");
+    if (!(c->adamw_beta1 >= 0.0 && c->adamw_beta1 < 1.0) || !(c->adamw_beta2 >= 0.0 && c->adamw_beta2 < 1.0))
+      return fail(LM_ERR_INVALID_ARG, "adamw_beta1/adamw_beta2 must lie in [0, 1)");
+    if (!finite(c->adamw_eps) || !(c->adamw_eps > 0)) return fail(LM_ERR_INVALID_ARG, "adamw_eps must be > 0");
+    if (!finite(c->adamw_weight_decay) || c->adamw_weight_decay < 0)
+      return fail(LM_ERR_INVALID_ARG, "adamw_weight_decay must be >= 0");
+  }
   return LM_OK;
 }
 
@@ -105,6 +115,24 @@ LionConsts lion_consts(const lm_config& c) {
   k.lam = (float)c.weight_decay;
   return k;
 }
+// AdamW constants of step t (update number t + 1): powers and the square
+// root in double, each constant rounded once to float.
+AdamConsts adamw_consts(const lm_config& c, int64_t t) {
+  const double k = (double)(t + 1);
+  const double bc1 = 1.0 - std::pow(c.adamw_beta1, k);
+  const double bc2 = 1.0 - std::pow(c.adamw_beta2, k);
+  AdamConsts a;
+  a.b1 = (float)c.adamw_beta1;
+  a.c1 = (float)(1.0 - c.adamw_beta1);
+  a.b2 = (float)c.adamw_beta2;
+  a.c2 = (float)(1.0 - c.adamw_beta2);
+  a.step = (float)(c.adamw_lr / bc1);
+  a.rbc2 = (float)(1.0 / std::sqrt(bc2));
+  a.lrwd = (float)(c.adamw_lr * c.adamw_weight_decay);
+  a.eps = (float)c.adamw_eps;
+  return a;
+}
+
 MuonConsts muon_consts(const lm_config& c) {
   MuonConsts k;
   k.b1 = (float)c.beta1;
@@ -148,7 +176,14 @@ struct NsBatch {
   int npairs[3] = {0, 0, 0};
 };
 
-void build_lion_chunks(const std::vector<LionTensor>& ts, std::vector<LionChunk>& out) {
+struct AdamTable {
+  AdamTensor* tensors = nullptr;
+  LionChunk* chunks = nullptr;
+  int nchunks = 0;
+};
+
+template <typename TensorT>
+void build_lion_chunks(const std::vector<TensorT>& ts, std::vector<LionChunk>& out) {
   for (size_t i = 0; i < ts.size(); ++i) {
     for (int64_t b = 0; b < ts[i].n; b += kLionChunk) {
       LionChunk c;
@@ -464,7 +499,12 @@ struct lm_state {
   const void** d_grads = nullptr;   // device grad-pointer table
   std::vector<const void*> h_grads; // what the device table holds
   bool grads_valid = false;
-  LionTable lion_all[2], lion_vec[2];
+  LionTable lion_all[2], lion_vec[2];   // lion_all: matrices only under LM_VECTOR_ADAMW
+  bool adamw = false;                   // 1-D parameters take AdamW
+  AdamTable adam[2];                    // per dtype, 1-D parameters
+  float* vmom = nullptr;                // AdamW second moments
+  std::vector<int64_t> v_off;           // element offset per parameter, -1 if none
+  size_t v_elems = 0;
   int lion_grid[2] = {0, 0};
   int nmat = 0;
   MatDesc* d_mats = nullptr;
@@ -496,6 +536,12 @@ void lm_config_default(lm_config* c) {
   c->shape_scale = 0.2;
   c->ns_precision = LM_BF16;
   c->ns_coeffs = nullptr;
+  c->vector_rule = LM_VECTOR_LION;
+  c->adamw_lr = 1e-3;
+  c->adamw_beta1 = 0.8;
+  c->adamw_beta2 = 0.999;
+  c->adamw_eps = 1e-8;
+  c->adamw_weight_decay = 0.1;
 }
 
 const char* lm_status_string(lm_status st) {
@@ -561,6 +607,18 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
     s->mom_elems += (size_t)numel(params[i]);
   }
   const size_t off_mom = ar.add(mom_elems_aligned * sizeof(float));
+  // AdamW second moments of the 1-D parameters
+  s->adamw = cfg->vector_rule == LM_VECTOR_ADAMW;
+  s->v_off.assign(n, -1);
+  size_t v_aligned = 0;
+  if (s->adamw)
+    for (int i = 0; i < n; ++i)
+      if (!is_matrix(params[i])) {
+        s->v_off[i] = (int64_t)v_aligned;
+        v_aligned = align_up(v_aligned + (size_t)numel(params[i]), 64);
+        s->v_elems += (size_t)numel(params[i]);
+      }
+  const size_t off_v = ar.add(v_aligned * sizeof(float));
   const size_t off_grads = ar.add((size_t)n * sizeof(void*));
   const size_t off_flags = ar.add(sizeof(unsigned));
 
@@ -574,8 +632,28 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
     t.n = numel(params[i]);
     t.grad_slot = i;
     t.pad = i;       // remember the param index until binding
-    lt_all[params[i].dtype].push_back(t);
+    if (!s->adamw || is_matrix(params[i])) lt_all[params[i].dtype].push_back(t);
     if (!is_matrix(params[i])) lt_vec[params[i].dtype].push_back(t);
+  }
+  // AdamW tables (per dtype) over the 1-D parameters
+  std::vector<AdamTensor> at[2];
+  std::vector<LionChunk> ac[2];
+  size_t off_at[2], off_ac[2];
+  for (int i = 0; s->adamw && i < n; ++i) {
+    if (numel(params[i]) == 0 || is_matrix(params[i])) continue;
+    AdamTensor t;
+    t.w = params[i].data;
+    t.m = nullptr;
+    t.v = nullptr;
+    t.n = numel(params[i]);
+    t.grad_slot = i;
+    t.pad = i;
+    at[params[i].dtype].push_back(t);
+  }
+  for (int d = 0; d < 2; ++d) {
+    build_lion_chunks(at[d], ac[d]);
+    off_at[d] = ar.add(at[d].size() * sizeof(AdamTensor));
+    off_ac[d] = ar.add(ac[d].size() * sizeof(LionChunk));
   }
   std::vector<LionChunk> lc_all[2], lc_vec[2];
   size_t off_lt_all[2], off_lc_all[2], off_lt_vec[2], off_lc_vec[2];
@@ -634,6 +712,17 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
     s->lion_vec[d] = {reinterpret_cast<LionTensor*>(base + off_lt_vec[d]),
                       reinterpret_cast<LionChunk*>(base + off_lc_vec[d]), (int)lc_vec[d].size()};
     s->lion_grid[d] = lion_grid_size((lm_dtype)d);
+  }
+  s->vmom = reinterpret_cast<float*>(base + off_v);
+  for (int d = 0; d < 2; ++d) {
+    for (auto& t : at[d]) {
+      t.m = s->mom + s->mom_off[t.pad];
+      t.v = s->vmom + s->v_off[t.pad];
+    }
+    if (!at[d].empty()) memcpy(img.data() + off_at[d], at[d].data(), at[d].size() * sizeof(AdamTensor));
+    if (!ac[d].empty()) memcpy(img.data() + off_ac[d], ac[d].data(), ac[d].size() * sizeof(LionChunk));
+    s->adam[d] = {reinterpret_cast<AdamTensor*>(base + off_at[d]), reinterpret_cast<LionChunk*>(base + off_ac[d]),
+                  (int)ac[d].size()};
   }
 
   bind_ns(s->ns, base, L, img);
@@ -718,6 +807,24 @@ static lm_status upload_grads(lm_state* s, const lm_tensor* grads, cudaStream_t 
   return LM_OK;
 }
 
+}  // extern "C"
+
+// AdamW over the 1-D parameters of both dtypes (LM_VECTOR_ADAMW).
+static lm_status run_adamw(lm_state* s, int64_t t, cudaStream_t stream) {
+  const AdamConsts ak = adamw_consts(s->cfg, t);
+  for (int d = 0; d < 2; ++d) {
+    if (s->adam[d].nchunks == 0) continue;
+    cudaError_t e = timed(&s->prof, LM_KERNEL_ADAMW, stream, [&]() {
+      return launch_adamw((lm_dtype)d, s->adam[d].tensors, s->adam[d].chunks, s->adam[d].nchunks, s->d_grads, ak,
+                          stream);
+    });
+    if (e != cudaSuccess) return cuda_fail(e, "AdamW kernel launch");
+  }
+  return LM_OK;
+}
+
+extern "C" {
+
 lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t, void* cuda_stream) {
   if (s == nullptr || grads == nullptr) return fail(LM_ERR_INVALID_ARG, "state/grads is NULL");
   if (n != s->n) return fail(LM_ERR_INVALID_ARG, "n = %d but the state has %d parameters", n, s->n);
@@ -749,7 +856,7 @@ lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t, void* c
       });
       if (e != cudaSuccess) return cuda_fail(e, "Lion kernel launch");
     }
-    return LM_OK;
+    return s->adamw ? run_adamw(s, t, stream) : LM_OK;
   }
   // Muon step: momentum + norm, Lion on the vectors, NS iterations, finalize.
   const MuonConsts mk = muon_consts(c);
@@ -767,7 +874,10 @@ lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t, void* c
       if (e != cudaSuccess) return cuda_fail(e, "momentum/norm kernel launch");
     }
   }
-  for (int d = 0; d < 2; ++d) {
+  if (s->adamw) {
+    if ((st = run_adamw(s, t, stream)) != LM_OK) return st;
+  }
+  for (int d = 0; d < 2 && !s->adamw; ++d) {
     if (s->lion_vec[d].nchunks == 0) continue;
     e = timed(P, LM_KERNEL_LION, stream, [&]() {
       return launch_lion((lm_dtype)d, s->lion_vec[d].tensors, s->lion_vec[d].chunks,
@@ -798,6 +908,41 @@ lm_status lm_set_lr(lm_state* s, double eta_muon, double eta_lion) {
     return fail(LM_ERR_INVALID_ARG, "learning rates must be finite and >= 0");
   s->cfg.eta_muon = eta_muon;
   s->cfg.eta_lion = eta_lion;
+  return LM_OK;
+}
+
+lm_status lm_set_adamw_lr(lm_state* s, double lr) {
+  if (s == nullptr) return fail(LM_ERR_INVALID_ARG, "state is NULL");
+  if (!std::isfinite(lr) || lr < 0) return fail(LM_ERR_INVALID_ARG, "learning rate must be finite and >= 0");
+  s->cfg.adamw_lr = lr;
+  return LM_OK;
+}
+
+lm_status lm_get_second_moment(const lm_state* s, int i, lm_tensor* view) {
+  if (s == nullptr || view == nullptr) return fail(LM_ERR_INVALID_ARG, "state/view is NULL");
+  if (i < 0 || i >= s->n) return fail(LM_ERR_INVALID_ARG, "index %d out of range", i);
+  if (s->v_off[i] < 0) return fail(LM_ERR_INVALID_ARG, "parameter %d has no AdamW second moment", i);
+  view->data = s->vmom + s->v_off[i];
+  view->rows = s->params[i].rows;
+  view->cols = s->params[i].cols;
+  view->dtype = LM_F32;
+  return LM_OK;
+}
+
+lm_status lm_set_second_moment(lm_state* s, int i, const lm_tensor* src, void* cuda_stream) {
+  if (s == nullptr || src == nullptr) return fail(LM_ERR_INVALID_ARG, "state/src is NULL");
+  if (i < 0 || i >= s->n) return fail(LM_ERR_INVALID_ARG, "index %d out of range", i);
+  if (s->v_off[i] < 0) return fail(LM_ERR_INVALID_ARG, "parameter %d has no AdamW second moment", i);
+  lm_status st = check_tensor(src, "src", 0);
+  if (st != LM_OK) return st;
+  if (src->dtype != LM_F32) return fail(LM_ERR_DTYPE, "second-moment source must be fp32");
+  if (src->rows != s->params[i].rows || src->cols != s->params[i].cols)
+    return fail(LM_ERR_INVALID_ARG, "second-moment source shape differs from the parameter's");
+  const size_t bytes = (size_t)numel(s->params[i]) * sizeof(float);
+  if (bytes == 0) return LM_OK;
+  cudaError_t e = cudaMemcpyAsync(s->vmom + s->v_off[i], src->data, bytes, cudaMemcpyDeviceToDevice,
+                                  static_cast<cudaStream_t>(cuda_stream));
+  if (e != cudaSuccess) return cuda_fail(e, "second-moment copy");
   return LM_OK;
 }
 
@@ -894,10 +1039,10 @@ lm_status lm_probe_bounded_wait(uint64_t limit_ns, uint32_t* device_flags, void*
                                : LM_OK;
 }
 
-size_t lm_state_bytes(const lm_state* s) { return s ? s->mom_elems * sizeof(float) : 0; }
+size_t lm_state_bytes(const lm_state* s) { return s ? (s->mom_elems + s->v_elems) * sizeof(float) : 0; }
 
 size_t lm_workspace_bytes(const lm_state* s) {
-  return s ? s->bytes - s->mom_elems * sizeof(float) : 0;
+  return s ? s->bytes - (s->mom_elems + s->v_elems) * sizeof(float) : 0;
 }
 
 void lm_destroy(lm_state* s) {

@@ -141,6 +141,42 @@ __global__ void __launch_bounds__(kLionThreads)
 }
 
 // ---------------------------------------------------------------------------
+// AdamW for 1-D parameters (Section 3's fallback for biases and norm gains).
+// The same fixed operation order as the float32 reference: every product,
+// sum, square root and quotient rounded once (IEEE __fsqrt_rn / __fdiv_rn).
+// 1-D parameters are a small share of any set (0.02% of the 720M-shaped one),
+// so the kernel streams one element per thread per trip.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void adamw_elem(float& w, float& m, float& v, float g, const AdamConsts& k) {
+  m = __fadd_rn(__fmul_rn(k.b1, m), __fmul_rn(k.c1, g));
+  v = __fadd_rn(__fmul_rn(k.b2, v), __fmul_rn(k.c2, __fmul_rn(g, g)));
+  w = __fsub_rn(w, __fmul_rn(k.lrwd, w));
+  const float den = __fadd_rn(__fmul_rn(__fsqrt_rn(v), k.rbc2), k.eps);
+  w = __fsub_rn(w, __fmul_rn(k.step, __fdiv_rn(m, den)));
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kLionThreads)
+    adamw_kernel(const AdamTensor* __restrict__ tensors, const LionChunk* __restrict__ chunks, int nchunks,
+                 const void* const* __restrict__ grads, AdamConsts k) {
+  for (int c = blockIdx.x; c < nchunks; c += gridDim.x) {
+    const LionChunk ch = chunks[c];
+    const AdamTensor t = tensors[ch.tensor];
+    T* w = static_cast<T*>(t.w) + ch.begin;
+    const T* g = static_cast<const T*>(grads[t.grad_slot]) + ch.begin;
+    float* m = t.m + ch.begin;
+    float* v = t.v + ch.begin;
+    for (int64_t e = threadIdx.x; e < ch.count; e += kLionThreads) {
+      float wf = to_f(w[e]), mf = m[e], vf = v[e];
+      adamw_elem(wf, mf, vf, to_f(g[e]), k);
+      w[e] = from_f<T>(wf);
+      m[e] = mf;
+      v[e] = vf;
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
 // Muon: momentum + Frobenius norm + X0, and finalize.  X keeps the
 // parameter's orientation (row pitch ldx), so both kernels stream element
 // ranges of a matrix: element e = r * cols + c of W, G, M is element
@@ -354,6 +390,21 @@ cudaError_t launch_lion(lm_dtype dt, const LionTensor* tensors, const LionChunk*
     lion_kernel<__nv_bfloat16><<<grid, kLionThreads, 0, st>>>(tensors, chunks, nchunks, grads, k);
   else
     lion_kernel<float><<<grid, kLionThreads, 0, st>>>(tensors, chunks, nchunks, grads, k);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_adamw(lm_dtype dt, const AdamTensor* tensors, const LionChunk* chunks, int nchunks,
+                         const void* const* grads, AdamConsts k, cudaStream_t st) {
+  if (nchunks <= 0) return cudaSuccess;
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int grid = nchunks < 4 * sms ? nchunks : 4 * sms;
+  count_launch();
+  if (dt == LM_BF16)
+    adamw_kernel<__nv_bfloat16><<<grid, kLionThreads, 0, st>>>(tensors, chunks, nchunks, grads, k);
+  else
+    adamw_kernel<float><<<grid, kLionThreads, 0, st>>>(tensors, chunks, nchunks, grads, k);
   return cudaGetLastError();
 }
 

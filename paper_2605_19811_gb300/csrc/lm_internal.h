@@ -32,6 +32,24 @@ struct LionConsts {
   float b1, c1, b2, c2, eL, lam;
 };
 
+// AdamW on 1-D parameters (the LM_VECTOR_ADAMW rule): parameter, first
+// moment (the momentum buffer), second moment, chunked like the Lion tables.
+struct AdamTensor {
+  void* w;
+  float* m;
+  float* v;
+  int64_t n;
+  int32_t grad_slot;
+  int32_t pad;
+};
+// float32 constants of one step: b1, 1-b1, b2, 1-b2, lr/(1-b1^k),
+// 1/sqrt(1-b2^k), lr*wd, eps (k = t + 1), each rounded once from double.
+struct AdamConsts {
+  float b1, c1, b2, c2, step, rbc2, lrwd, eps;
+};
+cudaError_t launch_adamw(lm_dtype dt, const AdamTensor* tensors, const LionChunk* chunks, int nchunks,
+                         const void* const* grads, AdamConsts k, cudaStream_t st);
+
 // Launch the Lion kernel over a chunk table whose tensors all have dtype dt.
 cudaError_t launch_lion(lm_dtype dt, const LionTensor* tensors, const LionChunk* chunks,
                         int nchunks, const void* const* grads, LionConsts k,

@@ -27,9 +27,11 @@ EXPORTED = ("lm_config_default", "lm_create", "lm_step", "lm_set_lr", "lm_msign_
             "lm_get_momentum", "lm_set_momentum", "lm_get_status", "lm_state_bytes",
             "lm_workspace_bytes", "lm_destroy", "lm_status_string", "lm_last_error",
             "lm_kernel_launch_count", "lm_profile_enable", "lm_profile_read",
-            "lm_msign_ns_noalloc", "lm_probe_bounded_wait", "lm_msign_ns_coeffs")
+            "lm_msign_ns_noalloc", "lm_probe_bounded_wait", "lm_msign_ns_coeffs",
+            "lm_set_adamw_lr", "lm_get_second_moment", "lm_set_second_moment")
 
-KERNEL_FAMILIES = ("lion", "momentum_norm", "ns_gram", "ns_poly", "ns_apply", "finalize", "other")
+KERNEL_FAMILIES = ("lion", "momentum_norm", "ns_gram", "ns_poly", "ns_apply", "finalize", "other", "adamw")
+LM_VECTOR_LION, LM_VECTOR_ADAMW = 0, 1
 
 
 class LmTensor(ctypes.Structure):
@@ -44,11 +46,14 @@ class LmConfig(ctypes.Structure):
                 ("ns_steps", ctypes.c_int), ("ns_a", ctypes.c_double), ("ns_b", ctypes.c_double),
                 ("ns_c", ctypes.c_double), ("ns_eps", ctypes.c_double),
                 ("shape_scale", ctypes.c_double), ("ns_precision", ctypes.c_int),
-                ("ns_coeffs", ctypes.POINTER(ctypes.c_double))]
+                ("ns_coeffs", ctypes.POINTER(ctypes.c_double)),
+                ("vector_rule", ctypes.c_int), ("adamw_lr", ctypes.c_double),
+                ("adamw_beta1", ctypes.c_double), ("adamw_beta2", ctypes.c_double),
+                ("adamw_eps", ctypes.c_double), ("adamw_weight_decay", ctypes.c_double)]
 
 
 class LmProfile(ctypes.Structure):
-    _fields_ = [("ms", ctypes.c_double * 7), ("launches", ctypes.c_uint64 * 7)]
+    _fields_ = [("ms", ctypes.c_double * 8), ("launches", ctypes.c_uint64 * 8)]
 
 
 class LionMuonError(RuntimeError):
@@ -89,6 +94,12 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib.lm_msign_ns_noalloc.argtypes = [P(LmTensor), P(LmTensor), c_int, c_double, c_double, c_double,
                                         c_double, c_int, c_void_p]
     lib.lm_msign_ns_noalloc.restype = c_int
+    lib.lm_set_adamw_lr.argtypes = [c_void_p, c_double]
+    lib.lm_set_adamw_lr.restype = c_int
+    lib.lm_get_second_moment.argtypes = [c_void_p, c_int, P(LmTensor)]
+    lib.lm_get_second_moment.restype = c_int
+    lib.lm_set_second_moment.argtypes = [c_void_p, c_int, P(LmTensor), c_void_p]
+    lib.lm_set_second_moment.restype = c_int
     lib.lm_get_momentum.argtypes = [c_void_p, c_int, P(LmTensor)]
     lib.lm_get_momentum.restype = c_int
     lib.lm_set_momentum.argtypes = [c_void_p, c_int, P(LmTensor), c_void_p]
@@ -215,6 +226,22 @@ class LionMuon:
         _check(self._lib, self._lib.lm_get_momentum(self._h, i, ctypes.byref(v)), "lm_get_momentum")
         shape = tuple(self.params[i].shape)
         return torch.as_tensor(_DeviceArray(v.data, shape, "<f4"), device=self.params[i].device)
+
+    def set_adamw_lr(self, lr: float) -> None:
+        _check(self._lib, self._lib.lm_set_adamw_lr(self._h, lr), "lm_set_adamw_lr")
+
+    def second_moment(self, i: int):
+        """Read-only torch view of 1-D parameter i's AdamW second moment."""
+        import torch
+        v = LmTensor()
+        _check(self._lib, self._lib.lm_get_second_moment(self._h, i, ctypes.byref(v)), "lm_get_second_moment")
+        shape = tuple(self.params[i].shape)
+        return torch.as_tensor(_DeviceArray(v.data, shape, "<f4"), device=self.params[i].device)
+
+    def set_second_moment(self, i: int, src, stream=None) -> None:
+        d = tensor_desc(src)
+        _check(self._lib, self._lib.lm_set_second_moment(self._h, i, ctypes.byref(d), _stream_handle(stream)),
+               "lm_set_second_moment")
 
     def set_momentum(self, i: int, src, stream=None) -> None:
         d = tensor_desc(src)
