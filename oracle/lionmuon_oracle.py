@@ -36,6 +36,10 @@ Readings taken where the paper is silent (each listed in the design doc):
   Table 5's 1-D learning rate 1e-3 and AdamW betas (0.8, 0.999), weight decay
   0.1 (Table 5's), eps 1e-8, bias correction with the update count t + 1.
 * P = infinity is encoded as ``period = 0``.
+* The adaptive schedule of Appendix G decides on M_{t-1}, the buffer at hand
+  when the step starts; its power iteration starts from a SplitMix64 vector
+  (seed a parameter), makes ``srank_iters`` passes (5 by default: "a few"),
+  and a zero buffer takes Muon.
 * Iteration-dependent NS coefficients (the minimax / Chebyshev-type msign
   iterations of Section 2) keep the Frobenius normalisation, so the first
   interval of singular values is [l_0, 1] with l_0 a parameter; the minimax
@@ -88,6 +92,13 @@ class Config:
     # "adamw" (Section 3's fallback for biases and norm gains, with Table 5's
     # 1-D learning rate 1e-3 and AdamW betas (0.8, 0.999)).
     vector_rule: str = "lion"
+    # Muon/Lion selection for matrices: "period" (Algorithm 1, t mod P) or
+    # "stable_rank" (Appendix G): Muon where the stable rank of M_{t-1},
+    # ||M||_F^2 / sigma_1_hat^2, is at most alpha * min(m, n).
+    schedule: str = "period"
+    srank_alpha: float = 0.01
+    srank_iters: int = 5        # passes over M of the power iteration
+    srank_seed: int = 0         # SplitMix64 seed of the start vector
     adamw_lr: float = 1e-3
     adamw_beta1: float = 0.8
     adamw_beta2: float = 0.999
@@ -340,25 +351,96 @@ def adamw_update(W, G, m_prev, v_prev, step: int, lr, beta1, beta2, eps, weight_
     return W_new, m, v
 
 
+# ---------------------------------------------------------------------------
+# Adaptive Muon/Lion selection (Appendix G)
+# ---------------------------------------------------------------------------
+
+_U64 = (1 << 64) - 1
+_GOLDEN = 0x9E3779B97F4A7C15
+
+
+def splitmix64(seed: int, count: int) -> List[int]:
+    """The first ``count`` outputs of SplitMix64 (Steele, Lea and Flood,
+    2014) started from ``seed``: the state advances by 0x9E3779B97F4A7C15 and
+    each output is the state passed through the two xor-shift-multiply
+    rounds (multipliers 0xBF58476D1CE4E5B9, 0x94D049BB133111EB) and a final
+    xor-shift by 31.  Output j depends only on seed + (j + 1) * golden, so it
+    is a counter-based generator."""
+    out = []
+    state = seed & _U64
+    for _ in range(count):
+        state = (state + _GOLDEN) & _U64
+        z = state
+        z = ((z ^ (z >> 30)) * 0xBF58476D1CE4E5B9) & _U64
+        z = ((z ^ (z >> 27)) * 0x94D049BB133111EB) & _U64
+        out.append(z ^ (z >> 31))
+    return out
+
+
+def power_start_vector(n: int, seed: int) -> np.ndarray:
+    """Start vector of the power iteration (the paper leaves it open):
+    entry j = 2 * (top 53 bits of SplitMix64 output j) / 2^53 - 1, in [-1, 1)."""
+    return np.array([2.0 * ((z >> 11) * 2.0 ** -53) - 1.0 for z in splitmix64(seed, n)], dtype=np.float64)
+
+
+def stable_rank_estimate(M: np.ndarray, iters: int, v0: np.ndarray):
+    """||M||_F^2 and the power-iteration estimate of sigma_1(M)^2 (Appendix G:
+    sigma_1 "approximated by a few power-iteration steps").  With
+    v = v0 / ||v0||, each of the ``iters`` passes forms u = M v and takes
+    ||u||^2 as the estimate; every pass but the last also forms w = M^T u and
+    v = w / ||w||.  So the estimate is the Rayleigh quotient of M^T M at
+    (M^T M)^(iters-1) v0, never above sigma_1^2.  Returns (fro2, sigma2)."""
+    M = np.asarray(M, dtype=np.float64)
+    fro2 = float(np.sum(M * M))
+    v = np.asarray(v0, dtype=np.float64)
+    v = v / np.linalg.norm(v)
+    sigma2 = 0.0
+    for k in range(iters):
+        u = M @ v
+        sigma2 = float(u @ u)
+        if k + 1 < iters:
+            w = M.T @ u
+            nw = np.linalg.norm(w)
+            if nw == 0.0:
+                break
+            v = w / nw
+    return fro2, sigma2
+
+
+def srank_takes_muon(M_prev: np.ndarray, cfg: "Config") -> bool:
+    """Appendix G's rule on the momentum buffer M_{t-1}: Muon iff the stable
+    rank estimate ||M||_F^2 / sigma_1_hat^2 <= alpha * min(m, n), decided as
+    ||M||_F^2 <= alpha * min(m, n) * sigma_1_hat^2.  A zero buffer (t = 0)
+    takes Muon, as step 0 does under the fixed period."""
+    m, n = np.shape(M_prev)
+    fro2, sigma2 = stable_rank_estimate(M_prev, cfg.srank_iters, power_start_vector(n, cfg.srank_seed))
+    if fro2 == 0.0:
+        return True
+    return fro2 <= cfg.srank_alpha * min(m, n) * sigma2
+
+
 def is_matrix(shape: Sequence[int]) -> bool:
     """A parameter is a hidden matrix (takes Muon steps) unless it is a vector
     (one of its two dimensions is 1)."""
     return len(shape) == 2 and shape[0] > 1 and shape[1] > 1
 
 
-def lionmuon_param_step(W, G, M_prev, t: int, cfg: Config, sign_in_f32: bool = False):
+def lionmuon_param_step(W, G, M_prev, t: int, cfg: Config, sign_in_f32: bool = False,
+                        take_muon: Optional[bool] = None):
     """One iteration of Algorithm 1 for one parameter, fp64.
 
     With ``sign_in_f32`` the Lion branch decides sign(G_hat) on the float32
     value of G_hat formed as fl(fl(b1*M) + fl(c1*G)) with float32 constants
     (the order the CUDA library uses), so both sides take the same integer
     decision near ties; the update itself stays fp64.
+    ``take_muon`` overrides the branch of a matrix (the adaptive schedule).
     Returns (W_{t+1}, M_t)."""
     W = np.asarray(W, dtype=np.float64)
     G = np.asarray(G, dtype=np.float64)
     M_prev = np.asarray(M_prev, dtype=np.float64)
     G_hat = interpolated_direction(M_prev, G, cfg.beta1)
-    if is_matrix(W.shape) and is_muon_step(t, cfg.period):
+    muon = is_muon_step(t, cfg.period) if take_muon is None else take_muon
+    if is_matrix(W.shape) and muon:
         W_new = muon_update(W, G_hat, cfg)
     else:
         direction = G_hat
@@ -420,6 +502,8 @@ def lionmuon_step(params: List[np.ndarray], grads: List[np.ndarray],
         raise ValueError("vector_rule must be 'lion' or 'adamw'")
     if adamw and seconds is None:
         raise ValueError("the AdamW rule needs the second moments")
+    if cfg.schedule not in ("period", "stable_rank"):
+        raise ValueError("schedule must be 'period' or 'stable_rank'")
     new_p, new_m, new_v = [], [], []
     for i, (W, G, M) in enumerate(zip(params, grads, moms)):
         if np.shape(W) != np.shape(G) or np.shape(W) != np.shape(M):
@@ -429,7 +513,11 @@ def lionmuon_step(params: List[np.ndarray], grads: List[np.ndarray],
             W1, M1, V1 = adamw_update(W, G, M, seconds[i], t + 1, cfg.adamw_lr, cfg.adamw_beta1,
                                       cfg.adamw_beta2, cfg.adamw_eps, cfg.adamw_weight_decay)
         else:
-            W1, M1 = lionmuon_param_step(W, G, M, t, cfg, sign_in_f32=param_dtypes is not None)
+            take = None
+            if cfg.schedule == "stable_rank" and is_matrix(np.shape(W)):
+                take = srank_takes_muon(M, cfg)
+            W1, M1 = lionmuon_param_step(W, G, M, t, cfg, sign_in_f32=param_dtypes is not None,
+                                         take_muon=take)
         if param_dtypes is not None:
             W1 = round_to_storage(W1, param_dtypes[i])
             M1 = round_to_storage(M1, "f32")

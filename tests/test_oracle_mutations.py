@@ -13,6 +13,7 @@ import oracle.lionmuon_oracle as OM
 from tests import test_oracle_pins as pins
 from tests import test_oracle_pins_msign_variants as vpins
 from tests import test_oracle_pins_adamw as apins
+from tests import test_oracle_pins_srank as spins
 
 # every pin, with representative arguments for the parametrised ones
 PIN_CALLS = [
@@ -51,6 +52,12 @@ PIN_CALLS = [
     (apins.test_adamw_constant_gradient_closed_form, ()),
     (apins.test_adamw_zero_gradient_is_pure_decay, ()),
     (apins.test_adamw_first_step_is_sign_like, ()),
+    (spins.test_splitmix64_published_outputs, ()),
+    (spins.test_power_estimate_closed_form_on_known_svd, (3,)),
+    (spins.test_exact_stable_ranks, ()),
+    (spins.test_threshold_and_zero_buffer, ()),
+    (spins.test_step_routes_matrices_by_stable_rank, ()),
+    (spins.test_decision_uses_the_buffer_before_the_update, ()),
 ]
 
 
@@ -104,6 +111,10 @@ def _mutations():
     muts["adamw_coupled_decay"] = [("adamw_update", _adamw_variant("coupled"))]
     muts["adamw_eps_inside_sqrt"] = [("adamw_update", _adamw_variant("eps_in_sqrt"))]
     muts["adamw_beta_swap"] = [("adamw_update", _adamw_variant("swap"))]
+    muts["srank_threshold_max_dim"] = [("srank_takes_muon", _srank_max_dim)]
+    muts["srank_estimate_from_w"] = [("stable_rank_estimate", _srank_estimate_w)]
+    muts["srank_post_update_buffer"] = [("lionmuon_step", _srank_post_update_step)]
+    muts["splitmix_shift_29"] = [("splitmix64", _splitmix_shift29)]
     return muts
 
 
@@ -151,12 +162,13 @@ def _schedule_fixed_interval(steps, lo, degree=5, safety=1.0):
     return (tr,) * steps
 
 
-def _post_update_step(W, G, M_prev, t, cfg, sign_in_f32=False):
+def _post_update_step(W, G, M_prev, t, cfg, sign_in_f32=False, take_muon=None):
     W = np.asarray(W, dtype=np.float64)
     G = np.asarray(G, dtype=np.float64)
     M_new = OM.momentum_update(np.asarray(M_prev, dtype=np.float64), G, cfg.beta2)
     G_hat = OM.interpolated_direction(M_new, G, cfg.beta1)
-    if OM.is_matrix(W.shape) and OM.is_muon_step(t, cfg.period):
+    muon = OM.is_muon_step(t, cfg.period) if take_muon is None else take_muon
+    if OM.is_matrix(W.shape) and muon:
         return OM.muon_update(W, G_hat, cfg), M_new
     return OM.lion_update(W, G_hat, cfg.eta_lion, cfg.weight_decay), M_new
 
@@ -186,6 +198,44 @@ def _adamw_variant(kind):
         decay = 0.0 if kind == "coupled" else lr * weight_decay * W
         return W - decay - lr * (m / bc1) / den, m, v
     return f
+
+
+def _srank_max_dim(M_prev, cfg):
+    m, n = np.shape(M_prev)
+    fro2, sig2 = OM.stable_rank_estimate(M_prev, cfg.srank_iters, OM.power_start_vector(n, cfg.srank_seed))
+    return fro2 == 0.0 or fro2 <= cfg.srank_alpha * max(m, n) * sig2
+
+
+def _srank_estimate_w(M, iters, v0):
+    M = np.asarray(M, dtype=np.float64)
+    v = v0 / np.linalg.norm(v0)
+    sig2 = 0.0
+    for _ in range(iters):
+        w = M.T @ (M @ v)
+        sig2 = float(np.linalg.norm(w))
+        v = w / np.linalg.norm(w)
+    return float(np.sum(M * M)), sig2
+
+
+def _srank_post_update_step(params, grads, moms, t, cfg, param_dtypes=None, seconds=None):
+    new_p, new_m = [], []
+    for W, G, M in zip(params, grads, moms):
+        M1 = OM.momentum_update(np.asarray(M, dtype=np.float64), np.asarray(G, dtype=np.float64), cfg.beta2)
+        take = OM.srank_takes_muon(M1, cfg) if OM.is_matrix(np.shape(W)) else None
+        W1, M1 = OM.lionmuon_param_step(W, G, M, t, cfg, take_muon=take)
+        new_p.append(W1)
+        new_m.append(M1)
+    return new_p, new_m
+
+
+def _splitmix_shift29(seed, count):
+    out, st, U = [], seed, (1 << 64) - 1
+    for _ in range(count):
+        st = (st + 0x9E3779B97F4A7C15) & U
+        z = ((st ^ (st >> 29)) * 0xBF58476D1CE4E5B9) & U
+        z = ((z ^ (z >> 27)) * 0x94D049BB133111EB) & U
+        out.append(z ^ (z >> 31))
+    return out
 
 
 def _storage_ns_unrounded_B(G, coeffs, eps=1e-7, storage="bf16"):
