@@ -46,6 +46,10 @@ def parse_args():
     ap.add_argument("--set", default="gpt_720m")
     ap.add_argument("--period", type=int, default=2)
     ap.add_argument("--precision", choices=["bf16", "f32"], default="bf16")
+    ap.add_argument("--schedule", choices=["period", "srank"], default="period",
+                    help="period: Algorithm 1's fixed P; srank: Appendix G's stable-rank selection")
+    ap.add_argument("--srank-alpha", type=float, default=0.01)
+    ap.add_argument("--srank-iters", type=int, default=5)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     return ap.parse_args()
@@ -309,7 +313,12 @@ def run_ours(args):
     torch.cuda.synchronize()
 
     prec = L.LM_BF16 if args.precision == "bf16" else L.LM_F32
-    opt = L.LionMuon(params, period=P, ns_precision=prec)
+    srank = args.schedule == "srank"
+    if srank:
+        opt = L.LionMuon(params, period=P, ns_precision=prec, schedule=L.LM_SCHEDULE_STABLE_RANK,
+                         srank_alpha=args.srank_alpha, srank_iters=args.srank_iters)
+    else:
+        opt = L.LionMuon(params, period=P, ns_precision=prec)
     n = len(params)
     gdesc = (L.LmTensor * n)(*[L.tensor_desc(g) for g in grads])
     stream = torch.cuda.current_stream()
@@ -323,7 +332,7 @@ def run_ours(args):
     for _ in range(args.warmup):
         opt.step_descs(gdesc, n, t, sh)
         t += 1
-    base = ((t + P - 1) // P) * P if P > 0 else t
+    base = ((t + P - 1) // P) * P if P > 0 and not srank else t
     torch.cuda.synchronize()
     barrier()
 
@@ -371,10 +380,11 @@ def run_ours(args):
                "what": "pinned-host gradients copied in, lm_step, updated parameters copied out, per step"}
     clk = clocks.stop()
     flags = opt.status()
+    took_last = opt.selection()[0] if srank else None
 
     # ---- roofline of the dominant kernel family ----
     peaks, peak_src = load_peaks()
-    n_muon = sum(1 for i in range(args.steps) if P > 0 and (base + i) % P == 0)
+    n_muon = 0 if srank else sum(1 for i in range(args.steps) if P > 0 and (base + i) % P == 0)
     n_lion = args.steps - n_muon
     ns_ms, ns_launches = prof["ns_gemm"]
     lion_ms, lion_launches = prof["lion"]
@@ -401,6 +411,16 @@ def run_ours(args):
                      "traffic": kernel_traffic("lion_kernel"), "kernel": "lion_kernel",
                      "per_launch_ms": lion_ms / max(lion_launches, 1),
                      "frac_of_8tbs": gbs / 8000.0, "peak_kind": f"HBM copy, {peak_src}"}
+    srank_roof = None
+    if srank and prof["srank"][0] > 0:
+        # every pass reads each fp32 momentum matrix once: 4 B per matrix element
+        sr_ms = prof["srank"][0]
+        gbs = 4.0 * mat_elems * args.srank_iters * args.steps / (sr_ms / 1e3) / 1e9
+        pk = peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
+        srank_roof = {"bound": "hbm", "achieved": gbs, "peak": pk, "unit": "GB/s", "frac": gbs / pk,
+                      "traffic": None, "kernel": "srank_pass_kernel",
+                      "per_step_ms": sr_ms / args.steps, "peak_kind": f"HBM copy, {peak_src}",
+                      "bytes": "4 B x matrix elements x passes (plus resets and the decision)"}
     fam_ms = {k: v[0] / args.steps for k, v in prof.items() if k != "ns_gemm"}
 
     cpu = None
@@ -418,11 +438,17 @@ def run_ours(args):
             "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
             "dtype": "bf16" if args.precision == "bf16" else "f32", "data": "synthetic",
             "config": {"workload": args.set, "params": numel, "matrices": len(mats),
-                       "period": P, "ns_steps": 5, "ns_precision": args.precision,
+                       "period": None if srank else P, "ns_steps": 5, "ns_precision": args.precision,
+                       **({"schedule": "stable_rank", "srank_alpha": args.srank_alpha,
+                           "srank_iters": args.srank_iters,
+                           "muon_matrices_last_step": sum(1 for i, s in enumerate(shapes)
+                                                          if len(s) == 2 and took_last[i])} if srank else {}),
                        "grads": f"{ps.grad_kind}, drawn on device, same gradients every step",
                        "l2": "inputs larger than L2 (14 B/param x %.0f M params streamed per Lion step)" % (numel / 1e6),
-                       "timed_steps": f"t = {base} .. {base + args.steps - 1} (whole periods from a Muon step)"},
-            "roofline": roof, "roofline_lion": lion_roof,
+                       "timed_steps": f"t = {base} .. {base + args.steps - 1}" +
+                                      ("" if srank else " (whole periods from a Muon step)")},
+            "roofline": srank_roof if srank else roof, "roofline_lion": lion_roof,
+            **({"roofline_ns": roof} if srank else {}),
             "kernel_ms_per_step": fam_ms,
             "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches, "clocks": clk,
             "device_flags": flags,

@@ -100,7 +100,25 @@ typedef struct {
    * 0.8, 0.999), adamw_eps > 0 (1e-8), adamw_weight_decay >= 0 (0.1). */
   int vector_rule;
   double adamw_lr, adamw_beta1, adamw_beta2, adamw_eps, adamw_weight_decay;
+  /* Choice between the Muon and Lion step for matrices: LM_SCHEDULE_PERIOD
+   * (Algorithm 1: Muon iff t mod period == 0, the default) or
+   * LM_SCHEDULE_STABLE_RANK, the adaptive rule of Appendix G: on every step
+   * a matrix takes the Muon step iff the stable rank of its momentum buffer
+   * M_{t-1}, ||M||_F^2 / sigma_1_hat^2, is at most srank_alpha * min(m, n)
+   * (a zero buffer takes Muon); sigma_1_hat^2 is the Rayleigh quotient of
+   * M^T M after srank_iters - 1 power-iteration steps from a SplitMix64
+   * start vector (seed srank_seed), srank_iters reads of M in all.
+   * srank_alpha > 0 (Appendix G sweeps 0.002 .. 0.01; default 0.01),
+   * srank_iters in [1, 64] (default 5); period is then ignored, and matrices
+   * may have at most 16384 columns. */
+  int schedule;
+  double srank_alpha;
+  int srank_iters;
+  uint64_t srank_seed;
 } lm_config;
+
+#define LM_SCHEDULE_PERIOD 0
+#define LM_SCHEDULE_STABLE_RANK 1
 
 #define LM_VECTOR_LION 0
 #define LM_VECTOR_ADAMW 1
@@ -136,6 +154,16 @@ lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t,
 /* Change the two learning rates (a caller-driven schedule); takes effect for
  * the next lm_step.  Errors: LM_ERR_INVALID_ARG (NULL, negative, non-finite). */
 lm_status lm_set_lr(lm_state* s, double eta_muon, double eta_lion);
+
+/* The branch each parameter took in the last lm_step, and under
+ * LM_SCHEDULE_STABLE_RANK the stable-rank estimate behind it (Appendix G).
+ * took_muon (n entries, or NULL): 1 where parameter i took the Muon step.
+ * srank (n entries, or NULL): ||M_{t-1}||_F^2 / sigma_1_hat^2 of matrix i
+ * (0 for a zero buffer), NaN for 1-D parameters and under the fixed period.
+ * Host memory; synchronises the state's last stream.  Errors:
+ * LM_ERR_INVALID_ARG (NULL state, n differs from the parameter count, no
+ * step taken yet), LM_ERR_CUDA. */
+lm_status lm_get_selection(lm_state* s, int n, unsigned char* took_muon, double* srank);
 
 /* Change the AdamW learning rate of 1-D parameters (LM_VECTOR_ADAMW); takes
  * effect for the next lm_step.  Errors: LM_ERR_INVALID_ARG (NULL, negative,
@@ -257,7 +285,8 @@ typedef enum {
   LM_KERNEL_FINALIZE = 5,      /* Muon: parameter write */
   LM_KERNEL_OTHER = 6,         /* gradient-pointer upload, norm reset */
   LM_KERNEL_ADAMW = 7,         /* AdamW on 1-D parameters (LM_VECTOR_ADAMW) */
-  LM_KERNEL_FAMILIES = 8
+  LM_KERNEL_SRANK = 8,         /* stable-rank selection: power iteration, decision */
+  LM_KERNEL_FAMILIES = 9
 } lm_kernel_family;
 
 typedef struct {

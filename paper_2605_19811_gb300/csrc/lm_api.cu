@@ -8,8 +8,10 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <limits>
 #include <map>
 #include <string>
+#include <tuple>
 #include <vector>
 
 #include "lm_internal.h"
@@ -79,6 +81,12 @@ lm_status check_config(const lm_config* c) {
   if (!finite(c->shape_scale) || c->shape_scale < 0) return fail(LM_ERR_INVALID_ARG, "shape_scale must be >= 0");
   if (c->ns_precision != LM_BF16 && c->ns_precision != LM_F32)
     return fail(LM_ERR_INVALID_ARG, "ns_precision must be LM_BF16 or LM_F32");
+  if (c->schedule != LM_SCHEDULE_PERIOD && c->schedule != LM_SCHEDULE_STABLE_RANK)
+    return fail(LM_ERR_INVALID_ARG, "schedule must be LM_SCHEDULE_PERIOD or LM_SCHEDULE_STABLE_RANK");
+  if (c->schedule == LM_SCHEDULE_STABLE_RANK) {
+    if (!finite(c->srank_alpha) || !(c->srank_alpha > 0)) return fail(LM_ERR_INVALID_ARG, "srank_alpha must be > 0");
+    if (c->srank_iters < 1 || c->srank_iters > 64) return fail(LM_ERR_INVALID_ARG, "srank_iters must be in [1, 64]");
+  }
   if (c->vector_rule != LM_VECTOR_LION && c->vector_rule != LM_VECTOR_ADAMW)
     return fail(LM_ERR_INVALID_ARG, "vector_rule must be LM_VECTOR_LION or LM_VECTOR_ADAMW");
   if (c->vector_rule == LM_VECTOR_ADAMW) {
@@ -113,6 +121,7 @@ LionConsts lion_consts(const lm_config& c) {
   k.c2 = (float)(1.0 - c.beta2);
   k.eL = (float)c.eta_lion;
   k.lam = (float)c.weight_decay;
+  k.skip = nullptr;
   return k;
 }
 // AdamW constants of step t (update number t + 1): powers and the square
@@ -143,6 +152,7 @@ MuonConsts muon_consts(const lm_config& c) {
   k.lam = (float)c.weight_decay;
   k.eps = (float)c.ns_eps;
   k.ns_steps = c.ns_steps;
+  k.active = nullptr;
   return k;
 }
 
@@ -461,7 +471,8 @@ static std::vector<NsCoeffs> ns_schedule(int steps, const double* table, double 
 }
 
 static lm_status run_ns(const NsEngine& E, int steps, const NsCoeffs* coeffs, unsigned* flags, cudaStream_t st,
-                        Profiler* P = nullptr, const FuseFinal* fuse = nullptr) {
+                        Profiler* P = nullptr, const FuseFinal* fuse = nullptr,
+                        const unsigned char* active = nullptr) {
   for (int it = 0; it < steps; ++it)
     for (const NsBatch& b : E.batches)
       for (int ph = 0; ph < 3; ++ph) {
@@ -470,9 +481,9 @@ static lm_status run_ns(const NsEngine& E, int steps, const NsCoeffs* coeffs, un
           if (E.xdt == LM_BF16)
             return launch_ns_tc((NsPhase)ph, it, b.ng, E.groups.data() + b.g0, E.maps.data() + b.g0,
                                 b.tiles[ph], b.ntiles[ph], b.offsets[ph], b.npairs[ph], E.d_norm2, co,
-                                flags, it == steps - 1 ? fuse : nullptr, st);
+                                flags, it == steps - 1 ? fuse : nullptr, st, active);
           return launch_ns_simt((NsPhase)ph, it, b.ng, E.d_groups + b.g0, b.tiles[ph], b.ntiles[ph],
-                                E.d_norm2, co, st);
+                                E.d_norm2, co, st, active);
         });
         if (e != cudaSuccess) return cuda_fail(e, "Newton-Schulz launch");
       }
@@ -505,6 +516,26 @@ struct lm_state {
   float* vmom = nullptr;                // AdamW second moments
   std::vector<int64_t> v_off;           // element offset per parameter, -1 if none
   size_t v_elems = 0;
+  // stable-rank selection (LM_SCHEDULE_STABLE_RANK)
+  struct SrLaunch {
+    int slots = 0, threads = 0;
+    bool vec4 = false;                  // rows are 16-byte multiples: the ring kernel
+    int64_t max_cols = 0;
+    SrItem* items = nullptr;
+    int nitems = 0;
+  };
+  bool srank = false;
+  SrMat* d_sr = nullptr;                // per matrix id
+  std::vector<SrLaunch> sr_launch;
+  float* sr_wa = nullptr;
+  float* sr_wb = nullptr;
+  size_t sr_w_elems = 0;                // floats in each of wa, wb
+  double* sr_acc = nullptr;             // nmat x (1 + srank_iters)
+  unsigned char* d_active = nullptr;    // per matrix id: takes Muon this step
+  unsigned char* d_skip = nullptr;      // per parameter: Lion kernel skips it
+  double* d_srank = nullptr;            // per matrix id: the estimate
+  std::vector<int> mat_param_of;        // matrix id -> parameter index
+  int64_t last_t = -1;
   int lion_grid[2] = {0, 0};
   int nmat = 0;
   MatDesc* d_mats = nullptr;
@@ -542,6 +573,10 @@ void lm_config_default(lm_config* c) {
   c->adamw_beta2 = 0.999;
   c->adamw_eps = 1e-8;
   c->adamw_weight_decay = 0.1;
+  c->schedule = LM_SCHEDULE_PERIOD;
+  c->srank_alpha = 0.01;
+  c->srank_iters = 5;
+  c->srank_seed = 0;
 }
 
 const char* lm_status_string(lm_status st) {
@@ -687,6 +722,72 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
   build_elem_chunks(mats, echunks_all);
   const size_t off_echunks = ar.add(echunks_all.size() * sizeof(ElemChunk));
 
+  // stable-rank selection: vectors v0 / wa / wb per matrix, accumulators,
+  // masks and the work items of each launch shape
+  s->srank = cfg->schedule == LM_SCHEDULE_STABLE_RANK && s->nmat > 0;
+  s->mat_param_of.resize(s->nmat);
+  for (int id = 0; id < s->nmat; ++id) s->mat_param_of[id] = mat_param[mat_order[id]];
+  std::vector<size_t> sr_voff(s->nmat, 0);
+  std::vector<std::vector<SrItem>> sr_items;
+  size_t off_srv0 = 0, off_srwa = 0, off_srwb = 0, off_sracc = 0, off_srmat = 0, off_active = 0, off_skip = 0,
+         off_srank = 0;
+  std::vector<size_t> off_sritems;
+  if (s->srank) {
+    std::map<std::tuple<int, int, bool>, int> shape_launch;
+    for (int id = 0; id < s->nmat; ++id) {
+      const lm_tensor& p = params[s->mat_param_of[id]];
+      int threads = 0;
+      const int slots = srank_slots(p.cols, &threads);
+      if (slots == 0) {
+        delete s;
+        return fail(LM_ERR_UNSUPPORTED, "stable-rank schedule: matrix with %lld columns (at most 16384)",
+                    (long long)p.cols);
+      }
+      sr_voff[id] = s->sr_w_elems;
+      s->sr_w_elems = align_up(s->sr_w_elems + (size_t)p.cols, 64);
+      const auto key = std::make_tuple(slots, threads, p.cols % 4 == 0);
+      auto it = shape_launch.find(key);
+      if (it == shape_launch.end()) {
+        it = shape_launch.emplace(key, (int)s->sr_launch.size()).first;
+        lm_state::SrLaunch L0;
+        L0.slots = slots;
+        L0.threads = threads;
+        L0.vec4 = p.cols % 4 == 0;
+        s->sr_launch.push_back(L0);
+        sr_items.emplace_back();
+      }
+      s->sr_launch[it->second].max_cols = std::max<int64_t>(s->sr_launch[it->second].max_cols, p.cols);
+      sr_items[it->second].push_back(SrItem{id, 0, (int32_t)p.rows, 0});   // split below
+    }
+    // Work items: runs of rows, sized per launch so that each launch has
+    // about eight per block (blocks: two per SM); longer runs mean fewer
+    // atomic additions into the M^T u vectors.
+    int sms = 0, dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    for (auto& list : sr_items) {
+      int64_t total = 0;
+      for (const SrItem& whole : list) total += whole.nrows;
+      const int64_t per = std::max<int64_t>(kSrankRows,
+                                            std::min<int64_t>(8 * kSrankRows, total / (16 * std::max(sms, 1))));
+      const int64_t rows_per_item = per / 16 * 16;
+      std::vector<SrItem> split;
+      for (const SrItem& whole : list)
+        for (int64_t r = 0; r < whole.nrows; r += rows_per_item)
+          split.push_back(SrItem{whole.m, (int32_t)r, (int32_t)std::min<int64_t>(rows_per_item, whole.nrows - r), 0});
+      list.swap(split);
+    }
+    off_srv0 = ar.add(s->sr_w_elems * sizeof(float));
+    off_srwa = ar.add(s->sr_w_elems * sizeof(float));
+    off_srwb = ar.add(s->sr_w_elems * sizeof(float));
+    off_sracc = ar.add((size_t)s->nmat * (1 + cfg->srank_iters) * sizeof(double));
+    off_srmat = ar.add((size_t)s->nmat * sizeof(SrMat));
+    off_active = ar.add((size_t)s->nmat);
+    off_skip = ar.add((size_t)n);
+    off_srank = ar.add((size_t)s->nmat * sizeof(double));
+    for (auto& v : sr_items) off_sritems.push_back(ar.add(v.size() * sizeof(SrItem)));
+  }
+
   cudaError_t e = cudaMalloc(&s->base, ar.total);
   if (e != cudaSuccess) {
     delete s;
@@ -749,6 +850,48 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
     }
   }
   if (s->nmat) memcpy(img.data() + off_mats, mats.data(), mats.size() * sizeof(MatDesc));
+  if (s->srank) {
+    float* v0 = reinterpret_cast<float*>(base + off_srv0);
+    s->sr_wa = reinterpret_cast<float*>(base + off_srwa);
+    s->sr_wb = reinterpret_cast<float*>(base + off_srwb);
+    s->sr_acc = reinterpret_cast<double*>(base + off_sracc);
+    s->d_sr = reinterpret_cast<SrMat*>(base + off_srmat);
+    s->d_active = reinterpret_cast<unsigned char*>(base + off_active);
+    s->d_skip = reinterpret_cast<unsigned char*>(base + off_skip);
+    s->d_srank = reinterpret_cast<double*>(base + off_srank);
+    std::vector<SrMat> srm(s->nmat);
+    float* hv0 = reinterpret_cast<float*>(img.data() + off_srv0);
+    for (int id = 0; id < s->nmat; ++id) {
+      const int pi = s->mat_param_of[id];
+      const lm_tensor& p = params[pi];
+      // start vector: entry j = 2 * (top 53 bits of SplitMix64 output j) / 2^53 - 1
+      uint64_t state = cfg->srank_seed;
+      for (int64_t j = 0; j < p.cols; ++j) {
+        state += 0x9E3779B97F4A7C15ull;
+        uint64_t z = state;
+        z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+        z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+        z ^= z >> 31;
+        hv0[sr_voff[id] + j] = (float)(2.0 * ((double)(z >> 11) * 0x1.0p-53) - 1.0);
+      }
+      SrMat& d = srm[id];
+      d.M = s->mom + s->mom_off[pi];
+      d.v0 = v0 + sr_voff[id];
+      d.wa = s->sr_wa + sr_voff[id];
+      d.wb = s->sr_wb + sr_voff[id];
+      d.acc = s->sr_acc + (size_t)id * (1 + cfg->srank_iters);
+      d.rows = p.rows;
+      d.cols = p.cols;
+      d.mat = id;
+      d.param = pi;
+    }
+    memcpy(img.data() + off_srmat, srm.data(), srm.size() * sizeof(SrMat));
+    for (size_t k = 0; k < s->sr_launch.size(); ++k) {
+      memcpy(img.data() + off_sritems[k], sr_items[k].data(), sr_items[k].size() * sizeof(SrItem));
+      s->sr_launch[k].items = reinterpret_cast<SrItem*>(base + off_sritems[k]);
+      s->sr_launch[k].nitems = (int)sr_items[k].size();
+    }
+  }
   {
     std::vector<ElemChunk> sorted;
     for (int dt = 0; dt < 2; ++dt) {
@@ -809,6 +952,41 @@ static lm_status upload_grads(lm_state* s, const lm_tensor* grads, cudaStream_t 
 
 }  // extern "C"
 
+// Stable-rank selection on M_{t-1} (Appendix G): srank_iters power-iteration
+// passes, then the per-matrix decision into d_active / d_skip.
+static lm_status run_srank(lm_state* s, cudaStream_t stream) {
+  const int passes = s->cfg.srank_iters;
+  Profiler* P = &s->prof;
+  cudaError_t e = timed(P, LM_KERNEL_SRANK, stream, [&]() {
+    cudaError_t r = cudaMemsetAsync(s->sr_acc, 0, (size_t)s->nmat * (1 + passes) * sizeof(double), stream);
+    if (r == cudaSuccess && passes > 1) r = cudaMemsetAsync(s->sr_wa, 0, s->sr_w_elems * sizeof(float), stream);
+    return r;
+  });
+  if (e != cudaSuccess) return cuda_fail(e, "selection buffer reset");
+  for (int k = 0; k < passes; ++k) {
+    const bool last = k == passes - 1;
+    if (k >= 1 && !last) {   // this pass's output vector starts at zero
+      float* out = (k & 1) ? s->sr_wb : s->sr_wa;
+      e = cudaMemsetAsync(out, 0, s->sr_w_elems * sizeof(float), stream);
+      if (e != cudaSuccess) return cuda_fail(e, "selection buffer reset");
+    }
+    for (const auto& L : s->sr_launch) {
+      e = timed(P, LM_KERNEL_SRANK, stream, [&]() {
+        if (L.vec4)
+          return launch_srank_ring((int)L.max_cols, s->d_sr, L.items, L.nitems, k, last, s->d_flags, stream);
+        return launch_srank_pass(L.slots, L.threads, L.vec4, s->d_sr, L.items, L.nitems, k, last, stream);
+      });
+      if (e != cudaSuccess) return cuda_fail(e, "power-iteration launch");
+    }
+  }
+  e = timed(P, LM_KERNEL_SRANK, stream, [&]() {
+    return launch_srank_decide(s->d_sr, s->nmat, s->cfg.srank_alpha, passes - 1, s->d_active, s->d_skip,
+                               s->d_srank, stream);
+  });
+  if (e != cudaSuccess) return cuda_fail(e, "selection launch");
+  return LM_OK;
+}
+
 // AdamW over the 1-D parameters of both dtypes (LM_VECTOR_ADAMW).
 static lm_status run_adamw(lm_state* s, int64_t t, cudaStream_t stream) {
   const AdamConsts ak = adamw_consts(s->cfg, t);
@@ -843,10 +1021,18 @@ lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t, void* c
   if ((st = upload_grads(s, grads, stream)) != LM_OK) return st;
   s->last_stream = stream;
   const lm_config& c = s->cfg;
-  const bool muon = c.period != 0 && (t % c.period) == 0;
-  const LionConsts lk = lion_consts(c);
+  // Under the stable-rank schedule every step is mixed: matrices take Muon
+  // or Lion as the device-side selection says, nothing returns to the host.
+  const bool mixed = s->srank;
+  const bool muon = mixed || (c.period != 0 && (t % c.period) == 0);
+  LionConsts lk = lion_consts(c);
   cudaError_t e;
   Profiler* P = &s->prof;
+  s->last_t = t;
+  if (mixed) {
+    if ((st = run_srank(s, stream)) != LM_OK) return st;
+    lk.skip = s->d_skip;
+  }
   if (!muon) {
     for (int d = 0; d < 2; ++d) {
       if (s->lion_all[d].nchunks == 0) continue;
@@ -859,7 +1045,8 @@ lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t, void* c
     return s->adamw ? run_adamw(s, t, stream) : LM_OK;
   }
   // Muon step: momentum + norm, Lion on the vectors, NS iterations, finalize.
-  const MuonConsts mk = muon_consts(c);
+  MuonConsts mk = muon_consts(c);
+  if (mixed) mk.active = s->d_active;
   if (s->nmat > 0) {
     e = timed(P, LM_KERNEL_OTHER, stream, [&]() {
       return cudaMemsetAsync(s->ns.d_norm2, 0, (size_t)s->nmat * sizeof(double), stream);
@@ -877,7 +1064,7 @@ lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t, void* c
   if (s->adamw) {
     if ((st = run_adamw(s, t, stream)) != LM_OK) return st;
   }
-  for (int d = 0; d < 2 && !s->adamw; ++d) {
+  for (int d = 0; d < 2 && !s->adamw && !mixed; ++d) {
     if (s->lion_vec[d].nchunks == 0) continue;
     e = timed(P, LM_KERNEL_LION, stream, [&]() {
       return launch_lion((lm_dtype)d, s->lion_vec[d].tensors, s->lion_vec[d].chunks,
@@ -885,10 +1072,20 @@ lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t, void* c
     });
     if (e != cudaSuccess) return cuda_fail(e, "Lion kernel launch (vectors)");
   }
+  // mixed step: the Lion table (with the vectors unless AdamW has them)
+  // minus the matrices selected for Muon
+  for (int d = 0; d < 2 && mixed; ++d) {
+    if (s->lion_all[d].nchunks == 0) continue;
+    e = timed(P, LM_KERNEL_LION, stream, [&]() {
+      return launch_lion((lm_dtype)d, s->lion_all[d].tensors, s->lion_all[d].chunks,
+                         s->lion_all[d].nchunks, s->d_grads, lk, s->lion_grid[d], stream);
+    });
+    if (e != cudaSuccess) return cuda_fail(e, "Lion kernel launch (mixed step)");
+  }
   if (s->nmat > 0) {
     const FuseFinal ff{s->d_mats, mk.eM, mk.lam};
-    if ((st = run_ns(s->ns, c.ns_steps, s->ns_co.data(), s->d_flags, stream, P, s->fuse_final ? &ff : nullptr)) !=
-        LM_OK)
+    if ((st = run_ns(s->ns, c.ns_steps, s->ns_co.data(), s->d_flags, stream, P, s->fuse_final ? &ff : nullptr,
+                     mixed ? s->d_active : nullptr)) != LM_OK)
       return st;
     for (int dt = 0; dt < 2 && !s->fuse_final; ++dt) {
       if (s->n_echunks[dt] == 0) continue;
@@ -908,6 +1105,35 @@ lm_status lm_set_lr(lm_state* s, double eta_muon, double eta_lion) {
     return fail(LM_ERR_INVALID_ARG, "learning rates must be finite and >= 0");
   s->cfg.eta_muon = eta_muon;
   s->cfg.eta_lion = eta_lion;
+  return LM_OK;
+}
+
+lm_status lm_get_selection(lm_state* s, int n, unsigned char* took_muon, double* srank) {
+  if (s == nullptr) return fail(LM_ERR_INVALID_ARG, "state is NULL");
+  if (n != s->n) return fail(LM_ERR_INVALID_ARG, "n = %d but the state has %d parameters", n, s->n);
+  if (s->last_t < 0) return fail(LM_ERR_INVALID_ARG, "no step taken yet");
+  const double nan = std::numeric_limits<double>::quiet_NaN();
+  std::vector<unsigned char> act(s->nmat, 0);
+  std::vector<double> est(s->nmat, nan);
+  if (s->srank) {
+    cudaError_t e = cudaStreamSynchronize(s->last_stream);
+    if (e == cudaSuccess) e = cudaMemcpy(act.data(), s->d_active, (size_t)s->nmat, cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess)
+      e = cudaMemcpy(est.data(), s->d_srank, (size_t)s->nmat * sizeof(double), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(e, "selection read-back");
+  } else {
+    const bool muon = s->cfg.period != 0 && (s->last_t % s->cfg.period) == 0;
+    std::fill(act.begin(), act.end(), muon ? 1 : 0);
+  }
+  for (int i = 0; i < n; ++i) {
+    if (took_muon) took_muon[i] = 0;
+    if (srank) srank[i] = nan;
+  }
+  for (int id = 0; id < s->nmat; ++id) {
+    const int pi = s->mat_param_of[id];
+    if (took_muon) took_muon[pi] = act[id];
+    if (srank) srank[pi] = est[id];
+  }
   return LM_OK;
 }
 

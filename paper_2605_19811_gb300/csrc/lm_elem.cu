@@ -90,6 +90,7 @@ __global__ void __launch_bounds__(kLionThreads)
   for (int c = blockIdx.x; c < nchunks; c += gridDim.x) {
     const LionChunk ch = chunks[c];
     const LionTensor t = tensors[ch.tensor];
+    if (k.skip != nullptr && k.skip[t.pad]) continue;   // this matrix takes the Muon step
     T* w = static_cast<T*>(t.w) + ch.begin;
     const T* g = static_cast<const T*>(grads[t.grad_slot]) + ch.begin;
     float* m = t.m + ch.begin;
@@ -276,6 +277,7 @@ __global__ void __launch_bounds__(kElemThreads, kMomCtas)
                          int nchunks, const void* const* __restrict__ grads, MuonConsts k) {
   for (int c = blockIdx.x; c < nchunks; c += gridDim.x) {
     const ElemChunk ch = chunks[c];
+    if (k.active != nullptr && !k.active[ch.mat]) continue;   // this matrix takes the Lion step
     const MatDesc& d = mats[ch.mat];
     const GT* src = static_cast<const GT*>(MODE == 0 ? grads[d.grad_slot] : d.w);
     float acc = momentum_chunk<XT>(d, ch.begin, ch.count, src, k, MODE);
@@ -347,6 +349,7 @@ __global__ void __launch_bounds__(kElemThreads, kFinCtas)
                     MuonConsts k, unsigned* flags) {
   for (int c = blockIdx.x; c < nchunks; c += gridDim.x) {
     const ElemChunk ch = chunks[c];
+    if (k.active != nullptr && !k.active[ch.mat]) continue;
     const MatDesc& d = mats[ch.mat];
     const float nrm = (float)sqrt(*d.norm2);
     if (threadIdx.x == 0 && ch.begin == 0 && !isfinite(nrm)) atomicOr(flags, LM_FLAG_NONFINITE);

@@ -30,6 +30,9 @@ struct LionChunk {
 };
 struct LionConsts {
   float b1, c1, b2, c2, eL, lam;
+  // Adaptive selection: skip[param] != 0 makes the Lion kernel leave that
+  // parameter alone (it takes the Muon step); NULL: no parameter skipped.
+  const unsigned char* skip;
 };
 
 // AdamW on 1-D parameters (the LM_VECTOR_ADAMW rule): parameter, first
@@ -88,6 +91,9 @@ struct MuonConsts {
   float eM, lam;          // Muon learning rate and weight decay
   float eps;              // NS normalisation eps
   int32_t ns_steps;
+  // Adaptive selection: active[mat] != 0 for the matrices that take the
+  // Muon step; NULL: every matrix does.
+  const unsigned char* active;
 };
 // mode 0: Muon momentum step (G_hat from grads + momentum, M update)
 // mode 1: msign input (G_hat = input tensor, no momentum)
@@ -163,14 +169,54 @@ struct FuseFinal {
 cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* groups,
                          const TcGroupMaps* maps, const NsTile* tiles, int ntiles,
                          const int* offsets, int npairs, const double* norm2, NsCoeffs co,
-                         unsigned* flags, const FuseFinal* fuse, cudaStream_t st);
+                         unsigned* flags, const FuseFinal* fuse, cudaStream_t st,
+                         const unsigned char* active = nullptr);
 
 // fp32 CUDA-core path.
 constexpr int kSimtBM = 64, kSimtBN = 64;
 int simt_pad(int x);
 cudaError_t launch_ns_simt(NsPhase ph, int iter, int ngroups, const NsGroup* dgroups,
                            const NsTile* tiles, int ntiles, const double* norm2, NsCoeffs co,
-                           cudaStream_t st);
+                           cudaStream_t st, const unsigned char* active = nullptr);
+// active (both NS paths): NULL, or active[first_mat + mat] != 0 for the
+// matrices whose tiles run; tiles of the others are skipped by every role.
+
+// Power iteration for the stable-rank selection (Appendix G).  One pass
+// reads each matrix M (fp32 momentum, row-major) once: with v the input
+// vector normalised, u = M v row by row, ||u||^2 into acc[1 + pass], and
+// (unless last) M^T u added into the output vector; pass 0 also adds
+// ||M||_F^2 into acc[0].  Pass k reads v0 (k = 0), wa (k odd) or wb (k even)
+// and writes wa (k even) or wb (k odd), which must be zero beforehand.
+struct SrMat {
+  const float* M;
+  const float* v0;
+  float* wa;
+  float* wb;
+  double* acc;            // 1 + passes doubles, zero before pass 0
+  int64_t rows, cols;
+  int32_t mat, param;     // matrix id (NS numbering) and parameter index
+};
+constexpr int kSrankRows = 64;   // rows per power-iteration work item
+struct SrItem {
+  int32_t m;              // index into the SrMat table
+  int32_t row0, nrows;    // rows of this work item
+  int32_t pad;
+};
+// Launch shape for a column count: slots per thread and threads per block;
+// slots = 0 means cols is too large (more than 16384).
+int srank_slots(int64_t cols, int* threads);
+cudaError_t launch_srank_pass(int slots, int threads, bool vec4, const SrMat* mats, const SrItem* items,
+                              int nitems, int pass, bool last, cudaStream_t st);
+// The same pass through the shared-memory ring (every matrix of the launch
+// with cols % 4 == 0, at most max_cols <= 16384 columns); a stalled copy sets
+// LM_FLAG_TIMEOUT in *flags.
+cudaError_t launch_srank_ring(int max_cols, const SrMat* mats, const SrItem* items, int nitems, int pass, bool last,
+                              unsigned* flags, cudaStream_t st);
+// Decide per matrix: Muon iff ||M||_F^2 == 0 or ||M||_F^2 <= alpha min(m, n)
+// sigma^2 (sigma^2 = acc[1 + last_pass]); writes active[mat], skip[param]
+// and the estimate srank[mat] = ||M||_F^2 / sigma^2.
+cudaError_t launch_srank_decide(const SrMat* mats, int nmat, double alpha, int last_pass, unsigned char* active,
+                                unsigned char* skip, double* srank, cudaStream_t st);
 constexpr int kMaxGroupsSimt = 64;
 
 // Launch accounting (lm_kernel_launch_count) and the thread's last-error text.

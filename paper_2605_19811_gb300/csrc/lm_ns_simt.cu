@@ -38,7 +38,7 @@ __device__ __forceinline__ void load_tile(float (*S)[BM + 4], const float* op, i
 __global__ void __launch_bounds__(kThreads)
     ns_simt_kernel(int phase, int iter, const NsGroup* __restrict__ groups,
                    const NsTile* __restrict__ tiles, int ntiles, const double* __restrict__ norm2,
-                   NsCoeffs co) {
+                   NsCoeffs co, const unsigned char* __restrict__ active) {
   __shared__ float As[BK][BM + 4];
   __shared__ float Bs[BK][BN + 4];
   const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
@@ -46,6 +46,7 @@ __global__ void __launch_bounds__(kThreads)
   for (int w = blockIdx.x; w < ntiles; w += gridDim.x) {
     const NsTile t = tiles[w];
     const NsGroup g = groups[t.group];
+    if (active != nullptr && !active[g.first_mat + t.mat]) continue;   // block-uniform
     const int cur = iter & 1;
     const bool tall = g.tall != 0;
     const int ldx = tall ? g.s_pad : g.l_pad;
@@ -134,7 +135,7 @@ int simt_pad(int x) { return (x + 63) / 64 * 64; }
 
 cudaError_t launch_ns_simt(NsPhase ph, int iter, int ngroups, const NsGroup* dgroups,
                            const NsTile* tiles, int ntiles, const double* norm2, NsCoeffs co,
-                           cudaStream_t st) {
+                           cudaStream_t st, const unsigned char* active) {
   (void)ngroups;
   if (ntiles <= 0) return cudaSuccess;
   int dev = 0, sms = 0;
@@ -143,7 +144,7 @@ cudaError_t launch_ns_simt(NsPhase ph, int iter, int ngroups, const NsGroup* dgr
   int grid = sms * 4;
   if (grid > ntiles) grid = ntiles;
   count_launch();
-  ns_simt_kernel<<<grid, kThreads, 0, st>>>((int)ph, iter, dgroups, tiles, ntiles, norm2, co);
+  ns_simt_kernel<<<grid, kThreads, 0, st>>>((int)ph, iter, dgroups, tiles, ntiles, norm2, co, active);
   return cudaGetLastError();
 }
 

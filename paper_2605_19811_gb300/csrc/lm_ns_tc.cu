@@ -80,7 +80,14 @@ struct TcParams {
   NsCoeffs co;
   unsigned* flags;
   FuseFinal fuse;       // fuse.mats != NULL: this APPLY writes the parameters
+  const unsigned char* active;   // NULL, or per matrix: 0 = skip its tiles
 };
+
+// Whether a tile's matrix runs in this launch; every role asks the same
+// question of the same tiles, so skipping keeps their pipelines in step.
+__device__ __forceinline__ bool tile_active(const TcParams& p, const NsTile& t) {
+  return p.active == nullptr || p.active[p.groups[t.group].first_mat + t.mat] != 0;
+}
 
 // ------------------------------- PTX wrappers -------------------------------
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -469,6 +476,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int w = w_begin; ok && w < w_end; w += w_step) {
         const NsTile t = p.tiles[w];
+        if (!tile_active(p, t)) continue;
         const NsGroup& g = p.groups[t.group];
         const TilePlan P = tile_plan(phase, g, p.maps[t.group], cur, t);
         const int row_a = t.tm * BM + (int)rank * kHalf;
@@ -508,6 +516,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int w = w_begin; ok && w < w_end; w += w_step) {
         const NsTile t = p.tiles[w];
+        if (!tile_active(p, t)) continue;
         const NsGroup& g = p.groups[t.group];
         const TilePlan P = tile_plan(phase, g, p.maps[t.group], cur, t);
         if (!mbar_wait(&accempty[ab], aph ^ 1u, abort_flag, kWaitLimitNs)) {
@@ -550,6 +559,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int w = w_begin; ok && w < w_end; w += w_step) {
         const NsTile t = p.tiles[w];
+        if (!tile_active(p, t)) continue;
         const TcGroupMaps& mp = p.maps[t.group];
         const CUtensorMap* map = (phase == NS_POLY) ? &mp.a : &mp.xk[cur];
         if (!mbar_wait(aux_empty, xph ^ 1u, abort_flag, kWaitLimitNs)) {
@@ -585,6 +595,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     uint32_t aph = 0, xph = 0;
     for (int w = w_begin; w < w_end; w += w_step) {
       const NsTile t = p.tiles[w];
+      if (!tile_active(p, t)) continue;
       const NsGroup& g = p.groups[t.group];
       const bool fused = phase == NS_APPLY && p.fuse.mats != nullptr;
       const MatDesc* fd = fused ? &p.fuse.mats[g.first_mat + t.mat] : nullptr;
@@ -814,7 +825,8 @@ int tc_max_pairs() {
 cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* groups,
                          const TcGroupMaps* maps, const NsTile* tiles, int ntiles,
                          const int* offsets, int npairs, const double* norm2, NsCoeffs co,
-                         unsigned* flags, const FuseFinal* fuse, cudaStream_t st) {
+                         unsigned* flags, const FuseFinal* fuse, cudaStream_t st,
+                         const unsigned char* active) {
   if (ntiles <= 0) return cudaSuccess;
   if (ngroups < 1 || ngroups > kMaxGroupsTc) return cudaErrorInvalidValue;
   static bool attr_set = false;
@@ -839,6 +851,7 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
   prm.co = co;
   prm.flags = flags;
   if (fuse != nullptr && ph == NS_APPLY) prm.fuse = *fuse;
+  prm.active = active;
   int pairs = npairs;
   if (offsets == nullptr) {
     pairs = tc_max_pairs();

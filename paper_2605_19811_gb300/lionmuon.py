@@ -28,10 +28,12 @@ EXPORTED = ("lm_config_default", "lm_create", "lm_step", "lm_set_lr", "lm_msign_
             "lm_workspace_bytes", "lm_destroy", "lm_status_string", "lm_last_error",
             "lm_kernel_launch_count", "lm_profile_enable", "lm_profile_read",
             "lm_msign_ns_noalloc", "lm_probe_bounded_wait", "lm_msign_ns_coeffs",
-            "lm_set_adamw_lr", "lm_get_second_moment", "lm_set_second_moment")
+            "lm_set_adamw_lr", "lm_get_second_moment", "lm_set_second_moment", "lm_get_selection")
 
-KERNEL_FAMILIES = ("lion", "momentum_norm", "ns_gram", "ns_poly", "ns_apply", "finalize", "other", "adamw")
+KERNEL_FAMILIES = ("lion", "momentum_norm", "ns_gram", "ns_poly", "ns_apply", "finalize", "other", "adamw",
+                   "srank")
 LM_VECTOR_LION, LM_VECTOR_ADAMW = 0, 1
+LM_SCHEDULE_PERIOD, LM_SCHEDULE_STABLE_RANK = 0, 1
 
 
 class LmTensor(ctypes.Structure):
@@ -49,11 +51,13 @@ class LmConfig(ctypes.Structure):
                 ("ns_coeffs", ctypes.POINTER(ctypes.c_double)),
                 ("vector_rule", ctypes.c_int), ("adamw_lr", ctypes.c_double),
                 ("adamw_beta1", ctypes.c_double), ("adamw_beta2", ctypes.c_double),
-                ("adamw_eps", ctypes.c_double), ("adamw_weight_decay", ctypes.c_double)]
+                ("adamw_eps", ctypes.c_double), ("adamw_weight_decay", ctypes.c_double),
+                ("schedule", ctypes.c_int), ("srank_alpha", ctypes.c_double), ("srank_iters", ctypes.c_int),
+                ("srank_seed", ctypes.c_uint64)]
 
 
 class LmProfile(ctypes.Structure):
-    _fields_ = [("ms", ctypes.c_double * 8), ("launches", ctypes.c_uint64 * 8)]
+    _fields_ = [("ms", ctypes.c_double * 9), ("launches", ctypes.c_uint64 * 9)]
 
 
 class LionMuonError(RuntimeError):
@@ -94,6 +98,8 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib.lm_msign_ns_noalloc.argtypes = [P(LmTensor), P(LmTensor), c_int, c_double, c_double, c_double,
                                         c_double, c_int, c_void_p]
     lib.lm_msign_ns_noalloc.restype = c_int
+    lib.lm_get_selection.argtypes = [c_void_p, c_int, P(ctypes.c_ubyte), P(c_double)]
+    lib.lm_get_selection.restype = c_int
     lib.lm_set_adamw_lr.argtypes = [c_void_p, c_double]
     lib.lm_set_adamw_lr.restype = c_int
     lib.lm_get_second_moment.argtypes = [c_void_p, c_int, P(LmTensor)]
@@ -226,6 +232,16 @@ class LionMuon:
         _check(self._lib, self._lib.lm_get_momentum(self._h, i, ctypes.byref(v)), "lm_get_momentum")
         shape = tuple(self.params[i].shape)
         return torch.as_tensor(_DeviceArray(v.data, shape, "<f4"), device=self.params[i].device)
+
+    def selection(self):
+        """(took_muon, srank) of the last step, one entry per parameter:
+        whether it took the Muon step, and under the stable-rank schedule the
+        estimate ||M||_F^2 / sigma_1_hat^2 behind it (NaN otherwise)."""
+        n = len(self.params)
+        took = (ctypes.c_ubyte * n)()
+        est = (ctypes.c_double * n)()
+        _check(self._lib, self._lib.lm_get_selection(self._h, n, took, est), "lm_get_selection")
+        return [bool(x) for x in took], [float(x) for x in est]
 
     def set_adamw_lr(self, lr: float) -> None:
         _check(self._lib, self._lib.lm_set_adamw_lr(self._h, lr), "lm_set_adamw_lr")
