@@ -410,6 +410,9 @@ __device__ __forceinline__ bool mma_range(int& stage, uint32_t& ph, uint8_t* sme
 }
 
 // ------------------------------- the kernel ---------------------------------
+// kMasked: the launch carries a per-matrix mask (stable-rank selection); the
+// unmasked instantiation keeps the fixed-period path free of the test.
+template <bool kMasked>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     ns_tc_kernel(const __grid_constant__ TcParams p) {
   extern __shared__ uint8_t smem_raw[];
@@ -476,7 +479,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int w = w_begin; ok && w < w_end; w += w_step) {
         const NsTile t = p.tiles[w];
-        if (!tile_active(p, t)) continue;
+        if (kMasked && !tile_active(p, t)) continue;
         const NsGroup& g = p.groups[t.group];
         const TilePlan P = tile_plan(phase, g, p.maps[t.group], cur, t);
         const int row_a = t.tm * BM + (int)rank * kHalf;
@@ -516,7 +519,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int w = w_begin; ok && w < w_end; w += w_step) {
         const NsTile t = p.tiles[w];
-        if (!tile_active(p, t)) continue;
+        if (kMasked && !tile_active(p, t)) continue;
         const NsGroup& g = p.groups[t.group];
         const TilePlan P = tile_plan(phase, g, p.maps[t.group], cur, t);
         if (!mbar_wait(&accempty[ab], aph ^ 1u, abort_flag, kWaitLimitNs)) {
@@ -559,7 +562,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int w = w_begin; ok && w < w_end; w += w_step) {
         const NsTile t = p.tiles[w];
-        if (!tile_active(p, t)) continue;
+        if (kMasked && !tile_active(p, t)) continue;
         const TcGroupMaps& mp = p.maps[t.group];
         const CUtensorMap* map = (phase == NS_POLY) ? &mp.a : &mp.xk[cur];
         if (!mbar_wait(aux_empty, xph ^ 1u, abort_flag, kWaitLimitNs)) {
@@ -595,7 +598,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     uint32_t aph = 0, xph = 0;
     for (int w = w_begin; w < w_end; w += w_step) {
       const NsTile t = p.tiles[w];
-      if (!tile_active(p, t)) continue;
+      if (kMasked && !tile_active(p, t)) continue;
       const NsGroup& g = p.groups[t.group];
       const bool fused = phase == NS_APPLY && p.fuse.mats != nullptr;
       const MatDesc* fd = fused ? &p.fuse.mats[g.first_mat + t.mat] : nullptr;
@@ -831,8 +834,10 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
   if (ngroups < 1 || ngroups > kMaxGroupsTc) return cudaErrorInvalidValue;
   static bool attr_set = false;
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(ns_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(ns_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)kSmemBytes);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(ns_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
@@ -859,7 +864,10 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
   }
   const int grid = 2 * (pairs > 0 ? pairs : 1);
   count_launch();
-  ns_tc_kernel<<<grid, kThreads, kSmemBytes, st>>>(prm);
+  if (active != nullptr)
+    ns_tc_kernel<true><<<grid, kThreads, kSmemBytes, st>>>(prm);
+  else
+    ns_tc_kernel<false><<<grid, kThreads, kSmemBytes, st>>>(prm);
   return cudaGetLastError();
 }
 
