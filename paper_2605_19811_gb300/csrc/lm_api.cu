@@ -3,6 +3,7 @@
 // grouped Newton-Schulz GEMMs, device tables, workspace, and the per-step
 // launch sequence of Algorithm 1 (Lion step, or Muon step on t mod P == 0).
 #include <algorithm>
+#include <array>
 #include <atomic>
 #include <cmath>
 #include <cstdarg>
@@ -184,6 +185,8 @@ struct NsBatch {
   int ntiles[3] = {0, 0, 0};
   int* offsets[3] = {nullptr, nullptr, nullptr};   // per-pair tile ranges (tensor-core path)
   int npairs[3] = {0, 0, 0};
+  NsSplitTarget* split_targets = nullptr;   // split Gram tiles of this batch
+  int nsplit = 0;
 };
 
 struct AdamTable {
@@ -283,6 +286,7 @@ struct NsEngine {
   NsGroup* d_groups = nullptr;       // fp32 path reads groups from device memory
   std::vector<NsBatch> batches;
   double* d_norm2 = nullptr;
+  float* d_split_ws = nullptr;       // fp32 partial sums of split Gram tiles
 };
 
 // Plan: group matrices by (s, l); returns matrix order (indices into shapes)
@@ -334,7 +338,45 @@ struct NsLayout {
   std::vector<size_t> off_offsets;
   size_t off_groups = 0;
   size_t off_norm = 0;
+  // split Gram tiles, per batch: (group, mat, tm, tn) of each target tile
+  std::vector<std::vector<std::array<int, 4>>> split_targets;
+  std::vector<size_t> off_split_targets;
+  size_t off_split_ws = 0;
 };
+
+// Split-K of the Gram phase: a tile longer than twice the average load of a
+// CTA pair (a long-K embedding Gram next to short hidden matrices, which would
+// otherwise set the length of the launch) is cut into parts of at most half
+// that load; each part is a tile of its own for the balancer and adds its
+// partial product into an fp32 workspace tile.  Tiles near the average stay
+// whole: splitting them costs the atomic additions and buys no balance.
+static void split_gram_tiles(const std::vector<NsGroup>& groups, int g0, std::vector<NsTile>& t,
+                             std::vector<std::array<int, 4>>& targets) {
+  int64_t total = 0;
+  for (const NsTile& x : t) total += groups[g0 + x.group].l_pad / kTcBK;
+  const int pairs = std::max(1, tc_max_pairs());
+  const int64_t avg = total / pairs;
+  const int64_t part = std::max<int64_t>(8, avg / 2);
+  std::vector<NsTile> out;
+  for (const NsTile& x : t) {
+    const int nk = groups[g0 + x.group].l_pad / kTcBK;
+    if (nk <= 2 * avg || (int64_t)targets.size() >= 65535) {
+      out.push_back(x);
+      continue;
+    }
+    const int nparts = (int)std::min<int64_t>(64, (nk + part - 1) / part);
+    targets.push_back({x.group, x.mat, x.tm, x.tn});
+    const int slot = (int)targets.size();   // 1-based
+    for (int k = 0; k < nparts; ++k) {
+      NsTile y = x;
+      y.kb0 = (uint16_t)((int64_t)nk * k / nparts);
+      y.kb1 = (uint16_t)((int64_t)nk * (k + 1) / nparts);
+      y.slot = (uint16_t)slot;
+      out.push_back(y);
+    }
+  }
+  t.swap(out);
+}
 
 static void layout_ns(std::vector<NsGroup>& groups, lm_dtype xdt, int nmat, Arena& ar, NsLayout& L,
                       std::vector<NsBatch>& batches) {
@@ -348,6 +390,7 @@ static void layout_ns(std::vector<NsGroup>& groups, lm_dtype xdt, int nmat, Aren
     L.off_b.push_back(ar.add(ab));
   }
   const int per = (xdt == LM_BF16) ? kMaxGroupsTc : kMaxGroupsSimt;
+  int max_split = 0;
   const int bm = (xdt == LM_BF16) ? kTcBM : kSimtBM;
   const int bn = (xdt == LM_BF16) ? kTcBN : kSimtBN;
   for (int g0 = 0; g0 < (int)groups.size(); g0 += per) {
@@ -358,12 +401,20 @@ static void layout_ns(std::vector<NsGroup>& groups, lm_dtype xdt, int nmat, Aren
       std::vector<NsTile> t;
       build_ns_tiles(groups, g0, b.ng, ph, bm, bn, t);
       std::vector<int> offs;
+      std::vector<std::array<int, 4>> targets;
+      if (xdt == LM_BF16 && ph == NS_GRAM) split_gram_tiles(groups, g0, t, targets);
+      if (ph == NS_GRAM) {
+        b.nsplit = (int)targets.size();
+        max_split = std::max(max_split, b.nsplit);
+        L.off_split_targets.push_back(ar.add(targets.size() * sizeof(NsSplitTarget)));
+        L.split_targets.push_back(std::move(targets));
+      }
       if (xdt == LM_BF16 && !t.empty()) {
         // cost of a tile: its K blocks plus an allowance for the epilogue
         std::vector<std::pair<int, NsTile>> sorted;
         for (const NsTile& x : t) {
           const NsGroup& g = groups[g0 + x.group];
-          const int nk = ((ph == NS_GRAM) ? g.l_pad : g.s_pad) / kTcBK;
+          const int nk = (ph == NS_GRAM) ? (x.kb1 != 0 ? x.kb1 - x.kb0 : g.l_pad / kTcBK) : g.s_pad / kTcBK;
           sorted.push_back({nk + 6, x});
         }
         std::stable_sort(sorted.begin(), sorted.end(),
@@ -385,6 +436,7 @@ static void layout_ns(std::vector<NsGroup>& groups, lm_dtype xdt, int nmat, Aren
   }
   L.off_groups = ar.add(groups.size() * sizeof(NsGroup));
   L.off_norm = ar.add((size_t)std::max(nmat, 1) * sizeof(double));
+  L.off_split_ws = ar.add((size_t)max_split * kTcBM * kTcBN * sizeof(float));
 }
 
 static void bind_ns(NsEngine& E, char* base, const NsLayout& L, std::vector<char>& host_img) {
@@ -405,6 +457,23 @@ static void bind_ns(NsEngine& E, char* base, const NsLayout& L, std::vector<char
         memcpy(host_img.data() + L.off_offsets[k], L.offsets[k].data(), L.offsets[k].size() * sizeof(int));
       }
     }
+  for (size_t bi = 0; bi < E.batches.size(); ++bi) {
+    const auto& tg = L.split_targets[bi];
+    std::vector<NsSplitTarget> st(tg.size());
+    for (size_t k = 0; k < tg.size(); ++k) {
+      const NsGroup& g = E.groups[E.batches[bi].g0 + tg[k][0]];
+      const size_t es = 2;   // bf16 A
+      char* a = static_cast<char*>(g.A) + (size_t)tg[k][1] * g.s_pad * g.s_pad * es;
+      st[k].a_tile = a + ((size_t)tg[k][2] * kTcBM * g.s_pad + (size_t)tg[k][3] * kTcBN) * es;
+      st[k].ld = g.s_pad;
+      st[k].nr = std::min(kTcBM, g.s_pad - tg[k][2] * kTcBM);
+      st[k].nc = std::min(kTcBN, g.s_pad - tg[k][3] * kTcBN);
+      st[k].slot = (int32_t)k;
+    }
+    E.batches[bi].split_targets = reinterpret_cast<NsSplitTarget*>(base + L.off_split_targets[bi]);
+    if (!st.empty()) memcpy(host_img.data() + L.off_split_targets[bi], st.data(), st.size() * sizeof(NsSplitTarget));
+  }
+  E.d_split_ws = reinterpret_cast<float*>(base + L.off_split_ws);
   E.d_groups = reinterpret_cast<NsGroup*>(base + L.off_groups);
   memcpy(host_img.data() + L.off_groups, E.groups.data(), E.groups.size() * sizeof(NsGroup));
   E.d_norm2 = reinterpret_cast<double*>(base + L.off_norm);
@@ -477,11 +546,19 @@ static lm_status run_ns(const NsEngine& E, int steps, const NsCoeffs* coeffs, un
     for (const NsBatch& b : E.batches)
       for (int ph = 0; ph < 3; ++ph) {
         const NsCoeffs co = coeffs[it];
+        const bool split = E.xdt == LM_BF16 && ph == NS_GRAM && b.nsplit > 0;
         cudaError_t e = timed(P, LM_KERNEL_NS_GRAM + ph, st, [&]() {
-          if (E.xdt == LM_BF16)
-            return launch_ns_tc((NsPhase)ph, it, b.ng, E.groups.data() + b.g0, E.maps.data() + b.g0,
-                                b.tiles[ph], b.ntiles[ph], b.offsets[ph], b.npairs[ph], E.d_norm2, co,
-                                flags, it == steps - 1 ? fuse : nullptr, st, active);
+          if (E.xdt == LM_BF16) {
+            cudaError_t r = cudaSuccess;
+            if (split)   // the split tiles' partial sums start at zero
+              r = cudaMemsetAsync(E.d_split_ws, 0, (size_t)b.nsplit * kTcBM * kTcBN * sizeof(float), st);
+            if (r == cudaSuccess)
+              r = launch_ns_tc((NsPhase)ph, it, b.ng, E.groups.data() + b.g0, E.maps.data() + b.g0, b.tiles[ph],
+                               b.ntiles[ph], b.offsets[ph], b.npairs[ph], E.d_norm2, co, flags,
+                               it == steps - 1 ? fuse : nullptr, st, active, E.d_split_ws);
+            if (r == cudaSuccess && split) r = launch_ns_split_finish(b.split_targets, b.nsplit, E.d_split_ws, st);
+            return r;
+          }
           return launch_ns_simt((NsPhase)ph, it, b.ng, E.d_groups + b.g0, b.tiles[ph], b.ntiles[ph],
                                 E.d_norm2, co, st, active);
         });

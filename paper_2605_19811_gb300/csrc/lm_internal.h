@@ -127,6 +127,19 @@ struct NsGroup {
 // Tile work item: group, matrix-in-group, tile row, tile col.
 struct NsTile {
   uint16_t group, mat, tm, tn;
+  // Split-K (Gram phase only): K blocks [kb0, kb1) of the tile, kb1 == 0 for
+  // all of them; slot != 0: the partial product is added in fp32 into
+  // workspace tile slot - 1 instead of being stored (NsSplitTarget finishes it).
+  uint16_t kb0, kb1, slot, pad;
+};
+// A split Gram tile: the fp32 sum of its parts in workspace tile `slot`
+// becomes bf16 A[tm * 256 + r][tn * 256 + c] for r < nr, c < nc (the part of
+// the tile inside s_pad x s_pad; a tile is 256 x 256 floats).
+struct NsSplitTarget {
+  void* a_tile;           // bf16 element (tm * 256, tn * 256) of the matrix's A
+  int32_t ld;             // s_pad
+  int32_t nr, nc;         // rows / columns of the tile inside the padded matrix
+  int32_t slot;
 };
 constexpr int kMaxGroupsTc = 8;   // groups per tensor-core launch
 
@@ -170,7 +183,9 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
                          const TcGroupMaps* maps, const NsTile* tiles, int ntiles,
                          const int* offsets, int npairs, const double* norm2, NsCoeffs co,
                          unsigned* flags, const FuseFinal* fuse, cudaStream_t st,
-                         const unsigned char* active = nullptr);
+                         const unsigned char* active = nullptr, float* split_ws = nullptr);
+// After a Gram launch with split tiles: A tiles from the fp32 workspace.
+cudaError_t launch_ns_split_finish(const NsSplitTarget* targets, int n, const float* ws, cudaStream_t st);
 
 // fp32 CUDA-core path.
 constexpr int kSimtBM = 64, kSimtBN = 64;

@@ -81,6 +81,7 @@ struct TcParams {
   unsigned* flags;
   FuseFinal fuse;       // fuse.mats != NULL: this APPLY writes the parameters
   const unsigned char* active;   // NULL, or per matrix: 0 = skip its tiles
+  float* split_ws;               // fp32 workspace of split Gram tiles (256 x 256 each)
 };
 
 // Whether a tile's matrix runs in this launch; every role asks the same
@@ -299,6 +300,7 @@ struct OpSeg {
 struct TilePlan {
   int nseg;
   int nk;
+  int kb_start;   // first K block (split Gram tiles start inside K)
   OpSeg seg[3];
 };
 __device__ __forceinline__ void plan_push(TilePlan& P, int kb_end, bool a_mn, bool b_mn,
@@ -311,10 +313,13 @@ __device__ __forceinline__ TilePlan tile_plan(int phase, const NsGroup& g, const
                                               const NsTile& t) {
   TilePlan P;
   P.nseg = 0;
+  P.kb_start = 0;
   if (phase == NS_GRAM) {
     P.nk = g.l_pad / BK;
-    if (g.tall) plan_push(P, P.nk, true, true, &mp.xmn[cur], &mp.xmn[cur]);
-    else plan_push(P, P.nk, false, false, &mp.xk[cur], &mp.xk[cur]);
+    const int kb_end = t.kb1 != 0 ? (int)t.kb1 : P.nk;
+    P.kb_start = t.kb1 != 0 ? (int)t.kb0 : 0;
+    if (g.tall) plan_push(P, kb_end, true, true, &mp.xmn[cur], &mp.xmn[cur]);
+    else plan_push(P, kb_end, false, false, &mp.xk[cur], &mp.xk[cur]);
     return P;
   }
   P.nk = g.s_pad / BK;
@@ -387,7 +392,7 @@ __device__ __forceinline__ bool produce_range(ProducerRing& R, uint8_t* smem, ui
 template <bool AMN, bool BMN>
 __device__ __forceinline__ bool mma_range(int& stage, uint32_t& ph, uint8_t* smem, uint64_t* full,
                                           uint64_t* empty, volatile int* abort_flag, int kb0, int kb1,
-                                          uint32_t d_tmem) {
+                                          uint32_t d_tmem, int kb_first) {
   const uint32_t idesc = make_idesc(BM, BN, AMN, BMN);
   for (int kb = kb0; kb < kb1; ++kb) {
     if (!mbar_wait(&full[stage], ph, abort_flag, kWaitLimitNs)) return false;
@@ -398,7 +403,7 @@ __device__ __forceinline__ bool mma_range(int& stage, uint32_t& ph, uint8_t* sme
     for (int kk = 0; kk < BK / 16; ++kk) {
       const uint64_t adesc = AMN ? sw128_desc(sa + kk * 2048, 64 * BK * 2, 1024) : sw128_desc(sa + kk * 32, 16, 1024);
       const uint64_t bdesc = BMN ? sw128_desc(sb + kk * 2048, 64 * BK * 2, 1024) : sw128_desc(sb + kk * 32, 16, 1024);
-      umma_bf16(d_tmem, adesc, bdesc, idesc, (kb | kk) != 0 ? 1u : 0u);
+      umma_bf16(d_tmem, adesc, bdesc, idesc, (kb != kb_first || kk != 0) ? 1u : 0u);
     }
     umma_commit_pair(&empty[stage]);
     if (++stage == kStages) {
@@ -484,7 +489,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         const TilePlan P = tile_plan(phase, g, p.maps[t.group], cur, t);
         const int row_a = t.tm * BM + (int)rank * kHalf;
         const int col_b = t.tn * BN + (int)rank * kHalf;
-        int kb0 = 0;
+        int kb0 = P.kb_start;
         for (int sg = 0; ok && sg < P.nseg; ++sg) {
           const OpSeg& S = P.seg[sg];
           if (!S.a_mn && !S.b_mn)
@@ -528,15 +533,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + (uint32_t)(ab * BN);
-        int kb0 = 0;
+        int kb0 = P.kb_start;
         for (int sg = 0; ok && sg < P.nseg; ++sg) {
           const OpSeg& S = P.seg[sg];
           if (!S.a_mn && !S.b_mn)
-            ok = mma_range<false, false>(stage, ph, smem, full, empty, abort_flag, kb0, S.kb_end, d_tmem);
+            ok = mma_range<false, false>(stage, ph, smem, full, empty, abort_flag, kb0, S.kb_end, d_tmem,
+                                            P.kb_start);
           else if (!S.a_mn)
-            ok = mma_range<false, true>(stage, ph, smem, full, empty, abort_flag, kb0, S.kb_end, d_tmem);
+            ok = mma_range<false, true>(stage, ph, smem, full, empty, abort_flag, kb0, S.kb_end, d_tmem,
+                                            P.kb_start);
           else
-            ok = mma_range<true, true>(stage, ph, smem, full, empty, abort_flag, kb0, S.kb_end, d_tmem);
+            ok = mma_range<true, true>(stage, ph, smem, full, empty, abort_flag, kb0, S.kb_end, d_tmem,
+                                            P.kb_start);
           kb0 = S.kb_end;
         }
         if (!ok) give_up();
@@ -628,6 +636,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const int r0 = t.tm * BM + (int)rank * kHalf + q * 32;   // first row of this warp
       const int i = r0 + lane;
       const bool warp_in = r0 < row_lim;        // rows past the padded matrix are skipped
+      const bool split = phase == NS_GRAM && t.slot != 0;
       if (fused && lane == 0 && q == 0 && half == 0 && rank == 0 && t.tm == 0 && t.tn == 0 &&
           !isfinite((float)sqrt(p.norm2[g.first_mat + t.mat])))
         atomicOr(p.flags, LM_FLAG_NONFINITE);
@@ -638,6 +647,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * BN + ch * 32), r);
         const int j0 = t.tn * BN + ch * 32;
         if (!warp_in || j0 >= jmax) continue;   // beyond the padded matrix
+        if (split) {
+          // partial Gram product of a split tile: add into the fp32 workspace
+          float* wrow = p.split_ws + (size_t)(t.slot - 1) * (BM * BN) + (size_t)((int)rank * kHalf + row) * BN +
+                        ch * 32;
+#pragma unroll
+          for (int e = 0; e < 32; ++e) {
+            const int j = j0 + e;
+            if (i < nrows && j < ncols) atomicAdd(wrow + e, __uint_as_float(r[e]) * nscale);
+          }
+          continue;
+        }
         // 16-byte chunk c of row r of a box sits at chunk position c ^ (r mod 8)
         uint4* abox = reinterpret_cast<uint4*>(auxbuf + (ch >> 1) * kAuxBoxBytes + row * 128);
         const int csub = (ch & 1) * 4;
@@ -720,7 +740,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             }
           }
         }
-      } else if (lane == 0 && warp_in) {
+      } else if (lane == 0 && warp_in && !split) {
         const TcGroupMaps& mp = p.maps[t.group];
         const CUtensorMap* dst = (phase == NS_GRAM) ? &mp.ast : (phase == NS_POLY ? &mp.bst : &mp.xst[cur ^ 1]);
 #pragma unroll
@@ -745,6 +765,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem_base, kTmemCols);
+  }
+}
+
+// Split Gram tiles: bf16 A tile = the fp32 sum of the parts (already scaled).
+__global__ void __launch_bounds__(256) ns_split_finish_kernel(const NsSplitTarget* __restrict__ targets,
+                                                              const float* __restrict__ ws) {
+  const NsSplitTarget T = targets[blockIdx.y];
+  const float* src = ws + (size_t)T.slot * (BM * BN);
+  __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(T.a_tile);
+  for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < BM * BN; e += gridDim.x * blockDim.x) {
+    const int r = e / BN, c = e % BN;
+    if (r < T.nr && c < T.nc) dst[(size_t)r * T.ld + c] = __float2bfloat16_rn(src[e]);
   }
 }
 
@@ -818,6 +850,13 @@ cudaError_t tc_encode_group_maps(const NsGroup& g, TcGroupMaps* maps) {
   return cudaSuccess;
 }
 
+cudaError_t launch_ns_split_finish(const NsSplitTarget* targets, int n, const float* ws, cudaStream_t st) {
+  if (n <= 0) return cudaSuccess;
+  count_launch();
+  ns_split_finish_kernel<<<dim3(32, n), 256, 0, st>>>(targets, ws);
+  return cudaGetLastError();
+}
+
 int tc_max_pairs() {
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
@@ -829,7 +868,7 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
                          const TcGroupMaps* maps, const NsTile* tiles, int ntiles,
                          const int* offsets, int npairs, const double* norm2, NsCoeffs co,
                          unsigned* flags, const FuseFinal* fuse, cudaStream_t st,
-                         const unsigned char* active) {
+                         const unsigned char* active, float* split_ws) {
   if (ntiles <= 0) return cudaSuccess;
   if (ngroups < 1 || ngroups > kMaxGroupsTc) return cudaErrorInvalidValue;
   static bool attr_set = false;
@@ -857,6 +896,7 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
   prm.flags = flags;
   if (fuse != nullptr && ph == NS_APPLY) prm.fuse = *fuse;
   prm.active = active;
+  prm.split_ws = split_ws;
   int pairs = npairs;
   if (offsets == nullptr) {
     pairs = tc_max_pairs();

@@ -91,3 +91,83 @@ def test_720m_muon_then_lion_sampled():
         np.testing.assert_array_equal(_host(opt.momentum(i)).view(np.uint32), m_ref.view(np.uint32))
     assert opt.status() == 0
     opt.close()
+
+
+def _muon_then_lion(set_name, period, check_shapes, spectrum_shape=None):
+    """One Muon step (t = 0) and one Lion step (t = 1, or t = period - 1 when
+    that is not a Muon step) of a whole parameter set in the bench's
+    configuration; sampled checks as in the 720M test above."""
+    import torch
+    from paper_2605_19811_gb300 import lionmuon as L
+    ps = synth.PARAM_SETS[set_name]
+    shapes = [tuple(s) for s in ps.shapes]
+    dev = torch.device("cuda", 0)
+    params = synth.device_weights_torch(shapes, seed=1, device=dev, dtype=torch.bfloat16)
+    g0 = synth.device_grads_torch(shapes, ps.grad_kind, seed=10, device=dev, dtype=torch.bfloat16)
+    idx = {s: next(i for i, x in enumerate(shapes) if x == s) for s in check_shapes}
+    vecs = [i for i, s in enumerate(shapes) if len(s) == 1][:1]
+    sample = list(idx.values()) + vecs + ([shapes.index(spectrum_shape)] if spectrum_shape else [])
+    W0 = {i: _host(params[i]) for i in sample}
+    G0 = {i: _host(g0[i]) for i in sample}
+    eta_M, eta_L, lam = 1.0, 1e-3, 0.0
+    opt = L.LionMuon(params, period=period, eta_muon=eta_M, eta_lion=eta_L, weight_decay=lam)
+    opt.step(g0, 0)
+    torch.cuda.synchronize()
+    W1 = {i: _host(params[i]) for i in sample}
+    M1 = {i: _host(opt.momentum(i)) for i in sample}
+    for i in sample:
+        _, m_ref = O.lion_step_f32(np.zeros_like(G0[i]), G0[i], np.zeros_like(G0[i]), 0.9, 0.99, 0.0, 0.0,
+                                   w_dtype="f32")
+        np.testing.assert_array_equal(M1[i].view(np.uint32), m_ref.view(np.uint32))
+    for i in vecs:
+        w_ref, _ = O.lion_step_f32(W0[i], G0[i], np.zeros_like(G0[i]), 0.9, 0.99, eta_L, lam)
+        np.testing.assert_array_equal(bits(torch.from_numpy(W1[i]).to(torch.bfloat16)),
+                                      bits(torch.from_numpy(w_ref).to(torch.bfloat16)))
+    for shp, i in idx.items():
+        s = 0.2 * math.sqrt(max(shp))
+        o_gpu = (W0[i].astype(np.float64) - W1[i].astype(np.float64)) / (eta_M * s)
+        o_ref = O.ns_polynomial(0.1 * G0[i].astype(np.float64), 5, *O.NS_QUINTIC, 1e-7)
+        slack = 2.0 ** -9 * np.linalg.norm(W1[i]) / (eta_M * s) / np.linalg.norm(o_ref)
+        assert rel_fro(o_gpu, o_ref) <= NS_TOL + slack, (set_name, shp, rel_fro(o_gpu, o_ref))
+    if spectrum_shape:
+        i = shapes.index(spectrum_shape)
+        s = 0.2 * math.sqrt(max(spectrum_shape))
+        o = (W0[i].astype(np.float64) - W1[i].astype(np.float64)) / (eta_M * s)
+        gh = 0.1 * G0[i].astype(np.float64)
+        sig_g = np.sqrt(np.clip(np.linalg.eigvalsh(gh.T @ gh), 0, None))
+        sig_o = np.sqrt(np.clip(np.linalg.eigvalsh(o.T @ o), 0, None))
+        want = np.sort(O.ns_scalar_map(sig_g / (np.linalg.norm(sig_g) + 1e-7), 5, *O.NS_QUINTIC))
+        slack = 2.0 ** -9 * np.linalg.norm(W1[i]) / (eta_M * s) / np.linalg.norm(want)
+        assert np.linalg.norm(np.sort(sig_o) - want) / np.linalg.norm(want) <= NS_TOL + slack
+    # a Lion step for every parameter: bit-exact on the samples
+    t1 = 1 if period != 1 else None
+    if t1 is not None:
+        g1 = synth.device_grads_torch(shapes, ps.grad_kind, seed=11, device=dev, dtype=torch.bfloat16)
+        G1 = {i: _host(g1[i]) for i in sample}
+        opt.step(g1, t1)
+        torch.cuda.synchronize()
+        for i in sample:
+            w_ref, m_ref = O.lion_step_f32(W1[i], G1[i], M1[i], 0.9, 0.99, eta_L, lam)
+            np.testing.assert_array_equal(bits(params[i]), bits(torch.from_numpy(w_ref).to(torch.bfloat16)))
+            np.testing.assert_array_equal(_host(opt.momentum(i)).view(np.uint32), m_ref.view(np.uint32))
+        del g1
+    assert opt.status() == 0
+    opt.close()
+    del params, g0
+    torch.cuda.empty_cache()
+
+
+def test_124m_muon_then_lion_sampled():
+    _muon_then_lion("gpt2_124m", 2, [(768, 2304), (768, 768), (3072, 768)], spectrum_shape=(50304, 768))
+
+
+@pytest.mark.parametrize("period", [1, 4])
+def test_355m_muon_then_lion_sampled(period):
+    _muon_then_lion("gpt_355m", period, [(1024, 3072), (4096, 1024)])
+
+
+def test_stress_7b_muon_then_lion_sampled():
+    """The 7B-style stress set (7.79 G parameters, outlier gradients, P = 8):
+    the Muon direction of a 4096 x 4096 and a 14336 x 4096 matrix against the
+    fp64 recurrence, the Lion step bit-exact."""
+    _muon_then_lion("stress_7b", 8, [(4096, 4096), (14336, 4096)])

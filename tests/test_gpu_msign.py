@@ -147,3 +147,14 @@ def test_msign_coefficient_table_argument_errors():
     assert e.value.status == 1
     with pytest.raises(L.LionMuonError):
         L.msign_ns_coeffs(x, out, [(1.0, 0.0, 0.0)] * 65)
+
+
+@pytest.mark.parametrize("shape", [(200, 20000), (20000, 200), (768, 50304)])
+def test_msign_parity_long_k_split_gram(shape):
+    """A matrix whose Gram tiles are far longer than a CTA pair's share of
+    the launch: the Gram phase splits them along K into parts that add fp32
+    partial sums (split-K); the result must match the oracle recurrence."""
+    xh = host_tensor(synth.draw_matrix(shape, seed=5 + shape[0]), "bf16")
+    got = _msign(xh, "bf16")
+    want = O.ns_polynomial(stored_values(xh), 5, *QUINTIC, 1e-7)
+    assert rel_fro(got, want) <= TOL["bf16"]
