@@ -196,3 +196,42 @@ def test_stable_rank_argument_errors():
     with pytest.raises(L.LionMuonError) as e:
         L.LionMuon(wide, schedule=L.LM_SCHEDULE_STABLE_RANK)
     assert e.value.status == 6                           # LM_ERR_UNSUPPORTED
+
+
+def test_stable_rank_schedule_with_adamw_vectors():
+    """Both options together: matrices take the branch the rule selects (Lion
+    ones bit-exact), the vector takes AdamW (bit-exact against the same-order
+    float32 AdamW step with its update count t + 1), momentum bit-exact."""
+    import torch
+    from paper_2605_19811_gb300 import lionmuon as L
+    kinds = ["lowrank", "noise", "lowrank", "noise", "lowrank", "noise", None]
+    opt, params, W0, M0 = _state(SHAPES, kinds, 21, srank_alpha=0.08, vector_rule=L.LM_VECTOR_ADAMW)
+    r = np.random.default_rng(22)
+    W = [stored_values(host_tensor(w, "bf16")).astype(np.float32) for w in W0]
+    M = [m.copy() for m in M0]
+    V = np.zeros(SHAPES[-1], np.float32)
+    cfg = O.Config(schedule="stable_rank", srank_alpha=0.08)
+    for t in (3, 4):
+        G = [stored_values(host_tensor(r.normal(size=s) * 1e-4, "bf16")).astype(np.float32) for s in SHAPES]
+        opt.step([host_tensor(x, "bf16").cuda() for x in G], t)
+        torch.cuda.synchronize()
+        took, _ = opt.selection()
+        assert took[:6] == [True, False, True, False, True, False]
+        for i, s in enumerate(SHAPES):
+            if len(s) == 1:
+                w_ref, m_ref, V = O.adamw_step_f32(W[i], G[i], M[i], V, t + 1, 1e-3, 0.8, 0.999, 1e-8, 0.1)
+                np.testing.assert_array_equal(bits(params[i]), bits(torch.from_numpy(w_ref).to(torch.bfloat16)))
+                np.testing.assert_array_equal(stored_values(opt.second_moment(i)).astype(np.float32).view(np.uint32),
+                                              V.view(np.uint32))
+            elif not took[i]:
+                w_ref, m_ref = O.lion_step_f32(W[i], G[i], M[i], 0.9, 0.99, 2e-5, 0.1)
+                np.testing.assert_array_equal(bits(params[i]), bits(torch.from_numpy(w_ref).to(torch.bfloat16)))
+            else:
+                _, m_ref = O.lion_step_f32(W[i], G[i], M[i], 0.9, 0.99, 0.0, 0.0, w_dtype="f32")
+                assert O.srank_takes_muon(M[i].astype(np.float64), cfg)
+            np.testing.assert_array_equal(stored_values(opt.momentum(i)).astype(np.float32).view(np.uint32),
+                                          m_ref.view(np.uint32))
+            W[i] = stored_values(params[i]).astype(np.float32)
+            M[i] = m_ref
+    assert opt.status() == 0
+    opt.close()
