@@ -427,13 +427,22 @@ def run_ours(args):
     roof = None
     if ns_ms > 0 and n_muon > 0:
         achieved = fl / (ns_ms / 1e3) / 1e12
-        pk = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
-        traffic = kernel_traffic("ns_tc_kernel")
-        roof = {"bound": "tensor", "achieved": achieved, "peak": pk, "unit": "TFLOP/s",
-                "frac": achieved / pk, "traffic": traffic, "kernel": "ns_tc_kernel",
+        if args.precision == "bf16":
+            pk = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+            bound, kernel, peak_kind = "tensor", "ns_tc_kernel", f"bf16 sustained, {peak_src}"
+        else:
+            # fp32 FMA on the CUDA cores: SMs x 128 lanes x 2 FLOP x the maximum SM clock
+            sms = torch.cuda.get_device_properties(dev).multi_processor_count
+            mhz = (clk or {}).get("sm_max_mhz") or 2070.0
+            pk = sms * 128 * 2 * mhz * 1e6 / 1e12
+            bound, kernel = "alu", "ns_simt_kernel"
+            peak_kind = f"fp32 FMA, derived: {sms} SMs x 128 lanes x 2 FLOP x {mhz:.0f} MHz"
+        traffic = kernel_traffic(kernel)
+        roof = {"bound": bound, "achieved": achieved, "peak": pk, "unit": "TFLOP/s",
+                "frac": achieved / pk, "traffic": traffic, "kernel": kernel,
                 "per_launch_ms": ns_ms / max(ns_launches, 1),
                 "per_launch_tflop": fl / max(ns_launches, 1) / 1e12,
-                "peak_kind": f"bf16 sustained, {peak_src}",
+                "peak_kind": peak_kind,
                 "flops": "symmetric count 3 s^2 l + s^3 per matrix per NS iteration"}
     lion_roof = None
     if lion_ms > 0:

@@ -338,42 +338,44 @@ struct NsLayout {
   std::vector<size_t> off_offsets;
   size_t off_groups = 0;
   size_t off_norm = 0;
-  // split Gram tiles, per batch: (group, mat, tm, tn) of each target tile
-  std::vector<std::vector<std::array<int, 4>>> split_targets;
+  // split Gram tiles, per batch: (group, mat, tm, tn, first part, parts) of each target tile
+  std::vector<std::vector<std::array<int, 6>>> split_targets;
   std::vector<size_t> off_split_targets;
   size_t off_split_ws = 0;
 };
 
 // Split-K of the Gram phase: a tile longer than twice the average load of a
-// CTA pair (a long-K embedding Gram next to short hidden matrices, which would
-// otherwise set the length of the launch) is cut into parts of at most half
-// that load; each part is a tile of its own for the balancer and adds its
-// partial product into an fp32 workspace tile.  Tiles near the average stay
-// whole: splitting them costs the atomic additions and buys no balance.
-static void split_gram_tiles(const std::vector<NsGroup>& groups, int g0, std::vector<NsTile>& t,
-                             std::vector<std::array<int, 4>>& targets) {
+// worker (a CTA pair on the tensor-core path, a block on the fp32 path) - a
+// long-K embedding Gram next to short hidden matrices, which would otherwise
+// set the length of the launch - is cut into parts of at most half that load.
+// Each part is a tile of its own for the scheduler and writes its partial
+// product to a workspace tile of its own (slot = part index + 1); the finish
+// kernel adds the parts in order, so the result does not depend on timing.
+// Tiles near the average stay whole: splitting them buys no balance.
+static void split_gram_tiles(const std::vector<NsGroup>& groups, int g0, std::vector<NsTile>& t, int kslice,
+                             int workers, std::vector<std::array<int, 6>>& targets, int& nparts_total) {
   int64_t total = 0;
-  for (const NsTile& x : t) total += groups[g0 + x.group].l_pad / kTcBK;
-  const int pairs = std::max(1, tc_max_pairs());
-  const int64_t avg = total / pairs;
+  for (const NsTile& x : t) total += groups[g0 + x.group].l_pad / kslice;
+  const int64_t avg = total / std::max(1, workers);
   const int64_t part = std::max<int64_t>(8, avg / 2);
   std::vector<NsTile> out;
+  nparts_total = 0;
   for (const NsTile& x : t) {
-    const int nk = groups[g0 + x.group].l_pad / kTcBK;
-    if (nk <= 2 * avg || (int64_t)targets.size() >= 65535) {
+    const int nk = groups[g0 + x.group].l_pad / kslice;
+    if (nk <= 2 * avg || nparts_total + 64 > 65535) {
       out.push_back(x);
       continue;
     }
     const int nparts = (int)std::min<int64_t>(64, (nk + part - 1) / part);
-    targets.push_back({x.group, x.mat, x.tm, x.tn});
-    const int slot = (int)targets.size();   // 1-based
+    targets.push_back({x.group, x.mat, x.tm, x.tn, nparts_total, nparts});
     for (int k = 0; k < nparts; ++k) {
       NsTile y = x;
       y.kb0 = (uint16_t)((int64_t)nk * k / nparts);
       y.kb1 = (uint16_t)((int64_t)nk * (k + 1) / nparts);
-      y.slot = (uint16_t)slot;
+      y.slot = (uint16_t)(nparts_total + k + 1);
       out.push_back(y);
     }
+    nparts_total += nparts;
   }
   t.swap(out);
 }
@@ -401,11 +403,19 @@ static void layout_ns(std::vector<NsGroup>& groups, lm_dtype xdt, int nmat, Aren
       std::vector<NsTile> t;
       build_ns_tiles(groups, g0, b.ng, ph, bm, bn, t);
       std::vector<int> offs;
-      std::vector<std::array<int, 4>> targets;
-      if (xdt == LM_BF16 && ph == NS_GRAM) split_gram_tiles(groups, g0, t, targets);
+      std::vector<std::array<int, 6>> targets;
       if (ph == NS_GRAM) {
+        int nparts = 0;
+        if (xdt == LM_BF16) {
+          split_gram_tiles(groups, g0, t, kTcBK, tc_max_pairs(), targets, nparts);
+        } else {
+          int dev = 0, sms = 0;
+          cudaGetDevice(&dev);
+          cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+          split_gram_tiles(groups, g0, t, 16, 2 * std::max(sms, 1), targets, nparts);
+        }
         b.nsplit = (int)targets.size();
-        max_split = std::max(max_split, b.nsplit);
+        max_split = std::max(max_split, nparts);
         L.off_split_targets.push_back(ar.add(targets.size() * sizeof(NsSplitTarget)));
         L.split_targets.push_back(std::move(targets));
       }
@@ -436,7 +446,8 @@ static void layout_ns(std::vector<NsGroup>& groups, lm_dtype xdt, int nmat, Aren
   }
   L.off_groups = ar.add(groups.size() * sizeof(NsGroup));
   L.off_norm = ar.add((size_t)std::max(nmat, 1) * sizeof(double));
-  L.off_split_ws = ar.add((size_t)max_split * kTcBM * kTcBN * sizeof(float));
+  const size_t tile_floats = (xdt == LM_BF16) ? (size_t)kTcBM * kTcBN : (size_t)kSimtBM * kSimtBN;
+  L.off_split_ws = ar.add((size_t)max_split * tile_floats * sizeof(float));
 }
 
 static void bind_ns(NsEngine& E, char* base, const NsLayout& L, std::vector<char>& host_img) {
@@ -460,15 +471,21 @@ static void bind_ns(NsEngine& E, char* base, const NsLayout& L, std::vector<char
   for (size_t bi = 0; bi < E.batches.size(); ++bi) {
     const auto& tg = L.split_targets[bi];
     std::vector<NsSplitTarget> st(tg.size());
+    const bool tc = E.xdt == LM_BF16;
+    const size_t es = tc ? 2 : 4;                 // A: bf16 (tensor cores) or fp32
+    const int tile = tc ? kTcBM : kSimtBM;
     for (size_t k = 0; k < tg.size(); ++k) {
       const NsGroup& g = E.groups[E.batches[bi].g0 + tg[k][0]];
-      const size_t es = 2;   // bf16 A
       char* a = static_cast<char*>(g.A) + (size_t)tg[k][1] * g.s_pad * g.s_pad * es;
-      st[k].a_tile = a + ((size_t)tg[k][2] * kTcBM * g.s_pad + (size_t)tg[k][3] * kTcBN) * es;
+      const int tm = tg[k][2], tn = tg[k][3];
+      st[k].a_tile = a + ((size_t)tm * tile * g.s_pad + (size_t)tn * tile) * es;
+      st[k].a_mirror = a + ((size_t)tn * tile * g.s_pad + (size_t)tm * tile) * es;
       st[k].ld = g.s_pad;
-      st[k].nr = std::min(kTcBM, g.s_pad - tg[k][2] * kTcBM);
-      st[k].nc = std::min(kTcBN, g.s_pad - tg[k][3] * kTcBN);
-      st[k].slot = (int32_t)k;
+      st[k].nr = std::min(tile, g.s_pad - tm * tile);
+      st[k].nc = std::min(tile, g.s_pad - tn * tile);
+      st[k].first = tg[k][4];
+      st[k].nparts = tg[k][5];
+      st[k].diag = tm == tn ? 1 : 0;
     }
     E.batches[bi].split_targets = reinterpret_cast<NsSplitTarget*>(base + L.off_split_targets[bi]);
     if (!st.empty()) memcpy(host_img.data() + L.off_split_targets[bi], st.data(), st.size() * sizeof(NsSplitTarget));
@@ -549,18 +566,17 @@ static lm_status run_ns(const NsEngine& E, int steps, const NsCoeffs* coeffs, un
         const bool split = E.xdt == LM_BF16 && ph == NS_GRAM && b.nsplit > 0;
         cudaError_t e = timed(P, LM_KERNEL_NS_GRAM + ph, st, [&]() {
           if (E.xdt == LM_BF16) {
-            cudaError_t r = cudaSuccess;
-            if (split)   // the split tiles' partial sums start at zero
-              r = cudaMemsetAsync(E.d_split_ws, 0, (size_t)b.nsplit * kTcBM * kTcBN * sizeof(float), st);
-            if (r == cudaSuccess)
-              r = launch_ns_tc((NsPhase)ph, it, b.ng, E.groups.data() + b.g0, E.maps.data() + b.g0, b.tiles[ph],
+            cudaError_t r = launch_ns_tc((NsPhase)ph, it, b.ng, E.groups.data() + b.g0, E.maps.data() + b.g0, b.tiles[ph],
                                b.ntiles[ph], b.offsets[ph], b.npairs[ph], E.d_norm2, co, flags,
                                it == steps - 1 ? fuse : nullptr, st, active, E.d_split_ws);
             if (r == cudaSuccess && split) r = launch_ns_split_finish(b.split_targets, b.nsplit, E.d_split_ws, st);
             return r;
           }
-          return launch_ns_simt((NsPhase)ph, it, b.ng, E.d_groups + b.g0, b.tiles[ph], b.ntiles[ph],
-                                E.d_norm2, co, st, active);
+          cudaError_t r = launch_ns_simt((NsPhase)ph, it, b.ng, E.d_groups + b.g0, b.tiles[ph], b.ntiles[ph],
+                                         E.d_norm2, co, st, active, E.d_split_ws);
+          if (r == cudaSuccess && ph == NS_GRAM && b.nsplit > 0)
+            r = launch_ns_split_finish_f32(b.split_targets, b.nsplit, E.d_split_ws, st);
+          return r;
         });
         if (e != cudaSuccess) return cuda_fail(e, "Newton-Schulz launch");
       }

@@ -128,18 +128,23 @@ struct NsGroup {
 struct NsTile {
   uint16_t group, mat, tm, tn;
   // Split-K (Gram phase only): K blocks [kb0, kb1) of the tile, kb1 == 0 for
-  // all of them; slot != 0: the partial product is added in fp32 into
-  // workspace tile slot - 1 instead of being stored (NsSplitTarget finishes it).
+  // all of them; slot != 0: the partial product is written in fp32 to
+  // workspace tile slot - 1 instead of A (NsSplitTarget sums the parts).
   uint16_t kb0, kb1, slot, pad;
 };
-// A split Gram tile: the fp32 sum of its parts in workspace tile `slot`
-// becomes bf16 A[tm * 256 + r][tn * 256 + c] for r < nr, c < nc (the part of
-// the tile inside s_pad x s_pad; a tile is 256 x 256 floats).
+// A split Gram tile (tile edge `tile`: 256 tensor-core, 128 fp32 path): the
+// parts in workspace tiles first .. first + nparts - 1 are summed in that
+// order (so the result does not depend on timing) and written to A at
+// (tm * tile + r, tn * tile + c) for r < nr, c < nc; the fp32 path, which keeps
+// A whole, also writes the mirror (tn * tile + c, tm * tile + r), and on a
+// diagonal tile only c >= r.
 struct NsSplitTarget {
-  void* a_tile;           // bf16 element (tm * 256, tn * 256) of the matrix's A
+  void* a_tile;           // element (tm * tile, tn * tile) of the matrix's A
+  void* a_mirror;         // element (tn * tile, tm * tile) (fp32 path)
   int32_t ld;             // s_pad
   int32_t nr, nc;         // rows / columns of the tile inside the padded matrix
-  int32_t slot;
+  int32_t first, nparts;
+  int32_t diag;
 };
 constexpr int kMaxGroupsTc = 8;   // groups per tensor-core launch
 
@@ -184,15 +189,17 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
                          const int* offsets, int npairs, const double* norm2, NsCoeffs co,
                          unsigned* flags, const FuseFinal* fuse, cudaStream_t st,
                          const unsigned char* active = nullptr, float* split_ws = nullptr);
-// After a Gram launch with split tiles: A tiles from the fp32 workspace.
+// After a Gram launch with split tiles: bf16 A tiles from the fp32 parts.
 cudaError_t launch_ns_split_finish(const NsSplitTarget* targets, int n, const float* ws, cudaStream_t st);
 
 // fp32 CUDA-core path.
-constexpr int kSimtBM = 64, kSimtBN = 64;
+constexpr int kSimtBM = 128, kSimtBN = 128;
 int simt_pad(int x);
 cudaError_t launch_ns_simt(NsPhase ph, int iter, int ngroups, const NsGroup* dgroups,
                            const NsTile* tiles, int ntiles, const double* norm2, NsCoeffs co,
-                           cudaStream_t st, const unsigned char* active = nullptr);
+                           cudaStream_t st, const unsigned char* active = nullptr, float* split_ws = nullptr);
+// fp32 path: A tiles (and mirrors) from the fp32 parts of split Gram tiles.
+cudaError_t launch_ns_split_finish_f32(const NsSplitTarget* targets, int n, const float* ws, cudaStream_t st);
 // active (both NS paths): NULL, or active[first_mat + mat] != 0 for the
 // matrices whose tiles run; tiles of the others are skipped by every role.
 

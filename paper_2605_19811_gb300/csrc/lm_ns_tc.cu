@@ -648,13 +648,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         const int j0 = t.tn * BN + ch * 32;
         if (!warp_in || j0 >= jmax) continue;   // beyond the padded matrix
         if (split) {
-          // partial Gram product of a split tile: add into the fp32 workspace
+          // partial Gram product of a split tile: its own fp32 workspace tile
           float* wrow = p.split_ws + (size_t)(t.slot - 1) * (BM * BN) + (size_t)((int)rank * kHalf + row) * BN +
                         ch * 32;
 #pragma unroll
-          for (int e = 0; e < 32; ++e) {
-            const int j = j0 + e;
-            if (i < nrows && j < ncols) atomicAdd(wrow + e, __uint_as_float(r[e]) * nscale);
+          for (int e = 0; e < 32; e += 4) {
+            float o[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+              const int j = j0 + e + u;
+              o[u] = (i < nrows && j < ncols) ? __uint_as_float(r[e + u]) * nscale : 0.f;
+            }
+            *reinterpret_cast<float4*>(wrow + e) = make_float4(o[0], o[1], o[2], o[3]);
           }
           continue;
         }
@@ -768,15 +773,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   }
 }
 
-// Split Gram tiles: bf16 A tile = the fp32 sum of the parts (already scaled).
+// Split Gram tiles: bf16 A tile = the sum of the fp32 parts (already scaled),
+// added in part order.
 __global__ void __launch_bounds__(256) ns_split_finish_kernel(const NsSplitTarget* __restrict__ targets,
                                                               const float* __restrict__ ws) {
   const NsSplitTarget T = targets[blockIdx.y];
-  const float* src = ws + (size_t)T.slot * (BM * BN);
   __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(T.a_tile);
   for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < BM * BN; e += gridDim.x * blockDim.x) {
     const int r = e / BN, c = e % BN;
-    if (r < T.nr && c < T.nc) dst[(size_t)r * T.ld + c] = __float2bfloat16_rn(src[e]);
+    if (r >= T.nr || c >= T.nc) continue;
+    float sum = 0.f;
+    for (int k = 0; k < T.nparts; ++k) sum += ws[(size_t)(T.first + k) * (BM * BN) + e];
+    dst[(size_t)r * T.ld + c] = __float2bfloat16_rn(sum);
   }
 }
 
