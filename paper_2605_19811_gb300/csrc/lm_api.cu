@@ -568,7 +568,7 @@ static lm_status run_ns(const NsEngine& E, int steps, const NsCoeffs* coeffs, un
           if (E.xdt == LM_BF16) {
             cudaError_t r = launch_ns_tc((NsPhase)ph, it, b.ng, E.groups.data() + b.g0, E.maps.data() + b.g0, b.tiles[ph],
                                b.ntiles[ph], b.offsets[ph], b.npairs[ph], E.d_norm2, co, flags,
-                               it == steps - 1 ? fuse : nullptr, st, active, E.d_split_ws);
+                               it == steps - 1 ? fuse : nullptr, st, active, split ? E.d_split_ws : nullptr);
             if (r == cudaSuccess && split) r = launch_ns_split_finish(b.split_targets, b.nsplit, E.d_split_ws, st);
             return r;
           }

@@ -189,6 +189,7 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
                          const int* offsets, int npairs, const double* norm2, NsCoeffs co,
                          unsigned* flags, const FuseFinal* fuse, cudaStream_t st,
                          const unsigned char* active = nullptr, float* split_ws = nullptr);
+// split_ws: non-NULL only for a Gram launch whose tiles include split-K parts.
 // After a Gram launch with split tiles: bf16 A tiles from the fp32 parts.
 cudaError_t launch_ns_split_finish(const NsSplitTarget* targets, int n, const float* ws, cudaStream_t st);
 

@@ -415,9 +415,10 @@ __device__ __forceinline__ bool mma_range(int& stage, uint32_t& ph, uint8_t* sme
 }
 
 // ------------------------------- the kernel ---------------------------------
-// kMasked: the launch carries a per-matrix mask (stable-rank selection); the
-// unmasked instantiation keeps the fixed-period path free of the test.
-template <bool kMasked>
+// kMasked: the launch carries a per-matrix mask (stable-rank selection);
+// kSplit: its Gram tiles include split-K parts.  The plain instantiation keeps
+// the common path free of both.
+template <bool kMasked, bool kSplit>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     ns_tc_kernel(const __grid_constant__ TcParams p) {
   extern __shared__ uint8_t smem_raw[];
@@ -636,7 +637,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const int r0 = t.tm * BM + (int)rank * kHalf + q * 32;   // first row of this warp
       const int i = r0 + lane;
       const bool warp_in = r0 < row_lim;        // rows past the padded matrix are skipped
-      const bool split = phase == NS_GRAM && t.slot != 0;
+      const bool split = kSplit && phase == NS_GRAM && t.slot != 0;
       if (fused && lane == 0 && q == 0 && half == 0 && rank == 0 && t.tm == 0 && t.tn == 0 &&
           !isfinite((float)sqrt(p.norm2[g.first_mat + t.mat])))
         atomicOr(p.flags, LM_FLAG_NONFINITE);
@@ -881,10 +882,17 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
   if (ngroups < 1 || ngroups > kMaxGroupsTc) return cudaErrorInvalidValue;
   static bool attr_set = false;
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(ns_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(ns_tc_kernel<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)kSmemBytes);
     if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(ns_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+      e = cudaFuncSetAttribute(ns_tc_kernel<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               (int)kSmemBytes);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(ns_tc_kernel<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               (int)kSmemBytes);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(ns_tc_kernel<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               (int)kSmemBytes);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
@@ -912,10 +920,14 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
   }
   const int grid = 2 * (pairs > 0 ? pairs : 1);
   count_launch();
-  if (active != nullptr)
-    ns_tc_kernel<true><<<grid, kThreads, kSmemBytes, st>>>(prm);
-  else
-    ns_tc_kernel<false><<<grid, kThreads, kSmemBytes, st>>>(prm);
+  const bool split = split_ws != nullptr && ph == NS_GRAM;
+  if (active != nullptr) {
+    if (split) ns_tc_kernel<true, true><<<grid, kThreads, kSmemBytes, st>>>(prm);
+    else ns_tc_kernel<true, false><<<grid, kThreads, kSmemBytes, st>>>(prm);
+  } else {
+    if (split) ns_tc_kernel<false, true><<<grid, kThreads, kSmemBytes, st>>>(prm);
+    else ns_tc_kernel<false, false><<<grid, kThreads, kSmemBytes, st>>>(prm);
+  }
   return cudaGetLastError();
 }
 
