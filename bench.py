@@ -50,6 +50,8 @@ def parse_args():
                     help="period: Algorithm 1's fixed P; srank: Appendix G's stable-rank selection")
     ap.add_argument("--srank-alpha", type=float, default=0.01)
     ap.add_argument("--srank-iters", type=int, default=5)
+    ap.add_argument("--vector-rule", choices=["lion", "adamw"], default="lion",
+                    help="1-D parameters: the Lion step, or the AdamW fallback of Section 3")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     return ap.parse_args()
@@ -314,11 +316,12 @@ def run_ours(args):
 
     prec = L.LM_BF16 if args.precision == "bf16" else L.LM_F32
     srank = args.schedule == "srank"
+    extra = {"vector_rule": L.LM_VECTOR_ADAMW} if args.vector_rule == "adamw" else {}
     if srank:
         opt = L.LionMuon(params, period=P, ns_precision=prec, schedule=L.LM_SCHEDULE_STABLE_RANK,
-                         srank_alpha=args.srank_alpha, srank_iters=args.srank_iters)
+                         srank_alpha=args.srank_alpha, srank_iters=args.srank_iters, **extra)
     else:
-        opt = L.LionMuon(params, period=P, ns_precision=prec)
+        opt = L.LionMuon(params, period=P, ns_precision=prec, **extra)
     n = len(params)
     gdesc = (L.LmTensor * n)(*[L.tensor_desc(g) for g in grads])
     stream = torch.cuda.current_stream()
@@ -483,6 +486,7 @@ def run_ours(args):
             "dtype": "bf16" if args.precision == "bf16" else "f32", "data": "synthetic",
             "config": {"workload": args.set, "params": numel, "matrices": len(mats),
                        "period": None if srank else P, "ns_steps": 5, "ns_precision": args.precision,
+                       **({"vector_rule": "adamw"} if args.vector_rule == "adamw" else {}),
                        **({"schedule": "stable_rank", "srank_alpha": args.srank_alpha,
                            "srank_iters": args.srank_iters,
                            "muon_matrices_last_step": sum(1 for i, s in enumerate(shapes)
