@@ -65,6 +65,18 @@ typedef struct {
 /* Device status flags read by lm_get_status. */
 #define LM_FLAG_NONFINITE 0x1u /* a matrix direction had a non-finite Frobenius norm */
 #define LM_FLAG_TIMEOUT 0x2u   /* a bounded device wait gave up */
+#define LM_FLAG_GUARD 0x4u     /* states created with LM_DEBUG=1: a workspace guard band was overwritten */
+
+/* Environment switches, read by lm_create for that state (host side; the
+ * device code is the same):
+ *   LM_DEBUG=1          a 256-byte guard band after every part of the state's
+ *                       workspace, filled with a fixed pattern and compared by
+ *                       lm_get_status (LM_FLAG_GUARD if one was overwritten)
+ *   LM_NVTX=1           NVTX ranges named after the kernel families around the
+ *                       library's launches
+ *   LM_FAULT=oom        lm_create returns LM_ERR_OOM as if the device allocation
+ *                       had failed (to exercise callers' error paths)
+ *   LM_NS_FORCE_FP32=1  the fp32 Newton-Schulz path whatever ns_precision says */
 
 /* Hyper-parameters: the Require line of Algorithm 1 plus the NS reading.
  * beta1, beta2 in [0, 1); eta_* >= 0; weight_decay >= 0;

@@ -8,12 +8,15 @@
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <limits>
 #include <map>
 #include <string>
 #include <tuple>
 #include <vector>
+
+#include <nvtx3/nvToolsExt.h>
 
 #include "lm_internal.h"
 
@@ -158,16 +161,41 @@ MuonConsts muon_consts(const lm_config& c) {
 }
 
 // Device-memory arena: one cudaMalloc, sub-allocated with 256-byte alignment.
+// With guard bands on (LM_DEBUG=1 when the state is created), every part is
+// followed by kGuardBytes of a fixed pattern, checked by lm_get_status.
+constexpr size_t kGuardBytes = 256;
+constexpr unsigned char kGuardByte = 0xA5;
 struct Arena {
   std::vector<std::pair<size_t, size_t>> parts;  // (offset, bytes)
   size_t total = 0;
+  bool guard = false;
+  std::vector<size_t> guards;                     // offsets of the guard bands
   size_t add(size_t bytes) {
     total = align_up(total, 256);
     size_t off = total;
     total += std::max<size_t>(bytes, 1);
+    if (guard) {
+      total = align_up(total, 256);
+      guards.push_back(total);
+      total += kGuardBytes;
+    }
     return off;
   }
 };
+
+// Debug switches read from the environment when a state is created (host
+// side only; none of them changes the device code):
+//   LM_DEBUG=1         guard bands around every workspace part
+//   LM_NVTX=1          NVTX ranges around every kernel family's launches
+//   LM_FAULT=oom       lm_create fails with LM_ERR_OOM as if the allocation had
+//   LM_NS_FORCE_FP32=1 the fp32 Newton-Schulz path whatever ns_precision says
+static bool env_is(const char* name, const char* value) {
+  const char* v = std::getenv(name);
+  return v != nullptr && std::strcmp(v, value) == 0;
+}
+static std::atomic<bool> g_nvtx{false};
+static const char* const kFamilyNames[LM_KERNEL_FAMILIES] = {
+    "lion", "momentum_norm", "ns_gram", "ns_poly", "ns_apply", "finalize", "other", "adamw", "srank"};
 
 constexpr int64_t kLionChunk = 32768;   // elements per Lion work chunk
 
@@ -533,7 +561,7 @@ struct Profiler {
 
 // Launch f() on st; with profiling on, bracket it by events of family fam.
 template <typename F>
-static cudaError_t timed(Profiler* P, int fam, cudaStream_t st, F&& f) {
+static cudaError_t timed_events(Profiler* P, int fam, cudaStream_t st, F&& f) {
   if (P == nullptr || !P->on) return f();
   cudaEvent_t a = P->next(), b = P->next();
   if (a == nullptr || b == nullptr) return f();
@@ -541,6 +569,16 @@ static cudaError_t timed(Profiler* P, int fam, cudaStream_t st, F&& f) {
   cudaError_t e = f();
   cudaEventRecord(b, st);
   P->recs.push_back({fam, a, b});
+  return e;
+}
+
+// timed_events plus an NVTX range named after the family when LM_NVTX=1.
+template <typename F>
+static cudaError_t timed(Profiler* P, int fam, cudaStream_t st, F&& f) {
+  const bool nvtx = g_nvtx.load(std::memory_order_relaxed);
+  if (nvtx) nvtxRangePushA(kFamilyNames[fam]);
+  cudaError_t e = timed_events(P, fam, st, std::forward<F>(f));
+  if (nvtx) nvtxRangePop();
   return e;
 }
 
@@ -629,6 +667,10 @@ struct lm_state {
   double* d_srank = nullptr;            // per matrix id: the estimate
   std::vector<int> mat_param_of;        // matrix id -> parameter index
   int64_t last_t = -1;
+  // LM_DEBUG guard bands: device list of their offsets
+  bool debug = false;
+  size_t* d_guard_offs = nullptr;
+  int n_guards = 0;
   int lion_grid[2] = {0, 0};
   int nmat = 0;
   MatDesc* d_mats = nullptr;
@@ -711,7 +753,9 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
   s->cfg.ns_coeffs = nullptr;   // the caller's table is not kept
   s->n = n;
   s->params.assign(params, params + n);
-  s->ns.xdt = (cfg->ns_precision == LM_F32) ? LM_F32 : LM_BF16;
+  s->ns.xdt = (cfg->ns_precision == LM_F32 || env_is("LM_NS_FORCE_FP32", "1")) ? LM_F32 : LM_BF16;
+  s->debug = env_is("LM_DEBUG", "1");
+  if (env_is("LM_NVTX", "1")) g_nvtx.store(true);
 
   // matrices and their shape groups
   std::vector<int> mat_param;
@@ -727,6 +771,7 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
 
   // arena layout
   Arena ar;
+  ar.guard = s->debug;
   s->mom_off.resize(n);
   size_t mom_elems_aligned = 0;
   for (int i = 0; i < n; ++i) {
@@ -881,6 +926,16 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
     for (auto& v : sr_items) off_sritems.push_back(ar.add(v.size() * sizeof(SrItem)));
   }
 
+  size_t off_guard_list = 0;
+  std::vector<size_t> guard_offs;
+  if (s->debug) {
+    off_guard_list = ar.add(ar.guards.size() * sizeof(size_t) + sizeof(size_t));
+    guard_offs = ar.guards;   // now including the list's own guard
+  }
+  if (env_is("LM_FAULT", "oom")) {
+    delete s;
+    return fail(LM_ERR_OOM, "injected allocation failure (LM_FAULT=oom)");
+  }
   cudaError_t e = cudaMalloc(&s->base, ar.total);
   if (e != cudaSuccess) {
     delete s;
@@ -888,6 +943,12 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
   }
   s->bytes = ar.total;
   std::vector<char> img(ar.total, 0);
+  if (s->debug) {
+    for (size_t g : guard_offs) memset(img.data() + g, kGuardByte, kGuardBytes);
+    memcpy(img.data() + off_guard_list, guard_offs.data(), guard_offs.size() * sizeof(size_t));
+    s->d_guard_offs = reinterpret_cast<size_t*>(s->base + off_guard_list);
+    s->n_guards = (int)guard_offs.size();
+  }
   char* base = s->base;
   s->mom = reinterpret_cast<float*>(base + off_mom);
   s->d_grads = reinterpret_cast<const void**>(base + off_grads);
@@ -1078,6 +1139,17 @@ static lm_status run_srank(lm_state* s, cudaStream_t stream) {
   });
   if (e != cudaSuccess) return cuda_fail(e, "selection launch");
   return LM_OK;
+}
+
+// LM_DEBUG: block k compares guard band k (kGuardBytes at offs[k]) with the
+// fill pattern and raises LM_FLAG_GUARD if any byte changed.
+__global__ void guard_check_kernel(const unsigned char* base, const size_t* offs, unsigned* flags) {
+  const uint4* g = reinterpret_cast<const uint4*>(base + offs[blockIdx.x]);
+  const uint32_t pat = 0x01010101u * kGuardByte;
+  for (int k = threadIdx.x; k < (int)(kGuardBytes / 16); k += blockDim.x) {
+    const uint4 v = g[k];
+    if (v.x != pat || v.y != pat || v.z != pat || v.w != pat) atomicOr(flags, LM_FLAG_GUARD);
+  }
 }
 
 // AdamW over the 1-D parameters of both dtypes (LM_VECTOR_ADAMW).
@@ -1293,6 +1365,13 @@ lm_status lm_set_momentum(lm_state* s, int i, const lm_tensor* src, void* cuda_s
 
 lm_status lm_get_status(lm_state* s, uint32_t* device_flags) {
   if (s == nullptr || device_flags == nullptr) return fail(LM_ERR_INVALID_ARG, "state/flags is NULL");
+  if (s->debug && s->n_guards > 0) {
+    count_launch();
+    guard_check_kernel<<<s->n_guards, 64, 0, s->last_stream>>>(reinterpret_cast<const unsigned char*>(s->base),
+                                                                s->d_guard_offs, s->d_flags);
+    cudaError_t g = cudaGetLastError();
+    if (g != cudaSuccess) return cuda_fail(g, "guard check launch");
+  }
   cudaError_t e = cudaStreamSynchronize(s->last_stream);
   if (e != cudaSuccess) return cuda_fail(e, "stream synchronize");
   unsigned f = 0;

@@ -18,6 +18,7 @@ LM_F32 = 0
 LM_BF16 = 1
 LM_FLAG_NONFINITE = 0x1
 LM_FLAG_TIMEOUT = 0x2
+LM_FLAG_GUARD = 0x4
 
 STATUS_NAMES = {0: "LM_OK", 1: "LM_ERR_INVALID_ARG", 2: "LM_ERR_DTYPE", 3: "LM_ERR_ALIGN",
                 4: "LM_ERR_OOM", 5: "LM_ERR_CUDA", 6: "LM_ERR_UNSUPPORTED", 7: "LM_ERR_TIMEOUT"}
