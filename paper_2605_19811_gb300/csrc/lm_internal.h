@@ -164,8 +164,8 @@ struct TcGroupMaps {
   CUtensorMap xk[2];    // K-major operand / aux loads: box 64 x 128
   CUtensorMap a;
   CUtensorMap b;
-  CUtensorMap xmn[2];   // MN-major operand loads: box 64 x 64
-  CUtensorMap amn;      // transposed reads of stored A / B tiles: box 64 x 64
+  CUtensorMap xmn[2];   // MN-major operand loads: 4-D box (64, 64, 2), a 128-wide half
+  CUtensorMap amn;      // transposed reads of stored A / B tiles: the same 4-D box
   CUtensorMap bmn;
   CUtensorMap xst[2];   // result stores: box 64 x 32
   CUtensorMap ast;

@@ -150,6 +150,17 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, u
       "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(c0), "r"(c1), "r"(c2)
       : "memory");
 }
+// 4-D tiled TMA load, signalled like tma_load_3d, for the MN-major operand
+// maps with dimensions (64 MN, K, MN / 64, matrix): one copy fills the two
+// 64-wide swizzle atoms of a 128-wide operand half.
+__device__ __forceinline__ void tma_load_4d(void* dst, const CUtensorMap* map, uint32_t bar_cluster,
+                                            int c0, int c1, int c2, int c3) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4, %5, %6}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+      : "memory");
+}
 // 3-D tiled TMA load signalling this CTA's own mbarrier.
 __device__ __forceinline__ void tma_load_3d_local(void* dst, const CUtensorMap* map, uint64_t* bar,
                                                   int c0, int c1, int c2) {
@@ -348,8 +359,9 @@ __device__ __forceinline__ uint32_t pack_bf2(float lo, float hi) {
 
 // Producer k-loop of one tile, specialised on the operand layouts (a loop
 // with per-block layout branches measured ~12% slower end to end).
-// K-major operand half: one 64 (K) x 128 box; MN-major: two 64 (MN) x 64 (K)
-// boxes.  Returns false if a wait gave up.
+// K-major operand half: one 64 (K) x 128 box; MN-major: one 4-D box that
+// fills both 64 (MN) x 64 (K) swizzle atoms (one copy instead of two
+// measured ~2% faster).  Returns false if a wait gave up.
 struct ProducerRing {
   int stage;
   uint32_t ph;
@@ -368,18 +380,10 @@ __device__ __forceinline__ bool produce_range(ProducerRing& R, uint8_t* smem, ui
     if (rank == 0) mbar_arrive_expect_tx(&full[R.stage], 2 * kStageBytes);
     R.armed[R.stage] = (int)R.ph;
     const int k0 = kb * BK;
-    if (!AMN) {
-      tma_load_3d(sa, map_a, fb, k0, row_a, mat);
-    } else {
-      tma_load_3d(sa, map_a, fb, row_a, k0, mat);
-      tma_load_3d(sa + 64 * BK * 2, map_a, fb, row_a + 64, k0, mat);
-    }
-    if (!BMN) {
-      tma_load_3d(sb, map_b, fb, k0, col_b, mat);
-    } else {
-      tma_load_3d(sb, map_b, fb, col_b, k0, mat);
-      tma_load_3d(sb + 64 * BK * 2, map_b, fb, col_b + 64, k0, mat);
-    }
+    if (!AMN) tma_load_3d(sa, map_a, fb, k0, row_a, mat);
+    else tma_load_4d(sa, map_a, fb, 0, k0, row_a >> 6, mat);
+    if (!BMN) tma_load_3d(sb, map_b, fb, k0, col_b, mat);
+    else tma_load_4d(sb, map_b, fb, 0, k0, col_b >> 6, mat);
     if (++R.stage == kStages) {
       R.stage = 0;
       R.ph ^= 1u;
@@ -830,6 +834,22 @@ cudaError_t encode_3d(CUtensorMap* m, void* base, uint64_t inner, uint64_t rows,
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
+// MN-major operand map: dimensions (64, rows, inner / 64, count), the third
+// 128 bytes apart, box (64, box_k, 2, 1): one copy reads a 128-wide half.
+cudaError_t encode_mn4d(CUtensorMap* m, void* base, uint64_t inner, uint64_t rows, uint64_t count,
+                        uint32_t box_k) {
+  PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode_fn();
+  if (enc == nullptr) return cudaErrorNotSupported;
+  const cuuint64_t dims[4] = {64, rows, inner / 64, count};
+  const cuuint64_t strides[3] = {inner * 2, 128, inner * rows * 2};
+  const cuuint32_t box[4] = {64, box_k, 2, 1};
+  const cuuint32_t estr[4] = {1, 1, 1, 1};
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, base, dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
 }  // namespace
 
 cudaError_t launch_bounded_wait_probe(uint64_t limit_ns, unsigned* flags, cudaStream_t st) {
@@ -848,12 +868,12 @@ cudaError_t tc_encode_group_maps(const NsGroup& g, TcGroupMaps* maps) {
   for (int b = 0; b < 2; ++b) {
     if ((e = encode_3d(&maps->xk[b], g.X[b], inner, rows, g.count, BK, kHalf)) != cudaSuccess) return e;
     if ((e = encode_3d(&maps->xst[b], g.X[b], inner, rows, g.count, 64, 32)) != cudaSuccess) return e;
-    if ((e = encode_3d(&maps->xmn[b], g.X[b], inner, rows, g.count, 64, BK)) != cudaSuccess) return e;
+    if ((e = encode_mn4d(&maps->xmn[b], g.X[b], inner, rows, g.count, BK)) != cudaSuccess) return e;
   }
   if ((e = encode_3d(&maps->a, g.A, g.s_pad, g.s_pad, g.count, BK, kHalf)) != cudaSuccess) return e;
   if ((e = encode_3d(&maps->b, g.B, g.s_pad, g.s_pad, g.count, BK, kHalf)) != cudaSuccess) return e;
-  if ((e = encode_3d(&maps->amn, g.A, g.s_pad, g.s_pad, g.count, 64, BK)) != cudaSuccess) return e;
-  if ((e = encode_3d(&maps->bmn, g.B, g.s_pad, g.s_pad, g.count, 64, BK)) != cudaSuccess) return e;
+  if ((e = encode_mn4d(&maps->amn, g.A, g.s_pad, g.s_pad, g.count, BK)) != cudaSuccess) return e;
+  if ((e = encode_mn4d(&maps->bmn, g.B, g.s_pad, g.s_pad, g.count, BK)) != cudaSuccess) return e;
   if ((e = encode_3d(&maps->ast, g.A, g.s_pad, g.s_pad, g.count, 64, 32)) != cudaSuccess) return e;
   if ((e = encode_3d(&maps->bst, g.B, g.s_pad, g.s_pad, g.count, 64, 32)) != cudaSuccess) return e;
   return cudaSuccess;
