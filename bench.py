@@ -363,59 +363,81 @@ def run_ours(args):
     # ---- end to end through the public API with host buffers ----
     # Every step copies its gradients in from pinned host memory and reads
     # the updated parameters back.  The copies are pipelined across steps:
-    # the gradients of step t+1 go into a second device buffer while step t
-    # and the read-back of its parameters run; step t+1 starts once its
-    # gradients are in and the read-back of W_t is done (W is updated in place).
+    # the gradients of step t+1 go into a free device buffer (three in a
+    # ring, so that the copy also overlaps a long Muon step followed by a
+    # short Lion step) while earlier steps run; after step t a
+    # device-to-device copy snapshots the parameters (W is updated in place
+    # by step t+1), and the snapshot is read back to the host while step t+1
+    # runs.  Warm-up steps run through the same pipeline before the timed
+    # region, as in a training loop that reuses its buffers.
     e2e = None
     if not args.no_e2e:
         g_host = torch.empty(flat_bytes // 2, dtype=torch.bfloat16, pin_memory=True)
         w_host = torch.empty(flat_bytes // 2, dtype=torch.bfloat16, pin_memory=True)
         g_host.copy_(gflat)
-        gflat2 = torch.empty_like(gflat)
-        gdesc2 = (L.LmTensor * n)(*[L.tensor_desc(g) for g in views(gflat2)])
-        gbufs, gdescs = (gflat, gflat2), (gdesc, gdesc2)
+        NG = 3
+        gbufs = [gflat] + [torch.empty_like(gflat) for _ in range(NG - 1)]
+        gdescs = [gdesc] + [(L.LmTensor * n)(*[L.tensor_desc(g) for g in views(gb)]) for gb in gbufs[1:]]
+        snaps = (torch.empty_like(wflat), torch.empty_like(wflat))
         # three non-default streams: the legacy default stream would serialise them
         s_cmp, s_h2d, s_d2h = (torch.cuda.Stream(device=dev) for _ in range(3))
         sh_cmp = ctypes.c_void_p(s_cmp.cuda_stream)
-        ev_in = [torch.cuda.Event() for _ in range(2)]      # gradients of a buffer are in
-        ev_used = [torch.cuda.Event() for _ in range(2)]    # the step reading a buffer is done
-        ev_out = torch.cuda.Event()                         # parameters read back
+        ev_in = [torch.cuda.Event() for _ in range(NG)]     # gradients of a buffer are in
+        ev_used = [torch.cuda.Event() for _ in range(NG)]   # the step reading a buffer is done
+        ev_snap = [torch.cuda.Event() for _ in range(2)]    # parameters copied into a snapshot
+        ev_out = [torch.cuda.Event() for _ in range(2)]     # a snapshot read back to the host
+        def pipelined(nsteps, t0):
+            """nsteps pipelined steps from step t0; returns the (start, end) events on s_cmp."""
+            ev_a, ev_b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            ev_a.record(s_cmp)
+            s_h2d.wait_event(ev_a)
+            with torch.cuda.stream(s_h2d):
+                gbufs[0].copy_(g_host, non_blocking=True)
+                ev_in[0].record(s_h2d)
+            for i in range(nsteps):
+                b, sb = i % NG, i & 1
+                if i + 1 < nsteps:          # next step's gradients, once their buffer is free
+                    nb = (i + 1) % NG
+                    if i + 1 >= NG:
+                        s_h2d.wait_event(ev_used[nb])
+                    with torch.cuda.stream(s_h2d):
+                        gbufs[nb].copy_(g_host, non_blocking=True)
+                        ev_in[nb].record(s_h2d)
+                s_cmp.wait_event(ev_in[b])
+                opt.step_descs(gdescs[b], n, t0 + i, sh_cmp)
+                ev_used[b].record(s_cmp)
+                if i >= 2:                  # the snapshot buffer's previous read-back is done
+                    s_cmp.wait_event(ev_out[sb])
+                with torch.cuda.stream(s_cmp):
+                    snaps[sb].copy_(wflat, non_blocking=True)
+                    ev_snap[sb].record(s_cmp)
+                s_d2h.wait_event(ev_snap[sb])
+                with torch.cuda.stream(s_d2h):
+                    w_host.copy_(snaps[sb], non_blocking=True)
+                    ev_out[sb].record(s_d2h)
+            s_cmp.wait_event(ev_out[(nsteps - 1) & 1])
+            ev_b.record(s_cmp)
+            return ev_a, ev_b
+
+        # untimed warm-up passes of the same pipeline (copies in both directions
+        # at once, streams, events), then the timed steps; whole periods from a
+        # Muon step in both
+        t_e2e = base + args.steps
+        nwarm = max(2, ((args.warmup + P - 1) // P) * P if P > 0 and not srank else args.warmup)
+        pipelined(nwarm, t_e2e)
+        t_e2e += nwarm
         torch.cuda.synchronize()
         barrier()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(s_cmp)
-        s_h2d.wait_event(e0)
-        with torch.cuda.stream(s_h2d):
-            gbufs[0].copy_(g_host, non_blocking=True)
-            ev_in[0].record(s_h2d)
-        for i in range(args.steps):
-            b = i & 1
-            if i + 1 < args.steps:          # next step's gradients, once the buffer is free
-                nb = b ^ 1
-                if i >= 1:
-                    s_h2d.wait_event(ev_used[nb])
-                with torch.cuda.stream(s_h2d):
-                    gbufs[nb].copy_(g_host, non_blocking=True)
-                    ev_in[nb].record(s_h2d)
-            s_cmp.wait_event(ev_in[b])
-            if i >= 1:
-                s_cmp.wait_event(ev_out)
-            opt.step_descs(gdescs[b], n, base + args.steps + i, sh_cmp)
-            ev_used[b].record(s_cmp)
-            s_d2h.wait_event(ev_used[b])
-            with torch.cuda.stream(s_d2h):
-                w_host.copy_(wflat, non_blocking=True)
-                ev_out.record(s_d2h)
-        s_cmp.wait_event(ev_out)
-        e1.record(s_cmp)
+        e0, e1 = pipelined(args.steps, t_e2e)
         torch.cuda.synchronize()
         barrier()
         e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
         e2e = {"value": e_ms / args.steps / world, "unit": "ms/step", "h2d_bytes_per_step": flat_bytes,
                "d2h_bytes_per_step": flat_bytes,
                "what": "pinned-host gradients copied in and updated parameters copied out every step, "
-                       "through lm_step; the next step's gradient copy overlaps the current step (two "
-                       "device gradient buffers)"}
+                       "through lm_step; the gradient copies and the read-back of a device snapshot of "
+                       "the parameters overlap the steps (three gradient and two snapshot buffers); "
+                       "the same pipeline runs untimed warm-up steps first"}
     clk = clocks.stop()
     flags = opt.status()
     took_last = opt.selection()[0] if srank else None
