@@ -45,7 +45,9 @@ def parse_args():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--set", default="gpt_720m")
     ap.add_argument("--period", type=int, default=2)
-    ap.add_argument("--precision", choices=["bf16", "f32"], default="bf16")
+    ap.add_argument("--precision", choices=["bf16", "f32", "f32tc"], default="bf16",
+                    help="NS precision: bf16 tensor cores, fp32 CUDA cores, or fp32 values as three "
+                         "bf16 pieces on the tensor cores")
     ap.add_argument("--schedule", choices=["period", "srank"], default="period",
                     help="period: Algorithm 1's fixed P; srank: Appendix G's stable-rank selection")
     ap.add_argument("--srank-alpha", type=float, default=0.01)
@@ -314,7 +316,7 @@ def run_ours(args):
         g.copy_(x)
     torch.cuda.synchronize()
 
-    prec = L.LM_BF16 if args.precision == "bf16" else L.LM_F32
+    prec = {"bf16": L.LM_BF16, "f32": L.LM_F32, "f32tc": L.LM_NS_F32_TC}[args.precision]
     srank = args.schedule == "srank"
     extra = {"vector_rule": L.LM_VECTOR_ADAMW} if args.vector_rule == "adamw" else {}
     if srank:
@@ -452,9 +454,17 @@ def run_ours(args):
     roof = None
     if ns_ms > 0 and n_muon > 0:
         achieved = fl / (ns_ms / 1e3) / 1e12
+        flops_note = "symmetric count 3 s^2 l + s^3 per matrix per NS iteration"
         if args.precision == "bf16":
             pk = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
             bound, kernel, peak_kind = "tensor", "ns_tc_kernel", f"bf16 sustained, {peak_src}"
+        elif args.precision == "f32tc":
+            # six bf16 piece products per fp32 product, on the bf16 tensor pipe
+            achieved *= 6
+            fl *= 6
+            pk = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+            bound, kernel, peak_kind = "tensor", "ns_tc_kernel", f"bf16 sustained, {peak_src}"
+            flops_note = "6 x the symmetric count 3 s^2 l + s^3 (six bf16 piece products per fp32 product)"
         else:
             # fp32 FMA on the CUDA cores: SMs x 128 lanes x 2 FLOP x the maximum SM clock
             sms = torch.cuda.get_device_properties(dev).multi_processor_count
@@ -462,13 +472,14 @@ def run_ours(args):
             pk = sms * 128 * 2 * mhz * 1e6 / 1e12
             bound, kernel = "alu", "ns_simt_kernel"
             peak_kind = f"fp32 FMA, derived: {sms} SMs x 128 lanes x 2 FLOP x {mhz:.0f} MHz"
-        traffic = kernel_traffic(kernel)
+        # the recorded ncu traffic is the bf16 workload's
+        traffic = kernel_traffic(kernel) if args.precision != "f32tc" else None
         roof = {"bound": bound, "achieved": achieved, "peak": pk, "unit": "TFLOP/s",
                 "frac": achieved / pk, "traffic": traffic, "kernel": kernel,
                 "per_launch_ms": ns_ms / max(ns_launches, 1),
                 "per_launch_tflop": fl / max(ns_launches, 1) / 1e12,
                 "peak_kind": peak_kind,
-                "flops": "symmetric count 3 s^2 l + s^3 per matrix per NS iteration"}
+                "flops": flops_note}
     lion_roof = None
     if lion_ms > 0:
         # Lion-step launches over all params: 14 B/param (bf16 W,G r/w W, fp32 M r/w)
@@ -505,7 +516,8 @@ def run_ours(args):
             "metric": METRIC, "value": value, "unit": "ms/step", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
             "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
-            "dtype": "bf16" if args.precision == "bf16" else "f32", "data": "synthetic",
+            "dtype": {"bf16": "bf16", "f32": "f32", "f32tc": "f32 (3 x bf16 pieces)"}[args.precision],
+            "data": "synthetic",
             "config": {"workload": args.set, "params": numel, "matrices": len(mats),
                        "period": None if srank else P, "ns_steps": 5, "ns_precision": args.precision,
                        **({"vector_rule": "adamw"} if args.vector_rule == "adamw" else {}),

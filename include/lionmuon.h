@@ -82,8 +82,11 @@ typedef struct {
  * beta1, beta2 in [0, 1); eta_* >= 0; weight_decay >= 0;
  * period >= 1, or 0 for P = infinity (never Muon);
  * ns_steps in [0, 64]; ns_eps >= 0; shape_scale >= 0;
- * ns_precision LM_BF16 (tensor-core bf16 GEMMs, fp32 accumulate) or LM_F32
- * (fp32 CUDA-core GEMMs).
+ * ns_precision LM_BF16 (tensor-core bf16 GEMMs, fp32 accumulate), LM_F32
+ * (fp32 CUDA-core GEMMs) or LM_NS_F32_TC (fp32 values on the tensor cores:
+ * each fp32 operand is stored exactly as three bf16 pieces hi + mid + lo and
+ * a product sums the six piece products down to order 2^-16, accumulated in
+ * fp32; the fast fp32 mode, at the cost of six bf16 products per product).
  * ns_coeffs: NULL for the same (ns_a, ns_b, ns_c) in every NS iteration, or
  * 3 * ns_steps finite values (a_k, b_k, c_k), k = 0 .. ns_steps - 1, for
  * iteration-dependent odd polynomials X <- a_k X + (b_k A + c_k A^2) X, the
@@ -131,6 +134,10 @@ typedef struct {
 
 #define LM_SCHEDULE_PERIOD 0
 #define LM_SCHEDULE_STABLE_RANK 1
+
+/* ns_precision / precision value for the three-piece tensor-core fp32 mode
+ * (LM_BF16 and LM_F32 are the other two). */
+#define LM_NS_F32_TC 2
 
 #define LM_VECTOR_LION 0
 #define LM_VECTOR_ADAMW 1
@@ -197,7 +204,8 @@ lm_status lm_set_second_moment(lm_state* s, int i, const lm_tensor* src,
  * wide orientation, with no 0.2 sqrt(max(m,n)) scaling.  in and out are
  * device tensors of equal shape (rows, cols >= 2 each), dtype LM_BF16 or
  * LM_F32 (may differ).  precision LM_BF16 uses the tensor-core path, LM_F32
- * the fp32 CUDA-core path.  Allocates its workspace with stream-ordered
+ * the fp32 CUDA-core path, LM_NS_F32_TC fp32 values on the tensor cores (as
+ * for lm_config::ns_precision).  Allocates its workspace with stream-ordered
  * allocation on cuda_stream and frees it the same way.
  * Errors: LM_ERR_INVALID_ARG, LM_ERR_DTYPE, LM_ERR_ALIGN, LM_ERR_OOM,
  * LM_ERR_CUDA. */
@@ -228,7 +236,8 @@ lm_status lm_msign_ns_coeffs(const lm_tensor* in, lm_tensor* out, int steps,
  * capture.  All calls share the one area, which keeps the last call's data:
  * each call clears what must start at zero, and calls whose GPU work may
  * overlap (unordered streams or threads) race on the area and must be
- * serialised by the caller.  Arguments and errors as for lm_msign_ns.
+ * serialised by the caller.  Arguments and errors as for lm_msign_ns, except
+ * that precision is LM_BF16 or LM_F32 only.
  * The paper has no counterpart of this call; it is a deployment variant. */
 lm_status lm_msign_ns_noalloc(const lm_tensor* in, lm_tensor* out, int steps,
                               double a, double b, double c, double eps,

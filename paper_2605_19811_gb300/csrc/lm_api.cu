@@ -83,8 +83,8 @@ lm_status check_config(const lm_config* c) {
       if (!finite(c->ns_coeffs[k])) return fail(LM_ERR_INVALID_ARG, "ns_coeffs[%d] is not finite", k);
   if (!finite(c->ns_eps) || c->ns_eps < 0) return fail(LM_ERR_INVALID_ARG, "ns_eps must be >= 0");
   if (!finite(c->shape_scale) || c->shape_scale < 0) return fail(LM_ERR_INVALID_ARG, "shape_scale must be >= 0");
-  if (c->ns_precision != LM_BF16 && c->ns_precision != LM_F32)
-    return fail(LM_ERR_INVALID_ARG, "ns_precision must be LM_BF16 or LM_F32");
+  if (c->ns_precision != LM_BF16 && c->ns_precision != LM_F32 && c->ns_precision != LM_NS_F32_TC)
+    return fail(LM_ERR_INVALID_ARG, "ns_precision must be LM_BF16, LM_F32 or LM_NS_F32_TC");
   if (c->schedule != LM_SCHEDULE_PERIOD && c->schedule != LM_SCHEDULE_STABLE_RANK)
     return fail(LM_ERR_INVALID_ARG, "schedule must be LM_SCHEDULE_PERIOD or LM_SCHEDULE_STABLE_RANK");
   if (c->schedule == LM_SCHEDULE_STABLE_RANK) {
@@ -309,6 +309,7 @@ lm_status set_error(lm_status st, const char* msg) { return fail(st, "%s", msg);
 // ---------------------------------------------------------------------------
 struct NsEngine {
   lm_dtype xdt = LM_BF16;            // workspace dtype: bf16 (tensor cores) or fp32
+  int pieces = 1;                    // tensor cores: 3 = fp32 values as three bf16 planes
   std::vector<NsGroup> groups;       // host copies (device pointers inside)
   std::vector<TcGroupMaps> maps;     // tensor-core path
   NsGroup* d_groups = nullptr;       // fp32 path reads groups from device memory
@@ -359,7 +360,7 @@ static void plan_groups(const std::vector<std::pair<int64_t, int64_t>>& shapes, 
 
 // Reserve workspace for the groups and the tile lists in the arena.
 struct NsLayout {
-  std::vector<size_t> off_x0, off_x1, off_a, off_b;
+  std::vector<size_t> off_x0, off_x1, off_a, off_b, off_xf;
   std::vector<std::vector<NsTile>> tiles;   // per batch*3 + phase
   std::vector<size_t> off_tiles;
   std::vector<std::vector<int>> offsets;    // per batch*3 + phase (tensor-core path)
@@ -409,8 +410,8 @@ static void split_gram_tiles(const std::vector<NsGroup>& groups, int g0, std::ve
 }
 
 static void layout_ns(std::vector<NsGroup>& groups, lm_dtype xdt, int nmat, Arena& ar, NsLayout& L,
-                      std::vector<NsBatch>& batches) {
-  const size_t es = dtype_size(xdt);
+                      std::vector<NsBatch>& batches, int pieces = 1) {
+  const size_t es = dtype_size(xdt) * (size_t)pieces;
   for (auto& g : groups) {
     const size_t xb = (size_t)g.count * g.s_pad * g.l_pad * es;
     const size_t ab = (size_t)g.count * g.s_pad * g.s_pad * es;
@@ -418,6 +419,8 @@ static void layout_ns(std::vector<NsGroup>& groups, lm_dtype xdt, int nmat, Aren
     L.off_x1.push_back(ar.add(xb));
     L.off_a.push_back(ar.add(ab));
     L.off_b.push_back(ar.add(ab));
+    // three-piece mode: fp32 X_0 / X_K
+    L.off_xf.push_back(pieces == 3 ? ar.add((size_t)g.count * g.s_pad * g.l_pad * sizeof(float)) : 0);
   }
   const int per = (xdt == LM_BF16) ? kMaxGroupsTc : kMaxGroupsSimt;
   int max_split = 0;
@@ -484,6 +487,7 @@ static void bind_ns(NsEngine& E, char* base, const NsLayout& L, std::vector<char
     E.groups[gi].X[1] = base + L.off_x1[gi];
     E.groups[gi].A = base + L.off_a[gi];
     E.groups[gi].B = base + L.off_b[gi];
+    E.groups[gi].Xf = E.pieces == 3 ? base + L.off_xf[gi] : nullptr;
   }
   for (size_t bi = 0; bi < E.batches.size(); ++bi)
     for (int ph = 0; ph < 3; ++ph) {
@@ -514,6 +518,7 @@ static void bind_ns(NsEngine& E, char* base, const NsLayout& L, std::vector<char
       st[k].first = tg[k][4];
       st[k].nparts = tg[k][5];
       st[k].diag = tm == tn ? 1 : 0;
+      st[k].plane = (tc && E.pieces == 3) ? (int64_t)g.count * g.s_pad * g.s_pad : 0;
     }
     E.batches[bi].split_targets = reinterpret_cast<NsSplitTarget*>(base + L.off_split_targets[bi]);
     if (!st.empty()) memcpy(host_img.data() + L.off_split_targets[bi], st.data(), st.size() * sizeof(NsSplitTarget));
@@ -528,7 +533,7 @@ static lm_status encode_maps(NsEngine& E) {
   if (E.xdt != LM_BF16) return LM_OK;
   E.maps.resize(E.groups.size());
   for (size_t gi = 0; gi < E.groups.size(); ++gi) {
-    cudaError_t e = tc_encode_group_maps(E.groups[gi], &E.maps[gi]);
+    cudaError_t e = tc_encode_group_maps(E.groups[gi], &E.maps[gi], E.pieces);
     if (e != cudaSuccess) return cuda_fail(e, "cuTensorMapEncodeTiled");
   }
   return LM_OK;
@@ -597,6 +602,14 @@ static std::vector<NsCoeffs> ns_schedule(int steps, const double* table, double 
 static lm_status run_ns(const NsEngine& E, int steps, const NsCoeffs* coeffs, unsigned* flags, cudaStream_t st,
                         Profiler* P = nullptr, const FuseFinal* fuse = nullptr,
                         const unsigned char* active = nullptr) {
+  // three-piece mode: X_0 (fp32, from the momentum kernel) -> bf16 planes
+  for (size_t gi = 0; E.pieces == 3 && steps > 0 && gi < E.groups.size(); ++gi) {
+    const NsGroup& g = E.groups[gi];
+    cudaError_t e = timed(P, LM_KERNEL_OTHER, st, [&]() {
+      return launch_split3(static_cast<const float*>(g.Xf), g.X[0], (size_t)g.count * g.s_pad * g.l_pad, st);
+    });
+    if (e != cudaSuccess) return cuda_fail(e, "three-piece split launch");
+  }
   for (int it = 0; it < steps; ++it)
     for (const NsBatch& b : E.batches)
       for (int ph = 0; ph < 3; ++ph) {
@@ -606,7 +619,8 @@ static lm_status run_ns(const NsEngine& E, int steps, const NsCoeffs* coeffs, un
           if (E.xdt == LM_BF16) {
             cudaError_t r = launch_ns_tc((NsPhase)ph, it, b.ng, E.groups.data() + b.g0, E.maps.data() + b.g0, b.tiles[ph],
                                b.ntiles[ph], b.offsets[ph], b.npairs[ph], E.d_norm2, co, flags,
-                               it == steps - 1 ? fuse : nullptr, st, active, split ? E.d_split_ws : nullptr);
+                               it == steps - 1 ? fuse : nullptr, st, active, split ? E.d_split_ws : nullptr,
+                               E.pieces, it == steps - 1 ? 1 : 0);
             if (r == cudaSuccess && split) r = launch_ns_split_finish(b.split_targets, b.nsplit, E.d_split_ws, st);
             return r;
           }
@@ -754,6 +768,7 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
   s->n = n;
   s->params.assign(params, params + n);
   s->ns.xdt = (cfg->ns_precision == LM_F32 || env_is("LM_NS_FORCE_FP32", "1")) ? LM_F32 : LM_BF16;
+  s->ns.pieces = (s->ns.xdt == LM_BF16 && cfg->ns_precision == LM_NS_F32_TC) ? 3 : 1;
   s->debug = env_is("LM_DEBUG", "1");
   if (env_is("LM_NVTX", "1")) g_nvtx.store(true);
 
@@ -841,7 +856,7 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
 
   // Muon tables
   NsLayout L;
-  layout_ns(s->ns.groups, s->ns.xdt, s->nmat, ar, L, s->ns.batches);
+  layout_ns(s->ns.groups, s->ns.xdt, s->nmat, ar, L, s->ns.batches, s->ns.pieces);
   const size_t off_mats = ar.add((size_t)std::max(s->nmat, 1) * sizeof(MatDesc));
   std::vector<MatDesc> mats(s->nmat);
   // matrices are numbered in group order
@@ -981,7 +996,8 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
   }
 
   bind_ns(s->ns, base, L, img);
-  const size_t es = dtype_size(s->ns.xdt);
+  const bool f32x = s->ns.pieces == 3;   // X_0 and X_K in the fp32 buffer Xf
+  const size_t es = f32x ? sizeof(float) : dtype_size(s->ns.xdt);
   for (size_t gi = 0; gi < s->ns.groups.size(); ++gi) {
     const NsGroup& g = s->ns.groups[gi];
     for (int k = 0; k < g.count; ++k) {
@@ -992,8 +1008,8 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
       const size_t xoff = (size_t)k * g.s_pad * g.l_pad * es;
       d.w = p.data;
       d.m = s->mom + s->mom_off[pi];
-      d.x = static_cast<char*>(g.X[0]) + xoff;
-      d.x_final = static_cast<char*>(g.X[cfg->ns_steps & 1]) + xoff;
+      d.x = static_cast<char*>(f32x ? g.Xf : g.X[0]) + xoff;
+      d.x_final = static_cast<char*>(f32x ? g.Xf : g.X[cfg->ns_steps & 1]) + xoff;
       d.out = nullptr;
       d.norm2 = s->ns.d_norm2 + id;
       d.ldx = g.tall ? g.s_pad : g.l_pad;
@@ -1059,7 +1075,7 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
   // The last APPLY can write the parameters when they are all bf16 with
   // 16-byte-aligned rows (the epilogue's vector accesses) and NS runs on the
   // tensor cores with at least one iteration.
-  s->fuse_final = s->ns.xdt == LM_BF16 && cfg->ns_steps > 0 && s->nmat > 0;
+  s->fuse_final = s->ns.xdt == LM_BF16 && s->ns.pieces == 1 && cfg->ns_steps > 0 && s->nmat > 0;
   for (const MatDesc& d : mats)
     if (d.wdt != LM_BF16 || (d.cols & 7) != 0) s->fuse_final = false;
   s->d_echunks[0] = reinterpret_cast<ElemChunk*>(base + off_echunks);
@@ -1220,8 +1236,8 @@ lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t, void* c
     for (int dt = 0; dt < 2; ++dt) {
       if (s->n_echunks[dt] == 0) continue;
       e = timed(P, LM_KERNEL_MOMENTUM_NORM, stream, [&]() {
-        return launch_momentum_norm(s->ns.xdt, (lm_dtype)dt, s->d_mats, s->d_echunks[dt], s->n_echunks[dt],
-                                    s->d_grads, mk, 0, stream);
+        return launch_momentum_norm(s->ns.pieces == 3 ? LM_F32 : s->ns.xdt, (lm_dtype)dt, s->d_mats,
+                                    s->d_echunks[dt], s->n_echunks[dt], s->d_grads, mk, 0, stream);
       });
       if (e != cudaSuccess) return cuda_fail(e, "momentum/norm kernel launch");
     }
@@ -1255,8 +1271,8 @@ lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t, void* c
     for (int dt = 0; dt < 2 && !s->fuse_final; ++dt) {
       if (s->n_echunks[dt] == 0) continue;
       e = timed(P, LM_KERNEL_FINALIZE, stream, [&]() {
-        return launch_finalize(s->ns.xdt, (lm_dtype)dt, s->d_mats, s->d_echunks[dt], s->n_echunks[dt], mk, 0,
-                               s->d_flags, stream);
+        return launch_finalize(s->ns.pieces == 3 ? LM_F32 : s->ns.xdt, (lm_dtype)dt, s->d_mats,
+                               s->d_echunks[dt], s->n_echunks[dt], mk, 0, s->d_flags, stream);
       });
       if (e != cudaSuccess) return cuda_fail(e, "finalize kernel launch");
     }
@@ -1470,11 +1486,13 @@ static lm_status msign_impl(const lm_tensor* in, lm_tensor* out, int steps, cons
 
   NsEngine E;
   E.xdt = precision == LM_F32 ? LM_F32 : LM_BF16;
+  E.pieces = precision == LM_NS_F32_TC ? 3 : 1;
+  const lm_dtype xio = E.pieces == 3 ? LM_F32 : E.xdt;   // X_0 / X_K buffer dtype
   std::vector<std::vector<int>> members;
   plan_groups({{in->rows, in->cols}}, E.xdt, E.groups, members);
   Arena ar;
   NsLayout L;
-  layout_ns(E.groups, E.xdt, 1, ar, L, E.batches);
+  layout_ns(E.groups, E.xdt, 1, ar, L, E.batches, E.pieces);
   const size_t off_mat = ar.add(sizeof(MatDesc));
   MatDesc d;
   memset(&d, 0, sizeof(d));
@@ -1493,8 +1511,8 @@ static lm_status msign_impl(const lm_tensor* in, lm_tensor* out, int steps, cons
   const NsGroup& g = E.groups[0];
   d.w = in->data;
   d.m = nullptr;
-  d.x = g.X[0];
-  d.x_final = g.X[steps & 1];
+  d.x = E.pieces == 3 ? g.Xf : g.X[0];
+  d.x_final = E.pieces == 3 ? g.Xf : g.X[steps & 1];
   d.out = out->data;
   d.norm2 = E.d_norm2;
   d.ldx = g.tall ? g.s_pad : g.l_pad;
@@ -1518,10 +1536,10 @@ static lm_status msign_impl(const lm_tensor* in, lm_tensor* out, int steps, cons
   MatDesc* dm = reinterpret_cast<MatDesc*>(base + off_mat);
   ElemChunk* de = reinterpret_cast<ElemChunk*>(base + off_et);
   unsigned* dflags = reinterpret_cast<unsigned*>(base + off_flags);
-  e = launch_momentum_norm(E.xdt, in->dtype, dm, de, (int)et.size(), nullptr, mk, 1, stream);
+  e = launch_momentum_norm(xio, in->dtype, dm, de, (int)et.size(), nullptr, mk, 1, stream);
   if (e != cudaSuccess) return cleanup(cuda_fail(e, "norm kernel launch"));
   if ((st = run_ns(E, steps, co.data(), dflags, stream)) != LM_OK) return cleanup(st);
-  e = launch_finalize(E.xdt, out->dtype, dm, de, (int)et.size(), mk, 1, dflags, stream);
+  e = launch_finalize(xio, out->dtype, dm, de, (int)et.size(), mk, 1, dflags, stream);
   if (e != cudaSuccess) return cleanup(cuda_fail(e, "output kernel launch"));
   return cleanup(LM_OK);
 }
@@ -1534,7 +1552,8 @@ lm_status lm_msign_ns(const lm_tensor* in, lm_tensor* out, int steps, double a, 
   if (steps < 0 || steps > 64) return fail(LM_ERR_INVALID_ARG, "steps must be in [0, 64]");
   if (!std::isfinite(a) || !std::isfinite(b) || !std::isfinite(c) || !std::isfinite(eps) || eps < 0)
     return fail(LM_ERR_INVALID_ARG, "coefficients must be finite, eps >= 0");
-  if (precision != LM_BF16 && precision != LM_F32) return fail(LM_ERR_INVALID_ARG, "precision must be LM_BF16 or LM_F32");
+  if (precision != LM_BF16 && precision != LM_F32 && precision != LM_NS_F32_TC)
+    return fail(LM_ERR_INVALID_ARG, "precision must be LM_BF16, LM_F32 or LM_NS_F32_TC");
   return msign_impl(in, out, steps, ns_schedule(steps, nullptr, a, b, c, eps), eps, precision, cuda_stream);
 }
 
@@ -1546,7 +1565,8 @@ lm_status lm_msign_ns_coeffs(const lm_tensor* in, lm_tensor* out, int steps, con
   for (int k = 0; k < 3 * steps; ++k)
     if (!std::isfinite(coeffs[k])) return fail(LM_ERR_INVALID_ARG, "coeffs[%d] is not finite", k);
   if (!std::isfinite(eps) || eps < 0) return fail(LM_ERR_INVALID_ARG, "eps must be finite and >= 0");
-  if (precision != LM_BF16 && precision != LM_F32) return fail(LM_ERR_INVALID_ARG, "precision must be LM_BF16 or LM_F32");
+  if (precision != LM_BF16 && precision != LM_F32 && precision != LM_NS_F32_TC)
+    return fail(LM_ERR_INVALID_ARG, "precision must be LM_BF16, LM_F32 or LM_NS_F32_TC");
   return msign_impl(in, out, steps, ns_schedule(steps, coeffs, 0, 0, 0, eps), eps, precision, cuda_stream);
 }
 

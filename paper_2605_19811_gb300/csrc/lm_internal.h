@@ -123,6 +123,10 @@ struct NsGroup {
   void* X[2];             // ping-pong X: count x (s_pad x l_pad, or l_pad x s_pad if tall)
   void* A;                // count x s_pad x s_pad
   void* B;                // count x s_pad x s_pad
+  // Three-piece tensor-core mode: X, A and B hold three bf16 planes (piece q
+  // of matrix k is matrix k + q * count of the buffer), and Xf is an fp32
+  // count x s_pad x l_pad buffer for X_0 (from the momentum kernel) and X_K.
+  void* Xf;
 };
 // Tile work item: group, matrix-in-group, tile row, tile col.
 struct NsTile {
@@ -145,6 +149,7 @@ struct NsSplitTarget {
   int32_t nr, nc;         // rows / columns of the tile inside the padded matrix
   int32_t first, nparts;
   int32_t diag;
+  int64_t plane;          // three-piece A: elements between its bf16 planes (0: one bf16 plane)
 };
 constexpr int kMaxGroupsTc = 8;   // groups per tensor-core launch
 
@@ -171,7 +176,8 @@ struct TcGroupMaps {
   CUtensorMap ast;
   CUtensorMap bst;
 };
-cudaError_t tc_encode_group_maps(const NsGroup& g, TcGroupMaps* maps);
+// pieces: 1 (bf16 buffers) or 3 (three bf16 planes per buffer)
+cudaError_t tc_encode_group_maps(const NsGroup& g, TcGroupMaps* maps, int pieces = 1);
 int tc_max_pairs();   // CTA pairs that fit the device (one CTA per SM)
 // One bounded wait on a barrier that is never signalled (failure-detection probe).
 cudaError_t launch_bounded_wait_probe(uint64_t limit_ns, unsigned* flags, cudaStream_t st);
@@ -188,8 +194,14 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
                          const TcGroupMaps* maps, const NsTile* tiles, int ntiles,
                          const int* offsets, int npairs, const double* norm2, NsCoeffs co,
                          unsigned* flags, const FuseFinal* fuse, cudaStream_t st,
-                         const unsigned char* active = nullptr, float* split_ws = nullptr);
+                         const unsigned char* active = nullptr, float* split_ws = nullptr, int pieces = 1,
+                         int final_f32 = 0);
 // split_ws: non-NULL only for a Gram launch whose tiles include split-K parts.
+// pieces = 3: fp32 operands as three bf16 pieces (no split tiles, no fused
+// parameter write); final_f32: this APPLY writes fp32 X to NsGroup::Xf.
+// fp32 -> three bf16 planes (hi, mid, lo; their sum is exactly the input):
+// n elements of src, plane q at dst + q * n.
+cudaError_t launch_split3(const float* src, void* dst, size_t n, cudaStream_t st);
 // After a Gram launch with split tiles: bf16 A tiles from the fp32 parts.
 cudaError_t launch_ns_split_finish(const NsSplitTarget* targets, int n, const float* ws, cudaStream_t st);
 

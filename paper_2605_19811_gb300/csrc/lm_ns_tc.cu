@@ -52,10 +52,8 @@ namespace {
 
 constexpr int BM = kTcBM, BN = kTcBN, BK = kTcBK;   // pair tile 256 x 256, K step 64
 constexpr int kHalf = 128;                           // A rows / B N-rows per CTA
-constexpr int kStages = 5;
 constexpr int kABytes = kHalf * BK * 2;              // 16 KB
 constexpr int kBBytes = kHalf * BK * 2;              // 16 KB
-constexpr int kStageBytes = kABytes + kBBytes;       // 32 KB per CTA
 constexpr int kEpiWarps = 8;
 constexpr int kAuxWarp = 2 + kEpiWarps;              // warp that loads the epilogue's aux tile
 constexpr int kThreads = 32 * (3 + kEpiWarps);
@@ -64,9 +62,18 @@ constexpr int kFuseBatch = 4;   // W loads in flight per thread in the fused par
 constexpr int kTmemCols = kAccBufs * BN;
 constexpr uint64_t kWaitLimitNs = 5000000000ull;     // 5 s
 constexpr int kAuxBoxBytes = kHalf * 64 * 2;         // one 64-column box of the CTA's rows: 16 KB
-constexpr size_t kAuxOffset = (size_t)kStages * kStageBytes;
-constexpr size_t kBarOffset = kAuxOffset + 4 * kAuxBoxBytes;
-constexpr size_t kSmemBytes = 1024 /*align slack*/ + kBarOffset + 256;
+// Shared-memory layout per operand precision.  kP = 1: bf16 operands, a
+// 5-stage ring of 32 KB per CTA and a 64 KB aux/staging buffer.  kP = 3:
+// fp32 operands held as three bf16 pieces (hi + mid + lo, exact), a 2-stage
+// ring of 96 KB per CTA, no aux buffer (that epilogue works from global memory).
+template <int kP>
+struct TcLayout {
+  static constexpr int kStages = kP == 1 ? 5 : 2;
+  static constexpr int kStageBytes = kP * (kABytes + kBBytes);
+  static constexpr size_t kAuxOffset = (size_t)kStages * kStageBytes;
+  static constexpr size_t kBarOffset = kAuxOffset + (kP == 1 ? 4 * kAuxBoxBytes : 0);
+  static constexpr size_t kSmemBytes = 1024 /*align slack*/ + kBarOffset + 256;
+};
 
 struct TcParams {
   TcGroupMaps maps[kMaxGroupsTc];
@@ -82,6 +89,7 @@ struct TcParams {
   FuseFinal fuse;       // fuse.mats != NULL: this APPLY writes the parameters
   const unsigned char* active;   // NULL, or per matrix: 0 = skip its tiles
   float* split_ws;               // fp32 workspace of split Gram tiles (256 x 256 each)
+  int final_f32;                 // three-piece operands: this APPLY writes fp32 X to NsGroup::Xf
 };
 
 // Whether a tile's matrix runs in this launch; every role asks the same
@@ -362,29 +370,40 @@ __device__ __forceinline__ uint32_t pack_bf2(float lo, float hi) {
 // K-major operand half: one 64 (K) x 128 box; MN-major: one 4-D box that
 // fills both 64 (MN) x 64 (K) swizzle atoms (one copy instead of two
 // measured ~2% faster).  Returns false if a wait gave up.
+template <int kS>
 struct ProducerRing {
   int stage;
   uint32_t ph;
-  int armed[kStages];
+  int armed[kS];
 };
-template <bool AMN, bool BMN>
-__device__ __forceinline__ bool produce_range(ProducerRing& R, uint8_t* smem, uint64_t* full, uint64_t* empty,
-                                              volatile int* abort_flag, uint32_t rank, int kb0, int kb1,
-                                              const CUtensorMap* map_a, const CUtensorMap* map_b,
-                                              int row_a, int col_b, int mat) {
+// kP pieces per operand: piece q of matrix mat is matrix mat + q * pstride
+// of the tensor map; a stage holds the kP A pieces, then the kP B pieces.
+template <bool AMN, bool BMN, int kP>
+__device__ __forceinline__ bool produce_range(ProducerRing<TcLayout<kP>::kStages>& R, uint8_t* smem,
+                                              uint64_t* full, uint64_t* empty, volatile int* abort_flag,
+                                              uint32_t rank, int kb0, int kb1, const CUtensorMap* map_a,
+                                              const CUtensorMap* map_b, int row_a, int col_b, int mat,
+                                              int pstride) {
+  using L = TcLayout<kP>;
   for (int kb = kb0; kb < kb1; ++kb) {
     if (!mbar_wait(&empty[R.stage], R.ph ^ 1u, abort_flag, kWaitLimitNs)) return false;
-    uint8_t* sa = smem + (size_t)R.stage * kStageBytes;
-    uint8_t* sb = sa + kABytes;
+    uint8_t* sa = smem + (size_t)R.stage * L::kStageBytes;
+    uint8_t* sb = sa + kP * kABytes;
     const uint32_t fb = peer_addr(&full[R.stage], 0);
-    if (rank == 0) mbar_arrive_expect_tx(&full[R.stage], 2 * kStageBytes);
+    if (rank == 0) mbar_arrive_expect_tx(&full[R.stage], 2 * L::kStageBytes);
     R.armed[R.stage] = (int)R.ph;
     const int k0 = kb * BK;
-    if (!AMN) tma_load_3d(sa, map_a, fb, k0, row_a, mat);
-    else tma_load_4d(sa, map_a, fb, 0, k0, row_a >> 6, mat);
-    if (!BMN) tma_load_3d(sb, map_b, fb, k0, col_b, mat);
-    else tma_load_4d(sb, map_b, fb, 0, k0, col_b >> 6, mat);
-    if (++R.stage == kStages) {
+#pragma unroll
+    for (int q = 0; q < kP; ++q) {
+      if (!AMN) tma_load_3d(sa + q * kABytes, map_a, fb, k0, row_a, mat + q * pstride);
+      else tma_load_4d(sa + q * kABytes, map_a, fb, 0, k0, row_a >> 6, mat + q * pstride);
+    }
+#pragma unroll
+    for (int q = 0; q < kP; ++q) {
+      if (!BMN) tma_load_3d(sb + q * kBBytes, map_b, fb, k0, col_b, mat + q * pstride);
+      else tma_load_4d(sb + q * kBBytes, map_b, fb, 0, k0, col_b >> 6, mat + q * pstride);
+    }
+    if (++R.stage == L::kStages) {
       R.stage = 0;
       R.ph ^= 1u;
     }
@@ -393,24 +412,35 @@ __device__ __forceinline__ bool produce_range(ProducerRing& R, uint8_t* smem, ui
 }
 
 // MMA issue for K blocks [kb0, kb1) of one tile with fixed operand layouts.
-template <bool AMN, bool BMN>
+// kP = 3: with A = A0 + A1 + A2 and B = B0 + B1 + B2 (each piece 2^-8 of the
+// previous in magnitude) the six products of order up to 2^-16 are summed,
+// A0B0 + A0B1 + A1B0 + A0B2 + A2B0 + A1B1; the dropped ones are of order 2^-24.
+template <bool AMN, bool BMN, int kP>
 __device__ __forceinline__ bool mma_range(int& stage, uint32_t& ph, uint8_t* smem, uint64_t* full,
                                           uint64_t* empty, volatile int* abort_flag, int kb0, int kb1,
                                           uint32_t d_tmem, int kb_first) {
+  using L = TcLayout<kP>;
+  constexpr int kProducts = kP == 1 ? 1 : 6;
+  constexpr int qa[6] = {0, 0, 1, 0, 2, 1};
+  constexpr int qb[6] = {0, 1, 0, 2, 0, 1};
   const uint32_t idesc = make_idesc(BM, BN, AMN, BMN);
   for (int kb = kb0; kb < kb1; ++kb) {
     if (!mbar_wait(&full[stage], ph, abort_flag, kWaitLimitNs)) return false;
     tc_fence_after();
-    const uint32_t sa = smem_u32(smem + (size_t)stage * kStageBytes);
-    const uint32_t sb = sa + kABytes;
+    const uint32_t sa = smem_u32(smem + (size_t)stage * L::kStageBytes);
+    const uint32_t sb = sa + kP * kABytes;
 #pragma unroll
     for (int kk = 0; kk < BK / 16; ++kk) {
-      const uint64_t adesc = AMN ? sw128_desc(sa + kk * 2048, 64 * BK * 2, 1024) : sw128_desc(sa + kk * 32, 16, 1024);
-      const uint64_t bdesc = BMN ? sw128_desc(sb + kk * 2048, 64 * BK * 2, 1024) : sw128_desc(sb + kk * 32, 16, 1024);
-      umma_bf16(d_tmem, adesc, bdesc, idesc, (kb != kb_first || kk != 0) ? 1u : 0u);
+#pragma unroll
+      for (int m = 0; m < kProducts; ++m) {
+        const uint32_t pa = sa + qa[m] * kABytes, pb = sb + qb[m] * kBBytes;
+        const uint64_t adesc = AMN ? sw128_desc(pa + kk * 2048, 64 * BK * 2, 1024) : sw128_desc(pa + kk * 32, 16, 1024);
+        const uint64_t bdesc = BMN ? sw128_desc(pb + kk * 2048, 64 * BK * 2, 1024) : sw128_desc(pb + kk * 32, 16, 1024);
+        umma_bf16(d_tmem, adesc, bdesc, idesc, (kb != kb_first || kk != 0 || m != 0) ? 1u : 0u);
+      }
     }
     umma_commit_pair(&empty[stage]);
-    if (++stage == kStages) {
+    if (++stage == L::kStages) {
       stage = 0;
       ph ^= 1u;
     }
@@ -418,18 +448,88 @@ __device__ __forceinline__ bool mma_range(int& stage, uint32_t& ph, uint8_t* sme
   return true;
 }
 
+// fp32 value v as hi + mid + lo bf16 pieces, exactly: each piece takes the
+// next 8 significant bits (the differences are exact in fp32).
+__device__ __forceinline__ void split3(float v, float& h, float& m, float& l) {
+  h = __bfloat162float(__float2bfloat16_rn(v));
+  const float r1 = v - h;
+  m = __bfloat162float(__float2bfloat16_rn(r1));
+  l = r1 - m;
+}
+// Epilogue of one 32-column chunk (columns j0 ..) of row i with three-piece
+// operands; the aux values and the results go through global memory.
+//   aux: the A (POLY) or X (APPLY) element, hi + mid + lo; out: the result's
+//   pieces, or fp32 in out_f32 (last APPLY).  plane = elements per piece.
+__device__ __forceinline__ void piece_chunk(const uint32_t (&r)[32], int phase, const NsCoeffs& co, float nscale,
+                                            const __nv_bfloat16* aux, __nv_bfloat16* out, float* out_f32,
+                                            size_t plane, size_t off, bool row_ok, int j0, int ncols) {
+  float v[32];
+  if (phase != NS_GRAM) {
+#pragma unroll
+    for (int e = 0; e < 32; ++e) v[e] = 0.f;
+#pragma unroll
+    for (int q = 0; q < 3; ++q) {
+      const uint4* src = reinterpret_cast<const uint4*>(aux + q * plane + off);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const uint4 a4 = src[u];
+        const uint32_t aw[4] = {a4.x, a4.y, a4.z, a4.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          v[u * 8 + 2 * e] += bf_lo(aw[e]);
+          v[u * 8 + 2 * e + 1] += bf_hi(aw[e]);
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int e = 0; e < 32; ++e) {
+    const float acc = __uint_as_float(r[e]);
+    float o;
+    if (phase == NS_GRAM) o = acc * nscale;
+    else if (phase == NS_POLY) o = co.b * v[e] + co.c * acc;
+    else o = (co.a * v[e] + acc) * nscale;
+    v[e] = (row_ok && j0 + e < ncols) ? o : 0.f;
+  }
+  if (out_f32 != nullptr) {
+    float4* dst = reinterpret_cast<float4*>(out_f32 + off);
+#pragma unroll
+    for (int u = 0; u < 8; ++u) dst[u] = make_float4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
+    return;
+  }
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    uint32_t w[3][4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      float h0, m0, l0, h1, m1, l1;
+      split3(v[u * 8 + 2 * e], h0, m0, l0);
+      split3(v[u * 8 + 2 * e + 1], h1, m1, l1);
+      w[0][e] = pack_bf2(h0, h1);
+      w[1][e] = pack_bf2(m0, m1);
+      w[2][e] = pack_bf2(l0, l1);
+    }
+#pragma unroll
+    for (int q = 0; q < 3; ++q)
+      reinterpret_cast<uint4*>(out + q * plane + off)[u] = make_uint4(w[q][0], w[q][1], w[q][2], w[q][3]);
+  }
+}
+
 // ------------------------------- the kernel ---------------------------------
 // kMasked: the launch carries a per-matrix mask (stable-rank selection);
 // kSplit: its Gram tiles include split-K parts.  The plain instantiation keeps
-// the common path free of both.
-template <bool kMasked, bool kSplit>
+// the common path free of both.  kP: bf16 pieces per operand value (1: bf16
+// operands; 3: fp32 operands as hi + mid + lo bf16 pieces, six products).
+template <bool kMasked, bool kSplit, int kP>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     ns_tc_kernel(const __grid_constant__ TcParams p) {
+  using L = TcLayout<kP>;
+  constexpr int kStages = L::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-  uint8_t* auxbuf = smem + kAuxOffset;   // 4 x (128 rows x 64 cols) bf16, 128-byte swizzled
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kBarOffset);
+  uint8_t* auxbuf = smem + L::kAuxOffset;   // kP = 1: 4 x (128 rows x 64 cols) bf16, 128-byte swizzled
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + L::kBarOffset);
   uint64_t* empty = full + kStages;
   uint64_t* accfull = empty + kStages;
   uint64_t* accempty = accfull + 2;
@@ -444,7 +544,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   const int cur = p.iter & 1;
   const uint32_t rank = cluster_rank();          // 0: MMA issuer of the pair
   const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
-  const bool aux_phase = phase != NS_GRAM;       // epilogue reads the A (POLY) or X (APPLY) tile
+  const bool aux_phase = kP == 1 && phase != NS_GRAM;   // epilogue reads the A (POLY) or X (APPLY) tile
   // this pair's tiles: a host-balanced range, or round robin
   const int w_begin = p.offsets ? p.offsets[pair] : pair;
   const int w_end = p.offsets ? p.offsets[pair + 1] : p.ntiles;
@@ -482,7 +582,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     // ------------------------------ producer ------------------------------
     if (lane == 0) {
-      ProducerRing R;
+      ProducerRing<kStages> R;
       R.stage = 0;
       R.ph = 0;
       for (int s = 0; s < kStages; ++s) R.armed[s] = -1;
@@ -498,14 +598,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         for (int sg = 0; ok && sg < P.nseg; ++sg) {
           const OpSeg& S = P.seg[sg];
           if (!S.a_mn && !S.b_mn)
-            ok = produce_range<false, false>(R, smem, full, empty, abort_flag, rank, kb0, S.kb_end, S.map_a,
-                                             S.map_b, row_a, col_b, t.mat);
+            ok = produce_range<false, false, kP>(R, smem, full, empty, abort_flag, rank, kb0, S.kb_end, S.map_a,
+                                             S.map_b, row_a, col_b, t.mat, g.count);
           else if (!S.a_mn)
-            ok = produce_range<false, true>(R, smem, full, empty, abort_flag, rank, kb0, S.kb_end, S.map_a,
-                                            S.map_b, row_a, col_b, t.mat);
+            ok = produce_range<false, true, kP>(R, smem, full, empty, abort_flag, rank, kb0, S.kb_end, S.map_a,
+                                            S.map_b, row_a, col_b, t.mat, g.count);
           else
-            ok = produce_range<true, true>(R, smem, full, empty, abort_flag, rank, kb0, S.kb_end, S.map_a,
-                                           S.map_b, row_a, col_b, t.mat);
+            ok = produce_range<true, true, kP>(R, smem, full, empty, abort_flag, rank, kb0, S.kb_end, S.map_a,
+                                           S.map_b, row_a, col_b, t.mat, g.count);
           kb0 = S.kb_end;
         }
         if (!ok) give_up();
@@ -542,13 +642,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         for (int sg = 0; ok && sg < P.nseg; ++sg) {
           const OpSeg& S = P.seg[sg];
           if (!S.a_mn && !S.b_mn)
-            ok = mma_range<false, false>(stage, ph, smem, full, empty, abort_flag, kb0, S.kb_end, d_tmem,
+            ok = mma_range<false, false, kP>(stage, ph, smem, full, empty, abort_flag, kb0, S.kb_end, d_tmem,
                                             P.kb_start);
           else if (!S.a_mn)
-            ok = mma_range<false, true>(stage, ph, smem, full, empty, abort_flag, kb0, S.kb_end, d_tmem,
+            ok = mma_range<false, true, kP>(stage, ph, smem, full, empty, abort_flag, kb0, S.kb_end, d_tmem,
                                             P.kb_start);
           else
-            ok = mma_range<true, true>(stage, ph, smem, full, empty, abort_flag, kb0, S.kb_end, d_tmem,
+            ok = mma_range<true, true, kP>(stage, ph, smem, full, empty, abort_flag, kb0, S.kb_end, d_tmem,
                                             P.kb_start);
           kb0 = S.kb_end;
         }
@@ -652,6 +752,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * BN + ch * 32), r);
         const int j0 = t.tn * BN + ch * 32;
         if (!warp_in || j0 >= jmax) continue;   // beyond the padded matrix
+        if (kP == 3 && !split) {
+          // rows of the output: s_pad or l_pad (APPLY tall); ld its row length
+          const size_t ld = (size_t)(phase == NS_APPLY ? (g.tall ? g.s_pad : g.l_pad) : g.s_pad);
+          const size_t msize = (size_t)(phase == NS_APPLY ? (size_t)g.s_pad * g.l_pad : (size_t)g.s_pad * g.s_pad);
+          const size_t off = (size_t)t.mat * msize + (size_t)i * ld + j0;
+          const size_t plane = (size_t)g.count * msize;
+          const __nv_bfloat16* aux = static_cast<const __nv_bfloat16*>(phase == NS_POLY ? g.A : g.X[cur]);
+          __nv_bfloat16* out = static_cast<__nv_bfloat16*>(phase == NS_GRAM ? g.A : (phase == NS_POLY ? g.B : g.X[cur ^ 1]));
+          float* out_f32 = (phase == NS_APPLY && p.final_f32) ? static_cast<float*>(g.Xf) : nullptr;
+          piece_chunk(r, phase, p.co, nscale, aux, out, out_f32, plane, off, i < nrows, j0, ncols);
+          continue;
+        }
         if (split) {
           // partial Gram product of a split tile: its own fp32 workspace tile
           float* wrow = p.split_ws + (size_t)(t.slot - 1) * (BM * BN) + (size_t)((int)rank * kHalf + row) * BN +
@@ -750,7 +862,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             }
           }
         }
-      } else if (lane == 0 && warp_in && !split) {
+      } else if (kP == 1 && lane == 0 && warp_in && !split) {
         const TcGroupMaps& mp = p.maps[t.group];
         const CUtensorMap* dst = (phase == NS_GRAM) ? &mp.ast : (phase == NS_POLY ? &mp.bst : &mp.xst[cur ^ 1]);
 #pragma unroll
@@ -789,7 +901,16 @@ __global__ void __launch_bounds__(256) ns_split_finish_kernel(const NsSplitTarge
     if (r >= T.nr || c >= T.nc) continue;
     float sum = 0.f;
     for (int k = 0; k < T.nparts; ++k) sum += ws[(size_t)(T.first + k) * (BM * BN) + e];
-    dst[(size_t)r * T.ld + c] = __float2bfloat16_rn(sum);
+    const size_t o = (size_t)r * T.ld + c;
+    if (T.plane == 0) {
+      dst[o] = __float2bfloat16_rn(sum);
+    } else {   // three bf16 planes
+      float h, m, l;
+      split3(sum, h, m, l);
+      dst[o] = __float2bfloat16_rn(h);
+      dst[T.plane + o] = __float2bfloat16_rn(m);
+      dst[2 * T.plane + o] = __float2bfloat16_rn(l);
+    }
   }
 }
 
@@ -861,22 +982,55 @@ cudaError_t launch_bounded_wait_probe(uint64_t limit_ns, unsigned* flags, cudaSt
 int tc_pad_s(int s) { return (s + kHalf - 1) / kHalf * kHalf; }
 int tc_pad_l(int l) { return (l + BN - 1) / BN * BN; }
 
-cudaError_t tc_encode_group_maps(const NsGroup& g, TcGroupMaps* maps) {
+cudaError_t tc_encode_group_maps(const NsGroup& g, TcGroupMaps* maps, int pieces) {
   cudaError_t e;
+  // three-piece buffers hold piece q of matrix k as matrix k + q * count
+  const uint64_t nm = (uint64_t)g.count * (uint64_t)pieces;
   // X buffers: s_pad x l_pad (wide) or l_pad x s_pad (tall), row-major
   const uint64_t inner = g.tall ? g.s_pad : g.l_pad, rows = g.tall ? g.l_pad : g.s_pad;
   for (int b = 0; b < 2; ++b) {
-    if ((e = encode_3d(&maps->xk[b], g.X[b], inner, rows, g.count, BK, kHalf)) != cudaSuccess) return e;
-    if ((e = encode_3d(&maps->xst[b], g.X[b], inner, rows, g.count, 64, 32)) != cudaSuccess) return e;
-    if ((e = encode_mn4d(&maps->xmn[b], g.X[b], inner, rows, g.count, BK)) != cudaSuccess) return e;
+    if ((e = encode_3d(&maps->xk[b], g.X[b], inner, rows, nm, BK, kHalf)) != cudaSuccess) return e;
+    if ((e = encode_3d(&maps->xst[b], g.X[b], inner, rows, nm, 64, 32)) != cudaSuccess) return e;
+    if ((e = encode_mn4d(&maps->xmn[b], g.X[b], inner, rows, nm, BK)) != cudaSuccess) return e;
   }
-  if ((e = encode_3d(&maps->a, g.A, g.s_pad, g.s_pad, g.count, BK, kHalf)) != cudaSuccess) return e;
-  if ((e = encode_3d(&maps->b, g.B, g.s_pad, g.s_pad, g.count, BK, kHalf)) != cudaSuccess) return e;
-  if ((e = encode_mn4d(&maps->amn, g.A, g.s_pad, g.s_pad, g.count, BK)) != cudaSuccess) return e;
-  if ((e = encode_mn4d(&maps->bmn, g.B, g.s_pad, g.s_pad, g.count, BK)) != cudaSuccess) return e;
-  if ((e = encode_3d(&maps->ast, g.A, g.s_pad, g.s_pad, g.count, 64, 32)) != cudaSuccess) return e;
-  if ((e = encode_3d(&maps->bst, g.B, g.s_pad, g.s_pad, g.count, 64, 32)) != cudaSuccess) return e;
+  if ((e = encode_3d(&maps->a, g.A, g.s_pad, g.s_pad, nm, BK, kHalf)) != cudaSuccess) return e;
+  if ((e = encode_3d(&maps->b, g.B, g.s_pad, g.s_pad, nm, BK, kHalf)) != cudaSuccess) return e;
+  if ((e = encode_mn4d(&maps->amn, g.A, g.s_pad, g.s_pad, nm, BK)) != cudaSuccess) return e;
+  if ((e = encode_mn4d(&maps->bmn, g.B, g.s_pad, g.s_pad, nm, BK)) != cudaSuccess) return e;
+  if ((e = encode_3d(&maps->ast, g.A, g.s_pad, g.s_pad, nm, 64, 32)) != cudaSuccess) return e;
+  if ((e = encode_3d(&maps->bst, g.B, g.s_pad, g.s_pad, nm, 64, 32)) != cudaSuccess) return e;
   return cudaSuccess;
+}
+
+namespace {
+__global__ void __launch_bounds__(256) split3_kernel(const float4* __restrict__ src, uint2* __restrict__ dst,
+                                                     size_t n4) {
+  for (size_t k = blockIdx.x * (size_t)blockDim.x + threadIdx.x; k < n4; k += (size_t)gridDim.x * blockDim.x) {
+    const float4 v = src[k];
+    float h[4], m[4], l[4];
+    split3(v.x, h[0], m[0], l[0]);
+    split3(v.y, h[1], m[1], l[1]);
+    split3(v.z, h[2], m[2], l[2]);
+    split3(v.w, h[3], m[3], l[3]);
+    dst[k] = make_uint2(pack_bf2(h[0], h[1]), pack_bf2(h[2], h[3]));
+    dst[n4 + k] = make_uint2(pack_bf2(m[0], m[1]), pack_bf2(m[2], m[3]));
+    dst[2 * n4 + k] = make_uint2(pack_bf2(l[0], l[1]), pack_bf2(l[2], l[3]));
+  }
+}
+}  // namespace
+
+cudaError_t launch_split3(const float* src, void* dst, size_t n, cudaStream_t st) {
+  if (n == 0) return cudaSuccess;
+  if (n % 4 != 0) return cudaErrorInvalidValue;
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const size_t n4 = n / 4;
+  size_t grid = (n4 + 255) / 256;
+  if (grid > (size_t)sms * 8) grid = (size_t)sms * 8;
+  count_launch();
+  split3_kernel<<<(unsigned)grid, 256, 0, st>>>(reinterpret_cast<const float4*>(src), static_cast<uint2*>(dst), n4);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_ns_split_finish(const NsSplitTarget* targets, int n, const float* ws, cudaStream_t st) {
@@ -893,26 +1047,31 @@ int tc_max_pairs() {
   return sms / 2 > 0 ? sms / 2 : 1;
 }
 
+template <bool kMasked, bool kSplit, int kP>
+static cudaError_t set_smem_attr() {
+  return cudaFuncSetAttribute(ns_tc_kernel<kMasked, kSplit, kP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)TcLayout<kP>::kSmemBytes);
+}
+
 cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* groups,
                          const TcGroupMaps* maps, const NsTile* tiles, int ntiles,
                          const int* offsets, int npairs, const double* norm2, NsCoeffs co,
                          unsigned* flags, const FuseFinal* fuse, cudaStream_t st,
-                         const unsigned char* active, float* split_ws) {
+                         const unsigned char* active, float* split_ws, int pieces, int final_f32) {
   if (ntiles <= 0) return cudaSuccess;
   if (ngroups < 1 || ngroups > kMaxGroupsTc) return cudaErrorInvalidValue;
+  if (pieces != 1 && pieces != 3) return cudaErrorInvalidValue;
+  if (pieces == 3 && fuse != nullptr) return cudaErrorInvalidValue;
   static bool attr_set = false;
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(ns_tc_kernel<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)kSmemBytes);
-    if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(ns_tc_kernel<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               (int)kSmemBytes);
-    if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(ns_tc_kernel<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               (int)kSmemBytes);
-    if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(ns_tc_kernel<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               (int)kSmemBytes);
+    cudaError_t e = set_smem_attr<false, false, 1>();
+    if (e == cudaSuccess) e = set_smem_attr<true, false, 1>();
+    if (e == cudaSuccess) e = set_smem_attr<false, true, 1>();
+    if (e == cudaSuccess) e = set_smem_attr<true, true, 1>();
+    if (e == cudaSuccess) e = set_smem_attr<false, false, 3>();
+    if (e == cudaSuccess) e = set_smem_attr<true, false, 3>();
+    if (e == cudaSuccess) e = set_smem_attr<false, true, 3>();
+    if (e == cudaSuccess) e = set_smem_attr<true, true, 3>();
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
@@ -933,6 +1092,7 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
   if (fuse != nullptr && ph == NS_APPLY) prm.fuse = *fuse;
   prm.active = active;
   prm.split_ws = split_ws;
+  prm.final_f32 = (pieces == 3 && ph == NS_APPLY && final_f32) ? 1 : 0;
   int pairs = npairs;
   if (offsets == nullptr) {
     pairs = tc_max_pairs();
@@ -941,12 +1101,24 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
   const int grid = 2 * (pairs > 0 ? pairs : 1);
   count_launch();
   const bool split = split_ws != nullptr && ph == NS_GRAM;
+  if (pieces == 3) {
+    constexpr size_t sm = TcLayout<3>::kSmemBytes;
+    if (active != nullptr) {
+      if (split) ns_tc_kernel<true, true, 3><<<grid, kThreads, sm, st>>>(prm);
+      else ns_tc_kernel<true, false, 3><<<grid, kThreads, sm, st>>>(prm);
+    } else {
+      if (split) ns_tc_kernel<false, true, 3><<<grid, kThreads, sm, st>>>(prm);
+      else ns_tc_kernel<false, false, 3><<<grid, kThreads, sm, st>>>(prm);
+    }
+    return cudaGetLastError();
+  }
+  constexpr size_t sm = TcLayout<1>::kSmemBytes;
   if (active != nullptr) {
-    if (split) ns_tc_kernel<true, true><<<grid, kThreads, kSmemBytes, st>>>(prm);
-    else ns_tc_kernel<true, false><<<grid, kThreads, kSmemBytes, st>>>(prm);
+    if (split) ns_tc_kernel<true, true, 1><<<grid, kThreads, sm, st>>>(prm);
+    else ns_tc_kernel<true, false, 1><<<grid, kThreads, sm, st>>>(prm);
   } else {
-    if (split) ns_tc_kernel<false, true><<<grid, kThreads, kSmemBytes, st>>>(prm);
-    else ns_tc_kernel<false, false><<<grid, kThreads, kSmemBytes, st>>>(prm);
+    if (split) ns_tc_kernel<false, true, 1><<<grid, kThreads, sm, st>>>(prm);
+    else ns_tc_kernel<false, false, 1><<<grid, kThreads, sm, st>>>(prm);
   }
   return cudaGetLastError();
 }

@@ -16,6 +16,7 @@ from . import build as _build
 LM_OK = 0
 LM_F32 = 0
 LM_BF16 = 1
+LM_NS_F32_TC = 2      # ns_precision: fp32 values as three bf16 pieces on the tensor cores
 LM_FLAG_NONFINITE = 0x1
 LM_FLAG_TIMEOUT = 0x2
 LM_FLAG_GUARD = 0x4

@@ -1,6 +1,10 @@
 """GPU parity of the Newton-Schulz msign approximation (lm_msign_ns) against
 the fp64 oracle recurrence on the same stored input: relative Frobenius error
-<= 2e-2 for the bf16 tensor-core path and <= 1e-5 for the fp32 path."""
+<= 2e-2 for the bf16 tensor-core path, <= 1e-5 for the fp32 CUDA-core path and
+<= 5e-5 for the three-piece tensor-core fp32 mode (LM_NS_F32_TC: each fp32
+operand is exactly hi + mid + lo in bf16, the dropped piece products are of
+order 2^-24 relative, and what remains is the tensor cores' fp32
+accumulation, measured at 1e-6 - 2.4e-5 up to 768 x 50304)."""
 
 import numpy as np
 import pytest
@@ -11,7 +15,11 @@ from tests.lm_testutil import host_tensor, rel_fro, stored_values
 
 pytestmark = pytest.mark.gpu
 
-TOL = {"bf16": 2e-2, "f32": 1e-5}
+TOL = {"bf16": 2e-2, "f32": 1e-5, "f32tc": 5e-5}
+
+
+def _prec(L, precision):
+    return {"bf16": L.LM_BF16, "f32": L.LM_F32, "f32tc": L.LM_NS_F32_TC}[precision]
 QUINTIC = O.NS_QUINTIC
 
 
@@ -21,13 +29,12 @@ def _msign(x_host, precision, steps=5, coeffs=QUINTIC, eps=1e-7, out_dtype="f32"
     x = x_host.cuda()
     out = torch.empty(x.shape, dtype={"f32": torch.float32, "bf16": torch.bfloat16}[out_dtype],
                       device="cuda")
-    prec = L.LM_BF16 if precision == "bf16" else L.LM_F32
-    L.msign_ns(x, out, steps, *coeffs, eps=eps, precision=prec)
+    L.msign_ns(x, out, steps, *coeffs, eps=eps, precision=_prec(L, precision))
     torch.cuda.synchronize()
     return stored_values(out)
 
 
-@pytest.mark.parametrize("precision", ["bf16", "f32"])
+@pytest.mark.parametrize("precision", ["bf16", "f32", "f32tc"])
 @pytest.mark.parametrize("shape", [(128, 256), (256, 128), (300, 700), (700, 300), (64, 64),
                                    (130, 1000), (1000, 130), (257, 257), (2, 3), (40, 9)])
 def test_msign_parity_quintic(precision, shape):
@@ -39,7 +46,7 @@ def test_msign_parity_quintic(precision, shape):
     assert rel_fro(got, want) <= TOL[precision]
 
 
-@pytest.mark.parametrize("precision", ["bf16", "f32"])
+@pytest.mark.parametrize("precision", ["bf16", "f32", "f32tc"])
 @pytest.mark.parametrize("coeffs,steps", [((0.0, 1.0, 0.0), 1), ((0.0, 0.0, 1.0), 1),
                                           ((1.5, -0.5, 0.0), 8), ((2.0, -1.3, 0.4), 3),
                                           (QUINTIC, 0), (QUINTIC, 1)])
@@ -54,7 +61,7 @@ def test_msign_parity_each_term(precision, coeffs, steps):
     assert rel_fro(got, want) <= TOL[precision]
 
 
-@pytest.mark.parametrize("precision", ["bf16", "f32"])
+@pytest.mark.parametrize("precision", ["bf16", "f32", "f32tc"])
 def test_msign_known_svd_closed_form(precision):
     """Input with exactly known SVD: output = U phi^K(sigma/||sigma||) V^T."""
     from tests.test_oracle_pins import known_svd_matrix
@@ -107,7 +114,7 @@ def table_tolerance(x, table, precision):
     polynomials (the minimax tables start near 8.5 x) amplify rounding of
     small singular values; the storage-modelled oracle measures by how much
     for this input, independently of the GPU."""
-    storage = "bf16" if precision == "bf16" else "f32"
+    storage = "bf16" if precision == "bf16" else "f32"   # the three-piece mode stores fp32 exactly
     d = rel_fro(O.ns_polynomial_schedule_storage(x, table, 1e-7, storage), O.ns_polynomial_schedule(x, table, 1e-7))
     return max(TOL[precision], 1.5 * d)
 
@@ -118,7 +125,7 @@ def _table(name):
             "mixed": MIXED_TABLE}[name]
 
 
-@pytest.mark.parametrize("precision", ["bf16", "f32"])
+@pytest.mark.parametrize("precision", ["bf16", "f32", "f32tc"])
 @pytest.mark.parametrize("name", ["polar_express", "chebyshev_cubic", "mixed"])
 @pytest.mark.parametrize("shape", [(256, 768), (768, 256), (300, 130), (64, 64)])
 def test_msign_coefficient_table_parity(precision, name, shape):
@@ -131,7 +138,7 @@ def test_msign_coefficient_table_parity(precision, name, shape):
     xh = host_tensor(synth.draw_matrix(shape, seed=11 + sum(shape)), in_dtype)
     x = xh.cuda()
     out = torch.empty(x.shape, dtype=torch.float32, device="cuda")
-    L.msign_ns_coeffs(x, out, table, precision=L.LM_BF16 if precision == "bf16" else L.LM_F32)
+    L.msign_ns_coeffs(x, out, table, precision=_prec(L, precision))
     torch.cuda.synchronize()
     want = O.ns_polynomial_schedule(stored_values(xh), table, 1e-7)
     assert rel_fro(stored_values(out), want) <= table_tolerance(stored_values(xh), table, precision)
@@ -149,12 +156,36 @@ def test_msign_coefficient_table_argument_errors():
         L.msign_ns_coeffs(x, out, [(1.0, 0.0, 0.0)] * 65)
 
 
+@pytest.mark.parametrize("precision", ["bf16", "f32tc"])
 @pytest.mark.parametrize("shape", [(200, 20000), (20000, 200), (768, 50304)])
-def test_msign_parity_long_k_split_gram(shape):
+def test_msign_parity_long_k_split_gram(shape, precision):
     """A matrix whose Gram tiles are far longer than a CTA pair's share of
     the launch: the Gram phase splits them along K into parts that add fp32
-    partial sums (split-K); the result must match the oracle recurrence."""
-    xh = host_tensor(synth.draw_matrix(shape, seed=5 + shape[0]), "bf16")
-    got = _msign(xh, "bf16")
+    partial sums (split-K; in the three-piece mode the finish kernel writes
+    the sum as three bf16 planes); the result must match the oracle."""
+    xh = host_tensor(synth.draw_matrix(shape, seed=5 + shape[0]), "bf16" if precision == "bf16" else "f32")
+    got = _msign(xh, precision)
     want = O.ns_polynomial(stored_values(xh), 5, *QUINTIC, 1e-7)
-    assert rel_fro(got, want) <= TOL["bf16"]
+    assert rel_fro(got, want) <= TOL[precision]
+
+
+@pytest.mark.parametrize("shape", [(300, 700), (700, 300), (130, 1000), (512, 2048)])
+def test_msign_three_piece_mode_agrees_with_fp32_path(shape):
+    """The two fp32 modes (CUDA cores, three-piece tensor cores) give the same
+    output within the three-piece tolerance, and both are far closer to the
+    exact recurrence than the bf16 tolerance."""
+    xh = host_tensor(synth.draw_matrix(shape, seed=3 * shape[0] + shape[1]), "f32")
+    a = _msign(xh, "f32")
+    b = _msign(xh, "f32tc")
+    assert rel_fro(b, a) <= TOL["f32tc"]
+
+
+def test_msign_three_piece_mode_not_in_noalloc_entry():
+    """lm_msign_ns_noalloc serves LM_BF16 and LM_F32 only."""
+    import torch
+    from paper_2605_19811_gb300 import lionmuon as L
+    x = torch.zeros((32, 48), device="cuda")
+    out = torch.empty_like(x)
+    with pytest.raises(L.LionMuonError) as e:
+        L.msign_ns_noalloc(x, out, 5, *QUINTIC, precision=L.LM_NS_F32_TC)
+    assert e.value.status == 1

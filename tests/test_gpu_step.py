@@ -1,7 +1,8 @@
 """GPU parity of whole LionMuon steps (Algorithm 1) through lm_create/lm_step
 against the storage-modelled fp64 oracle: weights within 1e-3 relative
 (Frobenius) after 8 steps with the fp32 Newton-Schulz path, and within the
-bound the 2e-2 NS tolerance implies with the bf16 tensor-core path; momentum
+bound the 2e-2 NS tolerance implies with the bf16 tensor-core path (and the
+5e-5 one with the three-piece tensor-core fp32 mode, ns_precision 2); momentum
 bit-exact (same-order fp32 EMA); the Muon direction itself within the NS
 tolerance; plus the state-size invariant, status flags and argument errors."""
 
@@ -25,6 +26,8 @@ def _cfg_pair(**kw):
 
 
 NS_TOL_BF16 = 2e-2     # relative Frobenius tolerance of the bf16 NS output
+NS_TOL_F32TC = 5e-5    # the same for the three-piece tensor-core fp32 mode
+F32TC = 2              # LM_NS_F32_TC
 BF16_ULP = 2.0 ** -8   # relative spacing of bf16 values (upper bound)
 
 
@@ -44,7 +47,7 @@ def _check(Wg, Wo, Mg, Mo, tol):
     return worst
 
 
-def _bf16_ns_bounds(W0, grads, dtype, cfg: O.Config, steps, Wo):
+def _bf16_ns_bounds(W0, grads, dtype, cfg: O.Config, steps, Wo, tau_ns=NS_TOL_BF16, storage="bf16", floor=1e-3):
     """Weight tolerance implied by the NS tolerance for the bf16 tensor-core
     path.  The gradients do not depend on W, so the momentum and G_hat are the
     same on both sides and a weight difference only comes from the Muon
@@ -53,7 +56,9 @@ def _bf16_ns_bounds(W0, grads, dtype, cfg: O.Config, steps, Wo):
     <= 1.  For bf16 parameters a pre-rounding difference d of relative size r
     also flips the bf16 rounding of about a fraction r/u of the entries (u the
     bf16 spacing), which adds sqrt(r u) in relative Frobenius terms.  The
-    bound per parameter is 1e-3 + r + sqrt(r u) (the last term for bf16)."""
+    bound per parameter is 1e-3 + r + sqrt(r u) (the last term for bf16).
+    tau_ns, storage, floor: the same bound for another NS mode (the
+    three-piece fp32 mode: 5e-5, fp32 storage, floor 1e-6 for fp32 W)."""
     P = [stored_values(host_tensor(w, dtype)) for w in W0]
     M = [np.zeros_like(p) for p in P]
     acc = [0.0] * len(P)
@@ -62,11 +67,11 @@ def _bf16_ns_bounds(W0, grads, dtype, cfg: O.Config, steps, Wo):
         for i, (p, g, m) in enumerate(zip(P, G, M)):
             if O.is_matrix(p.shape) and O.is_muon_step(t, cfg.period):
                 gh = O.interpolated_direction(m, g, cfg.beta1)
-                tau = NS_TOL_BF16
+                tau = tau_ns
                 if cfg.ns_coeffs is not None:
                     o = O.ns_polynomial_schedule(gh, cfg.ns_coeffs, cfg.ns_eps)
-                    # the table's own sensitivity to bf16 storage (see test_gpu_msign.table_tolerance)
-                    d = rel_fro(O.ns_polynomial_schedule_storage(gh, cfg.ns_coeffs, cfg.ns_eps, "bf16"), o)
+                    # the table's own sensitivity to storage (see test_gpu_msign.table_tolerance)
+                    d = rel_fro(O.ns_polynomial_schedule_storage(gh, cfg.ns_coeffs, cfg.ns_eps, storage), o)
                     tau = max(tau, 1.5 * d)
                 else:
                     o = O.ns_polynomial(gh, cfg.ns_steps, cfg.ns_a, cfg.ns_b, cfg.ns_c, cfg.ns_eps)
@@ -75,7 +80,7 @@ def _bf16_ns_bounds(W0, grads, dtype, cfg: O.Config, steps, Wo):
     out = []
     for a, w in zip(acc, Wo):
         r = a / max(np.linalg.norm(w), 1e-30)
-        out.append(1e-3 + r + (np.sqrt(r * BF16_ULP) if dtype == "bf16" else 0.0))
+        out.append(floor + r + (np.sqrt(r * BF16_ULP) if dtype == "bf16" else 0.0))
     return out
 
 
@@ -89,7 +94,12 @@ def _momentum_same_order(grads, shapes, beta2, steps):
     return M
 
 
-@pytest.mark.parametrize("precision", [1, 0])
+def _f32tc_bounds(W0, grads, dtype, cfg, steps, Wo):
+    return _bf16_ns_bounds(W0, grads, dtype, cfg, steps, Wo, tau_ns=NS_TOL_F32TC, storage="f32",
+                           floor=1e-3 if dtype == "bf16" else 1e-6)
+
+
+@pytest.mark.parametrize("precision", [1, 0, F32TC])
 def test_tiny_config_4_steps(precision):
     """The Tiny set: fp32 params, N(0,1) grads from seed 0, P=2, 4 steps,
     beta=(0.9,0.99), eta=0.02, lambda=0.1, NS per the paper (K=5)."""
@@ -101,7 +111,8 @@ def test_tiny_config_4_steps(precision):
     Wo, _ = run_trajectory_oracle(W0, grads, "f32", ocfg, steps)
     Mo = _momentum_same_order([[stored_values(host_tensor(g, "f32")).astype(np.float32) for g in gs]
                                for gs in grads], TINY.shapes, 0.99, steps)
-    tol = 1e-5 if precision == 0 else _bf16_ns_bounds(W0, grads, "f32", ocfg, steps, Wo)
+    tol = (1e-5 if precision == 0 else _f32tc_bounds(W0, grads, "f32", ocfg, steps, Wo) if precision == F32TC
+           else _bf16_ns_bounds(W0, grads, "f32", ocfg, steps, Wo))
     _check(Wg, Wo, Mg, Mo, tol)
     assert flags == 0
 
@@ -110,7 +121,7 @@ SMALL_GPT = synth.scaled_set("small_gpt", layers=2, d=128, vocab=1000)
 
 
 @pytest.mark.parametrize("period", [2, 1, 4])
-@pytest.mark.parametrize("precision", [1, 0])
+@pytest.mark.parametrize("precision", [1, 0, F32TC])
 def test_small_gpt_8_steps(period, precision):
     """bf16 GPT-style set (2 layers, d=128, vocab 1000, heavy-tailed grads):
     weights after 8 steps within 1e-3 of the storage-modelled oracle."""
@@ -123,12 +134,13 @@ def test_small_gpt_8_steps(period, precision):
     Wo, _ = run_trajectory_oracle(W0, grads, "bf16", ocfg, steps)
     Mo = _momentum_same_order([[stored_values(host_tensor(g, "bf16")).astype(np.float32) for g in gs]
                                for gs in grads], shapes, 0.99, steps)
-    tol = 1e-3 if precision == 0 else _bf16_ns_bounds(W0, grads, "bf16", ocfg, steps, Wo)
+    tol = (1e-3 if precision == 0 else _f32tc_bounds(W0, grads, "bf16", ocfg, steps, Wo) if precision == F32TC
+           else _bf16_ns_bounds(W0, grads, "bf16", ocfg, steps, Wo))
     _check(Wg, Wo, Mg, Mo, tol)
     assert flags == 0
 
 
-@pytest.mark.parametrize("precision,tau", [(1, NS_TOL_BF16), (0, 1e-5)])
+@pytest.mark.parametrize("precision,tau", [(1, NS_TOL_BF16), (0, 1e-5), (F32TC, NS_TOL_F32TC)])
 def test_muon_step_direction_within_ns_tolerance(precision, tau):
     """One Muon step on fp32 parameters (Algorithm 1, Muon branch): the
     direction recovered from the weight change,
@@ -275,7 +287,7 @@ def test_fused_parameter_write_matches_finalize_kernel_bit_exact():
         np.testing.assert_array_equal(a, b)
 
 
-@pytest.mark.parametrize("precision", [1, 0])
+@pytest.mark.parametrize("precision", [1, 0, F32TC])
 def test_small_gpt_8_steps_polar_express_table(precision):
     """Whole steps with an iteration-dependent NS table (the degree-5 minimax
     schedule from l_0 = 1e-3): weights after 8 steps against the
@@ -291,7 +303,8 @@ def test_small_gpt_8_steps_polar_express_table(precision):
     Wo, _ = run_trajectory_oracle(W0, grads, "bf16", ocfg, steps)
     Mo = _momentum_same_order([[stored_values(host_tensor(g, "bf16")).astype(np.float32) for g in gs]
                                for gs in grads], shapes, 0.99, steps)
-    tol = 1e-3 if precision == 0 else _bf16_ns_bounds(W0, grads, "bf16", ocfg, steps, Wo)
+    tol = (1e-3 if precision == 0 else _f32tc_bounds(W0, grads, "bf16", ocfg, steps, Wo) if precision == F32TC
+           else _bf16_ns_bounds(W0, grads, "bf16", ocfg, steps, Wo))
     _check(Wg, Wo, Mg, Mo, tol)
     assert flags == 0
 
