@@ -22,7 +22,8 @@
 // the shared-memory traffic per FLOP of a one-CTA 128 x 256 tile.
 //
 // CTA roles (352 threads, one CTA per SM):
-//   warp 0    TMA producer (one elected lane), 5-stage smem ring; both CTAs'
+//   warp 0    TMA producer (one elected lane), 5-stage smem ring (2 stages
+//             of three-piece operands in the fp32 mode, see TcLayout); both CTAs'
 //             copies signal CTA 0's full barrier
 //   warp 1    TMEM allocator (both CTAs) + MMA issuer (CTA 0, one lane)
 //   warps 2-9 epilogue: tcgen05.ld from TMEM, fused polynomial combination,
