@@ -381,17 +381,23 @@ struct NsLayout {
 // product to a workspace tile of its own (slot = part index + 1); the finish
 // kernel adds the parts in order, so the result does not depend on timing.
 // Tiles near the average stay whole: splitting them buys no balance.
+// kcap > 0 also splits every tile longer than kcap K slices into parts of at
+// most kcap: the three-piece fp32 mode bounds the length of each fp32
+// accumulation in TMEM that way (the parts are added in fp32 by the finish
+// kernel).
 static void split_gram_tiles(const std::vector<NsGroup>& groups, int g0, std::vector<NsTile>& t, int kslice,
-                             int workers, std::vector<std::array<int, 6>>& targets, int& nparts_total) {
+                             int workers, std::vector<std::array<int, 6>>& targets, int& nparts_total,
+                             int kcap = 0) {
   int64_t total = 0;
   for (const NsTile& x : t) total += groups[g0 + x.group].l_pad / kslice;
   const int64_t avg = total / std::max(1, workers);
-  const int64_t part = std::max<int64_t>(8, avg / 2);
+  int64_t part = std::max<int64_t>(8, avg / 2);
+  if (kcap > 0) part = std::min<int64_t>(part, kcap);
   std::vector<NsTile> out;
   nparts_total = 0;
   for (const NsTile& x : t) {
     const int nk = groups[g0 + x.group].l_pad / kslice;
-    if (nk <= 2 * avg || nparts_total + 64 > 65535) {
+    if ((nk <= 2 * avg && (kcap <= 0 || nk <= kcap)) || nparts_total + 64 > 65535) {
       out.push_back(x);
       continue;
     }
@@ -438,7 +444,8 @@ static void layout_ns(std::vector<NsGroup>& groups, lm_dtype xdt, int nmat, Aren
       if (ph == NS_GRAM) {
         int nparts = 0;
         if (xdt == LM_BF16) {
-          split_gram_tiles(groups, g0, t, kTcBK, tc_max_pairs(), targets, nparts);
+          // three-piece mode: no fp32 accumulation over more than 96 K blocks (6144)
+          split_gram_tiles(groups, g0, t, kTcBK, tc_max_pairs(), targets, nparts, pieces == 3 ? 96 : 0);
         } else {
           int dev = 0, sms = 0;
           cudaGetDevice(&dev);

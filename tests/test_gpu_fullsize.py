@@ -171,3 +171,53 @@ def test_stress_7b_muon_then_lion_sampled():
     the Muon direction of a 4096 x 4096 and a 14336 x 4096 matrix against the
     fp64 recurrence, the Lion step bit-exact."""
     _muon_then_lion("stress_7b", 8, [(4096, 4096), (14336, 4096)])
+
+
+def test_720m_three_piece_fp32_mode_directions_sampled():
+    """The 720M-shaped set with ns_precision = LM_NS_F32_TC and fp32
+    parameters and gradients (so that W's storage does not hide the NS
+    error): the Muon
+    direction of one matrix of each hidden shape against the fp64 recurrence
+    within the three-piece tolerance 5e-5, and the embedding's singular values
+    against the scalar map, after one Muon step of the whole set."""
+    import torch
+    from paper_2605_19811_gb300 import lionmuon as L
+    tol = 5e-5
+    ps = synth.PARAM_SETS["gpt_720m"]
+    shapes = [tuple(s) for s in ps.shapes]
+    dev = torch.device("cuda", 0)
+    params = synth.device_weights_torch(shapes, seed=1, device=dev, dtype=torch.float32)
+    g0 = synth.device_grads_torch(shapes, "student_t", seed=10, device=dev, dtype=torch.float32)
+
+    def first(shape):
+        return next(i for i, s in enumerate(shapes) if s == shape)
+    emb = first((50304, 1280))
+    mats = [first((1280, 1280)), first((1280, 3840)), first((1280, 5120)), first((5120, 1280))]
+    sample = mats + [emb]
+    W0 = {i: _host(params[i]) for i in sample}
+    G0 = {i: _host(g0[i]) for i in sample}
+    eta_M = 1.0
+    opt = L.LionMuon(params, period=1, eta_muon=eta_M, eta_lion=1e-3, weight_decay=0.0,
+                     ns_precision=L.LM_NS_F32_TC)
+    opt.step(g0, 0)
+    torch.cuda.synchronize()
+    W1 = {i: _host(params[i]) for i in sample}
+    for i in mats:
+        s = 0.2 * math.sqrt(max(shapes[i]))
+        o_gpu = (W0[i].astype(np.float64) - W1[i].astype(np.float64)) / (eta_M * s)
+        o_ref = O.ns_polynomial(0.1 * G0[i].astype(np.float64), 5, *O.NS_QUINTIC, 1e-7)
+        # fp32 W: its rounding adds up to 2^-24 (|W0| + |W1|) / (eta s)
+        slack = 2.0 ** -24 * (np.linalg.norm(W0[i]) + np.linalg.norm(W1[i])) / (eta_M * s) / np.linalg.norm(o_ref)
+        assert rel_fro(o_gpu, o_ref) <= tol + slack, (shapes[i], rel_fro(o_gpu, o_ref))
+    s = 0.2 * math.sqrt(50304)
+    o_emb = (W0[emb].astype(np.float64) - W1[emb].astype(np.float64)) / (eta_M * s)
+    gh = 0.1 * G0[emb].astype(np.float64)
+    sig_g = np.sqrt(np.clip(np.linalg.eigvalsh(gh.T @ gh), 0, None))
+    sig_o = np.sqrt(np.clip(np.linalg.eigvalsh(o_emb.T @ o_emb), 0, None))
+    want = np.sort(O.ns_scalar_map(sig_g / (np.linalg.norm(sig_g) + 1e-7), 5, *O.NS_QUINTIC))
+    slack = 2.0 ** -24 * (np.linalg.norm(W0[emb]) + np.linalg.norm(W1[emb])) / (eta_M * s) / np.linalg.norm(want)
+    assert np.linalg.norm(np.sort(sig_o) - want) / np.linalg.norm(want) <= tol + slack
+    assert opt.status() == 0
+    opt.close()
+    del params, g0
+    torch.cuda.empty_cache()
