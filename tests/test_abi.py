@@ -74,9 +74,10 @@ def test_create_rejects_bad_arguments_before_device_use(lib):
     bad = L.LmConfig.from_buffer_copy(cfg)
     bad.period = -1
     assert lib.lm_create(one, 1, ctypes.byref(bad), None, ctypes.byref(h)) == 1
-    bad = L.LmConfig.from_buffer_copy(cfg)
-    bad.ns_precision = 7
-    assert lib.lm_create(one, 1, ctypes.byref(bad), None, ctypes.byref(h)) == 1
+    for p in (7, 3, -1):          # LM_F32 (0), LM_BF16 (1) and LM_NS_F32_TC (2) are the valid values
+        bad = L.LmConfig.from_buffer_copy(cfg)
+        bad.ns_precision = p
+        assert lib.lm_create(one, 1, ctypes.byref(bad), None, ctypes.byref(h)) == 1
     misaligned = (L.LmTensor * 1)(_tensor(4098, 4, 4, L.LM_BF16))
     assert lib.lm_create(misaligned, 1, ctypes.byref(cfg), None, ctypes.byref(h)) == 3
     null = (L.LmTensor * 1)(_tensor(0, 4, 4, L.LM_BF16))
@@ -96,6 +97,9 @@ def test_msign_rejects_bad_arguments(lib):
     assert lib.lm_msign_ns(ctypes.byref(v), ctypes.byref(v), 5, 1, 1, 1, 0, 1, None) == 1
     assert lib.lm_msign_ns(ctypes.byref(a), ctypes.byref(a), -1, 1, 1, 1, 0, 1, None) == 1
     assert lib.lm_msign_ns(ctypes.byref(a), ctypes.byref(a), 5, 1, 1, 1, 0, 9, None) == 1
+    assert lib.lm_msign_ns(ctypes.byref(a), ctypes.byref(a), 5, 1, 1, 1, 0, 3, None) == 1
+    # the no-alloc entry point has no three-piece mode
+    assert lib.lm_msign_ns_noalloc(ctypes.byref(a), ctypes.byref(a), 5, 1, 1, 1, 0, L.LM_NS_F32_TC, None) == 1
 
 
 def test_null_handles_are_safe(lib):
