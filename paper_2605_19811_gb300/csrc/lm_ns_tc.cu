@@ -55,6 +55,7 @@ constexpr int BM = kTcBM, BN = kTcBN, BK = kTcBK;   // pair tile 256 x 256, K st
 constexpr int kHalf = 128;                           // A rows / B N-rows per CTA
 constexpr int kABytes = kHalf * BK * 2;              // 16 KB
 constexpr int kBBytes = kHalf * BK * 2;              // 16 KB
+static_assert(kABytes == kBBytes, "diagonal tiles read their A boxes as B");
 constexpr int kEpiWarps = 8;
 constexpr int kAuxWarp = 2 + kEpiWarps;              // warp that loads the epilogue's aux tile
 constexpr int kThreads = 32 * (3 + kEpiWarps);
@@ -379,19 +380,22 @@ struct ProducerRing {
 };
 // kP pieces per operand: piece q of matrix mat is matrix mat + q * pstride
 // of the tensor map; a stage holds the kP A pieces, then the kP B pieces.
+// same: both operands are the same rows of the same matrix (a diagonal Gram
+// or polynomial tile), so only the A boxes are loaded and the MMA reads them
+// as B too.
 template <bool AMN, bool BMN, int kP>
 __device__ __forceinline__ bool produce_range(ProducerRing<TcLayout<kP>::kStages>& R, uint8_t* smem,
                                               uint64_t* full, uint64_t* empty, volatile int* abort_flag,
                                               uint32_t rank, int kb0, int kb1, const CUtensorMap* map_a,
                                               const CUtensorMap* map_b, int row_a, int col_b, int mat,
-                                              int pstride) {
+                                              int pstride, bool same) {
   using L = TcLayout<kP>;
   for (int kb = kb0; kb < kb1; ++kb) {
     if (!mbar_wait(&empty[R.stage], R.ph ^ 1u, abort_flag, kWaitLimitNs)) return false;
     uint8_t* sa = smem + (size_t)R.stage * L::kStageBytes;
     uint8_t* sb = sa + kP * kABytes;
     const uint32_t fb = peer_addr(&full[R.stage], 0);
-    if (rank == 0) mbar_arrive_expect_tx(&full[R.stage], 2 * L::kStageBytes);
+    if (rank == 0) mbar_arrive_expect_tx(&full[R.stage], same ? 2 * kP * kABytes : 2 * L::kStageBytes);
     R.armed[R.stage] = (int)R.ph;
     const int k0 = kb * BK;
 #pragma unroll
@@ -400,7 +404,7 @@ __device__ __forceinline__ bool produce_range(ProducerRing<TcLayout<kP>::kStages
       else tma_load_4d(sa + q * kABytes, map_a, fb, 0, k0, row_a >> 6, mat + q * pstride);
     }
 #pragma unroll
-    for (int q = 0; q < kP; ++q) {
+    for (int q = 0; q < kP && !same; ++q) {
       if (!BMN) tma_load_3d(sb + q * kBBytes, map_b, fb, k0, col_b, mat + q * pstride);
       else tma_load_4d(sb + q * kBBytes, map_b, fb, 0, k0, col_b >> 6, mat + q * pstride);
     }
@@ -419,7 +423,7 @@ __device__ __forceinline__ bool produce_range(ProducerRing<TcLayout<kP>::kStages
 template <bool AMN, bool BMN, int kP>
 __device__ __forceinline__ bool mma_range(int& stage, uint32_t& ph, uint8_t* smem, uint64_t* full,
                                           uint64_t* empty, volatile int* abort_flag, int kb0, int kb1,
-                                          uint32_t d_tmem, int kb_first) {
+                                          uint32_t d_tmem, int kb_first, bool same) {
   using L = TcLayout<kP>;
   constexpr int kProducts = kP == 1 ? 1 : 6;
   constexpr int qa[6] = {0, 0, 1, 0, 2, 1};
@@ -429,7 +433,7 @@ __device__ __forceinline__ bool mma_range(int& stage, uint32_t& ph, uint8_t* sme
     if (!mbar_wait(&full[stage], ph, abort_flag, kWaitLimitNs)) return false;
     tc_fence_after();
     const uint32_t sa = smem_u32(smem + (size_t)stage * L::kStageBytes);
-    const uint32_t sb = sa + kP * kABytes;
+    const uint32_t sb = same ? sa : sa + kP * kABytes;   // kBBytes == kABytes
 #pragma unroll
     for (int kk = 0; kk < BK / 16; ++kk) {
 #pragma unroll
@@ -600,13 +604,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           const OpSeg& S = P.seg[sg];
           if (!S.a_mn && !S.b_mn)
             ok = produce_range<false, false, kP>(R, smem, full, empty, abort_flag, rank, kb0, S.kb_end, S.map_a,
-                                             S.map_b, row_a, col_b, t.mat, g.count);
+                                             S.map_b, row_a, col_b, t.mat, g.count,
+                                             S.map_a == S.map_b && row_a == col_b);
           else if (!S.a_mn)
             ok = produce_range<false, true, kP>(R, smem, full, empty, abort_flag, rank, kb0, S.kb_end, S.map_a,
-                                            S.map_b, row_a, col_b, t.mat, g.count);
+                                            S.map_b, row_a, col_b, t.mat, g.count,
+                                             S.map_a == S.map_b && row_a == col_b);
           else
             ok = produce_range<true, true, kP>(R, smem, full, empty, abort_flag, rank, kb0, S.kb_end, S.map_a,
-                                           S.map_b, row_a, col_b, t.mat, g.count);
+                                           S.map_b, row_a, col_b, t.mat, g.count,
+                                             S.map_a == S.map_b && row_a == col_b);
           kb0 = S.kb_end;
         }
         if (!ok) give_up();
@@ -644,13 +651,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           const OpSeg& S = P.seg[sg];
           if (!S.a_mn && !S.b_mn)
             ok = mma_range<false, false, kP>(stage, ph, smem, full, empty, abort_flag, kb0, S.kb_end, d_tmem,
-                                            P.kb_start);
+                                            P.kb_start, S.map_a == S.map_b && t.tm == t.tn);
           else if (!S.a_mn)
             ok = mma_range<false, true, kP>(stage, ph, smem, full, empty, abort_flag, kb0, S.kb_end, d_tmem,
-                                            P.kb_start);
+                                            P.kb_start, S.map_a == S.map_b && t.tm == t.tn);
           else
             ok = mma_range<true, true, kP>(stage, ph, smem, full, empty, abort_flag, kb0, S.kb_end, d_tmem,
-                                            P.kb_start);
+                                            P.kb_start, S.map_a == S.map_b && t.tm == t.tn);
           kb0 = S.kb_end;
         }
         if (!ok) give_up();
