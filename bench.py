@@ -55,6 +55,8 @@ def parse_args():
     ap.add_argument("--vector-rule", choices=["lion", "adamw"], default="lion",
                     help="1-D parameters: the Lion step, or the AdamW fallback of Section 3")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--cublas-context", action="store_true",
+                    help="also time the same NS iterations in torch.bmm/baddbmm (cuBLAS) for context")
     ap.add_argument("--no-cpu", action="store_true")
     return ap.parse_args()
 
@@ -81,6 +83,47 @@ def ns_flops_sym(mats, steps=5):
         s, l = min(a, b), max(a, b)
         tot += steps * (3.0 * s * s * l + 1.0 * s ** 3)
     return tot
+
+
+def cublas_ns_context(mats, dev, reps=5):
+    """Context only, not the library's path: the same five NS iterations in
+    torch.bmm / torch.baddbmm (cuBLAS) on the set's matrices (wide
+    orientation, batched per shape), bf16 operands: A = X X^T, B = b A + c A A,
+    X = a X + B X, with the symmetric products computed in full.  Returns ms
+    per Muon step's NS (CUDA events, after warm-up)."""
+    import torch
+    a, b, c = 3.4445, -4.7750, 2.0315
+    groups = {}
+    for m, n in mats:
+        key = (min(m, n), max(m, n))
+        groups[key] = groups.get(key, 0) + 1
+    bufs = []
+    for (sm, lg), cnt in groups.items():
+        x = torch.randn(cnt, sm, lg, device=dev, dtype=torch.bfloat16) / math.sqrt(sm * lg)
+        bufs.append([x, torch.empty_like(x), torch.empty(cnt, sm, sm, device=dev, dtype=torch.bfloat16),
+                     torch.empty(cnt, sm, sm, device=dev, dtype=torch.bfloat16)])
+
+    def ns():
+        for buf in bufs:
+            for _ in range(5):
+                x, y, A, B = buf
+                torch.bmm(x, x.transpose(1, 2), out=A)
+                torch.baddbmm(A, A, A, beta=b, alpha=c, out=B)
+                torch.baddbmm(x, B, x, beta=a, alpha=1.0, out=y)
+                buf[0], buf[1] = y, x
+    for _ in range(2):
+        ns()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(reps):
+        ns()
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / reps
+    del bufs
+    torch.cuda.empty_cache()
+    return ms
 
 
 def load_peaks():
@@ -443,6 +486,13 @@ def run_ours(args):
     clk = clocks.stop()
     flags = opt.status()
     took_last = opt.selection()[0] if srank else None
+    context = None
+    if args.cublas_context and rank == 0:
+        dense = sum(5 * (4.0 * min(m, n) ** 2 * max(m, n) + 2.0 * min(m, n) ** 3) for m, n in mats)
+        cms = cublas_ns_context(mats, dev)
+        context = {"what": "the same 5 NS iterations in torch.bmm/baddbmm (cuBLAS, bf16), full symmetric products, "
+                           "for context only (not the library's path)",
+                   "cublas_ms_per_muon_step": cms, "cublas_dense_tflops": dense / (cms / 1e3) / 1e12}
 
     # ---- roofline of the dominant kernel family ----
     peaks, peak_src = load_peaks()
@@ -502,6 +552,8 @@ def run_ours(args):
                       "per_step_ms": sr_ms / args.steps, "peak_kind": f"HBM copy, {peak_src}",
                       "bytes": "4 B x matrix elements x passes (plus resets and the decision)"}
     fam_ms = {k: v[0] / args.steps for k, v in prof.items() if k != "ns_gemm"}
+    if context is not None and n_muon > 0:
+        context["library_ns_ms_per_muon_step"] = ns_ms / n_muon
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
@@ -534,6 +586,7 @@ def run_ours(args):
             "kernel_ms_per_step": fam_ms,
             "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches, "clocks": clk,
             "device_flags": flags,
+            **({"context_cublas": context} if context else {}),
         }
         print(json.dumps(line), flush=True)
     opt.close()
