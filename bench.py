@@ -524,8 +524,11 @@ def run_ours(args):
             peak_kind = f"fp32 FMA, derived: {sms} SMs x 128 lanes x 2 FLOP x {mhz:.0f} MHz"
         # the recorded ncu traffic is the bf16 workload's
         traffic = kernel_traffic(kernel) if args.precision != "f32tc" else None
+        dense = sum(5 * (4.0 * min(m, n) ** 2 * max(m, n) + 2.0 * min(m, n) ** 3) for m, n in mats) * n_muon
         roof = {"bound": bound, "achieved": achieved, "peak": pk, "unit": "TFLOP/s",
                 "frac": achieved / pk, "traffic": traffic, "kernel": kernel,
+                # the same time over the dense count 4 s^2 l + 2 s^3 (both symmetric products in full)
+                "dense_equivalent_tflops": dense / (ns_ms / 1e3) / 1e12,
                 "per_launch_ms": ns_ms / max(ns_launches, 1),
                 "per_launch_tflop": fl / max(ns_launches, 1) / 1e12,
                 "peak_kind": peak_kind,
