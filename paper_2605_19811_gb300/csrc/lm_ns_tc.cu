@@ -67,13 +67,15 @@ constexpr int kAuxBoxBytes = kHalf * 64 * 2;         // one 64-column box of the
 // Shared-memory layout per operand precision.  kP = 1: bf16 operands, a
 // 5-stage ring of 32 KB per CTA and a 64 KB aux/staging buffer.  kP = 3:
 // fp32 operands held as three bf16 pieces (hi + mid + lo, exact), a 2-stage
-// ring of 96 KB per CTA, no aux buffer (that epilogue works from global memory).
+// ring of 96 KB per CTA and a 4 KB transpose tile per epilogue warp (that
+// epilogue reads its aux values and writes its results through global memory).
 template <int kP>
 struct TcLayout {
   static constexpr int kStages = kP == 1 ? 5 : 2;
   static constexpr int kStageBytes = kP * (kABytes + kBBytes);
   static constexpr size_t kAuxOffset = (size_t)kStages * kStageBytes;
-  static constexpr size_t kBarOffset = kAuxOffset + (kP == 1 ? 4 * kAuxBoxBytes : 0);
+  // kP = 1: the aux / staging boxes; kP = 3: a 32 x 33 fp32 transpose tile per epilogue warp
+  static constexpr size_t kBarOffset = kAuxOffset + (kP == 1 ? 4 * kAuxBoxBytes : 8 * 32 * 33 * 4);
   static constexpr size_t kSmemBytes = 1024 /*align slack*/ + kBarOffset + 256;
 };
 
@@ -461,31 +463,44 @@ __device__ __forceinline__ void split3(float v, float& h, float& m, float& l) {
   m = __bfloat162float(__float2bfloat16_rn(r1));
   l = r1 - m;
 }
-// Epilogue of one 32-column chunk (columns j0 ..) of row i with three-piece
-// operands; the aux values and the results go through global memory.
+// Epilogue of one 32 x 32 chunk (rows r0 .. r0 + 31, one per lane; columns
+// j0 ..) with three-piece operands; aux values and results go through global
+// memory, coalesced through the warp's transpose tile stg: lane l reads and
+// writes 16 bytes of row l / 4 + 8 k (k = 0 .. 3), so a warp access covers 8
+// rows x 64 bytes of one plane.
 //   aux: the A (POLY) or X (APPLY) element, hi + mid + lo; out: the result's
-//   pieces, or fp32 in out_f32 (last APPLY).  plane = elements per piece.
+//   pieces, or fp32 in out_f32 (last APPLY).  base: element (r0, j0) of the
+//   matrix in plane 0; ld: row length; plane: elements per piece.
 __device__ __forceinline__ void piece_chunk(const uint32_t (&r)[32], int phase, const NsCoeffs& co, float nscale,
                                             const __nv_bfloat16* aux, __nv_bfloat16* out, float* out_f32,
-                                            size_t plane, size_t off, bool row_ok, int j0, int ncols) {
+                                            size_t plane, size_t base, size_t ld, bool row_ok, int j0, int ncols,
+                                            float (*stg)[33], int lane) {
+  const int rr = lane >> 2, c8 = (lane & 3) * 8;
   float v[32];
   if (phase != NS_GRAM) {
 #pragma unroll
-    for (int e = 0; e < 32; ++e) v[e] = 0.f;
+    for (int k = 0; k < 4; ++k) {
+      const int row = rr + 8 * k;
+      float a8[8];
 #pragma unroll
-    for (int q = 0; q < 3; ++q) {
-      const uint4* src = reinterpret_cast<const uint4*>(aux + q * plane + off);
+      for (int t = 0; t < 8; ++t) a8[t] = 0.f;
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const uint4 a4 = src[u];
+      for (int q = 0; q < 3; ++q) {
+        const uint4 a4 = *reinterpret_cast<const uint4*>(aux + q * plane + base + (size_t)row * ld + c8);
         const uint32_t aw[4] = {a4.x, a4.y, a4.z, a4.w};
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-          v[u * 8 + 2 * e] += bf_lo(aw[e]);
-          v[u * 8 + 2 * e + 1] += bf_hi(aw[e]);
+          a8[2 * e] += bf_lo(aw[e]);
+          a8[2 * e + 1] += bf_hi(aw[e]);
         }
       }
+#pragma unroll
+      for (int t = 0; t < 8; ++t) stg[row][c8 + t] = a8[t];
     }
+    __syncwarp();
+#pragma unroll
+    for (int e = 0; e < 32; ++e) v[e] = stg[lane][e];
+    __syncwarp();
   }
 #pragma unroll
   for (int e = 0; e < 32; ++e) {
@@ -494,30 +509,37 @@ __device__ __forceinline__ void piece_chunk(const uint32_t (&r)[32], int phase, 
     if (phase == NS_GRAM) o = acc * nscale;
     else if (phase == NS_POLY) o = co.b * v[e] + co.c * acc;
     else o = (co.a * v[e] + acc) * nscale;
-    v[e] = (row_ok && j0 + e < ncols) ? o : 0.f;
+    stg[lane][e] = (row_ok && j0 + e < ncols) ? o : 0.f;
   }
-  if (out_f32 != nullptr) {
-    float4* dst = reinterpret_cast<float4*>(out_f32 + off);
+  __syncwarp();
 #pragma unroll
-    for (int u = 0; u < 8; ++u) dst[u] = make_float4(v[4 * u], v[4 * u + 1], v[4 * u + 2], v[4 * u + 3]);
-    return;
-  }
+  for (int k = 0; k < 4; ++k) {
+    const int row = rr + 8 * k;
+    float o8[8];
 #pragma unroll
-  for (int u = 0; u < 4; ++u) {
+    for (int t = 0; t < 8; ++t) o8[t] = stg[row][c8 + t];
+    const size_t off = base + (size_t)row * ld + c8;
+    if (out_f32 != nullptr) {
+      float4* dst = reinterpret_cast<float4*>(out_f32 + off);
+      dst[0] = make_float4(o8[0], o8[1], o8[2], o8[3]);
+      dst[1] = make_float4(o8[4], o8[5], o8[6], o8[7]);
+      continue;
+    }
     uint32_t w[3][4];
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
       float h0, m0, l0, h1, m1, l1;
-      split3(v[u * 8 + 2 * e], h0, m0, l0);
-      split3(v[u * 8 + 2 * e + 1], h1, m1, l1);
+      split3(o8[2 * e], h0, m0, l0);
+      split3(o8[2 * e + 1], h1, m1, l1);
       w[0][e] = pack_bf2(h0, h1);
       w[1][e] = pack_bf2(m0, m1);
       w[2][e] = pack_bf2(l0, l1);
     }
 #pragma unroll
     for (int q = 0; q < 3; ++q)
-      reinterpret_cast<uint4*>(out + q * plane + off)[u] = make_uint4(w[q][0], w[q][1], w[q][2], w[q][3]);
+      *reinterpret_cast<uint4*>(out + q * plane + off) = make_uint4(w[q][0], w[q][1], w[q][2], w[q][3]);
   }
+  __syncwarp();   // the tile is reused by the next chunk
 }
 
 // ------------------------------- the kernel ---------------------------------
@@ -764,12 +786,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           // rows of the output: s_pad or l_pad (APPLY tall); ld its row length
           const size_t ld = (size_t)(phase == NS_APPLY ? (g.tall ? g.s_pad : g.l_pad) : g.s_pad);
           const size_t msize = (size_t)(phase == NS_APPLY ? (size_t)g.s_pad * g.l_pad : (size_t)g.s_pad * g.s_pad);
-          const size_t off = (size_t)t.mat * msize + (size_t)i * ld + j0;
+          const size_t base = (size_t)t.mat * msize + (size_t)r0 * ld + j0;   // row r0 = this warp's first
           const size_t plane = (size_t)g.count * msize;
           const __nv_bfloat16* aux = static_cast<const __nv_bfloat16*>(phase == NS_POLY ? g.A : g.X[cur]);
           __nv_bfloat16* out = static_cast<__nv_bfloat16*>(phase == NS_GRAM ? g.A : (phase == NS_POLY ? g.B : g.X[cur ^ 1]));
           float* out_f32 = (phase == NS_APPLY && p.final_f32) ? static_cast<float*>(g.Xf) : nullptr;
-          piece_chunk(r, phase, p.co, nscale, aux, out, out_f32, plane, off, i < nrows, j0, ncols);
+          float (*stg)[33] = reinterpret_cast<float (*)[33]>(auxbuf) + (warp - 2) * 32;
+          piece_chunk(r, phase, p.co, nscale, aux, out, out_f32, plane, base, ld, i < nrows, j0, ncols, stg, lane);
           continue;
         }
         if (split) {
