@@ -445,8 +445,11 @@ cudaError_t launch_momentum_norm(lm_dtype xdt, lm_dtype gdt, const MatDesc* mats
                                  int nchunks, const void* const* grads, MuonConsts k, int mode,
                                  cudaStream_t st) {
   if (nchunks <= 0) return cudaSuccess;
-  static int grid_cap = 0;
+  static int grid_caps[kMaxDevices] = {};
+  const int slot = device_slot();
+  int grid_cap = slot >= 0 ? grid_caps[slot] : 0;
   if (grid_cap == 0) grid_cap = elem_grid_size(momentum_norm_kernel<__nv_bfloat16, __nv_bfloat16, 0>);
+  if (slot >= 0) grid_caps[slot] = grid_cap;
   const int grid = nchunks < grid_cap ? nchunks : grid_cap;
   count_launch();
   if (xdt == LM_BF16) {
@@ -462,8 +465,11 @@ cudaError_t launch_momentum_norm(lm_dtype xdt, lm_dtype gdt, const MatDesc* mats
 cudaError_t launch_finalize(lm_dtype xdt, lm_dtype pdt, const MatDesc* mats, const ElemChunk* chunks,
                             int nchunks, MuonConsts k, int mode, unsigned* flags, cudaStream_t st) {
   if (nchunks <= 0) return cudaSuccess;
-  static int grid_cap = 0;
+  static int grid_caps[kMaxDevices] = {};
+  const int slot = device_slot();
+  int grid_cap = slot >= 0 ? grid_caps[slot] : 0;
   if (grid_cap == 0) grid_cap = elem_grid_size(finalize_kernel<__nv_bfloat16, __nv_bfloat16, 0>);
+  if (slot >= 0) grid_caps[slot] = grid_cap;
   const int grid = nchunks < grid_cap ? nchunks : grid_cap;
   count_launch();
   if (xdt == LM_BF16) {

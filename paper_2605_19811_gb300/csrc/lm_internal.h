@@ -256,6 +256,11 @@ constexpr int kMaxGroupsSimt = 64;
 
 // Launch accounting (lm_kernel_launch_count) and the thread's last-error text.
 void count_launch();
+// Per-device slot for the launchers' one-time set-ups (kernel attributes set
+// and grid sizes read on each device the process uses): the current device,
+// or -1 when it cannot be used as an index (beyond kMaxDevices).
+constexpr int kMaxDevices = 64;
+int device_slot();
 lm_status set_error(lm_status st, const char* msg);
 
 // Pointer table upload (grads) as a kernel with the pointers in its parameters.

@@ -28,7 +28,6 @@ namespace {
 constexpr size_t kNoAllocScratchBytes = (size_t)64 << 20;   // 64 MiB
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
-constexpr int kMaxDevices = 64;
 std::mutex g_scratch_mu;
 char* g_scratch_addr[kMaxDevices] = {nullptr};
 

@@ -1093,8 +1093,9 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
   if (ngroups < 1 || ngroups > kMaxGroupsTc) return cudaErrorInvalidValue;
   if (pieces != 1 && pieces != 3) return cudaErrorInvalidValue;
   if (pieces == 3 && fuse != nullptr) return cudaErrorInvalidValue;
-  static bool attr_set = false;
-  if (!attr_set) {
+  static bool attr_set[kMaxDevices] = {};
+  const int slot = device_slot();
+  if (slot < 0 || !attr_set[slot]) {
     cudaError_t e = set_smem_attr<false, false, 1>();
     if (e == cudaSuccess) e = set_smem_attr<true, false, 1>();
     if (e == cudaSuccess) e = set_smem_attr<false, true, 1>();
@@ -1104,7 +1105,7 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
     if (e == cudaSuccess) e = set_smem_attr<false, true, 3>();
     if (e == cudaSuccess) e = set_smem_attr<true, true, 3>();
     if (e != cudaSuccess) return e;
-    attr_set = true;
+    if (slot >= 0) attr_set[slot] = true;
   }
   TcParams prm;
   memset(&prm, 0, sizeof(prm));

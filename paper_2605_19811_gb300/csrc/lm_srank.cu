@@ -497,11 +497,12 @@ cudaError_t ring_launch(const SrMat* mats, const SrItem* items, int nitems, int 
   const int stride = (max_cols + 3) / 4 * 4;
   const int nst = 3;
   const size_t smem = (size_t)nst * RB * stride * 4;
-  static bool attr_set = false;   // per instantiation
-  if (!attr_set) {
+  static bool attr_set[kMaxDevices] = {};   // per instantiation and device
+  const int slot = device_slot();
+  if (slot < 0 || !attr_set[slot]) {
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
     if (e != cudaSuccess) return e;
-    attr_set = true;
+    if (slot >= 0) attr_set[slot] = true;
   }
   int dev = 0, sms = 0, per_sm = 0;
   cudaGetDevice(&dev);
