@@ -551,7 +551,7 @@ def run_ours(args):
         gbs = 4.0 * mat_elems * args.srank_iters * args.steps / (sr_ms / 1e3) / 1e9
         pk = peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
         srank_roof = {"bound": "hbm", "achieved": gbs, "peak": pk, "unit": "GB/s", "frac": gbs / pk,
-                      "traffic": None, "kernel": "srank_pass_kernel",
+                      "traffic": None, "kernel": "srank_ring_kernel",
                       "per_step_ms": sr_ms / args.steps, "peak_kind": f"HBM copy, {peak_src}",
                       "bytes": "4 B x matrix elements x passes (plus resets and the decision)"}
     fam_ms = {k: v[0] / args.steps for k, v in prof.items() if k != "ns_gemm"}

@@ -692,6 +692,12 @@ struct lm_state {
   unsigned char* d_skip = nullptr;      // per parameter: Lion kernel skips it
   double* d_srank = nullptr;            // per matrix id: the estimate
   std::vector<int> mat_param_of;        // matrix id -> parameter index
+  // With two or more column-count launches per pass, launches after the
+  // first go to side streams forked from and joined back to the caller's
+  // stream, so that one launch's last blocks overlap the next launch.
+  cudaStream_t sr_side[2] = {nullptr, nullptr};
+  cudaEvent_t sr_fork = nullptr, sr_join[2] = {nullptr, nullptr};
+  int sr_nside = 0;
   int64_t last_t = -1;
   // LM_DEBUG guard bands: device list of their offsets
   bool debug = false;
@@ -709,6 +715,30 @@ struct lm_state {
   cudaStream_t last_stream = nullptr;
   Profiler prof;
 };
+
+// Side streams of the stable-rank passes (non-blocking, device of lm_create)
+// and the events that fork them from and join them to the caller's stream.
+static cudaError_t create_side_streams(lm_state* s) {
+  s->sr_nside = std::min<int>(2, (int)s->sr_launch.size() - 1);
+  cudaError_t e = cudaEventCreateWithFlags(&s->sr_fork, cudaEventDisableTiming);
+  for (int k = 0; e == cudaSuccess && k < s->sr_nside; ++k) {
+    e = cudaStreamCreateWithFlags(&s->sr_side[k], cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&s->sr_join[k], cudaEventDisableTiming);
+  }
+  return e;
+}
+
+static void destroy_side_streams(lm_state* s) {
+  for (int k = 0; k < 2; ++k) {
+    if (s->sr_join[k]) cudaEventDestroy(s->sr_join[k]);
+    if (s->sr_side[k]) cudaStreamDestroy(s->sr_side[k]);
+    s->sr_join[k] = nullptr;
+    s->sr_side[k] = nullptr;
+  }
+  if (s->sr_fork) cudaEventDestroy(s->sr_fork);
+  s->sr_fork = nullptr;
+  s->sr_nside = 0;
+}
 
 extern "C" {
 
@@ -1106,6 +1136,12 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
     delete s;
     return st;
   }
+  if (s->srank && s->sr_launch.size() >= 2 && (e = create_side_streams(s)) != cudaSuccess) {
+    destroy_side_streams(s);
+    cudaFree(s->base);
+    delete s;
+    return cuda_fail(e, "stable-rank side streams");
+  }
   s->last_stream = stream;
   *out = s;
   return LM_OK;
@@ -1152,14 +1188,30 @@ static lm_status run_srank(lm_state* s, cudaStream_t stream) {
       e = cudaMemsetAsync(out, 0, s->sr_w_elems * sizeof(float), stream);
       if (e != cudaSuccess) return cuda_fail(e, "selection buffer reset");
     }
-    for (const auto& L : s->sr_launch) {
-      e = timed(P, LM_KERNEL_SRANK, stream, [&]() {
-        if (L.vec4)
-          return launch_srank_ring((int)L.max_cols, s->d_sr, L.items, L.nitems, k, last, s->d_flags, stream);
-        return launch_srank_pass(L.slots, L.threads, L.vec4, s->d_sr, L.items, L.nitems, k, last, stream);
-      });
-      if (e != cudaSuccess) return cuda_fail(e, "power-iteration launch");
+    auto launch = [&](const lm_state::SrLaunch& L, cudaStream_t st) {
+      if (L.vec4) return launch_srank_ring((int)L.max_cols, s->d_sr, L.items, L.nitems, k, last, s->d_flags, st);
+      return launch_srank_pass(L.slots, L.threads, L.vec4, s->d_sr, L.items, L.nitems, k, last, st);
+    };
+    if (s->sr_nside == 0) {
+      for (const auto& L : s->sr_launch) {
+        e = timed(P, LM_KERNEL_SRANK, stream, [&]() { return launch(L, stream); });
+        if (e != cudaSuccess) return cuda_fail(e, "power-iteration launch");
+      }
+      continue;
     }
+    // The launches of one pass touch disjoint matrices: the first runs on the
+    // caller's stream, the others on the side streams, all after this pass's
+    // reset and before anything the caller enqueues next.
+    e = timed(P, LM_KERNEL_SRANK, stream, [&]() {
+      cudaError_t r = cudaEventRecord(s->sr_fork, stream);
+      for (int q = 0; r == cudaSuccess && q < s->sr_nside; ++q) r = cudaStreamWaitEvent(s->sr_side[q], s->sr_fork, 0);
+      for (size_t g = 0; r == cudaSuccess && g < s->sr_launch.size(); ++g)
+        r = launch(s->sr_launch[g], g == 0 ? stream : s->sr_side[(g - 1) % s->sr_nside]);
+      for (int q = 0; r == cudaSuccess && q < s->sr_nside; ++q) r = cudaEventRecord(s->sr_join[q], s->sr_side[q]);
+      for (int q = 0; r == cudaSuccess && q < s->sr_nside; ++q) r = cudaStreamWaitEvent(stream, s->sr_join[q], 0);
+      return r;
+    });
+    if (e != cudaSuccess) return cuda_fail(e, "power-iteration launch");
   }
   e = timed(P, LM_KERNEL_SRANK, stream, [&]() {
     return launch_srank_decide(s->d_sr, s->nmat, s->cfg.srank_alpha, passes - 1, s->d_active, s->d_skip,
@@ -1474,6 +1526,7 @@ size_t lm_workspace_bytes(const lm_state* s) {
 void lm_destroy(lm_state* s) {
   if (s == nullptr) return;
   cudaStreamSynchronize(s->last_stream);
+  destroy_side_streams(s);
   cudaFree(s->base);
   delete s;
 }

@@ -16,8 +16,9 @@
 // Matrices whose rows are 16-byte multiples (columns divisible by 4) go
 // through the ring kernel instead: a producer warp streams whole rows into a
 // shared-memory ring with 1-D bulk copies (cp.async.bulk, completion on an
-// mbarrier per stage), and eight consumer warps read their columns of each
-// staged row twice from shared memory (dot product, then the M^T u update).
+// mbarrier per stage), and eight or ten consumer warps read their columns of
+// each staged row twice from shared memory (dot product, then the M^T u
+// update).
 // Loads are thus decoupled from the per-batch reductions, and a batch can
 // hold many rows without using registers.  Every mbarrier wait is bounded;
 // a wait that gives up sets LM_FLAG_TIMEOUT and the block stops.
@@ -81,8 +82,9 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
       "l"(src), "r"(bytes), "r"(smem_addr(bar))
       : "memory");
 }
-// barrier over the 256 consumer threads only (the producer warp stays out)
-__device__ __forceinline__ void consumers_sync() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+// barrier over the NC consumer warps only (the producer warp stays out)
+template <int NC>
+__device__ __forceinline__ void consumers_sync() { asm volatile("bar.sync 1, %0;" ::"n"(32 * NC) : "memory"); }
 
 template <int TPB>
 __device__ __forceinline__ double block_sum(double x, double* red) {
@@ -235,40 +237,41 @@ __global__ void __launch_bounds__(TPB)
 }
 
 constexpr int kRingMaxStages = 4;
-constexpr int kRingThreads = 256 + 32;          // 8 consumer warps + 1 producer warp
 constexpr uint64_t kRingWaitNs = 2000000000ull;  // 2 s
 
+template <int NC>
 __device__ __forceinline__ double consumer_sum(double x, double* red) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = x;
-  consumers_sync();
+  consumers_sync<NC>();
   double s = 0.0;
 #pragma unroll
-  for (int w = 0; w < 8; ++w) s += red[w];
-  consumers_sync();
+  for (int w = 0; w < NC; ++w) s += red[w];
+  consumers_sync<NC>();
   return s;
 }
 
 // One pass over the items of this launch (all matrices have cols % 4 == 0 and
-// at most 1024 * S columns).  The ring holds nst stages of RB rows, each row at
+// at most 128 * NC * S columns: consumer thread t holds columns
+// 128 NC j + 4 t .. + 3, j < S; NC = 10 splits 1280 columns evenly).  The ring holds nst stages of RB rows, each row at
 // a pitch of `stride` floats; RB is a compile-time constant so that the RB
 // rows' dot products, shuffles and updates interleave.
-template <int S, int RB>
-__global__ void __launch_bounds__(kRingThreads, (S <= 8 ? 2 : 1))
+template <int S, int RB, int NC>
+__global__ void __launch_bounds__(32 * (NC + 1), (S <= 8 ? 2 : 1))
     srank_ring_kernel(const SrMat* __restrict__ mats, const SrItem* __restrict__ items, int nitems, int pass,
                       int last, int nst, int stride, unsigned* flags) {
   extern __shared__ __align__(128) unsigned char ring_raw[];
   float* ring = reinterpret_cast<float*>(ring_raw);
   __shared__ uint64_t full[kRingMaxStages], empty[kRingMaxStages];
-  __shared__ float red[2][RB][8];
-  __shared__ double dred[8];
+  __shared__ float red[2][RB][NC];
+  __shared__ double dred[NC];
   __shared__ int stop;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (tid == 0) {
     for (int k = 0; k < nst; ++k) {
       bar_init(&full[k], 1);
-      bar_init(&empty[k], 8);
+      bar_init(&empty[k], NC);
     }
     stop = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -276,7 +279,7 @@ __global__ void __launch_bounds__(kRingThreads, (S <= 8 ? 2 : 1))
   __syncthreads();
   volatile int* vstop = &stop;
 
-  if (warp == 8) {
+  if (warp == NC) {
     // ------------------------------ producer ------------------------------
     if (lane == 0) {
       int stage = 0;
@@ -330,7 +333,7 @@ __global__ void __launch_bounds__(kRingThreads, (S <= 8 ? 2 : 1))
     double ss = 0.0;
 #pragma unroll
     for (int j = 0; j < S; ++j) {
-      const int c0 = j * 1024 + 4 * tid;
+      const int c0 = j * 128 * NC + 4 * tid;
       if (c0 < cols) {
         const float4 q = *reinterpret_cast<const float4*>(vin + c0);
         v[j][0] = q.x; v[j][1] = q.y; v[j][2] = q.z; v[j][3] = q.w;
@@ -343,7 +346,7 @@ __global__ void __launch_bounds__(kRingThreads, (S <= 8 ? 2 : 1))
         w[j][e] = 0.f;
       }
     }
-    ss = consumer_sum(ss, dred);
+    ss = consumer_sum<NC>(ss, dred);
     const float inv = ss > 0.0 ? (float)(1.0 / sqrt(ss)) : 0.f;
 #pragma unroll
     for (int j = 0; j < S; ++j)
@@ -369,7 +372,7 @@ __global__ void __launch_bounds__(kRingThreads, (S <= 8 ? 2 : 1))
         if (b < n) {
 #pragma unroll
           for (int j = 0; j < S; ++j) {
-            const int c0 = j * 1024 + 4 * tid;
+            const int c0 = j * 128 * NC + 4 * tid;
             if (c0 < cols) {
               const float4 q = *reinterpret_cast<const float4*>(st + (size_t)b * stride + c0);
               ps[b] = fmaf(q.x, v[j][0], ps[b]); ps[b] = fmaf(q.y, v[j][1], ps[b]);
@@ -386,7 +389,7 @@ __global__ void __launch_bounds__(kRingThreads, (S <= 8 ? 2 : 1))
       if (lane == 0)
 #pragma unroll
         for (int b = 0; b < RB; ++b) red[buf][b][warp] = ps[b];
-      consumers_sync();
+      consumers_sync<NC>();
       if (*vstop) {        // every consumer reads the same value after the barrier
         aborted = true;
         break;
@@ -396,7 +399,7 @@ __global__ void __launch_bounds__(kRingThreads, (S <= 8 ? 2 : 1))
       for (int b = 0; b < RB; ++b) {
         u[b] = 0.f;
 #pragma unroll
-        for (int q = 0; q < 8; ++q) u[b] += red[buf][b][q];
+        for (int q = 0; q < NC; ++q) u[b] += red[buf][b][q];
         if (b >= n) u[b] = 0.f;
       }
       if (tid == 0)
@@ -408,7 +411,7 @@ __global__ void __launch_bounds__(kRingThreads, (S <= 8 ? 2 : 1))
           if (b < n) {
 #pragma unroll
             for (int j = 0; j < S; ++j) {
-              const int c0 = j * 1024 + 4 * tid;
+              const int c0 = j * 128 * NC + 4 * tid;
               if (c0 < cols) {
                 const float4 q = *reinterpret_cast<const float4*>(st + (size_t)b * stride + c0);
                 w[j][0] = fmaf(u[b], q.x, w[j][0]); w[j][1] = fmaf(u[b], q.y, w[j][1]);
@@ -430,13 +433,13 @@ __global__ void __launch_bounds__(kRingThreads, (S <= 8 ? 2 : 1))
     if (!last)
 #pragma unroll
       for (int j = 0; j < S; ++j) {
-        const int c0 = j * 1024 + 4 * tid;
+        const int c0 = j * 128 * NC + 4 * tid;
         if (c0 < cols)
 #pragma unroll
           for (int e = 0; e < 4; ++e) atomicAdd(&wout[c0 + e], w[j][e]);
       }
     if (pass == 0) {
-      const double f2s = consumer_sum((double)f2, dred);
+      const double f2s = consumer_sum<NC>((double)f2, dred);
       if (tid == 0) atomicAdd(&d.acc[0], f2s);
     }
     if (tid == 0) atomicAdd(&d.acc[1 + pass], u2);
@@ -489,10 +492,11 @@ cudaError_t dispatch(int slots, int threads, const SrMat* mats, const SrItem* it
   }
 }
 
-template <int S, int RB>
+template <int S, int RB, int NC = 8>
 cudaError_t ring_launch(const SrMat* mats, const SrItem* items, int nitems, int pass, bool last, int max_cols,
                         unsigned* flags, cudaStream_t st) {
-  auto kern = srank_ring_kernel<S, RB>;
+  auto kern = srank_ring_kernel<S, RB, NC>;
+  constexpr int kThreads = 32 * (NC + 1);   // NC consumer warps + 1 producer warp
   // 3 stages of RB rows (about 20-32 KB each), so that two blocks fit an SM
   const int stride = (max_cols + 3) / 4 * 4;
   const int nst = 3;
@@ -507,29 +511,55 @@ cudaError_t ring_launch(const SrMat* mats, const SrItem* items, int nitems, int 
   int dev = 0, sms = 0, per_sm = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kRingThreads, smem);
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, smem);
   int grid = sms * (per_sm > 0 ? per_sm : 1);
   if (grid > nitems) grid = nitems;
   count_launch();
-  kern<<<grid, kRingThreads, smem, st>>>(mats, items, nitems, pass, last ? 1 : 0, nst, stride, flags);
+  kern<<<grid, kThreads, smem, st>>>(mats, items, nitems, pass, last ? 1 : 0, nst, stride, flags);
   return cudaGetLastError();
+}
+
+// Rows per stage for S slots of NC consumer warps: the largest of 1, 2, 3,
+// 4, 6, 8 whose stage (rows of the full slot width, S * NC * 512 bytes) stays
+// within 32 KB, so that three stages of two blocks fit an SM.
+constexpr int ring_rows(int s, int nc) {
+  return 64 / (s * nc) >= 8 ? 8 : 64 / (s * nc) >= 6 ? 6 : 64 / (s * nc) >= 4 ? 4
+       : 64 / (s * nc) >= 3 ? 3 : 64 / (s * nc) >= 2 ? 2 : 1;
+}
+
+template <int S, int NC>
+cudaError_t ring_go(const SrMat* mats, const SrItem* items, int nitems, int pass, bool last, int max_cols,
+                    unsigned* flags, cudaStream_t st) {
+  return ring_launch<S, ring_rows(S, NC), NC>(mats, items, nitems, pass, last, max_cols, flags, st);
 }
 
 cudaError_t ring_dispatch(int max_cols, const SrMat* mats, const SrItem* items, int nitems, int pass, bool last,
                           unsigned* flags, cudaStream_t st) {
-  const int s = (max_cols + 1023) / 1024;
-  switch (s) {
-    case 1: return ring_launch<1, 12>(mats, items, nitems, pass, last, max_cols, flags, st);
-    case 2: return ring_launch<2, 6>(mats, items, nitems, pass, last, max_cols, flags, st);
-    case 3: return ring_launch<3, 2>(mats, items, nitems, pass, last, max_cols, flags, st);
-    case 4: return ring_launch<4, 2>(mats, items, nitems, pass, last, max_cols, flags, st);
-    case 5: return ring_launch<5, 1>(mats, items, nitems, pass, last, max_cols, flags, st);
-    case 6: return ring_launch<6, 1>(mats, items, nitems, pass, last, max_cols, flags, st);
-    case 7: case 8: return ring_launch<8, 1>(mats, items, nitems, pass, last, max_cols, flags, st);
+  // Ten consumer warps where they need fewer slots per thread than eight, up
+  // to three slots (1280 columns: one float4 per thread instead of two for a
+  // quarter of them); at 5120 columns four slots of ten warps measured no
+  // faster than five of eight.
+  const int s8 = (max_cols + 1023) / 1024, s10 = (max_cols + 1279) / 1280;
+  if (s10 < s8 && s10 <= 3) {
+    switch (s10) {
+      case 1: return ring_go<1, 10>(mats, items, nitems, pass, last, max_cols, flags, st);
+      case 2: return ring_go<2, 10>(mats, items, nitems, pass, last, max_cols, flags, st);
+      case 3: return ring_go<3, 10>(mats, items, nitems, pass, last, max_cols, flags, st);
+      default: break;
+    }
+  }
+  switch (s8) {
+    case 1: return ring_go<1, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
+    case 2: return ring_go<2, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
+    case 3: return ring_go<3, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
+    case 4: return ring_go<4, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
+    case 5: return ring_go<5, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
+    case 6: return ring_go<6, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
+    case 7: case 8: return ring_go<8, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
     case 9: case 10: case 11: case 12:
-      return ring_launch<12, 1>(mats, items, nitems, pass, last, max_cols, flags, st);
+      return ring_go<12, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
     case 13: case 14: case 15: case 16:
-      return ring_launch<16, 1>(mats, items, nitems, pass, last, max_cols, flags, st);
+      return ring_go<16, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
     default: return cudaErrorInvalidValue;
   }
 }
