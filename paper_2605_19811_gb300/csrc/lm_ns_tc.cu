@@ -577,6 +577,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   const int w_end = p.offsets ? p.offsets[pair + 1] : p.ntiles;
   const int w_step = p.offsets ? 1 : npairs;
 
+  if constexpr (kMasked) {
+    // A pair none of whose tiles belongs to a selected matrix leaves before
+    // any barrier, TMEM or cluster work (the roles would otherwise walk its
+    // tile list one dependent load chain at a time).  Both CTAs of the pair
+    // scan the same range of the same mask, so both leave or both stay.
+    int any = 0;
+    for (int w = w_begin + (int)threadIdx.x * w_step; !any && w < w_end; w += (int)blockDim.x * w_step)
+      any = tile_active(p, p.tiles[w]) ? 1 : 0;
+    if (!__syncthreads_or(any)) return;
+  }
+
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&full[s], 1);
