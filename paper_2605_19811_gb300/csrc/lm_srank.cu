@@ -22,6 +22,8 @@
 // Loads are thus decoupled from the per-batch reductions, and a batch can
 // hold many rows without using registers.  Every mbarrier wait is bounded;
 // a wait that gives up sets LM_FLAG_TIMEOUT and the block stops.
+#include <algorithm>
+
 #include "lm_internal.h"
 
 namespace lm {
@@ -237,6 +239,7 @@ __global__ void __launch_bounds__(TPB)
 }
 
 constexpr int kRingMaxStages = 4;
+constexpr size_t kRingBudget = 104 * 1024;      // ring bytes per block: two blocks per SM
 constexpr uint64_t kRingWaitNs = 2000000000ull;  // 2 s
 
 template <int NC>
@@ -497,10 +500,13 @@ cudaError_t ring_launch(const SrMat* mats, const SrItem* items, int nitems, int 
                         unsigned* flags, cudaStream_t st) {
   auto kern = srank_ring_kernel<S, RB, NC>;
   constexpr int kThreads = 32 * (NC + 1);   // NC consumer warps + 1 producer warp
-  // 3 stages of RB rows (about 20-32 KB each), so that two blocks fit an SM
+  // three or four stages of RB rows (at most 32 KB each), four where they
+  // fit the per-block budget: more rows in flight per block (a fifth stage
+  // measured slower at 5120 columns)
   const int stride = (max_cols + 3) / 4 * 4;
-  const int nst = 3;
-  const size_t smem = (size_t)nst * RB * stride * 4;
+  const size_t stage_bytes = (size_t)RB * stride * 4;
+  const int nst = (int)std::min<size_t>(kRingMaxStages, std::max<size_t>(3, kRingBudget / stage_bytes));
+  const size_t smem = (size_t)nst * stage_bytes;
   static bool attr_set[kMaxDevices] = {};   // per instantiation and device
   const int slot = device_slot();
   if (slot < 0 || !attr_set[slot]) {
