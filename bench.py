@@ -55,6 +55,8 @@ def parse_args():
     ap.add_argument("--vector-rule", choices=["lion", "adamw"], default="lion",
                     help="1-D parameters: the Lion step, or the AdamW fallback of Section 3")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-graph", action="store_true",
+                    help="skip timing the same steps replayed from CUDA graphs")
     ap.add_argument("--cublas-context", action="store_true",
                     help="also time the same NS iterations in torch.bmm/baddbmm (cuBLAS) for context")
     ap.add_argument("--no-cpu", action="store_true")
@@ -405,6 +407,30 @@ def run_ours(args):
     ms_per_step = ms_total / args.steps
     value = ms_per_step / world
 
+    # ---- the same steps replayed from CUDA graphs, one per step phase ----
+    # (t enters the Lion/Muon rules only mod P; AdamW's bias correction uses
+    # t itself, so that rule is not captured)
+    graph = None
+    if not args.no_graph and args.vector_rule != "adamw":
+        graphs = opt.capture_steps(grads, base)
+        nph = len(graphs)
+        for i in range(2 * nph):
+            graphs[i % nph].replay()
+        torch.cuda.synchronize()
+        barrier()
+        g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        g0.record(stream)
+        for i in range(args.steps):
+            graphs[i % nph].replay()
+        g1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        g_ms = max_over_ranks(g0.elapsed_time(g1), world, dev) / args.steps
+        graph = {"ms_per_step": g_ms / world,
+                 "what": "the same K steps replayed from CUDA graphs of lm_step (one per phase t mod P), "
+                         "captured once; inputs resident in HBM as for value"}
+        del graphs
+
     # ---- end to end through the public API with host buffers ----
     # Every step copies its gradients in from pinned host memory and reads
     # the updated parameters back.  The copies are pipelined across steps:
@@ -587,7 +613,7 @@ def run_ours(args):
             "roofline": srank_roof if srank else roof, "roofline_lion": lion_roof,
             **({"roofline_ns": roof} if srank else {}),
             "kernel_ms_per_step": fam_ms,
-            "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches, "clocks": clk,
+            "cpu_baseline": cpu, "e2e": e2e, "graph": graph, "gpu_launches": launches, "clocks": clk,
             "device_flags": flags,
             **({"context_cublas": context} if context else {}),
         }

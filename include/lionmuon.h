@@ -165,6 +165,14 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg,
 /* One LionMuon step t >= 0 (Algorithm 1 body).  grads[i] must have the shape
  * and dtype of params[i]; they are read-only device memory borrowed until the
  * enqueued work completes.  Muon iff period != 0 and t % period == 0.
+ * The work may be captured into a CUDA graph (stream capture on a non-NULL
+ * stream): the graph keeps the gradient pointers, the learning rates and t
+ * of the capture.  Under the Lion/Muon rules t matters only mod period, so
+ * a graph of step k (0 <= k < period) serves every later step t with
+ * t % period == k; the AdamW rule for vectors uses t itself (bias
+ * correction).
+ * After a captured step every later lm_step re-uploads its gradient pointers.
+ * Replays and lm_step calls on one state must not overlap on the GPU.
  * Errors: LM_ERR_INVALID_ARG (n mismatch, t < 0, shape mismatch, NULL),
  * LM_ERR_DTYPE, LM_ERR_ALIGN, LM_ERR_CUDA. */
 lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t,

@@ -713,6 +713,7 @@ struct lm_state {
   std::vector<NsCoeffs> ns_co;      // coefficients of each NS iteration
   unsigned* d_flags = nullptr;
   cudaStream_t last_stream = nullptr;
+  bool captured = false;             // a step of this state was captured into a graph
   Profiler prof;
 };
 
@@ -1148,7 +1149,14 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
 }
 
 static lm_status upload_grads(lm_state* s, const lm_tensor* grads, cudaStream_t st) {
-  bool same = s->grads_valid;
+  // A step captured into a CUDA graph carries its own pointer upload, and a
+  // replay rewrites the device table behind the host's copy: from the first
+  // captured step on, every step uploads its pointers.  (The legacy stream
+  // cannot be captured.)
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  if (st != nullptr && cudaStreamIsCapturing(st, &cap) == cudaSuccess && cap != cudaStreamCaptureStatusNone)
+    s->captured = true;
+  bool same = s->grads_valid && !s->captured;
   for (int i = 0; same && i < s->n; ++i) same = s->h_grads[i] == grads[i].data;
   if (same) return LM_OK;
   s->h_grads.resize(s->n);

@@ -224,6 +224,38 @@ class LionMuon:
         """lm_step with pre-built descriptors (no per-call marshalling)."""
         _check(self._lib, self._lib.lm_step(self._h, descs, n, int(t), stream_handle), "lm_step")
 
+    def capture_steps(self, grads: Sequence, t0: int = 0) -> list:
+        """Capture one step of each phase into torch.cuda.CUDAGraph objects:
+        graphs[k] runs step t0 + k, for k < P (P = period; one graph when
+        P = 0 or under the stable-rank schedule).  The steps depend on t only
+        through t mod P, so with t0 % P == 0 step t replays graphs[t % P].
+        The graphs read ``grads`` (write each step's gradients into them
+        before its replay) and keep the learning rates of the capture.  The
+        AdamW rule for vectors uses t itself and is refused.  Capturing runs
+        nothing; each replay runs one step."""
+        import torch
+        c = self.config
+        if c.vector_rule == LM_VECTOR_ADAMW:
+            raise ValueError("capture_steps: the AdamW vector rule depends on t (bias correction)")
+        period = int(c.period)
+        if c.schedule == LM_SCHEDULE_STABLE_RANK or period == 0:
+            nphase = 1
+        else:
+            nphase = period
+            if t0 % period != 0:
+                raise ValueError("capture_steps: t0 must be a multiple of the period")
+        descs = (LmTensor * len(grads))(*[tensor_desc(g) for g in grads])
+        side = torch.cuda.Stream()
+        side.wait_stream(torch.cuda.current_stream())
+        graphs = []
+        for k in range(nphase):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=side):
+                self.step_descs(descs, len(grads), t0 + k, ctypes.c_void_p(side.cuda_stream))
+            graphs.append(g)
+        torch.cuda.current_stream().wait_stream(side)
+        return graphs
+
     def set_lr(self, eta_muon: float, eta_lion: float) -> None:
         _check(self._lib, self._lib.lm_set_lr(self._h, eta_muon, eta_lion), "lm_set_lr")
 
