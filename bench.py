@@ -390,7 +390,6 @@ def run_ours(args):
     clocks.start()
     time.sleep(0.3)
     launches0 = L.kernel_launch_count()
-    opt.profile(True)
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize()
     barrier()
@@ -401,18 +400,28 @@ def run_ours(args):
     torch.cuda.synchronize()
     barrier()
     launches = L.kernel_launch_count() - launches0
-    prof = opt.profile_read()
-    opt.profile(False)
     ms_total = max_over_ranks(ev0.elapsed_time(ev1), world, dev)
     ms_per_step = ms_total / args.steps
     value = ms_per_step / world
+
+    # The same K steps again, from the same phase, with the library's
+    # per-launch events on: the per-kernel split and the rooflines come from
+    # this pass, so that its events stay out of the timed region above.
+    base_p = base + (((args.steps + P - 1) // P) * P if P > 0 and not srank else args.steps)
+    opt.profile(True)
+    for i in range(args.steps):
+        opt.step_descs(gdesc, n, base_p + i, sh)
+    torch.cuda.synchronize()
+    prof = opt.profile_read()
+    opt.profile(False)
+    base_g = base_p + (base_p - base)   # next aligned start, for the graph capture
 
     # ---- the same steps replayed from CUDA graphs, one per step phase ----
     # (t enters the Lion/Muon rules only mod P; AdamW's bias correction uses
     # t itself, so that rule is not captured)
     graph = None
     if not args.no_graph and args.vector_rule != "adamw":
-        graphs = opt.capture_steps(grads, base)
+        graphs = opt.capture_steps(grads, base_g)
         nph = len(graphs)
         for i in range(2 * nph):
             graphs[i % nph].replay()

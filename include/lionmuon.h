@@ -323,7 +323,8 @@ typedef struct {
   uint64_t launches[LM_KERNEL_FAMILIES];  /* launches timed */
 } lm_profile;
 
-/* Turn event timing on (on != 0) or off for the state's later lm_step calls.
+/* Turn event timing on (on != 0) or off for the state's later lm_step calls
+ * (steps captured into a CUDA graph are not timed).
  * Errors: LM_ERR_INVALID_ARG. */
 lm_status lm_profile_enable(lm_state* s, int on);
 

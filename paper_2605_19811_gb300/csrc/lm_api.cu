@@ -580,6 +580,11 @@ struct Profiler {
 template <typename F>
 static cudaError_t timed_events(Profiler* P, int fam, cudaStream_t st, F&& f) {
   if (P == nullptr || !P->on) return f();
+  // launches being captured into a graph are not timed (their events would
+  // be graph nodes, not measurements)
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  if (st != nullptr && cudaStreamIsCapturing(st, &cap) == cudaSuccess && cap != cudaStreamCaptureStatusNone)
+    return f();
   cudaEvent_t a = P->next(), b = P->next();
   if (a == nullptr || b == nullptr) return f();
   cudaEventRecord(a, st);

@@ -117,3 +117,22 @@ def test_capture_refuses_adamw_and_misaligned_start():
     with pytest.raises(ValueError):
         o.capture_steps(grads[0], 1)
     o.close()
+
+
+def test_capture_with_profiling_on_records_no_events():
+    """Profiling left on during a capture: the captured launches are not
+    timed, and eager steps afterwards are."""
+    dev, params, grads = _setup(seed=7)
+    o = L.LionMuon([p.clone() for p in params], period=2)
+    o.profile(True)
+    graphs = o.capture_steps(grads[0], 0)
+    graphs[0].replay()
+    graphs[1].replay()
+    torch.cuda.synchronize()
+    prof = o.profile_read()
+    assert all(v[1] == 0 for v in prof.values()), prof
+    o.step(grads[1], 2)
+    prof = o.profile_read()
+    assert prof["ns_gemm"][1] > 0 and prof["lion"][1] > 0
+    assert o.status() == 0
+    o.close()
