@@ -16,7 +16,9 @@ from paper_2605_19811_gb300 import synth
 
 pytestmark = pytest.mark.gpu
 
-SHAPES = [(256, 768), (768, 256), (512, 512), (1280, 384), (1024,)]
+# rows of 256-1024, 1280 and 3072 columns: three power-iteration launches per
+# pass under the stable-rank schedule, so its side streams take part
+SHAPES = [(256, 768), (768, 256), (512, 512), (384, 1280), (256, 3072), (1024,)]
 
 
 def _setup(seed=1):
