@@ -102,6 +102,43 @@ __device__ __forceinline__ double block_sum(double x, double* red) {
   return s;
 }
 
+// Sum of squares of this thread's entries of v, returned in fp64 but formed
+// in fp32 (this GPU's fp64 rate is a small fraction of its fp32 rate): the
+// entries are first scaled by the power of two that brings the largest to
+// [1, 2), so no square overflows or underflows.  Zero, infinite or NaN
+// entries take the plain fp64 sum.
+template <int S>
+__device__ __forceinline__ double sumsq_scaled(const float (&v)[S][4]) {
+  float mx = 0.f;
+#pragma unroll
+  for (int j = 0; j < S; ++j)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) mx = fmaxf(mx, fabsf(v[j][e]));
+  bool plain = !(mx > 0.f) || !isfinite(mx);
+#pragma unroll
+  for (int j = 0; j < S; ++j)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) plain = plain || isnan(v[j][e]);
+  if (plain) {
+    double s = 0.0;
+#pragma unroll
+    for (int j = 0; j < S; ++j)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) s += (double)v[j][e] * v[j][e];
+    return s;
+  }
+  const int ex = ilogbf(mx);
+  float s = 0.f;
+#pragma unroll
+  for (int j = 0; j < S; ++j)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const float x = scalbnf(v[j][e], -ex);
+      s = fmaf(x, x, s);
+    }
+  return ldexp((double)s, 2 * ex);
+}
+
 // Rows [r0, r0 + RB) of the item (zeros past nrows), this thread's columns.
 template <int S, int TPB, int RB, bool VEC>
 __device__ __forceinline__ void load_rows(float (&m)[RB][S][4], const float* M, int64_t cols, int row0, int r0,
@@ -132,9 +169,10 @@ __device__ __forceinline__ void row_batch(const float (&m)[RB][S][4], const floa
                                           int last, double& f2, double& u2) {
   constexpr int NW = TPB / 32;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  float sq = 0.f;   // this batch's squares: one fp64 addition per batch
 #pragma unroll
   for (int b = 0; b < RB; ++b) {
-    float ps = 0.f, sq = 0.f;
+    float ps = 0.f;
 #pragma unroll
     for (int j = 0; j < S; ++j)
 #pragma unroll
@@ -142,11 +180,11 @@ __device__ __forceinline__ void row_batch(const float (&m)[RB][S][4], const floa
         ps = fmaf(m[b][j][e], v[j][e], ps);
         sq = fmaf(m[b][j][e], m[b][j][e], sq);
       }
-    if (pass == 0) f2 += (double)sq;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) ps += __shfl_xor_sync(0xffffffffu, ps, o);
     if (lane == 0) red[buf][b][warp] = ps;
   }
+  if (pass == 0) f2 += (double)sq;
   __syncthreads();
   float u[RB];
 #pragma unroll
@@ -157,10 +195,13 @@ __device__ __forceinline__ void row_batch(const float (&m)[RB][S][4], const floa
     u[b] = x;
   }
   buf ^= 1;   // the next batch writes the other buffer: no second barrier
-  if (threadIdx.x == 0)
+  if (threadIdx.x == 0) {
+    float us = 0.f;
 #pragma unroll
     for (int b = 0; b < RB; ++b)
-      if (r0 + b < nrows) u2 += (double)u[b] * u[b];
+      if (r0 + b < nrows) us = fmaf(u[b], u[b], us);
+    u2 += (double)us;
+  }
   if (!last)
 #pragma unroll
     for (int b = 0; b < RB; ++b)
@@ -187,16 +228,14 @@ __global__ void __launch_bounds__(TPB)
 
     // normalised input vector, this thread's columns
     float v[S][4];
-    double ss = 0.0;
 #pragma unroll
     for (int j = 0; j < S; ++j)
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
         const int64_t c = (int64_t)j * 4 * TPB + 4 * tid + e;
         v[j][e] = c < cols ? vin[c] : 0.f;
-        ss += (double)v[j][e] * v[j][e];
       }
-    ss = block_sum<TPB>(ss, dred);
+    const double ss = block_sum<TPB>(sumsq_scaled<S>(v), dred);
     const float inv = ss > 0.0 ? (float)(1.0 / sqrt(ss)) : 0.f;
 #pragma unroll
     for (int j = 0; j < S; ++j)
@@ -333,7 +372,6 @@ __global__ void __launch_bounds__(32 * (NC + 1), (S <= 8 ? 2 : 1))
     float* wout = (pass & 1) ? d.wb : d.wa;
     const int cols = (int)d.cols;
     float v[S][4], w[S][4];
-    double ss = 0.0;
 #pragma unroll
     for (int j = 0; j < S; ++j) {
       const int c0 = j * 128 * NC + 4 * tid;
@@ -344,12 +382,9 @@ __global__ void __launch_bounds__(32 * (NC + 1), (S <= 8 ? 2 : 1))
         v[j][0] = v[j][1] = v[j][2] = v[j][3] = 0.f;
       }
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        ss += (double)v[j][e] * v[j][e];
-        w[j][e] = 0.f;
-      }
+      for (int e = 0; e < 4; ++e) w[j][e] = 0.f;
     }
-    ss = consumer_sum<NC>(ss, dred);
+    const double ss = consumer_sum<NC>(sumsq_scaled<S>(v), dred);
     const float inv = ss > 0.0 ? (float)(1.0 / sqrt(ss)) : 0.f;
 #pragma unroll
     for (int j = 0; j < S; ++j)
@@ -405,9 +440,14 @@ __global__ void __launch_bounds__(32 * (NC + 1), (S <= 8 ? 2 : 1))
         for (int q = 0; q < NC; ++q) u[b] += red[buf][b][q];
         if (b >= n) u[b] = 0.f;
       }
-      if (tid == 0)
+      if (tid == 0) {   // one fp64 addition per stage (this GPU's fp64 rate is a
+                        // small fraction of its fp32 rate); u_b^2 is of the order
+                        // of the squares in ||M||_F^2, which are summed in fp32
+        float us = 0.f;
 #pragma unroll
-        for (int b = 0; b < RB; ++b) u2 += (double)u[b] * u[b];
+        for (int b = 0; b < RB; ++b) us = fmaf(u[b], u[b], us);
+        u2 += (double)us;
+      }
       if (!last) {
 #pragma unroll
         for (int b = 0; b < RB; ++b) {

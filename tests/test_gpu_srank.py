@@ -41,6 +41,31 @@ def _state(shapes, kinds, seed, **cfg):
     return opt, params, W0, M0
 
 
+@pytest.mark.parametrize("scale", [1e-16, 1e9])
+def test_estimates_hold_at_extreme_momentum_scales(scale):
+    """Momentum entries of 1e-16 or 1e9 (the power-iteration vectors M^T u then
+    have entries near 1e-30 or 1e21, whose squares leave the fp32 range): the
+    estimates still match the fp64 oracle."""
+    import torch
+    kinds = ["lowrank", "noise", "lowrank", "noise", "lowrank", "noise", None]
+    opt, params, _, M0 = _state(SHAPES, kinds, 4, srank_alpha=0.08, srank_iters=5)
+    for i, m in enumerate(M0):
+        M0[i] = (m.astype(np.float64) * (scale / 1e-3)).astype(np.float32)
+        opt.set_momentum(i, torch.from_numpy(M0[i]).cuda())
+    g = [torch.zeros(s, dtype=torch.bfloat16, device="cuda") for s in SHAPES]
+    opt.step(g, 3)
+    took, est = opt.selection()
+    for i, s in enumerate(SHAPES):
+        if len(s) == 1:
+            continue
+        M = M0[i].astype(np.float64)
+        fro2, sig2 = O.stable_rank_estimate(M, 5, O.power_start_vector(s[1], 0))
+        want = fro2 / sig2
+        assert np.isfinite(est[i]) and abs(est[i] - want) <= 1e-4 * want, (s, scale, est[i], want)
+    assert opt.status() == 0
+    opt.close()
+
+
 @pytest.mark.parametrize("iters", [1, 2, 5])
 def test_estimates_and_decisions_match_oracle(iters):
     import torch
