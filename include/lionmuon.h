@@ -125,7 +125,12 @@ typedef struct {
    * start vector (seed srank_seed), srank_iters reads of M in all.
    * srank_alpha > 0 (Appendix G sweeps 0.002 .. 0.01; default 0.01),
    * srank_iters in [1, 64] (default 5); period is then ignored, and matrices
-   * may have at most 16384 columns. */
+   * may have at most 16384 columns.  When the matrices' column counts need
+   * more than one power-iteration launch per pass, lm_create also creates
+   * two non-blocking streams (freed by lm_destroy) on which lm_step runs
+   * those launches, forked from and joined back to the caller's stream by
+   * events: work enqueued on the caller's stream after lm_step still sees
+   * all of it. */
   int schedule;
   double srank_alpha;
   int srank_iters;
