@@ -183,6 +183,35 @@ def test_mixed_step_muon_matrices_equal_plain_muon_step(precision):
     opt_b.close()
 
 
+def test_no_matrix_selected_equals_pure_lion_steps():
+    """With an alpha no buffer meets, every step is a Lion step: three mixed
+    steps end bit-identical (weights and momentum) to three steps with
+    period 0 (P = infinity, Algorithm 1's pure Lion reduction).  The masked
+    Newton-Schulz launches then hold no selected tile anywhere, and every CTA
+    pair leaves before any set-up."""
+    import torch
+    from paper_2605_19811_gb300 import lionmuon as L
+    kinds = ["lowrank", "noise", "lowrank", "noise", "lowrank", "noise", None]
+    opt_a, pa, W0, M0 = _state(SHAPES, kinds, 21, srank_alpha=1e-12)
+    pb = [host_tensor(w, "bf16").cuda() for w in W0]
+    opt_b = L.LionMuon(pb, period=0)
+    for i, m in enumerate(M0):
+        opt_b.set_momentum(i, torch.from_numpy(m).cuda())
+    r = np.random.default_rng(22)
+    for t in range(1, 4):
+        G = [host_tensor(r.normal(size=s) * 1e-3, "bf16").cuda() for s in SHAPES]
+        opt_a.step(G, t)
+        opt_b.step(G, t)
+        torch.cuda.synchronize()
+        assert not any(opt_a.selection()[0]), t
+    for i in range(len(SHAPES)):
+        np.testing.assert_array_equal(bits(pa[i]), bits(pb[i]))
+        assert torch.equal(opt_a.momentum(i), opt_b.momentum(i)), i
+    assert opt_a.status() == 0 and opt_b.status() == 0
+    opt_a.close()
+    opt_b.close()
+
+
 def test_zero_buffer_takes_muon_at_t0():
     import torch
     from paper_2605_19811_gb300 import lionmuon as L
