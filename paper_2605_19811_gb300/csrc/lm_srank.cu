@@ -581,14 +581,14 @@ cudaError_t ring_go(const SrMat* mats, const SrItem* items, int nitems, int pass
 
 cudaError_t ring_dispatch(int max_cols, const SrMat* mats, const SrItem* items, int nitems, int pass, bool last,
                           unsigned* flags, cudaStream_t st) {
+  // Six consumer warps for rows of at most 768 columns: every thread holds
+  // a float4 (eight warps would leave a quarter of them idle at 768).
+  if (max_cols <= 768) return ring_go<1, 6>(mats, items, nitems, pass, last, max_cols, flags, st);
   // Ten consumer warps where they need fewer slots per thread than eight, up
   // to three slots (1280 columns: one float4 per thread instead of two for a
   // quarter of them); at 5120 columns four slots of ten warps measured no
   // faster than five of eight.
   const int s8 = (max_cols + 1023) / 1024, s10 = (max_cols + 1279) / 1280;
-  // six consumer warps for rows of at most 768 columns: every thread holds
-  // a float4 (eight warps would leave a quarter of them idle at 768)
-  if (max_cols <= 768) return ring_go<1, 6>(mats, items, nitems, pass, last, max_cols, flags, st);
   if (s10 < s8 && s10 <= 3) {
     switch (s10) {
       case 1: return ring_go<1, 10>(mats, items, nitems, pass, last, max_cols, flags, st);
