@@ -946,7 +946,10 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
       }
       sr_voff[id] = s->sr_w_elems;
       s->sr_w_elems = align_up(s->sr_w_elems + (size_t)p.cols, 64);
-      const auto key = std::make_tuple(slots, threads, p.cols % 4 == 0);
+      // rows of 16-byte multiples share a launch per ring-kernel shape, the
+      // others per register-kernel shape
+      const bool vec4 = p.cols % 4 == 0;
+      const auto key = std::make_tuple(vec4 ? srank_ring_shape(p.cols) : slots, threads, vec4);
       auto it = shape_launch.find(key);
       if (it == shape_launch.end()) {
         it = shape_launch.emplace(key, (int)s->sr_launch.size()).first;

@@ -245,6 +245,10 @@ cudaError_t launch_srank_pass(int slots, int threads, bool vec4, const SrMat* ma
 // The same pass through the shared-memory ring (every matrix of the launch
 // with cols % 4 == 0, at most max_cols <= 16384 columns); a stalled copy sets
 // LM_FLAG_TIMEOUT in *flags.
+// Launch shape of the ring kernel for rows of `cols` columns as one code
+// (100 x consumer warps + slots per thread; 0 beyond 16384 columns): rows
+// with the same code share a launch.
+int srank_ring_shape(int64_t cols);
 cudaError_t launch_srank_ring(int max_cols, const SrMat* mats, const SrItem* items, int nitems, int pass, bool last,
                               unsigned* flags, cudaStream_t st);
 // Decide per matrix: Muon iff ||M||_F^2 == 0 or ||M||_F^2 <= alpha min(m, n)

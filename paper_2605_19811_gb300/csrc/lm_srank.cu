@@ -579,41 +579,58 @@ cudaError_t ring_go(const SrMat* mats, const SrItem* items, int nitems, int pass
   return ring_launch<S, ring_rows(S, NC), NC>(mats, items, nitems, pass, last, max_cols, flags, st);
 }
 
-cudaError_t ring_dispatch(int max_cols, const SrMat* mats, const SrItem* items, int nitems, int pass, bool last,
-                          unsigned* flags, cudaStream_t st) {
+// Launch shape of the ring kernel for rows of max_cols columns, as
+// (slots per thread S, consumer warps NC).
+struct RingShape {
+  int s, nc;
+};
+RingShape ring_shape(int max_cols) {
   // Six consumer warps for rows of at most 768 columns: every thread holds
   // a float4 (eight warps would leave a quarter of them idle at 768).
-  if (max_cols <= 768) return ring_go<1, 6>(mats, items, nitems, pass, last, max_cols, flags, st);
+  if (max_cols <= 768) return {1, 6};
   // Ten consumer warps where they need fewer slots per thread than eight, up
   // to three slots (1280 columns: one float4 per thread instead of two for a
   // quarter of them); at 5120 columns four slots of ten warps measured no
   // faster than five of eight.
   const int s8 = (max_cols + 1023) / 1024, s10 = (max_cols + 1279) / 1280;
-  if (s10 < s8 && s10 <= 3) {
-    switch (s10) {
+  if (s10 < s8 && s10 <= 3) return {s10, 10};
+  return {s8 <= 6 ? s8 : s8 <= 8 ? 8 : s8 <= 12 ? 12 : 16, 8};
+}
+
+cudaError_t ring_dispatch(int max_cols, const SrMat* mats, const SrItem* items, int nitems, int pass, bool last,
+                          unsigned* flags, cudaStream_t st) {
+  if (max_cols > 16 * 1024) return cudaErrorInvalidValue;
+  const RingShape sh = ring_shape(max_cols);
+  if (sh.nc == 6) return ring_go<1, 6>(mats, items, nitems, pass, last, max_cols, flags, st);
+  if (sh.nc == 10) {
+    switch (sh.s) {
       case 1: return ring_go<1, 10>(mats, items, nitems, pass, last, max_cols, flags, st);
       case 2: return ring_go<2, 10>(mats, items, nitems, pass, last, max_cols, flags, st);
       case 3: return ring_go<3, 10>(mats, items, nitems, pass, last, max_cols, flags, st);
-      default: break;
+      default: return cudaErrorInvalidValue;
     }
   }
-  switch (s8) {
+  switch (sh.s) {
     case 1: return ring_go<1, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
     case 2: return ring_go<2, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
     case 3: return ring_go<3, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
     case 4: return ring_go<4, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
     case 5: return ring_go<5, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
     case 6: return ring_go<6, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
-    case 7: case 8: return ring_go<8, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
-    case 9: case 10: case 11: case 12:
-      return ring_go<12, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
-    case 13: case 14: case 15: case 16:
-      return ring_go<16, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
+    case 8: return ring_go<8, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
+    case 12: return ring_go<12, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
+    case 16: return ring_go<16, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
     default: return cudaErrorInvalidValue;
   }
 }
 
 }  // namespace
+
+int srank_ring_shape(int64_t cols) {
+  if (cols <= 0 || cols > 16 * 1024) return 0;
+  const RingShape sh = ring_shape((int)cols);
+  return sh.nc * 100 + sh.s;
+}
 
 cudaError_t launch_srank_ring(int max_cols, const SrMat* mats, const SrItem* items, int nitems, int pass, bool last,
                               unsigned* flags, cudaStream_t st) {
