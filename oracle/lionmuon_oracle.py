@@ -21,7 +21,7 @@ names the passage of the paper it restates:
   scaling 0.2 * sqrt(max(m, n)).
 * Section 3, Implementation notes: one persisted buffer per parameter.
 
-Readings taken where the paper is silent (each listed in the design doc):
+Readings taken where the paper is silent:
 
 * NS coefficients: the paper gives none; the default is the widely used
   quintic (a, b, c) = (3.4445, -4.7750, 2.0315), constant over iterations.
