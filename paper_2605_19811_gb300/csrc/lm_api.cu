@@ -963,6 +963,24 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
       s->sr_launch[it->second].max_cols = std::max<int64_t>(s->sr_launch[it->second].max_cols, p.cols);
       sr_items[it->second].push_back(SrItem{id, 0, (int32_t)p.rows, 0});   // split below
     }
+    // Largest launch first: the launches of a pass run concurrently, and the
+    // last to finish (whose end no other launch covers) is then the smallest.
+    {
+      std::vector<int64_t> elems(s->sr_launch.size(), 0);
+      for (size_t k = 0; k < sr_items.size(); ++k)
+        for (const SrItem& whole : sr_items[k]) elems[k] += (int64_t)whole.nrows * params[s->mat_param_of[whole.m]].cols;
+      std::vector<size_t> order(s->sr_launch.size());
+      for (size_t k = 0; k < order.size(); ++k) order[k] = k;
+      std::stable_sort(order.begin(), order.end(), [&](size_t a, size_t b) { return elems[a] > elems[b]; });
+      std::vector<lm_state::SrLaunch> sl;
+      std::vector<std::vector<SrItem>> si;
+      for (size_t k : order) {
+        sl.push_back(s->sr_launch[k]);
+        si.push_back(std::move(sr_items[k]));
+      }
+      s->sr_launch.swap(sl);
+      sr_items.swap(si);
+    }
     // Work items: runs of rows, sized per launch so that each launch has
     // about eight per block (blocks: two per SM); longer runs mean fewer
     // atomic additions into the M^T u vectors.
