@@ -19,7 +19,11 @@
  * Conventions for every call:
  *   - Device pointers are CUDA device memory of the current device; host
  *     pointers are ordinary host memory.  Tensors are dense, row-major,
- *     contiguous and 16-byte aligned (LM_ERR_ALIGN otherwise).
+ *     contiguous and 16-byte aligned (LM_ERR_ALIGN otherwise).  A tensor
+ *     whose data is host memory (page-locked or not) or another device's
+ *     memory is refused with LM_ERR_INVALID_ARG (managed memory is
+ *     accepted); lm_step checks each gradient pointer the first time it
+ *     sees it.
  *   - Calls return an lm_status; nothing unwinds across the ABI.  Arguments
  *     are validated before any work is enqueued: on an error return nothing
  *     was enqueued and no state changed.  An asynchronous CUDA error surfaces

@@ -73,6 +73,25 @@ lm_status check_tensor(const lm_tensor* t, const char* what, int i) {
   return LM_OK;
 }
 
+// The tensor's data must be device (or managed) memory of device `dev`: a
+// host pointer handed to a kernel would fault or read the wrong memory.
+lm_status check_device_memory(const lm_tensor* t, const char* what, int i, int dev) {
+  if (numel(*t) == 0) return LM_OK;
+  cudaPointerAttributes a{};
+  cudaError_t e = cudaPointerGetAttributes(&a, t->data);
+  if (e != cudaSuccess) {
+    cudaGetLastError();   // an unknown pointer is an argument error, not a sticky CUDA error
+    return fail(LM_ERR_INVALID_ARG, "%s[%d]: not a CUDA pointer (%s)", what, i, cudaGetErrorString(e));
+  }
+  if (a.type != cudaMemoryTypeDevice && a.type != cudaMemoryTypeManaged)
+    return fail(LM_ERR_INVALID_ARG, "%s[%d]: data is %s memory, not device memory", what, i,
+                a.type == cudaMemoryTypeHost ? "page-locked host" : "unregistered host");
+  if (a.type == cudaMemoryTypeDevice && a.device != dev)
+    return fail(LM_ERR_INVALID_ARG, "%s[%d]: data lives on device %d, the call runs on device %d", what, i,
+                a.device, dev);
+  return LM_OK;
+}
+
 lm_status check_config(const lm_config* c) {
   auto finite = [](double x) { return std::isfinite(x); };
   if (!(c->beta1 >= 0.0 && c->beta1 < 1.0) || !(c->beta2 >= 0.0 && c->beta2 < 1.0))
@@ -671,6 +690,7 @@ struct lm_state {
   float* mom = nullptr;
   const void** d_grads = nullptr;   // device grad-pointer table
   std::vector<const void*> h_grads; // what the device table holds
+  std::vector<const void*> grads_checked;   // gradient pointers found to be device memory
   bool grads_valid = false;
   LionTable lion_all[2], lion_vec[2];   // lion_all: matrices only under LM_VECTOR_ADAMW
   bool adamw = false;                   // 1-D parameters take AdamW
@@ -806,6 +826,8 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
     if ((st = check_tensor(&params[i], "params", i)) != LM_OK) return st;
   int dev = 0;
   if ((st = check_device(&dev)) != LM_OK) return st;
+  for (int i = 0; i < n; ++i)
+    if ((st = check_device_memory(&params[i], "params", i, dev)) != LM_OK) return st;
   cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
 
   lm_state* s = new lm_state();
@@ -1296,6 +1318,12 @@ lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t, void* c
     if (grads[i].dtype != s->params[i].dtype)
       return fail(LM_ERR_DTYPE, "grads[%d] dtype differs from the parameter's", i);
   }
+  // device memory: checked once per new gradient pointer
+  s->grads_checked.resize(n, nullptr);
+  for (int i = 0; i < n; ++i)
+    if (grads[i].data != s->grads_checked[i] && (st = check_device_memory(&grads[i], "grads", i, s->device)) != LM_OK)
+      return st;
+  for (int i = 0; i < n; ++i) s->grads_checked[i] = grads[i].data;
   cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
   if ((st = upload_grads(s, grads, stream)) != LM_OK) return st;
   s->last_stream = stream;
@@ -1443,6 +1471,7 @@ lm_status lm_set_second_moment(lm_state* s, int i, const lm_tensor* src, void* c
   if (src->dtype != LM_F32) return fail(LM_ERR_DTYPE, "second-moment source must be fp32");
   if (src->rows != s->params[i].rows || src->cols != s->params[i].cols)
     return fail(LM_ERR_INVALID_ARG, "second-moment source shape differs from the parameter's");
+  if ((st = check_device_memory(src, "src", 0, s->device)) != LM_OK) return st;
   const size_t bytes = (size_t)numel(s->params[i]) * sizeof(float);
   if (bytes == 0) return LM_OK;
   cudaError_t e = cudaMemcpyAsync(s->vmom + s->v_off[i], src->data, bytes, cudaMemcpyDeviceToDevice,
@@ -1469,6 +1498,7 @@ lm_status lm_set_momentum(lm_state* s, int i, const lm_tensor* src, void* cuda_s
   if (src->dtype != LM_F32) return fail(LM_ERR_DTYPE, "momentum source must be fp32");
   if (src->rows != s->params[i].rows || src->cols != s->params[i].cols)
     return fail(LM_ERR_INVALID_ARG, "momentum source shape differs from the parameter's");
+  if ((st = check_device_memory(src, "src", 0, s->device)) != LM_OK) return st;
   const size_t bytes = (size_t)numel(s->params[i]) * sizeof(float);
   if (bytes == 0) return LM_OK;
   cudaError_t e = cudaMemcpyAsync(s->mom + s->mom_off[i], src->data, bytes, cudaMemcpyDeviceToDevice,
@@ -1581,6 +1611,8 @@ static lm_status msign_impl(const lm_tensor* in, lm_tensor* out, int steps, cons
     return fail(LM_ERR_UNSUPPORTED, "matrix too large for lm_msign_ns");
   int dev = 0;
   if ((st = check_device(&dev)) != LM_OK) return st;
+  if ((st = check_device_memory(in, "in", 0, dev)) != LM_OK) return st;
+  if ((st = check_device_memory(out, "out", 0, dev)) != LM_OK) return st;
   cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
 
   NsEngine E;

@@ -137,6 +137,16 @@ extern "C" lm_status lm_msign_ns_noalloc(const lm_tensor* in, lm_tensor* out, in
   cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
   if (major != 10 || minor != 3) return set_error(LM_ERR_UNSUPPORTED, "device is not sm_103");
   if (dev >= kMaxDevices) return set_error(LM_ERR_UNSUPPORTED, "device ordinal above 63");
+  // in and out must be memory of this device (a host pointer would reach the kernels)
+  for (const lm_tensor* t : {in, static_cast<const lm_tensor*>(out)}) {
+    cudaPointerAttributes pa{};
+    if (cudaPointerGetAttributes(&pa, t->data) != cudaSuccess) {
+      cudaGetLastError();
+      return set_error(LM_ERR_INVALID_ARG, "in/out is not a CUDA pointer");
+    }
+    if (!(pa.type == cudaMemoryTypeManaged || (pa.type == cudaMemoryTypeDevice && pa.device == dev)))
+      return set_error(LM_ERR_INVALID_ARG, "in/out is not device memory of the current device");
+  }
 
   // Layout of this call inside the scratch area.
   const lm_dtype xdt = precision == LM_F32 ? LM_F32 : LM_BF16;
