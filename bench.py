@@ -9,10 +9,14 @@ periods.  Prints one JSON line (rank 0).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
-Under torchrun every rank runs an independent replica (the optimizer step
-has no exchange between parameter sets: weak scaling); the time is the max
-over ranks.  ``--impl reference`` times the CPU oracle on bounded samples of
-the same workload instead (rank 0 only).
+Under torchrun the N ranks share one parameter set by layer sharding
+(Section 5.4): every rank holds all parameters, gradients and momentum and
+runs the same step, each matrix's Muon update (momentum, Newton-Schulz,
+parameter write) runs on its owner rank only, and after every Muon step each
+rank broadcasts the matrices it owns (NCCL, inside the timed region).  The
+work per step is fixed as N grows (strong scaling); the time is the max over
+ranks.  ``--impl reference`` times the CPU oracle on bounded samples of the
+same workload instead (rank 0 only).
 """
 
 from __future__ import annotations
@@ -327,6 +331,7 @@ def run_ours(args):
     import torch.distributed as dist
     from paper_2605_19811_gb300 import build as B
     from paper_2605_19811_gb300 import lionmuon as L
+    from paper_2605_19811_gb300 import shard
     from paper_2605_19811_gb300 import synth
 
     rank, world, local = dist_env()
@@ -340,30 +345,39 @@ def run_ours(args):
 
     ps, shapes, mats, numel, mat_elems = workload(args.set)
     P = args.period
+    srank = args.schedule == "srank"
+    sharded = world > 1
+    if sharded and srank:
+        raise SystemExit("the stable-rank schedule is not layer-sharded; run it on one GPU")
+    owner = shard.owners(shapes, world) if sharded else [0 if len(s) == 2 and min(s) > 1 else -1 for s in shapes]
+    own_mats = [s for s, o in zip(shapes, owner) if o == rank]
     # Parameters and gradients live in two flat device buffers (views per
     # tensor, 256-byte aligned) so that the end-to-end leg moves each with one
-    # copy.
+    # copy; sharded, each rank's matrices are adjacent, so that the exchange
+    # is one broadcast per rank.
     elt = 2
-    offs, cur = [], 0
-    for s in shapes:
-        offs.append(cur)
-        cur += (int(math.prod(s)) * elt + 255) // 256 * 256
+    offs, cur = [0] * len(shapes), 0
+    for i in (shard.owner_order(shapes, owner) if sharded else range(len(shapes))):
+        offs[i] = cur
+        cur += (int(math.prod(shapes[i])) * elt + 255) // 256 * 256
     flat_bytes = cur
     wflat = torch.empty(flat_bytes // 2, dtype=torch.bfloat16, device=dev)
     gflat = torch.empty(flat_bytes // 2, dtype=torch.bfloat16, device=dev)
     def views(flat):
         return [flat[o // 2: o // 2 + int(math.prod(s))].view(s) for o, s in zip(offs, shapes)]
     params, grads = views(wflat), views(gflat)
-    for p, w in zip(params, synth.device_weights_torch(shapes, seed=1 + rank, device=dev, dtype=torch.bfloat16)):
+    # the same parameters and (already reduced) gradients on every rank
+    for p, w in zip(params, synth.device_weights_torch(shapes, seed=1, device=dev, dtype=torch.bfloat16)):
         p.copy_(w)
-    for g, x in zip(grads, synth.device_grads_torch(shapes, ps.grad_kind, seed=100 + rank, device=dev,
+    for g, x in zip(grads, synth.device_grads_torch(shapes, ps.grad_kind, seed=100, device=dev,
                                                      dtype=torch.bfloat16)):
         g.copy_(x)
     torch.cuda.synchronize()
 
     prec = {"bf16": L.LM_BF16, "f32": L.LM_F32, "f32tc": L.LM_NS_F32_TC}[args.precision]
-    srank = args.schedule == "srank"
     extra = {"vector_rule": L.LM_VECTOR_ADAMW} if args.vector_rule == "adamw" else {}
+    if sharded:
+        extra.update(shard_rank=rank, shard_world=world)
     if srank:
         opt = L.LionMuon(params, period=P, ns_precision=prec, schedule=L.LM_SCHEDULE_STABLE_RANK,
                          srank_alpha=args.srank_alpha, srank_iters=args.srank_iters, **extra)
@@ -373,14 +387,22 @@ def run_ours(args):
     gdesc = (L.LmTensor * n)(*[L.tensor_desc(g) for g in grads])
     stream = torch.cuda.current_stream()
     sh = ctypes.c_void_p(stream.cuda_stream)
+    ex = shard.Exchange(params, owner) if sharded else None
 
     def barrier():
         if world > 1:
             dist.barrier()
 
+    def step(descs, t, handle):
+        """One step; sharded, a Muon step ends with the exchange (NCCL waits
+        for the step's work on torch's current stream, which it runs on)."""
+        opt.step_descs(descs, n, t, handle)
+        if ex is not None and shard.is_muon_step(t, P):
+            ex.run()
+
     t = 0
     for _ in range(args.warmup):
-        opt.step_descs(gdesc, n, t, sh)
+        step(gdesc, t, sh)
         t += 1
     base = ((t + P - 1) // P) * P if P > 0 and not srank else t
     torch.cuda.synchronize()
@@ -395,14 +417,14 @@ def run_ours(args):
     barrier()
     ev0.record(stream)
     for i in range(args.steps):
-        opt.step_descs(gdesc, n, base + i, sh)
+        step(gdesc, base + i, sh)
     ev1.record(stream)
     torch.cuda.synchronize()
     barrier()
     launches = L.kernel_launch_count() - launches0
     ms_total = max_over_ranks(ev0.elapsed_time(ev1), world, dev)
     ms_per_step = ms_total / args.steps
-    value = ms_per_step / world
+    value = ms_per_step          # one parameter set, whatever N
 
     # The same K steps again, from the same phase, with the library's
     # per-launch events on: the per-kernel split and the rooflines come from
@@ -410,7 +432,7 @@ def run_ours(args):
     base_p = base + (((args.steps + P - 1) // P) * P if P > 0 and not srank else args.steps)
     opt.profile(True)
     for i in range(args.steps):
-        opt.step_descs(gdesc, n, base_p + i, sh)
+        step(gdesc, base_p + i, sh)
     torch.cuda.synchronize()
     prof = opt.profile_read()
     opt.profile(False)
@@ -420,7 +442,7 @@ def run_ours(args):
     # (t enters the Lion/Muon rules only mod P; AdamW's bias correction uses
     # t itself, so that rule is not captured)
     graph = None
-    if not args.no_graph and args.vector_rule != "adamw":
+    if not args.no_graph and args.vector_rule != "adamw" and not sharded:
         graphs = opt.capture_steps(grads, base_g)
         nph = len(graphs)
         for i in range(2 * nph):
@@ -435,7 +457,7 @@ def run_ours(args):
         torch.cuda.synchronize()
         barrier()
         g_ms = max_over_ranks(g0.elapsed_time(g1), world, dev) / args.steps
-        graph = {"ms_per_step": g_ms / world,
+        graph = {"ms_per_step": g_ms,
                  "what": "the same K steps replayed from CUDA graphs of lm_step (one per phase t mod P), "
                          "captured once; inputs resident in HBM as for value"}
         del graphs
@@ -449,9 +471,10 @@ def run_ours(args):
     # device-to-device copy snapshots the parameters (W is updated in place
     # by step t+1), and the snapshot is read back to the host while step t+1
     # runs.  Warm-up steps run through the same pipeline before the timed
-    # region, as in a training loop that reuses its buffers.
+    # region, as in a training loop that reuses its buffers.  (Sharded, the
+    # exchange of a Muon step belongs to NCCL and is not in this pipeline.)
     e2e = None
-    if not args.no_e2e:
+    if not args.no_e2e and not sharded:
         g_host = torch.empty(flat_bytes // 2, dtype=torch.bfloat16, pin_memory=True)
         w_host = torch.empty(flat_bytes // 2, dtype=torch.bfloat16, pin_memory=True)
         g_host.copy_(gflat)
@@ -512,7 +535,7 @@ def run_ours(args):
         torch.cuda.synchronize()
         barrier()
         e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
-        e2e = {"value": e_ms / args.steps / world, "unit": "ms/step", "h2d_bytes_per_step": flat_bytes,
+        e2e = {"value": e_ms / args.steps, "unit": "ms/step", "h2d_bytes_per_step": flat_bytes,
                "d2h_bytes_per_step": flat_bytes,
                "what": "pinned-host gradients copied in and updated parameters copied out every step, "
                        "through lm_step; the gradient copies and the read-back of a device snapshot of "
@@ -535,20 +558,29 @@ def run_ours(args):
     n_lion = args.steps - n_muon
     ns_ms, ns_launches = prof["ns_gemm"]
     lion_ms, lion_launches = prof["lion"]
-    fl = ns_flops_sym(mats) * n_muon
+    ns_mats = own_mats if sharded else mats      # sharded: this rank's Newton-Schulz work
+    fl = ns_flops_sym(ns_mats) * n_muon
+    # The burst peak applies to a kernel timed in a short region, the
+    # sustained one (the power cap's) to one inside a seconds-long loop.
+    pk_burst = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
+    pk_sust = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+    long_region = ms_total >= 1000.0
+    pk_bf16 = pk_sust if long_region else pk_burst
+    bf16_kind = (f"bf16 {'sustained' if long_region else 'burst'} ({ms_total / 1e3:.2f} s timed region), "
+                 f"{peak_src}")
     roof = None
     if ns_ms > 0 and n_muon > 0:
         achieved = fl / (ns_ms / 1e3) / 1e12
         flops_note = "symmetric count 3 s^2 l + s^3 per matrix per NS iteration"
         if args.precision == "bf16":
-            pk = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
-            bound, kernel, peak_kind = "tensor", "ns_tc_kernel", f"bf16 sustained, {peak_src}"
+            pk = pk_bf16
+            bound, kernel, peak_kind = "tensor", "ns_tc_kernel", bf16_kind
         elif args.precision == "f32tc":
             # six bf16 piece products per fp32 product, on the bf16 tensor pipe
             achieved *= 6
             fl *= 6
-            pk = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
-            bound, kernel, peak_kind = "tensor", "ns_tc_kernel", f"bf16 sustained, {peak_src}"
+            pk = pk_bf16
+            bound, kernel, peak_kind = "tensor", "ns_tc_kernel", bf16_kind
             flops_note = "6 x the symmetric count 3 s^2 l + s^3 (six bf16 piece products per fp32 product)"
         else:
             # fp32 FMA on the CUDA cores: SMs x 128 lanes x 2 FLOP x the maximum SM clock
@@ -559,9 +591,24 @@ def run_ours(args):
             peak_kind = f"fp32 FMA, derived: {sms} SMs x 128 lanes x 2 FLOP x {mhz:.0f} MHz"
         # the recorded ncu traffic is the bf16 workload's
         traffic = kernel_traffic(kernel) if args.precision != "f32tc" else None
-        dense = sum(5 * (4.0 * min(m, n) ** 2 * max(m, n) + 2.0 * min(m, n) ** 3) for m, n in mats) * n_muon
+        dense = sum(5 * (4.0 * min(m, n) ** 2 * max(m, n) + 2.0 * min(m, n) ** 3) for m, n in ns_mats) * n_muon
+        # per phase: GRAM s^2 l, POLY s^3 (the symmetric products once), APPLY 2 s^2 l per iteration
+        ph_fl = {"ns_gram": sum(min(a, b) ** 2 * max(a, b) for a, b in ns_mats),
+                 "ns_poly": sum(min(a, b) ** 3 for a, b in ns_mats),
+                 "ns_apply": sum(2.0 * min(a, b) ** 2 * max(a, b) for a, b in ns_mats)}
+        mult = 6 if args.precision == "f32tc" else 1
+        phases = {}
+        for k, f1 in ph_fl.items():
+            ms_k, n_k = prof[k]
+            if ms_k > 0:
+                tf = mult * 5 * f1 * n_muon / (ms_k / 1e3) / 1e12
+                phases[k] = {"ms_per_launch": ms_k / max(n_k, 1), "tflops": tf,
+                             **({"frac": tf / pk} if bound == "tensor" else {})}
         roof = {"bound": bound, "achieved": achieved, "peak": pk, "unit": "TFLOP/s",
                 "frac": achieved / pk, "traffic": traffic, "kernel": kernel,
+                **({"frac_of_sustained": achieved / pk_sust, "frac_of_burst": achieved / pk_burst}
+                   if bound == "tensor" else {}),
+                "phases": phases,
                 # the same time over the dense count 4 s^2 l + 2 s^3 (both symmetric products in full)
                 "dense_equivalent_tflops": dense / (ns_ms / 1e3) / 1e12,
                 "per_launch_ms": ns_ms / max(ns_launches, 1),
@@ -571,13 +618,14 @@ def run_ours(args):
     lion_roof = None
     if lion_ms > 0:
         # Lion-step launches over all params: 14 B/param (bf16 W,G r/w W, fp32 M r/w)
-        lion_full_ms = lion_ms - 0.0
         bytes_moved = 14.0 * numel * n_lion + 14.0 * (numel - mat_elems) * n_muon
-        gbs = bytes_moved / (lion_full_ms / 1e3) / 1e9
+        gbs = bytes_moved / (lion_ms / 1e3) / 1e9
         pk = peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
         lion_roof = {"bound": "hbm", "achieved": gbs, "peak": pk, "unit": "GB/s", "frac": gbs / pk,
                      "traffic": kernel_traffic("lion_kernel"), "kernel": "lion_kernel",
-                     "per_launch_ms": lion_ms / max(lion_launches, 1),
+                     # per full-set launch (one per Lion step); the vector-only launches of the
+                     # Muon steps (0.02% of the parameters) are inside the sum
+                     "per_launch_ms": lion_ms / max(n_lion, 1),
                      "frac_of_8tbs": gbs / 8000.0, "peak_kind": f"HBM copy, {peak_src}"}
     srank_roof = None
     if srank and prof["srank"][0] > 0:
@@ -605,7 +653,7 @@ def run_ours(args):
         line = {
             "metric": METRIC, "value": value, "unit": "ms/step", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
-            "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
+            "higher_is_better": False, "scaling": "strong", "vs_baseline": None,
             "dtype": {"bf16": "bf16", "f32": "f32", "f32tc": "f32 (3 x bf16 pieces)"}[args.precision],
             "data": "synthetic",
             "config": {"workload": args.set, "params": numel, "matrices": len(mats),
@@ -618,7 +666,14 @@ def run_ours(args):
                        "grads": f"{ps.grad_kind}, drawn on device, same gradients every step",
                        "l2": "inputs larger than L2 (14 B/param x %.0f M params streamed per Lion step)" % (numel / 1e6),
                        "timed_steps": f"t = {base} .. {base + args.steps - 1}" +
-                                      ("" if srank else " (whole periods from a Muon step)")},
+                                      ("" if srank else " (whole periods from a Muon step)"),
+                       "parallelism": (f"layer-sharded Muon over {world} GPUs (each matrix's Muon update on "
+                                       "its owner, owners' matrices broadcast after each Muon step; Lion "
+                                       "steps on every GPU)") if sharded else "one GPU"},
+            **({"exchange": {"bytes_received_per_muon_step_rank0": ex.received_bytes(0),
+                             "broadcasts_per_muon_step": len(ex.items),
+                             "ns_tflop_per_muon_step_rank0": ns_flops_sym(own_mats) / 1e12,
+                             "ns_tflop_per_muon_step_total": ns_flops_sym(mats) / 1e12}} if sharded else {}),
             "roofline": srank_roof if srank else roof, "roofline_lion": lion_roof,
             **({"roofline_ns": roof} if srank else {}),
             "kernel_ms_per_step": fam_ms,

@@ -80,7 +80,19 @@ typedef struct {
  *                       library's launches
  *   LM_FAULT=oom        lm_create returns LM_ERR_OOM as if the device allocation
  *                       had failed (to exercise callers' error paths)
- *   LM_NS_FORCE_FP32=1  the fp32 Newton-Schulz path whatever ns_precision says */
+ *   LM_NS_FORCE_FP32=1  the fp32 Newton-Schulz path whatever ns_precision says
+ *   LM_NS_TILES=wide    bf16 Newton-Schulz tiles of two 256-column blocks per
+ *                       CTA pair (the default is one block); same results bit
+ *                       for bit, slower on the GPT-style parameter sets
+ *   LM_PDL=0            no programmatic dependent launch between the
+ *                       Newton-Schulz launches (same results)
+ *   LM_WAIT_LIMIT_NS=n  limit of every bounded device wait in ns (default 5 s;
+ *                       also read by lm_msign_ns and lm_msign_ns_noalloc).  A
+ *                       wait that runs out raises LM_FLAG_TIMEOUT; every kernel
+ *                       of this state (or call) launched after it reads the
+ *                       flag at entry and does nothing, so a step stops within
+ *                       about one limit and writes no parameter after the
+ *                       give-up, until lm_get_status clears the flag. */
 
 /* Hyper-parameters: the Require line of Algorithm 1 plus the NS reading.
  * beta1, beta2 in [0, 1); eta_* >= 0; weight_decay >= 0;
@@ -139,6 +151,21 @@ typedef struct {
   double srank_alpha;
   int srank_iters;
   uint64_t srank_seed;
+  /* Layer-sharded Muon (Section 5.4: a Muon step needs each matrix whole,
+   * a Lion step is element-wise).  With shard_world > 1 this state is rank
+   * shard_rank of shard_world ranks that each hold all parameters, the
+   * (already reduced) gradients and the momentum.  Every matrix has one owner
+   * rank (lm_shard_owners).  On a Muon step a rank runs the momentum, Newton-
+   * Schulz and parameter write only for the matrices it owns, and for the
+   * others the momentum update M = beta2 M + (1 - beta2) G alone; the caller
+   * then copies each matrix from its owner to the other ranks (a broadcast
+   * per matrix, on Muon steps only).  Lion steps and 1-D parameters run the
+   * same on every rank and exchange nothing.  The Newton-Schulz workspace
+   * covers the owned matrices only.  shard_world 0 or 1: no sharding (the
+   * default 1); otherwise shard_world <= 4096, 0 <= shard_rank < shard_world,
+   * and schedule must be LM_SCHEDULE_PERIOD. */
+  int shard_rank;
+  int shard_world;
 } lm_config;
 
 #define LM_SCHEDULE_PERIOD 0
@@ -159,6 +186,24 @@ typedef struct lm_state lm_state; /* opaque */
  * (3.4445, -4.7750, 2.0315) with eps 1e-7 (the paper gives none; this is the
  * stated reading), shape_scale 0.2 (Table 5), ns_precision LM_BF16. */
 void lm_config_default(lm_config* cfg);
+
+/* sizeof(lm_config) as this library was built: a binding that lays the
+ * struct out itself compares it with its own size before any call that
+ * takes an lm_config (a mismatch would make those calls read or write past
+ * the caller's struct). */
+size_t lm_config_size(void);
+
+/* Owner rank of each parameter under layer sharding over `world` ranks
+ * (lm_config::shard_world, Section 5.4): matrices (rows, cols >= 2) are
+ * dealt out whole, largest Newton-Schulz cost 3 s^2 l + s^3 first (s, l the
+ * smaller and larger dimension; the FLOPs of one iteration counting the
+ * symmetric products once), each to the rank with the least cost so far (the
+ * lowest such rank), ties in cost taken in parameter order; 1-D parameters
+ * get -1 (every rank updates them).  The same inputs give the same owners on
+ * every rank.  Reads only the shapes (no device access; usable without a
+ * GPU).  owner: n ints of host memory.
+ * Errors: LM_ERR_INVALID_ARG (NULL, n < 1, world outside [1, 4096]). */
+lm_status lm_shard_owners(const lm_tensor* params, int n, int world, int* owner);
 
 /* Create an optimizer state over n parameter tensors (Algorithm 1, Require:
  * W_0 given, M_{-1} = 0).  params[i].data is caller-owned device memory that
@@ -223,9 +268,12 @@ lm_status lm_set_second_moment(lm_state* s, int i, const lm_tensor* src,
  * LM_F32 (may differ).  precision LM_BF16 uses the tensor-core path, LM_F32
  * the fp32 CUDA-core path, LM_NS_F32_TC fp32 values on the tensor cores (as
  * for lm_config::ns_precision).  Allocates its workspace with stream-ordered
- * allocation on cuda_stream and frees it the same way.
+ * allocation on cuda_stream and frees it the same way.  A testing entry
+ * point: it synchronises cuda_stream before it returns, to read its own
+ * status word.
  * Errors: LM_ERR_INVALID_ARG, LM_ERR_DTYPE, LM_ERR_ALIGN, LM_ERR_OOM,
- * LM_ERR_CUDA. */
+ * LM_ERR_CUDA, LM_ERR_TIMEOUT (a bounded device wait gave up; the kernels
+ * after it did nothing and out holds no result). */
 lm_status lm_msign_ns(const lm_tensor* in, lm_tensor* out, int steps, double a,
                       double b, double c, double eps, int precision,
                       void* cuda_stream);
@@ -246,19 +294,34 @@ lm_status lm_msign_ns_coeffs(const lm_tensor* in, lm_tensor* out, int steps,
  * 64 MiB area inside the library (a static device array that every GPU which
  * loads the library holds until the process exits); a matrix whose workspace
  * does not fit is rejected with LM_ERR_UNSUPPORTED and a message giving the
- * bytes needed.  Roughly: bf16 precision fits up to 1280 x 5120, fp32
- * precision up to 1024 x 4096.  The caller still provides in and out.
- * The first call on a device looks up the area's device address on that
- * device (cudaGetSymbolAddress); make that first call before any stream
- * capture.  All calls share the one area, which keeps the last call's data:
- * each call clears what must start at zero, and calls whose GPU work may
- * overlap (unordered streams or threads) race on the area and must be
- * serialised by the caller.  Arguments and errors as for lm_msign_ns, except
- * that precision is LM_BF16 or LM_F32 only.
+ * bytes needed.  The workspace is (2 s_p l_p + 2 s_p^2) e bytes plus about
+ * 1 KB of descriptors, 24 bytes per 32768 elements of the matrix and 16
+ * bytes per tile, where s = min(rows, cols), l = max(rows, cols); with
+ * precision LM_BF16: e = 2, s_p = s rounded up to 128, l_p = l rounded up
+ * to 256 (so 2048 x 5120 fits, 2048 x 8192 does not); with LM_F32: e = 4 and
+ * both rounded up to 128.  The caller still provides in and out.
+ * The first call on a device (and the first after its context was
+ * destroyed and made again, as by cudaDeviceReset) looks up the area's
+ * device address on that device (cudaGetSymbolAddress); make that first call
+ * before any stream capture.  All calls share the one area, which keeps the
+ * last call's data: each call clears what must start at zero, and calls
+ * whose GPU work may overlap (unordered streams or threads) race on the area
+ * and must be serialised by the caller.  Unlike lm_msign_ns the call does not
+ * synchronise: lm_msign_ns_noalloc_status reports its status word.
+ * Arguments and errors as for lm_msign_ns, except that precision is LM_BF16
+ * or LM_F32 only.
  * The paper has no counterpart of this call; it is a deployment variant. */
 lm_status lm_msign_ns_noalloc(const lm_tensor* in, lm_tensor* out, int steps,
                               double a, double b, double c, double eps,
                               int precision, void* cuda_stream);
+
+/* Status of the last lm_msign_ns_noalloc call on the current device:
+ * synchronises cuda_stream (the stream of that call), then stores its status
+ * word (LM_FLAG_*) in *device_flags, without allocating.  Returns
+ * LM_ERR_TIMEOUT when a bounded device wait of that call gave up (out then
+ * holds no result).  The paper has no counterpart; deployment variant.
+ * Errors: LM_ERR_INVALID_ARG (NULL), LM_ERR_CUDA, LM_ERR_TIMEOUT. */
+lm_status lm_msign_ns_noalloc_status(uint32_t* device_flags, void* cuda_stream);
 
 /* A read-only view of parameter i's momentum buffer (fp32, the shape of
  * params[i], device memory owned by the state).  For checkpointing and tests.

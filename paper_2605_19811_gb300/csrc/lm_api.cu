@@ -29,6 +29,13 @@ int device_slot() {
   if (cudaGetDevice(&dev) != cudaSuccess) return -1;
   return (dev >= 0 && dev < kMaxDevices) ? dev : -1;
 }
+uint64_t env_wait_limit_ns() {
+  const char* v = std::getenv("LM_WAIT_LIMIT_NS");
+  if (v == nullptr || *v == '\0') return kDefaultWaitNs;
+  char* end = nullptr;
+  const unsigned long long x = std::strtoull(v, &end, 10);
+  return (end != nullptr && *end == '\0' && x > 0) ? (uint64_t)x : kDefaultWaitNs;
+}
 
 namespace {
 
@@ -115,6 +122,12 @@ lm_status check_config(const lm_config* c) {
     if (!finite(c->srank_alpha) || !(c->srank_alpha > 0)) return fail(LM_ERR_INVALID_ARG, "srank_alpha must be > 0");
     if (c->srank_iters < 1 || c->srank_iters > 64) return fail(LM_ERR_INVALID_ARG, "srank_iters must be in [1, 64]");
   }
+  const int world = c->shard_world == 0 ? 1 : c->shard_world;
+  if (world < 1 || world > 4096) return fail(LM_ERR_INVALID_ARG, "shard_world must be in [0, 4096]");
+  if (c->shard_rank < 0 || c->shard_rank >= world)
+    return fail(LM_ERR_INVALID_ARG, "shard_rank %d is not in [0, %d)", c->shard_rank, world);
+  if (world > 1 && c->schedule != LM_SCHEDULE_PERIOD)
+    return fail(LM_ERR_UNSUPPORTED, "layer sharding needs schedule LM_SCHEDULE_PERIOD");
   if (c->vector_rule != LM_VECTOR_LION && c->vector_rule != LM_VECTOR_ADAMW)
     return fail(LM_ERR_INVALID_ARG, "vector_rule must be LM_VECTOR_LION or LM_VECTOR_ADAMW");
   if (c->vector_rule == LM_VECTOR_ADAMW) {
@@ -150,6 +163,7 @@ LionConsts lion_consts(const lm_config& c) {
   k.eL = (float)c.eta_lion;
   k.lam = (float)c.weight_decay;
   k.skip = nullptr;
+  k.flags = nullptr;
   return k;
 }
 // AdamW constants of step t (update number t + 1): powers and the square
@@ -167,6 +181,7 @@ AdamConsts adamw_consts(const lm_config& c, int64_t t) {
   a.rbc2 = (float)(1.0 / std::sqrt(bc2));
   a.lrwd = (float)(c.adamw_lr * c.adamw_weight_decay);
   a.eps = (float)c.adamw_eps;
+  a.flags = nullptr;
   return a;
 }
 
@@ -181,6 +196,7 @@ MuonConsts muon_consts(const lm_config& c) {
   k.eps = (float)c.ns_eps;
   k.ns_steps = c.ns_steps;
   k.active = nullptr;
+  k.flags = nullptr;
   return k;
 }
 
@@ -207,21 +223,34 @@ struct Arena {
   }
 };
 
-// Debug switches read from the environment when a state is created (host
-// side only; none of them changes the device code):
+// Switches read from the environment when a state is created (or an msign
+// call starts; host side only, none of them changes the device code):
 //   LM_DEBUG=1         guard bands around every workspace part
 //   LM_NVTX=1          NVTX ranges around every kernel family's launches
 //   LM_FAULT=oom       lm_create fails with LM_ERR_OOM as if the allocation had
 //   LM_NS_FORCE_FP32=1 the fp32 Newton-Schulz path whatever ns_precision says
+//   LM_NS_TILES=wide   two-block (256 x 512) Newton-Schulz tiles wherever
+//                      they fit, run by the wide-tile kernel; the default
+//                      (or LM_NS_TILES=narrow) is one-block tiles.  The
+//                      results are the same bit for bit
+//   LM_PDL=0           no programmatic dependent launch between NS launches
+//   LM_WAIT_LIMIT_NS=n limit of every bounded device wait (default 5 s; a
+//                      short limit makes waits give up, for failure tests)
 static bool env_is(const char* name, const char* value) {
   const char* v = std::getenv(name);
   return v != nullptr && std::strcmp(v, value) == 0;
+}
+static int env_tiles_mode() {
+  if (env_is("LM_NS_TILES", "narrow")) return 1;
+  if (env_is("LM_NS_TILES", "wide")) return 2;
+  return 0;
 }
 static std::atomic<bool> g_nvtx{false};
 static const char* const kFamilyNames[LM_KERNEL_FAMILIES] = {
     "lion", "momentum_norm", "ns_gram", "ns_poly", "ns_apply", "finalize", "other", "adamw", "srank"};
 
 constexpr int64_t kLionChunk = 32768;   // elements per Lion work chunk
+constexpr uint64_t kRingWaitNs = 2000000000ull;   // the power-iteration ring's waits: 2 s unless set shorter
 
 struct LionTable {
   LionTensor* tensors = nullptr;
@@ -235,6 +264,7 @@ struct NsBatch {
   int g0 = 0, ng = 0;
   NsTile* tiles[3] = {nullptr, nullptr, nullptr};
   int ntiles[3] = {0, 0, 0};
+  bool wide[3] = {false, false, false};            // tiles of two 256-column blocks: the wide-tile kernel
   int* offsets[3] = {nullptr, nullptr, nullptr};   // per-pair tile ranges (tensor-core path)
   int npairs[3] = {0, 0, 0};
   NsSplitTarget* split_targets = nullptr;   // split Gram tiles of this batch
@@ -287,8 +317,12 @@ void balance_tiles(const std::vector<std::pair<int, NsTile>>& sorted, int worker
   }
 }
 
+// wide: a tile covers column blocks tn and tn + 1 where both exist (nh = 2).
+// APPLY pairs blocks 2k and 2k + 1; the symmetric phases pair the blocks of
+// a row from its diagonal block on, (tm, tm + 1), (tm + 2, tm + 3), ..., so
+// that every stored block is computed exactly once.
 void build_ns_tiles(const std::vector<NsGroup>& groups, int g0, int ng, int phase, int bm, int bn,
-                    std::vector<NsTile>& out) {
+                    std::vector<NsTile>& out, bool wide = false) {
   std::vector<std::pair<int, NsTile>> v;
   for (int gi = g0; gi < g0 + ng; ++gi) {
     const NsGroup& g = groups[gi];
@@ -298,16 +332,22 @@ void build_ns_tiles(const std::vector<NsGroup>& groups, int g0, int ng, int phas
     const int K = (phase == NS_GRAM) ? g.l_pad : g.s_pad;
     const int tms = (nrow + bm - 1) / bm, tns = (ncol + bn - 1) / bn;
     for (int m = 0; m < g.count; ++m)
-      for (int tm = 0; tm < tms; ++tm)
-        for (int tn = 0; tn < tns; ++tn) {
-          if (phase != NS_APPLY && (int64_t)(tn + 1) * bn <= (int64_t)tm * bm) continue;
+      for (int tm = 0; tm < tms; ++tm) {
+        int tn = 0;
+        if (phase != NS_APPLY)   // first block reaching the diagonal
+          while (tn < tns && (int64_t)(tn + 1) * bn <= (int64_t)tm * bm) ++tn;
+        while (tn < tns) {
           NsTile t;
+          memset(&t, 0, sizeof(t));
           t.group = (uint16_t)(gi - g0);
           t.mat = (uint16_t)m;
           t.tm = (uint16_t)tm;
           t.tn = (uint16_t)tn;
+          t.nh = (uint16_t)((wide && tn + 1 < tns) ? 2 : 1);
           v.push_back({K, t});
+          tn += t.nh;
         }
+      }
   }
   std::stable_sort(v.begin(), v.end(), [](const std::pair<int, NsTile>& a, const std::pair<int, NsTile>& b) {
     return a.first > b.first;
@@ -340,6 +380,8 @@ struct NsEngine {
   std::vector<NsBatch> batches;
   double* d_norm2 = nullptr;
   float* d_split_ws = nullptr;       // fp32 partial sums of split Gram tiles
+  bool pdl = true;                   // programmatic dependent launch between NS launches
+  uint64_t wait_ns = kDefaultWaitNs; // limit of the kernels' bounded waits
 };
 
 // Plan: group matrices by (s, l); returns matrix order (indices into shapes)
@@ -413,34 +455,45 @@ static void split_gram_tiles(const std::vector<NsGroup>& groups, int g0, std::ve
                              int workers, std::vector<std::array<int, 6>>& targets, int& nparts_total,
                              int kcap = 0) {
   int64_t total = 0;
-  for (const NsTile& x : t) total += groups[g0 + x.group].l_pad / kslice;
+  for (const NsTile& x : t) total += (int64_t)(groups[g0 + x.group].l_pad / kslice) * (x.nh == 2 ? 2 : 1);
   const int64_t avg = total / std::max(1, workers);
   int64_t part = std::max<int64_t>(8, avg / 2);
   if (kcap > 0) part = std::min<int64_t>(part, kcap);
   std::vector<NsTile> out;
   nparts_total = 0;
-  for (const NsTile& x : t) {
-    const int nk = groups[g0 + x.group].l_pad / kslice;
-    if ((nk <= 2 * avg && (kcap <= 0 || nk <= kcap)) || nparts_total + 64 > 65535) {
-      out.push_back(x);
+  for (const NsTile& x0 : t) {
+    const int nk = groups[g0 + x0.group].l_pad / kslice;
+    const int nh = x0.nh == 2 ? 2 : 1;
+    // decided per 256-column block, so that one- and two-block tiles split
+    // the same blocks into the same parts (and give the same sums)
+    if ((nk <= 2 * avg && (kcap <= 0 || nk <= kcap)) || nparts_total + 128 > 65535) {
+      out.push_back(x0);
       continue;
     }
-    const int nparts = (int)std::min<int64_t>(64, (nk + part - 1) / part);
-    targets.push_back({x.group, x.mat, x.tm, x.tn, nparts_total, nparts});
-    for (int k = 0; k < nparts; ++k) {
-      NsTile y = x;
-      y.kb0 = (uint16_t)((int64_t)nk * k / nparts);
-      y.kb1 = (uint16_t)((int64_t)nk * (k + 1) / nparts);
-      y.slot = (uint16_t)(nparts_total + k + 1);
-      out.push_back(y);
+    // a split tile is one block wide: a two-block tile is split per block
+    for (int h = 0; h < nh; ++h) {
+      NsTile x = x0;
+      x.tn = (uint16_t)(x0.tn + h);
+      x.nh = 1;
+      const int nparts = (int)std::min<int64_t>(64, (nk + part - 1) / part);
+      targets.push_back({x.group, x.mat, x.tm, x.tn, nparts_total, nparts});
+      for (int k = 0; k < nparts; ++k) {
+        NsTile y = x;
+        y.kb0 = (uint16_t)((int64_t)nk * k / nparts);
+        y.kb1 = (uint16_t)((int64_t)nk * (k + 1) / nparts);
+        y.slot = (uint16_t)(nparts_total + k + 1);
+        out.push_back(y);
+      }
+      nparts_total += nparts;
     }
-    nparts_total += nparts;
   }
   t.swap(out);
 }
 
+// tiles_mode: 0 or 1 one-block tiles, 2 two-block tiles wherever a row has
+// two blocks left (bf16 operands).
 static void layout_ns(std::vector<NsGroup>& groups, lm_dtype xdt, int nmat, Arena& ar, NsLayout& L,
-                      std::vector<NsBatch>& batches, int pieces = 1) {
+                      std::vector<NsBatch>& batches, int pieces = 1, int tiles_mode = 0) {
   const size_t es = dtype_size(xdt) * (size_t)pieces;
   for (auto& g : groups) {
     const size_t xb = (size_t)g.count * g.s_pad * g.l_pad * es;
@@ -463,6 +516,16 @@ static void layout_ns(std::vector<NsGroup>& groups, lm_dtype xdt, int nmat, Aren
     for (int ph = 0; ph < 3; ++ph) {
       std::vector<NsTile> t;
       build_ns_tiles(groups, g0, b.ng, ph, bm, bn, t);
+      // Two-block tiles stage a quarter fewer bytes per FLOP, but they take
+      // both accumulators (the epilogue of one tile no longer overlaps the
+      // next tile's main loop), leave room for a 3- or 4-stage ring only and
+      // put twice as many matrices in flight in a launch (a larger L2 working
+      // set): measured slower on the GPT-style sets, so used only on request.
+      if (xdt == LM_BF16 && pieces == 1 && tiles_mode == 2) {
+        t.clear();
+        build_ns_tiles(groups, g0, b.ng, ph, bm, bn, t, true);
+        b.wide[ph] = true;
+      }
       std::vector<int> offs;
       std::vector<std::array<int, 6>> targets;
       if (ph == NS_GRAM) {
@@ -487,7 +550,7 @@ static void layout_ns(std::vector<NsGroup>& groups, lm_dtype xdt, int nmat, Aren
         for (const NsTile& x : t) {
           const NsGroup& g = groups[g0 + x.group];
           const int nk = (ph == NS_GRAM) ? (x.kb1 != 0 ? x.kb1 - x.kb0 : g.l_pad / kTcBK) : g.s_pad / kTcBK;
-          sorted.push_back({nk + 6, x});
+          sorted.push_back({(nk + 6) * (x.nh == 2 ? 2 : 1), x});
         }
         std::stable_sort(sorted.begin(), sorted.end(),
                          [](const std::pair<int, NsTile>& a, const std::pair<int, NsTile>& c) {
@@ -642,7 +705,7 @@ static lm_status run_ns(const NsEngine& E, int steps, const NsCoeffs* coeffs, un
   for (size_t gi = 0; E.pieces == 3 && steps > 0 && gi < E.groups.size(); ++gi) {
     const NsGroup& g = E.groups[gi];
     cudaError_t e = timed(P, LM_KERNEL_OTHER, st, [&]() {
-      return launch_split3(static_cast<const float*>(g.Xf), g.X[0], (size_t)g.count * g.s_pad * g.l_pad, st);
+      return launch_split3(static_cast<const float*>(g.Xf), g.X[0], (size_t)g.count * g.s_pad * g.l_pad, flags, st);
     });
     if (e != cudaSuccess) return cuda_fail(e, "three-piece split launch");
   }
@@ -656,14 +719,15 @@ static lm_status run_ns(const NsEngine& E, int steps, const NsCoeffs* coeffs, un
             cudaError_t r = launch_ns_tc((NsPhase)ph, it, b.ng, E.groups.data() + b.g0, E.maps.data() + b.g0, b.tiles[ph],
                                b.ntiles[ph], b.offsets[ph], b.npairs[ph], E.d_norm2, co, flags,
                                it == steps - 1 ? fuse : nullptr, st, active, split ? E.d_split_ws : nullptr,
-                               E.pieces, it == steps - 1 ? 1 : 0);
-            if (r == cudaSuccess && split) r = launch_ns_split_finish(b.split_targets, b.nsplit, E.d_split_ws, st);
+                               E.pieces, it == steps - 1 ? 1 : 0, b.wide[ph], E.pdl, E.wait_ns);
+            if (r == cudaSuccess && split)
+              r = launch_ns_split_finish(b.split_targets, b.nsplit, E.d_split_ws, flags, st);
             return r;
           }
           cudaError_t r = launch_ns_simt((NsPhase)ph, it, b.ng, E.d_groups + b.g0, b.tiles[ph], b.ntiles[ph],
-                                         E.d_norm2, co, st, active, E.d_split_ws);
+                                         E.d_norm2, co, st, active, E.d_split_ws, flags);
           if (r == cudaSuccess && ph == NS_GRAM && b.nsplit > 0)
-            r = launch_ns_split_finish_f32(b.split_targets, b.nsplit, E.d_split_ws, st);
+            r = launch_ns_split_finish_f32(b.split_targets, b.nsplit, E.d_split_ws, flags, st);
           return r;
         });
         if (e != cudaSuccess) return cuda_fail(e, "Newton-Schulz launch");
@@ -674,6 +738,29 @@ static lm_status run_ns(const NsEngine& E, int steps, const NsCoeffs* coeffs, un
 }  // namespace lm
 
 using namespace lm;
+
+// Layer sharding (Section 5.4): whole matrices dealt out to `world` ranks,
+// largest Newton-Schulz cost 3 s^2 l + s^3 first, each to the least-loaded
+// rank (the lowest on a tie); ties in cost keep parameter order.  1-D
+// parameters: -1.
+static void shard_owners(const lm_tensor* params, int n, int world, std::vector<int>& owner) {
+  owner.assign(n, -1);
+  std::vector<std::pair<double, int>> cost;
+  for (int i = 0; i < n; ++i)
+    if (is_matrix(params[i])) {
+      const double s = (double)std::min(params[i].rows, params[i].cols);
+      const double l = (double)std::max(params[i].rows, params[i].cols);
+      cost.push_back({3.0 * s * s * l + s * s * s, i});
+    }
+  std::stable_sort(cost.begin(), cost.end(),
+                   [](const std::pair<double, int>& a, const std::pair<double, int>& b) { return a.first > b.first; });
+  std::vector<double> load(std::max(world, 1), 0.0);
+  for (const auto& c : cost) {
+    const int r = (int)(std::min_element(load.begin(), load.end()) - load.begin());
+    owner[c.second] = r;
+    load[r] += c.first;
+  }
+}
 
 // ---------------------------------------------------------------------------
 // the state
@@ -693,6 +780,9 @@ struct lm_state {
   std::vector<const void*> grads_checked;   // gradient pointers found to be device memory
   bool grads_valid = false;
   LionTable lion_all[2], lion_vec[2];   // lion_all: matrices only under LM_VECTOR_ADAMW
+  int world = 1, rank = 0;              // layer sharding: this state's rank of `world`
+  std::vector<int> owner;               // owner rank per parameter (-1: 1-D), sharded states
+  LionTable ema[2];                     // matrices other ranks own: momentum update on Muon steps
   bool adamw = false;                   // 1-D parameters take AdamW
   AdamTable adam[2];                    // per dtype, 1-D parameters
   float* vmom = nullptr;                // AdamW second moments
@@ -794,7 +884,11 @@ void lm_config_default(lm_config* c) {
   c->srank_alpha = 0.01;
   c->srank_iters = 5;
   c->srank_seed = 0;
+  c->shard_rank = 0;
+  c->shard_world = 1;
 }
+
+size_t lm_config_size(void) { return sizeof(lm_config); }
 
 const char* lm_status_string(lm_status st) {
   switch (st) {
@@ -813,6 +907,18 @@ const char* lm_status_string(lm_status st) {
 const char* lm_last_error(void) { return g_last_error.c_str(); }
 
 uint64_t lm_kernel_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+lm_status lm_shard_owners(const lm_tensor* params, int n, int world, int* owner) {
+  if (params == nullptr || owner == nullptr) return fail(LM_ERR_INVALID_ARG, "params/owner is NULL");
+  if (n < 1) return fail(LM_ERR_INVALID_ARG, "n must be >= 1");
+  if (world < 1 || world > 4096) return fail(LM_ERR_INVALID_ARG, "world must be in [1, 4096]");
+  for (int i = 0; i < n; ++i)
+    if (params[i].rows < 0 || params[i].cols < 0) return fail(LM_ERR_INVALID_ARG, "params[%d] has a negative size", i);
+  std::vector<int> o;
+  shard_owners(params, n, world, o);
+  std::copy(o.begin(), o.end(), owner);
+  return LM_OK;
+}
 
 lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* cuda_stream,
                     lm_state** out) {
@@ -842,11 +948,16 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
   s->debug = env_is("LM_DEBUG", "1");
   if (env_is("LM_NVTX", "1")) g_nvtx.store(true);
 
-  // matrices and their shape groups
+  // matrices and their shape groups (under layer sharding: the matrices this
+  // rank owns; the others only take the momentum update on Muon steps)
+  s->world = cfg->shard_world > 1 ? cfg->shard_world : 1;
+  s->rank = s->world > 1 ? cfg->shard_rank : 0;
+  if (s->world > 1) shard_owners(params, n, s->world, s->owner);
+  auto owned = [&](int i) { return s->world == 1 || s->owner[i] == s->rank; };
   std::vector<int> mat_param;
   std::vector<std::pair<int64_t, int64_t>> mat_shapes;
   for (int i = 0; i < n; ++i)
-    if (is_matrix(params[i])) {
+    if (is_matrix(params[i]) && owned(i)) {
       mat_param.push_back(i);
       mat_shapes.push_back({params[i].rows, params[i].cols});
     }
@@ -913,20 +1024,37 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
     off_at[d] = ar.add(at[d].size() * sizeof(AdamTensor));
     off_ac[d] = ar.add(ac[d].size() * sizeof(LionChunk));
   }
-  std::vector<LionChunk> lc_all[2], lc_vec[2];
-  size_t off_lt_all[2], off_lc_all[2], off_lt_vec[2], off_lc_vec[2];
+  // momentum-only table: matrices another rank owns (layer sharding)
+  std::vector<LionTensor> lt_ema[2];
+  for (int i = 0; i < n; ++i) {
+    if (numel(params[i]) == 0 || !is_matrix(params[i]) || owned(i)) continue;
+    LionTensor t;
+    t.w = params[i].data;
+    t.m = nullptr;
+    t.n = numel(params[i]);
+    t.grad_slot = i;
+    t.pad = i;
+    lt_ema[params[i].dtype].push_back(t);
+  }
+  std::vector<LionChunk> lc_all[2], lc_vec[2], lc_ema[2];
+  size_t off_lt_all[2], off_lc_all[2], off_lt_vec[2], off_lc_vec[2], off_lt_ema[2], off_lc_ema[2];
   for (int d = 0; d < 2; ++d) {
     build_lion_chunks(lt_all[d], lc_all[d]);
     build_lion_chunks(lt_vec[d], lc_vec[d]);
+    build_lion_chunks(lt_ema[d], lc_ema[d]);
     off_lt_all[d] = ar.add(lt_all[d].size() * sizeof(LionTensor));
     off_lc_all[d] = ar.add(lc_all[d].size() * sizeof(LionChunk));
     off_lt_vec[d] = ar.add(lt_vec[d].size() * sizeof(LionTensor));
     off_lc_vec[d] = ar.add(lc_vec[d].size() * sizeof(LionChunk));
+    off_lt_ema[d] = ar.add(lt_ema[d].size() * sizeof(LionTensor));
+    off_lc_ema[d] = ar.add(lc_ema[d].size() * sizeof(LionChunk));
   }
 
   // Muon tables
   NsLayout L;
-  layout_ns(s->ns.groups, s->ns.xdt, s->nmat, ar, L, s->ns.batches, s->ns.pieces);
+  layout_ns(s->ns.groups, s->ns.xdt, s->nmat, ar, L, s->ns.batches, s->ns.pieces, env_tiles_mode());
+  s->ns.pdl = !env_is("LM_PDL", "0");
+  s->ns.wait_ns = env_wait_limit_ns();
   const size_t off_mats = ar.add((size_t)std::max(s->nmat, 1) * sizeof(MatDesc));
   std::vector<MatDesc> mats(s->nmat);
   // matrices are numbered in group order
@@ -1063,11 +1191,16 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
   for (int d = 0; d < 2; ++d) {
     for (auto& t : lt_all[d]) { t.m = s->mom + s->mom_off[t.pad]; }
     for (auto& t : lt_vec[d]) { t.m = s->mom + s->mom_off[t.pad]; }
+    for (auto& t : lt_ema[d]) { t.m = s->mom + s->mom_off[t.pad]; }
     auto put = [&](size_t off, const void* src, size_t bytes) { if (bytes) memcpy(img.data() + off, src, bytes); };
     put(off_lt_all[d], lt_all[d].data(), lt_all[d].size() * sizeof(LionTensor));
     put(off_lc_all[d], lc_all[d].data(), lc_all[d].size() * sizeof(LionChunk));
     put(off_lt_vec[d], lt_vec[d].data(), lt_vec[d].size() * sizeof(LionTensor));
     put(off_lc_vec[d], lc_vec[d].data(), lc_vec[d].size() * sizeof(LionChunk));
+    put(off_lt_ema[d], lt_ema[d].data(), lt_ema[d].size() * sizeof(LionTensor));
+    put(off_lc_ema[d], lc_ema[d].data(), lc_ema[d].size() * sizeof(LionChunk));
+    s->ema[d] = {reinterpret_cast<LionTensor*>(base + off_lt_ema[d]),
+                 reinterpret_cast<LionChunk*>(base + off_lc_ema[d]), (int)lc_ema[d].size()};
     s->lion_all[d] = {reinterpret_cast<LionTensor*>(base + off_lt_all[d]),
                       reinterpret_cast<LionChunk*>(base + off_lc_all[d]), (int)lc_all[d].size()};
     s->lion_vec[d] = {reinterpret_cast<LionTensor*>(base + off_lt_vec[d]),
@@ -1245,8 +1378,10 @@ static lm_status run_srank(lm_state* s, cudaStream_t stream) {
       if (e != cudaSuccess) return cuda_fail(e, "selection buffer reset");
     }
     auto launch = [&](const lm_state::SrLaunch& L, cudaStream_t st) {
-      if (L.vec4) return launch_srank_ring((int)L.max_cols, s->d_sr, L.items, L.nitems, k, last, s->d_flags, st);
-      return launch_srank_pass(L.slots, L.threads, L.vec4, s->d_sr, L.items, L.nitems, k, last, st);
+      if (L.vec4)
+        return launch_srank_ring((int)L.max_cols, s->d_sr, L.items, L.nitems, k, last, s->d_flags,
+                                 std::min<uint64_t>(kRingWaitNs, s->ns.wait_ns), st);
+      return launch_srank_pass(L.slots, L.threads, L.vec4, s->d_sr, L.items, L.nitems, k, last, s->d_flags, st);
     };
     if (s->sr_nside == 0) {
       for (const auto& L : s->sr_launch) {
@@ -1271,7 +1406,7 @@ static lm_status run_srank(lm_state* s, cudaStream_t stream) {
   }
   e = timed(P, LM_KERNEL_SRANK, stream, [&]() {
     return launch_srank_decide(s->d_sr, s->nmat, s->cfg.srank_alpha, passes - 1, s->d_active, s->d_skip,
-                               s->d_srank, stream);
+                               s->d_srank, s->d_flags, stream);
   });
   if (e != cudaSuccess) return cuda_fail(e, "selection launch");
   return LM_OK;
@@ -1290,7 +1425,8 @@ __global__ void guard_check_kernel(const unsigned char* base, const size_t* offs
 
 // AdamW over the 1-D parameters of both dtypes (LM_VECTOR_ADAMW).
 static lm_status run_adamw(lm_state* s, int64_t t, cudaStream_t stream) {
-  const AdamConsts ak = adamw_consts(s->cfg, t);
+  AdamConsts ak = adamw_consts(s->cfg, t);
+  ak.flags = s->d_flags;
   for (int d = 0; d < 2; ++d) {
     if (s->adam[d].nchunks == 0) continue;
     cudaError_t e = timed(&s->prof, LM_KERNEL_ADAMW, stream, [&]() {
@@ -1333,6 +1469,7 @@ lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t, void* c
   const bool mixed = s->srank;
   const bool muon = mixed || (c.period != 0 && (t % c.period) == 0);
   LionConsts lk = lion_consts(c);
+  lk.flags = s->d_flags;
   cudaError_t e;
   Profiler* P = &s->prof;
   s->last_t = t;
@@ -1353,6 +1490,7 @@ lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t, void* c
   }
   // Muon step: momentum + norm, Lion on the vectors, NS iterations, finalize.
   MuonConsts mk = muon_consts(c);
+  mk.flags = s->d_flags;
   if (mixed) mk.active = s->d_active;
   if (s->nmat > 0) {
     e = timed(P, LM_KERNEL_OTHER, stream, [&]() {
@@ -1367,6 +1505,16 @@ lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t, void* c
       });
       if (e != cudaSuccess) return cuda_fail(e, "momentum/norm kernel launch");
     }
+  }
+  // layer sharding: the matrices other ranks own take the momentum update
+  // here and their new values from their owners afterwards
+  for (int d = 0; d < 2; ++d) {
+    if (s->ema[d].nchunks == 0) continue;
+    e = timed(P, LM_KERNEL_MOMENTUM_NORM, stream, [&]() {
+      return launch_ema((lm_dtype)d, s->ema[d].tensors, s->ema[d].chunks, s->ema[d].nchunks, s->d_grads, lk,
+                        s->lion_grid[d], stream);
+    });
+    if (e != cudaSuccess) return cuda_fail(e, "momentum kernel launch (matrices of other ranks)");
   }
   if (s->adamw) {
     if ((st = run_adamw(s, t, stream)) != LM_OK) return st;
@@ -1432,8 +1580,11 @@ lm_status lm_get_selection(lm_state* s, int n, unsigned char* took_muon, double*
     const bool muon = s->cfg.period != 0 && (s->last_t % s->cfg.period) == 0;
     std::fill(act.begin(), act.end(), muon ? 1 : 0);
   }
+  const bool muon_step = !s->srank && s->cfg.period != 0 && (s->last_t % s->cfg.period) == 0;
   for (int i = 0; i < n; ++i) {
-    if (took_muon) took_muon[i] = 0;
+    // under layer sharding a matrix another rank owns also took the Muon
+    // step (there, with this rank's momentum update)
+    if (took_muon) took_muon[i] = (muon_step && is_matrix(s->params[i])) ? 1 : 0;
     if (srank) srank[i] = nan;
   }
   for (int id = 0; id < s->nmat; ++id) {
@@ -1623,7 +1774,9 @@ static lm_status msign_impl(const lm_tensor* in, lm_tensor* out, int steps, cons
   plan_groups({{in->rows, in->cols}}, E.xdt, E.groups, members);
   Arena ar;
   NsLayout L;
-  layout_ns(E.groups, E.xdt, 1, ar, L, E.batches, E.pieces);
+  layout_ns(E.groups, E.xdt, 1, ar, L, E.batches, E.pieces, env_tiles_mode());
+  E.pdl = !env_is("LM_PDL", "0");
+  E.wait_ns = env_wait_limit_ns();
   const size_t off_mat = ar.add(sizeof(MatDesc));
   MatDesc d;
   memset(&d, 0, sizeof(d));
@@ -1667,12 +1820,21 @@ static lm_status msign_impl(const lm_tensor* in, lm_tensor* out, int steps, cons
   MatDesc* dm = reinterpret_cast<MatDesc*>(base + off_mat);
   ElemChunk* de = reinterpret_cast<ElemChunk*>(base + off_et);
   unsigned* dflags = reinterpret_cast<unsigned*>(base + off_flags);
+  mk.flags = dflags;
   e = launch_momentum_norm(xio, in->dtype, dm, de, (int)et.size(), nullptr, mk, 1, stream);
   if (e != cudaSuccess) return cleanup(cuda_fail(e, "norm kernel launch"));
   if ((st = run_ns(E, steps, co.data(), dflags, stream)) != LM_OK) return cleanup(st);
   e = launch_finalize(xio, out->dtype, dm, de, (int)et.size(), mk, 1, dflags, stream);
   if (e != cudaSuccess) return cleanup(cuda_fail(e, "output kernel launch"));
-  return cleanup(LM_OK);
+  // the call's status word: read back before the workspace goes
+  unsigned hflags = 0;
+  e = cudaMemcpyAsync(&hflags, dflags, sizeof(unsigned), cudaMemcpyDeviceToHost, stream);
+  cudaFreeAsync(base, stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return cuda_fail(e, "msign status read");
+  if (hflags & LM_FLAG_TIMEOUT)
+    return fail(LM_ERR_TIMEOUT, "a bounded device wait gave up; out was not written (LM_FLAG_TIMEOUT)");
+  return LM_OK;
 }
 
 extern "C" {

@@ -87,6 +87,9 @@ template <typename T>
 __global__ void __launch_bounds__(kLionThreads)
     lion_kernel(const LionTensor* __restrict__ tensors, const LionChunk* __restrict__ chunks,
                 int nchunks, const void* const* __restrict__ grads, LionConsts k) {
+  if (lm_stopped(k.flags)) return;
+  // the next kernel on the stream may start its set-up (programmatic launch)
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   for (int c = blockIdx.x; c < nchunks; c += gridDim.x) {
     const LionChunk ch = chunks[c];
     const LionTensor t = tensors[ch.tensor];
@@ -141,6 +144,34 @@ __global__ void __launch_bounds__(kLionThreads)
   }
 }
 
+// Momentum update alone, M <- beta2 M + (1 - beta2) G (the last line of
+// Algorithm 1's loop body), for the matrices another rank owns on a layer-
+// sharded Muon step: the same float32 operations as lion_elem, so every
+// rank's momentum stays equal to the owner's bit for bit.
+template <typename T>
+__global__ void __launch_bounds__(kLionThreads)
+    ema_kernel(const LionTensor* __restrict__ tensors, const LionChunk* __restrict__ chunks, int nchunks,
+               const void* const* __restrict__ grads, LionConsts k) {
+  if (lm_stopped(k.flags)) return;
+  for (int c = blockIdx.x; c < nchunks; c += gridDim.x) {
+    const LionChunk ch = chunks[c];
+    const LionTensor t = tensors[ch.tensor];
+    const T* g = static_cast<const T*>(grads[t.grad_slot]) + ch.begin;
+    float* m = t.m + ch.begin;
+    const int64_t nvec = ch.count >> 3;
+    for (int64_t v = threadIdx.x; v < nvec; v += kLionThreads) {
+      float gv[8], mv[8];
+      load8(g + v * 8, gv);
+      load8(m + v * 8, mv);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) mv[e] = __fadd_rn(__fmul_rn(k.b2, mv[e]), __fmul_rn(k.c2, gv[e]));
+      store8(m + v * 8, mv);
+    }
+    for (int64_t e = (nvec << 3) + threadIdx.x; e < ch.count; e += kLionThreads)
+      m[e] = __fadd_rn(__fmul_rn(k.b2, m[e]), __fmul_rn(k.c2, to_f(g[e])));
+  }
+}
+
 // ---------------------------------------------------------------------------
 // AdamW for 1-D parameters (Section 3's fallback for biases and norm gains).
 // The same fixed operation order as the float32 reference: every product,
@@ -160,6 +191,7 @@ template <typename T>
 __global__ void __launch_bounds__(kLionThreads)
     adamw_kernel(const AdamTensor* __restrict__ tensors, const LionChunk* __restrict__ chunks, int nchunks,
                  const void* const* __restrict__ grads, AdamConsts k) {
+  if (lm_stopped(k.flags)) return;
   for (int c = blockIdx.x; c < nchunks; c += gridDim.x) {
     const LionChunk ch = chunks[c];
     const AdamTensor t = tensors[ch.tensor];
@@ -275,6 +307,8 @@ template <typename XT, typename GT, int MODE>
 __global__ void __launch_bounds__(kElemThreads, kMomCtas)
     momentum_norm_kernel(const MatDesc* __restrict__ mats, const ElemChunk* __restrict__ chunks,
                          int nchunks, const void* const* __restrict__ grads, MuonConsts k) {
+  if (lm_stopped(k.flags)) return;
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   for (int c = blockIdx.x; c < nchunks; c += gridDim.x) {
     const ElemChunk ch = chunks[c];
     if (k.active != nullptr && !k.active[ch.mat]) continue;   // this matrix takes the Lion step
@@ -347,6 +381,9 @@ template <typename XT, typename PT, int MODE>
 __global__ void __launch_bounds__(kElemThreads, kFinCtas)
     finalize_kernel(const MatDesc* __restrict__ mats, const ElemChunk* __restrict__ chunks, int nchunks,
                     MuonConsts k, unsigned* flags) {
+  // the NS launches before it may be programmatic: wait for their results
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  if (lm_stopped(flags)) return;
   for (int c = blockIdx.x; c < nchunks; c += gridDim.x) {
     const ElemChunk ch = chunks[c];
     if (k.active != nullptr && !k.active[ch.mat]) continue;
@@ -393,6 +430,18 @@ cudaError_t launch_lion(lm_dtype dt, const LionTensor* tensors, const LionChunk*
     lion_kernel<__nv_bfloat16><<<grid, kLionThreads, 0, st>>>(tensors, chunks, nchunks, grads, k);
   else
     lion_kernel<float><<<grid, kLionThreads, 0, st>>>(tensors, chunks, nchunks, grads, k);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_ema(lm_dtype dt, const LionTensor* tensors, const LionChunk* chunks, int nchunks,
+                       const void* const* grads, LionConsts k, int grid, cudaStream_t st) {
+  if (nchunks <= 0) return cudaSuccess;
+  if (grid > nchunks) grid = nchunks;
+  count_launch();
+  if (dt == LM_BF16)
+    ema_kernel<__nv_bfloat16><<<grid, kLionThreads, 0, st>>>(tensors, chunks, nchunks, grads, k);
+  else
+    ema_kernel<float><<<grid, kLionThreads, 0, st>>>(tensors, chunks, nchunks, grads, k);
   return cudaGetLastError();
 }
 

@@ -12,6 +12,15 @@ namespace lm {
 
 constexpr int kPtrsPerUpload = 1024;   // pointers per pointer-upload launch
 
+#ifdef __CUDACC__
+// Every kernel of a step reads the status word at entry: once a bounded wait
+// has given up (LM_FLAG_TIMEOUT), the rest of the step, and every later
+// step until the flag is cleared, does nothing.  NULL: no status word.
+__device__ __forceinline__ bool lm_stopped(const unsigned* flags) {
+  return flags != nullptr && (*reinterpret_cast<const volatile unsigned*>(flags) & LM_FLAG_TIMEOUT) != 0u;
+}
+#endif
+
 // ---------------------------------------------------------------------------
 // Lion multi-tensor step (Algorithm 1, Lion branch + momentum update)
 // ---------------------------------------------------------------------------
@@ -33,6 +42,7 @@ struct LionConsts {
   // Adaptive selection: skip[param] != 0 makes the Lion kernel leave that
   // parameter alone (it takes the Muon step); NULL: no parameter skipped.
   const unsigned char* skip;
+  const unsigned* flags;   // status word read at entry (lm_stopped), or NULL
 };
 
 // AdamW on 1-D parameters (the LM_VECTOR_ADAMW rule): parameter, first
@@ -49,6 +59,7 @@ struct AdamTensor {
 // 1/sqrt(1-b2^k), lr*wd, eps (k = t + 1), each rounded once from double.
 struct AdamConsts {
   float b1, c1, b2, c2, step, rbc2, lrwd, eps;
+  const unsigned* flags;   // status word read at entry (lm_stopped), or NULL
 };
 cudaError_t launch_adamw(lm_dtype dt, const AdamTensor* tensors, const LionChunk* chunks, int nchunks,
                          const void* const* grads, AdamConsts k, cudaStream_t st);
@@ -58,6 +69,10 @@ cudaError_t launch_lion(lm_dtype dt, const LionTensor* tensors, const LionChunk*
                         int nchunks, const void* const* grads, LionConsts k,
                         int grid, cudaStream_t st);
 int lion_grid_size(lm_dtype dt);
+// Momentum update alone over a chunk table (matrices another rank owns on a
+// layer-sharded Muon step); k.b2, k.c2 and k.flags are used.
+cudaError_t launch_ema(lm_dtype dt, const LionTensor* tensors, const LionChunk* chunks, int nchunks,
+                       const void* const* grads, LionConsts k, int grid, cudaStream_t st);
 
 // ---------------------------------------------------------------------------
 // Muon element-wise kernels: momentum + norm -> X0 (K2), finalize (K6)
@@ -94,6 +109,7 @@ struct MuonConsts {
   // Adaptive selection: active[mat] != 0 for the matrices that take the
   // Muon step; NULL: every matrix does.
   const unsigned char* active;
+  const unsigned* flags;   // status word read at entry (lm_stopped), or NULL
 };
 // mode 0: Muon momentum step (G_hat from grads + momentum, M update)
 // mode 1: msign input (G_hat = input tensor, no momentum)
@@ -134,7 +150,10 @@ struct NsTile {
   // Split-K (Gram phase only): K blocks [kb0, kb1) of the tile, kb1 == 0 for
   // all of them; slot != 0: the partial product is written in fp32 to
   // workspace tile slot - 1 instead of A (NsSplitTarget sums the parts).
-  uint16_t kb0, kb1, slot, pad;
+  uint16_t kb0, kb1, slot;
+  // 256-column output blocks of the tile, starting at block tn: 2 only in
+  // the wide-tile kernel's launches (0 and 1 both mean one block).
+  uint16_t nh;
 };
 // A split Gram tile (tile edge `tile`: 256 tensor-core, 128 fp32 path): the
 // parts in workspace tiles first .. first + nparts - 1 are summed in that
@@ -188,6 +207,11 @@ struct FuseFinal {
   const MatDesc* mats;
   float eM, lam;
 };
+// Limit of a bounded device wait unless the state sets another
+// (LM_WAIT_LIMIT_NS at lm_create): a wait that runs out gives up and raises
+// LM_FLAG_TIMEOUT; every later kernel then does nothing until the flag is cleared.
+constexpr uint64_t kDefaultWaitNs = 5000000000ull;   // 5 s
+uint64_t env_wait_limit_ns();   // LM_WAIT_LIMIT_NS if set to a positive integer, else kDefaultWaitNs
 // offsets: NULL (round robin over tiles) or npairs + 1 range starts;
 // fuse: NULL, or the parameter write of the last APPLY phase.
 cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* groups,
@@ -195,24 +219,32 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
                          const int* offsets, int npairs, const double* norm2, NsCoeffs co,
                          unsigned* flags, const FuseFinal* fuse, cudaStream_t st,
                          const unsigned char* active = nullptr, float* split_ws = nullptr, int pieces = 1,
-                         int final_f32 = 0);
+                         int final_f32 = 0, bool wide = false, bool pdl = false,
+                         uint64_t wait_ns = kDefaultWaitNs);
 // split_ws: non-NULL only for a Gram launch whose tiles include split-K parts.
 // pieces = 3: fp32 operands as three bf16 pieces (no split tiles, no fused
 // parameter write); final_f32: this APPLY writes fp32 X to NsGroup::Xf.
+// wide: the tile list may hold two-block tiles (NsTile::nh = 2), run by the
+// wide-tile kernel (bf16 only); pdl: programmatic dependent launch (the
+// kernel may start while the previous kernel on the stream finishes).
+// Both kernels do nothing when LM_FLAG_TIMEOUT is already set in *flags.
 // fp32 -> three bf16 planes (hi, mid, lo; their sum is exactly the input):
 // n elements of src, plane q at dst + q * n.
-cudaError_t launch_split3(const float* src, void* dst, size_t n, cudaStream_t st);
+cudaError_t launch_split3(const float* src, void* dst, size_t n, const unsigned* flags, cudaStream_t st);
 // After a Gram launch with split tiles: bf16 A tiles from the fp32 parts.
-cudaError_t launch_ns_split_finish(const NsSplitTarget* targets, int n, const float* ws, cudaStream_t st);
+cudaError_t launch_ns_split_finish(const NsSplitTarget* targets, int n, const float* ws, const unsigned* flags,
+                                   cudaStream_t st);
 
 // fp32 CUDA-core path.
 constexpr int kSimtBM = 128, kSimtBN = 128;
 int simt_pad(int x);
 cudaError_t launch_ns_simt(NsPhase ph, int iter, int ngroups, const NsGroup* dgroups,
                            const NsTile* tiles, int ntiles, const double* norm2, NsCoeffs co,
-                           cudaStream_t st, const unsigned char* active = nullptr, float* split_ws = nullptr);
+                           cudaStream_t st, const unsigned char* active = nullptr, float* split_ws = nullptr,
+                           const unsigned* flags = nullptr);
 // fp32 path: A tiles (and mirrors) from the fp32 parts of split Gram tiles.
-cudaError_t launch_ns_split_finish_f32(const NsSplitTarget* targets, int n, const float* ws, cudaStream_t st);
+cudaError_t launch_ns_split_finish_f32(const NsSplitTarget* targets, int n, const float* ws, const unsigned* flags,
+                                       cudaStream_t st);
 // active (both NS paths): NULL, or active[first_mat + mat] != 0 for the
 // matrices whose tiles run; tiles of the others are skipped by every role.
 
@@ -241,7 +273,7 @@ struct SrItem {
 // slots = 0 means cols is too large (more than 16384).
 int srank_slots(int64_t cols, int* threads);
 cudaError_t launch_srank_pass(int slots, int threads, bool vec4, const SrMat* mats, const SrItem* items,
-                              int nitems, int pass, bool last, cudaStream_t st);
+                              int nitems, int pass, bool last, const unsigned* flags, cudaStream_t st);
 // The same pass through the shared-memory ring (every matrix of the launch
 // with cols % 4 == 0, at most max_cols <= 16384 columns); a stalled copy sets
 // LM_FLAG_TIMEOUT in *flags.
@@ -250,12 +282,12 @@ cudaError_t launch_srank_pass(int slots, int threads, bool vec4, const SrMat* ma
 // with the same code share a launch.
 int srank_ring_shape(int64_t cols);
 cudaError_t launch_srank_ring(int max_cols, const SrMat* mats, const SrItem* items, int nitems, int pass, bool last,
-                              unsigned* flags, cudaStream_t st);
+                              unsigned* flags, uint64_t wait_ns, cudaStream_t st);
 // Decide per matrix: Muon iff ||M||_F^2 == 0 or ||M||_F^2 <= alpha min(m, n)
 // sigma^2 (sigma^2 = acc[1 + last_pass]); writes active[mat], skip[param]
 // and the estimate srank[mat] = ||M||_F^2 / sigma^2.
 cudaError_t launch_srank_decide(const SrMat* mats, int nmat, double alpha, int last_pass, unsigned char* active,
-                                unsigned char* skip, double* srank, cudaStream_t st);
+                                unsigned char* skip, double* srank, const unsigned* flags, cudaStream_t st);
 constexpr int kMaxGroupsSimt = 64;
 
 // Launch accounting (lm_kernel_launch_count) and the thread's last-error text.

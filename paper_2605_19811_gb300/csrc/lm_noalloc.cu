@@ -5,9 +5,11 @@
 // The scratch is a file-scope __device__ array of kNoAllocScratchBytes.  Every
 // GPU that loads this library holds it until the process exits.  Host code
 // cannot use the array's name as a device address (on the host it names a
-// stand-in object), so the device address is looked up once per device with
+// stand-in object), so the device address is looked up with
 // cudaGetSymbolAddress, with that device current, on the first call made on
-// that device, and cached.
+// that device, and cached together with the device's current context: a call
+// that finds another context (the old one destroyed and a new one made, as
+// by cudaDeviceReset, which reloads the module) looks the address up again.
 //
 // All calls share the array and it keeps what the last call left there: the
 // parts that must start at zero (the padded X0 buffer, the norm accumulator,
@@ -20,6 +22,8 @@
 #include <cstring>
 #include <mutex>
 
+#include <cudaTypedefs.h>
+
 #include "lm_internal.h"
 
 namespace lm {
@@ -29,17 +33,43 @@ constexpr size_t kNoAllocScratchBytes = (size_t)64 << 20;   // 64 MiB
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
 std::mutex g_scratch_mu;
-char* g_scratch_addr[kMaxDevices] = {nullptr};
+struct ScratchSlot {
+  CUcontext ctx;   // context the address was looked up in
+  char* addr;
+};
+ScratchSlot g_scratch[kMaxDevices] = {};
+
+// The calling thread's current context (the device's primary context for
+// runtime-API callers), through the driver entry point the runtime exposes.
+CUcontext current_context() {
+  static PFN_cuCtxGetCurrent_v4000 fn = nullptr;
+  static bool looked = false;
+  if (!looked) {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f, 4000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(f);
+    looked = true;
+  }
+  CUcontext c = nullptr;
+  if (fn != nullptr && fn(&c) != CUDA_SUCCESS) c = nullptr;
+  return c;
+}
 
 cudaError_t scratch_address(int dev, char** out) {
   std::lock_guard<std::mutex> lock(g_scratch_mu);
-  if (g_scratch_addr[dev] == nullptr) {
+  // the pointer checks before this made the device's context current
+  const CUcontext ctx = current_context();
+  ScratchSlot& sl = g_scratch[dev];
+  if (sl.addr == nullptr || ctx == nullptr || sl.ctx != ctx) {   // no context handle: look up every call
     void* p = nullptr;
     cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
     if (e != cudaSuccess) return e;
-    g_scratch_addr[dev] = static_cast<char*>(p);
+    sl.addr = static_cast<char*>(p);
+    sl.ctx = ctx;
   }
-  *out = g_scratch_addr[dev];
+  *out = sl.addr;
   return cudaSuccess;
 }
 
@@ -249,6 +279,7 @@ extern "C" lm_status lm_msign_ns_noalloc(const lm_tensor* in, lm_tensor* out, in
   memset(&mk, 0, sizeof(mk));
   mk.eps = (float)eps;
   mk.ns_steps = steps;
+  mk.flags = ba.d_flags;
   e = launch_momentum_norm(xdt, in->dtype, ba.d_mat, ba.d_chunks, n_et, nullptr, mk, 1, stream);
   if (e != cudaSuccess) return set_error(LM_ERR_CUDA, cudaGetErrorString(e));
   const NsCoeffs co{(float)a, (float)b, (float)c, (float)eps};
@@ -256,13 +287,33 @@ extern "C" lm_status lm_msign_ns_noalloc(const lm_tensor* in, lm_tensor* out, in
     for (int ph = 0; ph < 3; ++ph) {
       if (xdt == LM_BF16)
         e = launch_ns_tc((NsPhase)ph, it, 1, &g, &maps, ba.d_tiles[ph], ntiles[ph], nullptr, 0,
-                         d.norm2, co, ba.d_flags, nullptr, stream);
+                         d.norm2, co, ba.d_flags, nullptr, stream, nullptr, nullptr, 1, 0, false, false,
+                         env_wait_limit_ns());
       else
         e = launch_ns_simt((NsPhase)ph, it, 1, ba.d_group, ba.d_tiles[ph], ntiles[ph], d.norm2, co,
-                           stream);
+                           stream, nullptr, nullptr, ba.d_flags);
       if (e != cudaSuccess) return set_error(LM_ERR_CUDA, cudaGetErrorString(e));
     }
   e = launch_finalize(xdt, out->dtype, ba.d_mat, ba.d_chunks, n_et, mk, 1, ba.d_flags, stream);
   if (e != cudaSuccess) return set_error(LM_ERR_CUDA, cudaGetErrorString(e));
+  return LM_OK;
+}
+
+extern "C" lm_status lm_msign_ns_noalloc_status(uint32_t* device_flags, void* cuda_stream) {
+  if (device_flags == nullptr) return set_error(LM_ERR_INVALID_ARG, "device_flags is NULL");
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return set_error(LM_ERR_CUDA, "no CUDA device");
+  if (dev >= kMaxDevices) return set_error(LM_ERR_UNSUPPORTED, "device ordinal above 63");
+  char* base = nullptr;
+  cudaError_t e = scratch_address(dev, &base);
+  if (e != cudaSuccess) return set_error(LM_ERR_CUDA, cudaGetErrorString(e));
+  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+  unsigned h = 0;   // the status word sits at offset 0 of every call's layout
+  e = cudaStreamSynchronize(stream);
+  if (e == cudaSuccess) e = cudaMemcpy(&h, base, sizeof(unsigned), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return set_error(LM_ERR_CUDA, cudaGetErrorString(e));
+  *device_flags = h;
+  if (h & LM_FLAG_TIMEOUT)
+    return set_error(LM_ERR_TIMEOUT, "a bounded device wait of the last lm_msign_ns_noalloc call gave up");
   return LM_OK;
 }

@@ -61,7 +61,9 @@ __device__ __forceinline__ void store_slice(float (*S)[BM + kPadS], const SliceR
 __global__ void __launch_bounds__(kThreads, 2)   // two blocks per SM: at most 128 registers
     ns_simt_kernel(int phase, int iter, const NsGroup* __restrict__ groups,
                    const NsTile* __restrict__ tiles, int ntiles, const double* __restrict__ norm2,
-                   NsCoeffs co, const unsigned char* __restrict__ active, float* __restrict__ split_ws) {
+                   NsCoeffs co, const unsigned char* __restrict__ active, float* __restrict__ split_ws,
+                   const unsigned* flags) {
+  if (lm_stopped(flags)) return;
   __shared__ __align__(16) float As[2][BK][BM + kPadS];
   __shared__ __align__(16) float Bs[2][BK][BN + kPadS];
   const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
@@ -182,7 +184,7 @@ int simt_pad(int x) { return (x + BM - 1) / BM * BM; }
 
 cudaError_t launch_ns_simt(NsPhase ph, int iter, int ngroups, const NsGroup* dgroups,
                            const NsTile* tiles, int ntiles, const double* norm2, NsCoeffs co,
-                           cudaStream_t st, const unsigned char* active, float* split_ws) {
+                           cudaStream_t st, const unsigned char* active, float* split_ws, const unsigned* flags) {
   (void)ngroups;
   if (ntiles <= 0) return cudaSuccess;
   int dev = 0, sms = 0;
@@ -192,7 +194,7 @@ cudaError_t launch_ns_simt(NsPhase ph, int iter, int ngroups, const NsGroup* dgr
   if (grid > ntiles) grid = ntiles;
   count_launch();
   ns_simt_kernel<<<grid, kThreads, 0, st>>>((int)ph, iter, dgroups, tiles, ntiles, norm2, co, active,
-                                            split_ws);
+                                            split_ws, flags);
   return cudaGetLastError();
 }
 
@@ -200,7 +202,9 @@ namespace {
 // fp32 A from the parts of split Gram tiles, summed in part order; the tile
 // and its mirror (a diagonal tile: its upper triangle and the mirror of it).
 __global__ void __launch_bounds__(256) ns_split_finish_f32_kernel(const NsSplitTarget* __restrict__ targets,
-                                                                  const float* __restrict__ ws) {
+                                                                  const float* __restrict__ ws,
+                                                                  const unsigned* flags) {
+  if (lm_stopped(flags)) return;
   const NsSplitTarget T = targets[blockIdx.y];
   float* dst = static_cast<float*>(T.a_tile);
   float* mir = static_cast<float*>(T.a_mirror);
@@ -215,10 +219,11 @@ __global__ void __launch_bounds__(256) ns_split_finish_f32_kernel(const NsSplitT
 }
 }  // namespace
 
-cudaError_t launch_ns_split_finish_f32(const NsSplitTarget* targets, int n, const float* ws, cudaStream_t st) {
+cudaError_t launch_ns_split_finish_f32(const NsSplitTarget* targets, int n, const float* ws, const unsigned* flags,
+                                       cudaStream_t st) {
   if (n <= 0) return cudaSuccess;
   count_launch();
-  ns_split_finish_f32_kernel<<<dim3(16, n), 256, 0, st>>>(targets, ws);
+  ns_split_finish_f32_kernel<<<dim3(16, n), 256, 0, st>>>(targets, ws, flags);
   return cudaGetLastError();
 }
 

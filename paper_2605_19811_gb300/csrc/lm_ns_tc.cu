@@ -46,24 +46,17 @@
 #include <cuda_bf16.h>
 #include <cudaTypedefs.h>
 
-#include "lm_internal.h"
+#include "lm_ns_tc_shared.cuh"
 
 namespace lm {
 namespace {
 
-constexpr int BM = kTcBM, BN = kTcBN, BK = kTcBK;   // pair tile 256 x 256, K step 64
-constexpr int kHalf = 128;                           // A rows / B N-rows per CTA
-constexpr int kABytes = kHalf * BK * 2;              // 16 KB
-constexpr int kBBytes = kHalf * BK * 2;              // 16 KB
-static_assert(kABytes == kBBytes, "diagonal tiles read their A boxes as B");
-constexpr int kEpiWarps = 8;
-constexpr int kAuxWarp = 2 + kEpiWarps;              // warp that loads the epilogue's aux tile
-constexpr int kThreads = 32 * (3 + kEpiWarps);
-constexpr int kAccBufs = 2;                          // accumulators in TMEM
+using namespace tc;    // PTX wrappers (lm_tc_ptx.cuh)
+using namespace tcs;   // constants, stop check and end-of-launch handshake (lm_ns_tc_shared.cuh)
+
+constexpr int kAccBufs = 2;                          // 256-column accumulators in TMEM
 constexpr int kFuseBatch = 4;   // W loads in flight per thread in the fused parameter write
 constexpr int kTmemCols = kAccBufs * BN;
-constexpr uint64_t kWaitLimitNs = 5000000000ull;     // 5 s
-constexpr int kAuxBoxBytes = kHalf * 64 * 2;         // one 64-column box of the CTA's rows: 16 KB
 // Shared-memory layout per operand precision.  kP = 1: bf16 operands, a
 // 5-stage ring of 32 KB per CTA and a 64 KB aux/staging buffer.  kP = 3:
 // fp32 operands held as three bf16 pieces (hi + mid + lo, exact), a 2-stage
@@ -78,229 +71,6 @@ struct TcLayout {
   static constexpr size_t kBarOffset = kAuxOffset + (kP == 1 ? 4 * kAuxBoxBytes : 8 * 32 * 33 * 4);
   static constexpr size_t kSmemBytes = 1024 /*align slack*/ + kBarOffset + 256;
 };
-
-struct TcParams {
-  TcGroupMaps maps[kMaxGroupsTc];
-  NsGroup groups[kMaxGroupsTc];
-  const NsTile* tiles;
-  const int* offsets;   // tiles of pair k: [offsets[k], offsets[k+1]); NULL: round robin
-  int ntiles;
-  int phase;
-  int iter;
-  const double* norm2;
-  NsCoeffs co;
-  unsigned* flags;
-  FuseFinal fuse;       // fuse.mats != NULL: this APPLY writes the parameters
-  const unsigned char* active;   // NULL, or per matrix: 0 = skip its tiles
-  float* split_ws;               // fp32 workspace of split Gram tiles (256 x 256 each)
-  int final_f32;                 // three-piece operands: this APPLY writes fp32 X to NsGroup::Xf
-};
-
-// Whether a tile's matrix runs in this launch; every role asks the same
-// question of the same tiles, so skipping keeps their pipelines in step.
-__device__ __forceinline__ bool tile_active(const TcParams& p, const NsTile& t) {
-  return p.active == nullptr || p.active[p.groups[t.group].first_mat + t.mat] != 0;
-}
-
-// ------------------------------- PTX wrappers -------------------------------
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-__device__ __forceinline__ uint64_t globaltimer() {
-  uint64_t t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
-}
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
-}
-__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
-               "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(smem_u32(bar)), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-// Bounded wait for the phase with the given parity.  Returns false if the
-// time limit passed or another role asked to stop.  The first probe is
-// inlined; the slow path is a call.
-__device__ __noinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                            uint64_t limit_ns) {
-  const uint64_t t0 = globaltimer();
-  for (uint32_t i = 1;; ++i) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if ((i & 255u) == 0) {
-      if (*abort_flag) return false;
-      if (globaltimer() - t0 > limit_ns) return false;
-    }
-  }
-}
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                          uint64_t limit_ns) {
-  if (mbar_try_wait(bar, parity)) return true;
-  return mbar_wait_slow(bar, parity, abort_flag, limit_ns);
-}
-// 3-D tiled TMA load into this CTA's shared memory; completion is signalled
-// on the mbarrier at shared::cluster address bar_cluster (either CTA of the pair).
-__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, uint32_t bar_cluster,
-                                            int c0, int c1, int c2) {
-  asm volatile(
-      "cp.async.bulk.tensor.3d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(smem_u32(dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(c0), "r"(c1), "r"(c2)
-      : "memory");
-}
-// 4-D tiled TMA load, signalled like tma_load_3d, for the MN-major operand
-// maps with dimensions (64 MN, K, MN / 64, matrix): one copy fills the two
-// 64-wide swizzle atoms of a 128-wide operand half.
-__device__ __forceinline__ void tma_load_4d(void* dst, const CUtensorMap* map, uint32_t bar_cluster,
-                                            int c0, int c1, int c2, int c3) {
-  asm volatile(
-      "cp.async.bulk.tensor.4d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%3, %4, %5, %6}], [%2];" ::"r"(smem_u32(dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
-      : "memory");
-}
-// 3-D tiled TMA load signalling this CTA's own mbarrier.
-__device__ __forceinline__ void tma_load_3d_local(void* dst, const CUtensorMap* map, uint64_t* bar,
-                                                  int c0, int c1, int c2) {
-  asm volatile(
-      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(smem_u32(dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "r"(c2)
-      : "memory");
-}
-// 3-D tiled TMA store from this CTA's shared memory (bulk-group completion).
-__device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, const void* src, int c0, int c1,
-                                             int c2) {
-  asm volatile(
-      "cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
-          reinterpret_cast<uint64_t>(map)),
-      "r"(smem_u32(src)), "r"(c0), "r"(c1), "r"(c2)
-      : "memory");
-}
-__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
-__device__ __forceinline__ void bulk_wait_read() {
-  asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
-}
-__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
-// Make this thread's generic-proxy shared-memory writes visible to the TMA.
-__device__ __forceinline__ void fence_proxy_async_smem() {
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
-__device__ __forceinline__ uint32_t cluster_rank() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-  return r;
-}
-// shared::cluster address of the same shared variable in CTA `rank`
-__device__ __forceinline__ uint32_t peer_addr(const void* p, uint32_t rank) {
-  uint32_t r;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_u32(p)), "r"(rank));
-  return r;
-}
-__device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar_cluster) {
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster)
-               : "memory");
-}
-__device__ __forceinline__ void cluster_sync() {
-  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::
-                   : "memory");
-}
-__device__ __forceinline__ void tc_fence_before() {
-  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void tc_fence_after() {
-  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void tmem_alloc(uint32_t* dst, uint32_t ncols) {
-  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                   smem_u32(dst)),
-               "r"(ncols)
-               : "memory");
-}
-__device__ __forceinline__ void tmem_relinquish() {
-  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
-}
-__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
-  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
-               : "memory");
-}
-__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
-                                          uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-// Arrive on the barrier at the same shared-memory offset in both CTAs of the
-// pair once all previously issued MMAs of this thread have completed.
-__device__ __forceinline__ void umma_commit_pair(uint64_t* bar) {
-  asm volatile(
-      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
-      " [%0], %1;" ::"r"(smem_u32(bar)), "h"((uint16_t)0x3)
-      : "memory");
-}
-__device__ __forceinline__ void umma_commit_local(uint64_t* bar) {
-  asm volatile(
-      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-          smem_u32(bar))
-      : "memory");
-}
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32"
-      " {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15,"
-      " %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31},"
-      " [%32];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
-        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
-        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
-        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-}
-
-// Shared-memory matrix descriptor (tcgen05), 128-byte swizzle.
-//   bits 0-13  start address >> 4
-//   bits 16-29 leading-dimension byte offset >> 4
-//   bits 32-45 stride-dimension byte offset >> 4
-//   bits 46-47 descriptor version (1)
-//   bits 61-63 layout: 2 = 128-byte swizzle
-// K-major: rows of 128 B (64 bf16 of K), 8-row groups 1024 B apart (SBO);
-//          LBO unused.  MN-major: 64 MN-elements per 128-B row, one row per K,
-//          8-K-row groups 1024 B apart (SBO), 64-element MN atoms LBO apart.
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
-  uint64_t d = 0;
-  d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
-  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
-  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
-  d |= (uint64_t)1 << 46;
-  d |= (uint64_t)2 << 61;
-  return d;
-}
-// Instruction descriptor, kind::f16: D fp32, A and B bf16, A K-major,
-// B K-major or MN-major, N >> 3 at bit 17, M >> 4 at bit 24 (M = 256 for a
-// CTA pair).
-__host__ __device__ constexpr uint32_t make_idesc(int m, int n, bool a_mn_major, bool b_mn_major) {
-  return (1u << 4) | (1u << 7) | (1u << 10) | ((a_mn_major ? 1u : 0u) << 15) |
-         ((b_mn_major ? 1u : 0u) << 16) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
-}
 
 // Operands of one tile.  Wide groups hold X as s x l, tall groups as l x s
 // (the parameter's own orientation):
@@ -362,12 +132,6 @@ __device__ __forceinline__ TilePlan tile_plan(int phase, const NsGroup& g, const
   return P;
 }
 
-__device__ __forceinline__ float bf_lo(uint32_t v) { return __uint_as_float(v << 16); }
-__device__ __forceinline__ float bf_hi(uint32_t v) { return __uint_as_float(v & 0xFFFF0000u); }
-__device__ __forceinline__ uint32_t pack_bf2(float lo, float hi) {
-  __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
-  return *reinterpret_cast<uint32_t*>(&h);
-}
 
 // Producer k-loop of one tile, specialised on the operand layouts (a loop
 // with per-block layout branches measured ~12% slower end to end).
@@ -386,19 +150,25 @@ struct ProducerRing {
 // or polynomial tile), so only the A boxes are loaded and the MMA reads them
 // as B too.
 template <bool AMN, bool BMN, int kP>
-__device__ __forceinline__ bool produce_range(ProducerRing<TcLayout<kP>::kStages>& R, uint8_t* smem,
+__device__ __forceinline__ bool produce_range(ProducerRing<TcLayout<kP>::kStages>& R,
+                                              ProducerLog<TcLayout<kP>::kStages>& log, uint8_t* smem,
                                               uint64_t* full, uint64_t* empty, volatile int* abort_flag,
-                                              uint32_t rank, int kb0, int kb1, const CUtensorMap* map_a,
-                                              const CUtensorMap* map_b, int row_a, int col_b, int mat,
-                                              int pstride, bool same) {
+                                              uint64_t wait_ns, uint32_t rank, int kb0, int kb1,
+                                              const CUtensorMap* map_a, const CUtensorMap* map_b, int row_a,
+                                              int col_b, int mat, int pstride, bool same) {
   using L = TcLayout<kP>;
+  const uint32_t own = same ? (uint32_t)(kP * kABytes) : (uint32_t)L::kStageBytes;   // this CTA's bytes
   for (int kb = kb0; kb < kb1; ++kb) {
-    if (!mbar_wait(&empty[R.stage], R.ph ^ 1u, abort_flag, kWaitLimitNs)) return false;
+    if (!mbar_wait(&empty[R.stage], R.ph ^ 1u, abort_flag, wait_ns)) return false;
     uint8_t* sa = smem + (size_t)R.stage * L::kStageBytes;
     uint8_t* sb = sa + kP * kABytes;
     const uint32_t fb = peer_addr(&full[R.stage], 0);
-    if (rank == 0) mbar_arrive_expect_tx(&full[R.stage], same ? 2 * kP * kABytes : 2 * L::kStageBytes);
-    R.armed[R.stage] = (int)R.ph;
+    if (rank == 0) {
+      mbar_arrive_expect_tx(&full[R.stage], 2u * own);
+      R.armed[R.stage] = (int)R.ph;
+    }
+    log.bytes[R.stage] = own;
+    log.n += 1u;
     const int k0 = kb * BK;
 #pragma unroll
     for (int q = 0; q < kP; ++q) {
@@ -422,17 +192,24 @@ __device__ __forceinline__ bool produce_range(ProducerRing<TcLayout<kP>::kStages
 // kP = 3: with A = A0 + A1 + A2 and B = B0 + B1 + B2 (each piece 2^-8 of the
 // previous in magnitude) the six products of order up to 2^-16 are summed,
 // A0B0 + A0B1 + A1B0 + A0B2 + A2B0 + A1B1; the dropped ones are of order 2^-24.
+// A0B0 goes into the accumulator d_tmem and the five smaller products into
+// d_cross; the epilogue adds the two in fp32.  The tensor cores' fp32
+// accumulation loses about one unit of the last place of the accumulator per
+// MMA, in the same direction (measured: the error grows with the number of
+// MMAs summed, 2.2e-5 relative for a 1280-deep product with all six in one
+// accumulator), so the large accumulator takes a sixth of the additions and
+// the errors of the other are 2^-8 smaller.
 template <bool AMN, bool BMN, int kP>
 __device__ __forceinline__ bool mma_range(int& stage, uint32_t& ph, uint8_t* smem, uint64_t* full,
-                                          uint64_t* empty, volatile int* abort_flag, int kb0, int kb1,
-                                          uint32_t d_tmem, int kb_first, bool same) {
+                                          uint64_t* empty, volatile int* abort_flag, uint64_t wait_ns, int kb0,
+                                          int kb1, uint32_t d_tmem, uint32_t d_cross, int kb_first, bool same) {
   using L = TcLayout<kP>;
   constexpr int kProducts = kP == 1 ? 1 : 6;
   constexpr int qa[6] = {0, 0, 1, 0, 2, 1};
   constexpr int qb[6] = {0, 1, 0, 2, 0, 1};
   const uint32_t idesc = make_idesc(BM, BN, AMN, BMN);
   for (int kb = kb0; kb < kb1; ++kb) {
-    if (!mbar_wait(&full[stage], ph, abort_flag, kWaitLimitNs)) return false;
+    if (!mbar_wait(&full[stage], ph, abort_flag, wait_ns)) return false;
     tc_fence_after();
     const uint32_t sa = smem_u32(smem + (size_t)stage * L::kStageBytes);
     const uint32_t sb = same ? sa : sa + kP * kABytes;   // kBBytes == kABytes
@@ -443,7 +220,8 @@ __device__ __forceinline__ bool mma_range(int& stage, uint32_t& ph, uint8_t* sme
         const uint32_t pa = sa + qa[m] * kABytes, pb = sb + qb[m] * kBBytes;
         const uint64_t adesc = AMN ? sw128_desc(pa + kk * 2048, 64 * BK * 2, 1024) : sw128_desc(pa + kk * 32, 16, 1024);
         const uint64_t bdesc = BMN ? sw128_desc(pb + kk * 2048, 64 * BK * 2, 1024) : sw128_desc(pb + kk * 32, 16, 1024);
-        umma_bf16(d_tmem, adesc, bdesc, idesc, (kb != kb_first || kk != 0 || m != 0) ? 1u : 0u);
+        const bool first = kb == kb_first && kk == 0 && m <= 1;   // first product into each accumulator
+        umma_bf16(m == 0 ? d_tmem : d_cross, adesc, bdesc, idesc, first ? 0u : 1u);
       }
     }
     umma_commit_pair(&empty[stage]);
@@ -552,6 +330,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     ns_tc_kernel(const __grid_constant__ TcParams p) {
   using L = TcLayout<kP>;
   constexpr int kStages = L::kStages;
+  // tiles in flight in TMEM: kP = 1 double-buffers two accumulators; kP = 3
+  // gives one tile both (main and cross products)
+  constexpr int kAccRing = kP == 1 ? kAccBufs : 1;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -563,8 +344,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   uint64_t* aux_full = accempty + 2;
   uint64_t* aux_empty = aux_full + 1;
   uint64_t* done = aux_empty + 1;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+  ProducerLog<kStages>* log = reinterpret_cast<ProducerLog<kStages>*>(done + 1);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(log + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  uint32_t* stop_word = tmem_slot + 2;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int phase = p.phase;
@@ -573,7 +356,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
   const bool aux_phase = kP == 1 && phase != NS_GRAM;   // epilogue reads the A (POLY) or X (APPLY) tile
   // this pair's tiles: a host-balanced range, or round robin
-  const int w_begin = p.offsets ? p.offsets[pair] : pair;
+  int w_begin = p.offsets ? p.offsets[pair] : pair;
   const int w_end = p.offsets ? p.offsets[pair + 1] : p.ntiles;
   const int w_step = p.offsets ? 1 : npairs;
 
@@ -581,11 +364,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     // A pair none of whose tiles belongs to a selected matrix leaves before
     // any barrier, TMEM or cluster work (the roles would otherwise walk its
     // tile list one dependent load chain at a time).  Both CTAs of the pair
-    // scan the same range of the same mask, so both leave or both stay.
+    // scan the same range of the same mask, so both leave or both stay.  The
+    // mask comes from a kernel this launch may overlap: wait for it first.
+    griddep_wait();
     int any = 0;
     for (int w = w_begin + (int)threadIdx.x * w_step; !any && w < w_end; w += (int)blockDim.x * w_step)
       any = tile_active(p, p.tiles[w]) ? 1 : 0;
-    if (!__syncthreads_or(any)) return;
+    if (!__syncthreads_or(any)) {
+      griddep_launch_dependents();
+      return;
+    }
   }
 
   if (threadIdx.x == 0) {
@@ -600,6 +388,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     mbar_init(aux_full, 1);
     mbar_init(aux_empty, kEpiWarps);
     mbar_init(done, 1);
+    log->n = 0;
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -607,23 +396,23 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     tmem_alloc(tmem_slot, kTmemCols);
     tmem_relinquish();
   }
-  tc_fence_before();
-  cluster_sync();     // barriers of both CTAs initialised before any remote use
-  tc_fence_after();
+  if (pair_start(p, stop_word, rank)) w_begin = w_end;   // an earlier launch gave up: no tiles
   const uint32_t tmem_base = *tmem_slot;
+  const uint64_t wait_ns = p.wait_ns;
 
   auto give_up = [&]() {
     *abort_flag = 1;
     atomicOr(p.flags, LM_FLAG_TIMEOUT);
   };
 
+  ProducerRing<kStages> R;   // producer lane: ring position and armed phases
+  R.stage = 0;
+  R.ph = 0;
+  for (int s = 0; s < kStages; ++s) R.armed[s] = -1;
+
   if (warp == 0) {
     // ------------------------------ producer ------------------------------
     if (lane == 0) {
-      ProducerRing<kStages> R;
-      R.stage = 0;
-      R.ph = 0;
-      for (int s = 0; s < kStages; ++s) R.armed[s] = -1;
       bool ok = true;
       for (int w = w_begin; ok && w < w_end; w += w_step) {
         const NsTile t = p.tiles[w];
@@ -636,28 +425,20 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         for (int sg = 0; ok && sg < P.nseg; ++sg) {
           const OpSeg& S = P.seg[sg];
           if (!S.a_mn && !S.b_mn)
-            ok = produce_range<false, false, kP>(R, smem, full, empty, abort_flag, rank, kb0, S.kb_end, S.map_a,
+            ok = produce_range<false, false, kP>(R, *log, smem, full, empty, abort_flag, wait_ns, rank, kb0, S.kb_end, S.map_a,
                                              S.map_b, row_a, col_b, t.mat, g.count,
                                              S.map_a == S.map_b && row_a == col_b);
           else if (!S.a_mn)
-            ok = produce_range<false, true, kP>(R, smem, full, empty, abort_flag, rank, kb0, S.kb_end, S.map_a,
+            ok = produce_range<false, true, kP>(R, *log, smem, full, empty, abort_flag, wait_ns, rank, kb0, S.kb_end, S.map_a,
                                             S.map_b, row_a, col_b, t.mat, g.count,
                                              S.map_a == S.map_b && row_a == col_b);
           else
-            ok = produce_range<true, true, kP>(R, smem, full, empty, abort_flag, rank, kb0, S.kb_end, S.map_a,
+            ok = produce_range<true, true, kP>(R, *log, smem, full, empty, abort_flag, wait_ns, rank, kb0, S.kb_end, S.map_a,
                                            S.map_b, row_a, col_b, t.mat, g.count,
                                              S.map_a == S.map_b && row_a == col_b);
           kb0 = S.kb_end;
         }
         if (!ok) give_up();
-      }
-      if (!ok && rank == 0) {
-        // let the copies already issued land before the CTA exits
-        for (int s = 0; s < kStages; ++s)
-          if (R.armed[s] >= 0) {
-            volatile int never = 0;
-            mbar_wait(&full[s], (uint32_t)R.armed[s], &never, 100000000ull);
-          }
       }
     }
   } else if (warp == 1) {
@@ -673,30 +454,33 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         if (kMasked && !tile_active(p, t)) continue;
         const NsGroup& g = p.groups[t.group];
         const TilePlan P = tile_plan(phase, g, p.maps[t.group], cur, t);
-        if (!mbar_wait(&accempty[ab], aph ^ 1u, abort_flag, kWaitLimitNs)) {
+        if (!mbar_wait(&accempty[ab], aph ^ 1u, abort_flag, wait_ns)) {
           give_up();
           break;
         }
         tc_fence_after();
+        // kP = 1: accumulator ab; kP = 3: the main products in the first 256
+        // columns, the cross products in the second
         const uint32_t d_tmem = tmem_base + (uint32_t)(ab * BN);
+        const uint32_t d_cross = tmem_base + (uint32_t)BN;
         int kb0 = P.kb_start;
         for (int sg = 0; ok && sg < P.nseg; ++sg) {
           const OpSeg& S = P.seg[sg];
           if (!S.a_mn && !S.b_mn)
-            ok = mma_range<false, false, kP>(stage, ph, smem, full, empty, abort_flag, kb0, S.kb_end, d_tmem,
+            ok = mma_range<false, false, kP>(stage, ph, smem, full, empty, abort_flag, wait_ns, kb0, S.kb_end, d_tmem, d_cross,
                                             P.kb_start, S.map_a == S.map_b && t.tm == t.tn);
           else if (!S.a_mn)
-            ok = mma_range<false, true, kP>(stage, ph, smem, full, empty, abort_flag, kb0, S.kb_end, d_tmem,
+            ok = mma_range<false, true, kP>(stage, ph, smem, full, empty, abort_flag, wait_ns, kb0, S.kb_end, d_tmem, d_cross,
                                             P.kb_start, S.map_a == S.map_b && t.tm == t.tn);
           else
-            ok = mma_range<true, true, kP>(stage, ph, smem, full, empty, abort_flag, kb0, S.kb_end, d_tmem,
+            ok = mma_range<true, true, kP>(stage, ph, smem, full, empty, abort_flag, wait_ns, kb0, S.kb_end, d_tmem, d_cross,
                                             P.kb_start, S.map_a == S.map_b && t.tm == t.tn);
           kb0 = S.kb_end;
         }
         if (!ok) give_up();
         if (!ok) break;
         umma_commit_pair(&accfull[ab]);
-        if (++ab == kAccBufs) {
+        if (++ab == kAccRing) {
           ab = 0;
           aph ^= 1u;
         }
@@ -704,7 +488,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       // all issued MMAs complete before TMEM is released
       umma_commit_local(done);
       volatile int never = 0;
-      mbar_wait(done, 0, &never, 100000000ull);
+      mbar_wait(done, 0, &never, kCleanupWaitNs);
     }
   } else if (warp == kAuxWarp) {
     // --------------------------- aux tile loader ---------------------------
@@ -719,7 +503,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         if (kMasked && !tile_active(p, t)) continue;
         const TcGroupMaps& mp = p.maps[t.group];
         const CUtensorMap* map = (phase == NS_POLY) ? &mp.a : &mp.xk[cur];
-        if (!mbar_wait(aux_empty, xph ^ 1u, abort_flag, kWaitLimitNs)) {
+        if (!mbar_wait(aux_empty, xph ^ 1u, abort_flag, wait_ns)) {
           give_up();
           ok = false;
           break;
@@ -734,7 +518,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       }
       if (!ok && armed >= 0) {
         volatile int never = 0;
-        mbar_wait(aux_full, (uint32_t)armed, &never, 100000000ull);
+        mbar_wait(aux_full, (uint32_t)armed, &never, kCleanupWaitNs);
       }
     }
   } else {
@@ -747,7 +531,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     const int half = (warp - 2) >> 2;         // which 128 columns of the tile
     const int row = q * 32 + lane;            // row of this CTA's half tile
     const uint32_t acc_empty0 = peer_addr(&accempty[0], 0);
-    const uint32_t acc_empty1 = peer_addr(&accempty[kAccBufs - 1], 0);
+    const uint32_t acc_empty1 = peer_addr(&accempty[kAccRing - 1], 0);
     int ab = 0;
     uint32_t aph = 0, xph = 0;
     for (int w = w_begin; w < w_end; w += w_step) {
@@ -756,10 +540,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const NsGroup& g = p.groups[t.group];
       const bool fused = phase == NS_APPLY && p.fuse.mats != nullptr;
       const MatDesc* fd = fused ? &p.fuse.mats[g.first_mat + t.mat] : nullptr;
+      // a tile whose epilogue starts after a give-up was recorded leaves W alone
+      const unsigned flags_now = fused && lane == 0 ? *reinterpret_cast<volatile unsigned*>(p.flags) : 0u;
+      const bool write_w = fused && __shfl_sync(0xffffffffu, flags_now, 0) == 0u;
       bool ok = true;
       if (lane == 0) {
-        ok = mbar_wait(&accfull[ab], aph, abort_flag, kWaitLimitNs);
-        if (ok && aux_phase) ok = mbar_wait(aux_full, xph, abort_flag, kWaitLimitNs);
+        ok = mbar_wait(&accfull[ab], aph, abort_flag, wait_ns);
+        if (ok && aux_phase) ok = mbar_wait(aux_full, xph, abort_flag, wait_ns);
       }
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
       if (!ok) {
@@ -791,6 +578,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         uint32_t r[32];
         __syncwarp();   // tcgen05.ld is warp-collective: reconverge first
         tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * BN + ch * 32), r);
+        if (kP == 3) {   // main + cross accumulators
+          uint32_t rc[32];
+          tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(BN + ch * 32), rc);
+#pragma unroll
+          for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) + __uint_as_float(rc[e]));
+        }
         const int j0 = t.tn * BN + ch * 32;
         if (!warp_in || j0 >= jmax) continue;   // beyond the padded matrix
         if (kP == 3 && !split) {
@@ -857,7 +650,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_cluster(ab == 0 ? acc_empty0 : acc_empty1);
-      if (++ab == kAccBufs) {
+      if (++ab == kAccRing) {
         ab = 0;
         aph ^= 1u;
       }
@@ -868,7 +661,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         // Last APPLY: W <- W - eta_M (s X_K + lambda W), with X_K the bf16
         // values just written to auxbuf.  Half-warp h covers row 2k + h of the
         // warp's 32 rows, 16 lanes x 8 columns = 256 contiguous bytes of W.
-        if (warp_in) {
+        if (warp_in && write_w) {
           const int cc = lane & 15;
           const int jc = t.tn * BN + half * 128 + cc * 8;
           const unsigned char* box = auxbuf + (2 * half + (cc >> 3)) * kAuxBoxBytes;
@@ -924,8 +717,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   }
 
   __syncwarp();
-  tc_fence_before();
-  cluster_sync();     // neither CTA leaves while its peer may still signal it
+  pair_finish<kStages>(*log, abort_flag, full, R.armed, rank);
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem_base, kTmemCols);
@@ -935,7 +727,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 // Split Gram tiles: bf16 A tile = the sum of the fp32 parts (already scaled),
 // added in part order.
 __global__ void __launch_bounds__(256) ns_split_finish_kernel(const NsSplitTarget* __restrict__ targets,
-                                                              const float* __restrict__ ws) {
+                                                              const float* __restrict__ ws, const unsigned* flags) {
+  asm volatile("griddepcontrol.wait;" ::: "memory");   // the Gram launch before it may be programmatic
+  if (lm_stopped(flags)) return;
   const NsSplitTarget T = targets[blockIdx.y];
   __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(T.a_tile);
   for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < BM * BN; e += gridDim.x * blockDim.x) {
@@ -1046,7 +840,8 @@ cudaError_t tc_encode_group_maps(const NsGroup& g, TcGroupMaps* maps, int pieces
 
 namespace {
 __global__ void __launch_bounds__(256) split3_kernel(const float4* __restrict__ src, uint2* __restrict__ dst,
-                                                     size_t n4) {
+                                                     size_t n4, const unsigned* flags) {
+  if (lm_stopped(flags)) return;
   for (size_t k = blockIdx.x * (size_t)blockDim.x + threadIdx.x; k < n4; k += (size_t)gridDim.x * blockDim.x) {
     const float4 v = src[k];
     float h[4], m[4], l[4];
@@ -1061,7 +856,7 @@ __global__ void __launch_bounds__(256) split3_kernel(const float4* __restrict__ 
 }
 }  // namespace
 
-cudaError_t launch_split3(const float* src, void* dst, size_t n, cudaStream_t st) {
+cudaError_t launch_split3(const float* src, void* dst, size_t n, const unsigned* flags, cudaStream_t st) {
   if (n == 0) return cudaSuccess;
   if (n % 4 != 0) return cudaErrorInvalidValue;
   int dev = 0, sms = 0;
@@ -1071,14 +866,15 @@ cudaError_t launch_split3(const float* src, void* dst, size_t n, cudaStream_t st
   size_t grid = (n4 + 255) / 256;
   if (grid > (size_t)sms * 8) grid = (size_t)sms * 8;
   count_launch();
-  split3_kernel<<<(unsigned)grid, 256, 0, st>>>(reinterpret_cast<const float4*>(src), static_cast<uint2*>(dst), n4);
+  split3_kernel<<<(unsigned)grid, 256, 0, st>>>(reinterpret_cast<const float4*>(src), static_cast<uint2*>(dst), n4, flags);
   return cudaGetLastError();
 }
 
-cudaError_t launch_ns_split_finish(const NsSplitTarget* targets, int n, const float* ws, cudaStream_t st) {
+cudaError_t launch_ns_split_finish(const NsSplitTarget* targets, int n, const float* ws, const unsigned* flags,
+                                   cudaStream_t st) {
   if (n <= 0) return cudaSuccess;
   count_launch();
-  ns_split_finish_kernel<<<dim3(32, n), 256, 0, st>>>(targets, ws);
+  ns_split_finish_kernel<<<dim3(32, n), 256, 0, st>>>(targets, ws, flags);
   return cudaGetLastError();
 }
 
@@ -1099,11 +895,13 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
                          const TcGroupMaps* maps, const NsTile* tiles, int ntiles,
                          const int* offsets, int npairs, const double* norm2, NsCoeffs co,
                          unsigned* flags, const FuseFinal* fuse, cudaStream_t st,
-                         const unsigned char* active, float* split_ws, int pieces, int final_f32) {
+                         const unsigned char* active, float* split_ws, int pieces, int final_f32, bool wide,
+                         bool pdl, uint64_t wait_ns) {
   if (ntiles <= 0) return cudaSuccess;
   if (ngroups < 1 || ngroups > kMaxGroupsTc) return cudaErrorInvalidValue;
   if (pieces != 1 && pieces != 3) return cudaErrorInvalidValue;
-  if (pieces == 3 && fuse != nullptr) return cudaErrorInvalidValue;
+  if (pieces == 3 && (fuse != nullptr || wide)) return cudaErrorInvalidValue;
+  if (wait_ns == 0) return cudaErrorInvalidValue;
   static bool attr_set[kMaxDevices] = {};
   const int slot = device_slot();
   if (slot < 0 || !attr_set[slot]) {
@@ -1136,34 +934,33 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
   prm.active = active;
   prm.split_ws = split_ws;
   prm.final_f32 = (pieces == 3 && ph == NS_APPLY && final_f32) ? 1 : 0;
+  prm.wait_ns = wait_ns;
   int pairs = npairs;
   if (offsets == nullptr) {
     pairs = tc_max_pairs();
     if (pairs > ntiles) pairs = ntiles;
   }
   const int grid = 2 * (pairs > 0 ? pairs : 1);
-  count_launch();
   const bool split = split_ws != nullptr && ph == NS_GRAM;
+  const bool masked = active != nullptr;
+  if (wide) return launch_ns_wide(prm, grid, masked, split, pdl, st);
+  count_launch();
   if (pieces == 3) {
     constexpr size_t sm = TcLayout<3>::kSmemBytes;
-    if (active != nullptr) {
-      if (split) ns_tc_kernel<true, true, 3><<<grid, kThreads, sm, st>>>(prm);
-      else ns_tc_kernel<true, false, 3><<<grid, kThreads, sm, st>>>(prm);
-    } else {
-      if (split) ns_tc_kernel<false, true, 3><<<grid, kThreads, sm, st>>>(prm);
-      else ns_tc_kernel<false, false, 3><<<grid, kThreads, sm, st>>>(prm);
+    if (masked) {
+      if (split) return launch_tc_kernel(ns_tc_kernel<true, true, 3>, grid, sm, pdl, st, prm);
+      return launch_tc_kernel(ns_tc_kernel<true, false, 3>, grid, sm, pdl, st, prm);
     }
-    return cudaGetLastError();
+    if (split) return launch_tc_kernel(ns_tc_kernel<false, true, 3>, grid, sm, pdl, st, prm);
+    return launch_tc_kernel(ns_tc_kernel<false, false, 3>, grid, sm, pdl, st, prm);
   }
   constexpr size_t sm = TcLayout<1>::kSmemBytes;
-  if (active != nullptr) {
-    if (split) ns_tc_kernel<true, true, 1><<<grid, kThreads, sm, st>>>(prm);
-    else ns_tc_kernel<true, false, 1><<<grid, kThreads, sm, st>>>(prm);
-  } else {
-    if (split) ns_tc_kernel<false, true, 1><<<grid, kThreads, sm, st>>>(prm);
-    else ns_tc_kernel<false, false, 1><<<grid, kThreads, sm, st>>>(prm);
+  if (masked) {
+    if (split) return launch_tc_kernel(ns_tc_kernel<true, true, 1>, grid, sm, pdl, st, prm);
+    return launch_tc_kernel(ns_tc_kernel<true, false, 1>, grid, sm, pdl, st, prm);
   }
-  return cudaGetLastError();
+  if (split) return launch_tc_kernel(ns_tc_kernel<false, true, 1>, grid, sm, pdl, st, prm);
+  return launch_tc_kernel(ns_tc_kernel<false, false, 1>, grid, sm, pdl, st, prm);
 }
 
 }  // namespace lm

@@ -214,7 +214,8 @@ __device__ __forceinline__ void row_batch(const float (&m)[RB][S][4], const floa
 template <int S, int TPB, int RB, bool VEC>
 __global__ void __launch_bounds__(TPB)
     srank_pass_kernel(const SrMat* __restrict__ mats, const SrItem* __restrict__ items, int nitems, int pass,
-                      int last) {
+                      int last, const unsigned* flags) {
+  if (lm_stopped(flags)) return;
   constexpr int NW = TPB / 32;
   __shared__ float red[2][RB][NW];
   __shared__ double dred[NW];
@@ -279,7 +280,6 @@ __global__ void __launch_bounds__(TPB)
 
 constexpr int kRingMaxStages = 4;
 constexpr size_t kRingBudget = 104 * 1024;      // ring bytes per block: two blocks per SM
-constexpr uint64_t kRingWaitNs = 2000000000ull;  // 2 s
 
 template <int NC>
 __device__ __forceinline__ double consumer_sum(double x, double* red) {
@@ -302,13 +302,14 @@ __device__ __forceinline__ double consumer_sum(double x, double* red) {
 template <int S, int RB, int NC>
 __global__ void __launch_bounds__(32 * (NC + 1), (S <= 8 ? 2 : 1))
     srank_ring_kernel(const SrMat* __restrict__ mats, const SrItem* __restrict__ items, int nitems, int pass,
-                      int last, int nst, int stride, unsigned* flags) {
+                      int last, int nst, int stride, unsigned* flags, uint64_t wait_ns) {
   extern __shared__ __align__(128) unsigned char ring_raw[];
   float* ring = reinterpret_cast<float*>(ring_raw);
   __shared__ uint64_t full[kRingMaxStages], empty[kRingMaxStages];
   __shared__ float red[2][RB][NC];
   __shared__ double dred[NC];
   __shared__ int stop;
+  if (lm_stopped(flags)) return;   // block-uniform: before any barrier
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (tid == 0) {
     for (int k = 0; k < nst; ++k) {
@@ -333,7 +334,7 @@ __global__ void __launch_bounds__(32 * (NC + 1), (S <= 8 ? 2 : 1))
         const SrItem I = items[it];
         const SrMat& d = mats[I.m];
         for (int r0 = 0; r0 < I.nrows; r0 += RB) {
-          if (!bar_wait(&empty[stage], ph ^ 1u, vstop, kRingWaitNs)) {
+          if (!bar_wait(&empty[stage], ph ^ 1u, vstop, wait_ns)) {
             ok = false;
             break;
           }
@@ -396,7 +397,7 @@ __global__ void __launch_bounds__(32 * (NC + 1), (S <= 8 ? 2 : 1))
     for (int r0 = 0; r0 < I.nrows; r0 += RB) {
       const int n = min(RB, I.nrows - r0);
       bool ok = true;
-      if (lane == 0) ok = bar_wait(&full[stage], ph, vstop, kRingWaitNs);
+      if (lane == 0) ok = bar_wait(&full[stage], ph, vstop, wait_ns);
       ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
       if (!ok && lane == 0) {
         *vstop = 1;
@@ -490,9 +491,10 @@ __global__ void __launch_bounds__(32 * (NC + 1), (S <= 8 ? 2 : 1))
 }
 
 __global__ void srank_decide_kernel(const SrMat* __restrict__ mats, int nmat, double alpha, int last_pass,
-                                    unsigned char* active, unsigned char* skip, double* srank) {
+                                    unsigned char* active, unsigned char* skip, double* srank,
+                                    const unsigned* flags) {
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= nmat) return;
+  if (i >= nmat || lm_stopped(flags)) return;
   const SrMat d = mats[i];
   const double f2 = d.acc[0], s2 = d.acc[1 + last_pass];
   const double smin = (double)(d.rows < d.cols ? d.rows : d.cols);
@@ -504,7 +506,7 @@ __global__ void srank_decide_kernel(const SrMat* __restrict__ mats, int nmat, do
 
 template <int S, int TPB, int RB, bool VEC>
 cudaError_t launch_one(const SrMat* mats, const SrItem* items, int nitems, int pass, bool last,
-                       cudaStream_t st) {
+                       const unsigned* flags, cudaStream_t st) {
   auto kern = srank_pass_kernel<S, TPB, RB, VEC>;
   int dev = 0, sms = 0, per_sm = 0;
   cudaGetDevice(&dev);
@@ -513,31 +515,31 @@ cudaError_t launch_one(const SrMat* mats, const SrItem* items, int nitems, int p
   int grid = sms * (per_sm > 0 ? per_sm : 1);
   if (grid > nitems) grid = nitems;
   count_launch();
-  kern<<<grid, TPB, 0, st>>>(mats, items, nitems, pass, last ? 1 : 0);
+  kern<<<grid, TPB, 0, st>>>(mats, items, nitems, pass, last ? 1 : 0, flags);
   return cudaGetLastError();
 }
 
 template <bool VEC>
 cudaError_t dispatch(int slots, int threads, const SrMat* mats, const SrItem* items, int nitems, int pass,
-                     bool last, cudaStream_t st) {
+                     bool last, const unsigned* flags, cudaStream_t st) {
   // rows per batch: about 8 floats x 4 per thread in each of the two sets
-  if (threads == 512) return launch_one<8, 512, 1, VEC>(mats, items, nitems, pass, last, st);
+  if (threads == 512) return launch_one<8, 512, 1, VEC>(mats, items, nitems, pass, last, flags, st);
   switch (slots) {
-    case 1: return launch_one<1, 256, 8, VEC>(mats, items, nitems, pass, last, st);
-    case 2: return launch_one<2, 256, 4, VEC>(mats, items, nitems, pass, last, st);
-    case 3: return launch_one<3, 256, 2, VEC>(mats, items, nitems, pass, last, st);
-    case 4: return launch_one<4, 256, 2, VEC>(mats, items, nitems, pass, last, st);
-    case 5: return launch_one<5, 256, 1, VEC>(mats, items, nitems, pass, last, st);
-    case 6: return launch_one<6, 256, 1, VEC>(mats, items, nitems, pass, last, st);
-    case 7: return launch_one<7, 256, 1, VEC>(mats, items, nitems, pass, last, st);
-    case 8: return launch_one<8, 256, 1, VEC>(mats, items, nitems, pass, last, st);
+    case 1: return launch_one<1, 256, 8, VEC>(mats, items, nitems, pass, last, flags, st);
+    case 2: return launch_one<2, 256, 4, VEC>(mats, items, nitems, pass, last, flags, st);
+    case 3: return launch_one<3, 256, 2, VEC>(mats, items, nitems, pass, last, flags, st);
+    case 4: return launch_one<4, 256, 2, VEC>(mats, items, nitems, pass, last, flags, st);
+    case 5: return launch_one<5, 256, 1, VEC>(mats, items, nitems, pass, last, flags, st);
+    case 6: return launch_one<6, 256, 1, VEC>(mats, items, nitems, pass, last, flags, st);
+    case 7: return launch_one<7, 256, 1, VEC>(mats, items, nitems, pass, last, flags, st);
+    case 8: return launch_one<8, 256, 1, VEC>(mats, items, nitems, pass, last, flags, st);
     default: return cudaErrorInvalidValue;
   }
 }
 
 template <int S, int RB, int NC = 8>
 cudaError_t ring_launch(const SrMat* mats, const SrItem* items, int nitems, int pass, bool last, int max_cols,
-                        unsigned* flags, cudaStream_t st) {
+                        unsigned* flags, uint64_t wait_ns, cudaStream_t st) {
   auto kern = srank_ring_kernel<S, RB, NC>;
   constexpr int kThreads = 32 * (NC + 1);   // NC consumer warps + 1 producer warp
   // three or four stages of RB rows (at most 32 KB each), four where they
@@ -561,7 +563,7 @@ cudaError_t ring_launch(const SrMat* mats, const SrItem* items, int nitems, int 
   int grid = sms * (per_sm > 0 ? per_sm : 1);
   if (grid > nitems) grid = nitems;
   count_launch();
-  kern<<<grid, kThreads, smem, st>>>(mats, items, nitems, pass, last ? 1 : 0, nst, stride, flags);
+  kern<<<grid, kThreads, smem, st>>>(mats, items, nitems, pass, last ? 1 : 0, nst, stride, flags, wait_ns);
   return cudaGetLastError();
 }
 
@@ -575,8 +577,8 @@ constexpr int ring_rows(int s, int nc) {
 
 template <int S, int NC>
 cudaError_t ring_go(const SrMat* mats, const SrItem* items, int nitems, int pass, bool last, int max_cols,
-                    unsigned* flags, cudaStream_t st) {
-  return ring_launch<S, ring_rows(S, NC), NC>(mats, items, nitems, pass, last, max_cols, flags, st);
+                    unsigned* flags, uint64_t wait_ns, cudaStream_t st) {
+  return ring_launch<S, ring_rows(S, NC), NC>(mats, items, nitems, pass, last, max_cols, flags, wait_ns, st);
 }
 
 // Launch shape of the ring kernel for rows of max_cols columns, as
@@ -598,28 +600,28 @@ RingShape ring_shape(int max_cols) {
 }
 
 cudaError_t ring_dispatch(int max_cols, const SrMat* mats, const SrItem* items, int nitems, int pass, bool last,
-                          unsigned* flags, cudaStream_t st) {
+                          unsigned* flags, uint64_t wait_ns, cudaStream_t st) {
   if (max_cols > 16 * 1024) return cudaErrorInvalidValue;
   const RingShape sh = ring_shape(max_cols);
-  if (sh.nc == 6) return ring_go<1, 6>(mats, items, nitems, pass, last, max_cols, flags, st);
+  if (sh.nc == 6) return ring_go<1, 6>(mats, items, nitems, pass, last, max_cols, flags, wait_ns, st);
   if (sh.nc == 10) {
     switch (sh.s) {
-      case 1: return ring_go<1, 10>(mats, items, nitems, pass, last, max_cols, flags, st);
-      case 2: return ring_go<2, 10>(mats, items, nitems, pass, last, max_cols, flags, st);
-      case 3: return ring_go<3, 10>(mats, items, nitems, pass, last, max_cols, flags, st);
+      case 1: return ring_go<1, 10>(mats, items, nitems, pass, last, max_cols, flags, wait_ns, st);
+      case 2: return ring_go<2, 10>(mats, items, nitems, pass, last, max_cols, flags, wait_ns, st);
+      case 3: return ring_go<3, 10>(mats, items, nitems, pass, last, max_cols, flags, wait_ns, st);
       default: return cudaErrorInvalidValue;
     }
   }
   switch (sh.s) {
-    case 1: return ring_go<1, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
-    case 2: return ring_go<2, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
-    case 3: return ring_go<3, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
-    case 4: return ring_go<4, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
-    case 5: return ring_go<5, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
-    case 6: return ring_go<6, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
-    case 8: return ring_go<8, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
-    case 12: return ring_go<12, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
-    case 16: return ring_go<16, 8>(mats, items, nitems, pass, last, max_cols, flags, st);
+    case 1: return ring_go<1, 8>(mats, items, nitems, pass, last, max_cols, flags, wait_ns, st);
+    case 2: return ring_go<2, 8>(mats, items, nitems, pass, last, max_cols, flags, wait_ns, st);
+    case 3: return ring_go<3, 8>(mats, items, nitems, pass, last, max_cols, flags, wait_ns, st);
+    case 4: return ring_go<4, 8>(mats, items, nitems, pass, last, max_cols, flags, wait_ns, st);
+    case 5: return ring_go<5, 8>(mats, items, nitems, pass, last, max_cols, flags, wait_ns, st);
+    case 6: return ring_go<6, 8>(mats, items, nitems, pass, last, max_cols, flags, wait_ns, st);
+    case 8: return ring_go<8, 8>(mats, items, nitems, pass, last, max_cols, flags, wait_ns, st);
+    case 12: return ring_go<12, 8>(mats, items, nitems, pass, last, max_cols, flags, wait_ns, st);
+    case 16: return ring_go<16, 8>(mats, items, nitems, pass, last, max_cols, flags, wait_ns, st);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -633,9 +635,9 @@ int srank_ring_shape(int64_t cols) {
 }
 
 cudaError_t launch_srank_ring(int max_cols, const SrMat* mats, const SrItem* items, int nitems, int pass, bool last,
-                              unsigned* flags, cudaStream_t st) {
+                              unsigned* flags, uint64_t wait_ns, cudaStream_t st) {
   if (nitems <= 0) return cudaSuccess;
-  return ring_dispatch(max_cols, mats, items, nitems, pass, last, flags, st);
+  return ring_dispatch(max_cols, mats, items, nitems, pass, last, flags, wait_ns, st);
 }
 
 int srank_slots(int64_t cols, int* threads) {
@@ -652,17 +654,17 @@ int srank_slots(int64_t cols, int* threads) {
 }
 
 cudaError_t launch_srank_pass(int slots, int threads, bool vec4, const SrMat* mats, const SrItem* items,
-                              int nitems, int pass, bool last, cudaStream_t st) {
+                              int nitems, int pass, bool last, const unsigned* flags, cudaStream_t st) {
   if (nitems <= 0) return cudaSuccess;
-  return vec4 ? dispatch<true>(slots, threads, mats, items, nitems, pass, last, st)
-              : dispatch<false>(slots, threads, mats, items, nitems, pass, last, st);
+  return vec4 ? dispatch<true>(slots, threads, mats, items, nitems, pass, last, flags, st)
+              : dispatch<false>(slots, threads, mats, items, nitems, pass, last, flags, st);
 }
 
 cudaError_t launch_srank_decide(const SrMat* mats, int nmat, double alpha, int last_pass, unsigned char* active,
-                                unsigned char* skip, double* srank, cudaStream_t st) {
+                                unsigned char* skip, double* srank, const unsigned* flags, cudaStream_t st) {
   if (nmat <= 0) return cudaSuccess;
   count_launch();
-  srank_decide_kernel<<<(nmat + 127) / 128, 128, 0, st>>>(mats, nmat, alpha, last_pass, active, skip, srank);
+  srank_decide_kernel<<<(nmat + 127) / 128, 128, 0, st>>>(mats, nmat, alpha, last_pass, active, skip, srank, flags);
   return cudaGetLastError();
 }
 

@@ -30,7 +30,8 @@ EXPORTED = ("lm_config_default", "lm_create", "lm_step", "lm_set_lr", "lm_msign_
             "lm_workspace_bytes", "lm_destroy", "lm_status_string", "lm_last_error",
             "lm_kernel_launch_count", "lm_profile_enable", "lm_profile_read",
             "lm_msign_ns_noalloc", "lm_probe_bounded_wait", "lm_msign_ns_coeffs",
-            "lm_set_adamw_lr", "lm_get_second_moment", "lm_set_second_moment", "lm_get_selection")
+            "lm_set_adamw_lr", "lm_get_second_moment", "lm_set_second_moment", "lm_get_selection",
+            "lm_msign_ns_noalloc_status", "lm_shard_owners", "lm_config_size")
 
 KERNEL_FAMILIES = ("lion", "momentum_norm", "ns_gram", "ns_poly", "ns_apply", "finalize", "other", "adamw",
                    "srank")
@@ -55,7 +56,7 @@ class LmConfig(ctypes.Structure):
                 ("adamw_beta1", ctypes.c_double), ("adamw_beta2", ctypes.c_double),
                 ("adamw_eps", ctypes.c_double), ("adamw_weight_decay", ctypes.c_double),
                 ("schedule", ctypes.c_int), ("srank_alpha", ctypes.c_double), ("srank_iters", ctypes.c_int),
-                ("srank_seed", ctypes.c_uint64)]
+                ("srank_seed", ctypes.c_uint64), ("shard_rank", ctypes.c_int), ("shard_world", ctypes.c_int)]
 
 
 class LmProfile(ctypes.Structure):
@@ -83,6 +84,11 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib = ctypes.CDLL(p)
     c_void_p, c_int, c_int64, c_double = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_double
     P = ctypes.POINTER
+    lib.lm_config_size.argtypes = []
+    lib.lm_config_size.restype = ctypes.c_size_t
+    if lib.lm_config_size() != ctypes.sizeof(LmConfig):
+        raise RuntimeError(f"{p}: lm_config is {lib.lm_config_size()} bytes in the library but "
+                           f"{ctypes.sizeof(LmConfig)} in this binding (rebuild the library)")
     lib.lm_config_default.argtypes = [P(LmConfig)]
     lib.lm_config_default.restype = None
     lib.lm_create.argtypes = [P(LmTensor), c_int, P(LmConfig), c_void_p, P(c_void_p)]
@@ -100,6 +106,10 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
     lib.lm_msign_ns_noalloc.argtypes = [P(LmTensor), P(LmTensor), c_int, c_double, c_double, c_double,
                                         c_double, c_int, c_void_p]
     lib.lm_msign_ns_noalloc.restype = c_int
+    lib.lm_shard_owners.argtypes = [P(LmTensor), c_int, c_int, P(c_int)]
+    lib.lm_shard_owners.restype = c_int
+    lib.lm_msign_ns_noalloc_status.argtypes = [P(ctypes.c_uint32), c_void_p]
+    lib.lm_msign_ns_noalloc_status.restype = c_int
     lib.lm_get_selection.argtypes = [c_void_p, c_int, P(ctypes.c_ubyte), P(c_double)]
     lib.lm_get_selection.restype = c_int
     lib.lm_set_adamw_lr.argtypes = [c_void_p, c_double]
@@ -382,3 +392,12 @@ def msign_ns_noalloc(x, out, steps: int = 5, a: float = 3.4445, b: float = -4.77
     _check(lib, lib.lm_msign_ns_noalloc(ctypes.byref(di), ctypes.byref(do), steps, a, b, c, eps,
                                         precision, _stream_handle(stream)), "lm_msign_ns_noalloc")
     return out
+
+
+def msign_ns_noalloc_status(stream=None):
+    """Synchronise the stream of the last lm_msign_ns_noalloc call and return
+    (status, device flags) of that call (lm_msign_ns_noalloc_status)."""
+    lib = load_library()
+    f = ctypes.c_uint32()
+    st = lib.lm_msign_ns_noalloc_status(ctypes.byref(f), _stream_handle(stream))
+    return st, int(f.value)

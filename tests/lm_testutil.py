@@ -75,3 +75,31 @@ def make_problem(shapes, grad_kind, steps, wseed=1, gseed=0, w_std=0.02):
     W0 = synth.init_weights(shapes, seed=wseed, std=w_std)
     grads = [synth.draw_grads(shapes, grad_kind, seed=gseed, step=t) for t in range(steps)]
     return W0, grads
+
+
+def ns_closed_form_rows(G_hat: np.ndarray, steps: int, a: float, b: float, c: float, eps: float = 1e-7,
+                        rows=None) -> np.ndarray:
+    """NS_steps(G_hat) (Section 2's odd-polynomial iteration with the
+    Frobenius pre-normalisation) through its closed form on the SVD, in fp64:
+    with X0 = G_hat / (||G_hat||_F + eps) = U diag(s) V^T,
+    NS(X0) = U diag(phi^K(s)) V^T = X0 V diag(phi^K(s) / s) V^T, computed
+    in the tall orientation (a wide input as its transpose, NS(X^T) =
+    NS(X)^T) from the eigen-decomposition of the small Gram X0^T X0.  Returns
+    the rows ``rows`` (all if None) of the tall-orientation result, so a large
+    matrix can be checked element-wise on a sample of its long dimension.
+    Agrees with oracle.ns_polynomial to fp64 rounding (pinned on the CPU)."""
+    import oracle as O
+    X0 = np.asarray(G_hat, dtype=np.float64)
+    X0 = X0 / (np.linalg.norm(X0) + eps)
+    Xt = X0 if X0.shape[0] >= X0.shape[1] else X0.T
+    lam, V = np.linalg.eigh(Xt.T @ Xt)
+    sig = np.sqrt(np.clip(lam, 0.0, None))
+    safe = np.where(sig > 0, sig, 1.0)
+    f = np.where(sig > 0, O.ns_scalar_map(sig, steps, a, b, c) / safe, 0.0)
+    Xr = Xt if rows is None else Xt[rows]
+    return ((Xr @ V) * f) @ V.T
+
+
+def tall(x: np.ndarray) -> np.ndarray:
+    """The tall orientation of a matrix (its transpose if it is wide)."""
+    return x if x.shape[0] >= x.shape[1] else x.T

@@ -1,10 +1,12 @@
 """GPU parity of the Newton-Schulz msign approximation (lm_msign_ns) against
 the fp64 oracle recurrence on the same stored input: relative Frobenius error
 <= 2e-2 for the bf16 tensor-core path, <= 1e-5 for the fp32 CUDA-core path and
-<= 5e-5 for the three-piece tensor-core fp32 mode (LM_NS_F32_TC: each fp32
-operand is exactly hi + mid + lo in bf16, the dropped piece products are of
-order 2^-24 relative, and what remains is the tensor cores' fp32
-accumulation, measured at 1e-6 - 2.4e-5 up to 768 x 50304)."""
+<= 2e-5 for the three-piece tensor-core mode (LM_NS_F32_TC: each fp32 operand
+is exactly hi + mid + lo in bf16, the dropped piece products are of order
+2^-24 relative, and what remains is the tensor cores' fp32 accumulation, which
+loses about a unit of the last place per MMA; with the largest products in an
+accumulator of their own it measures 1.3e-6 - 1.8e-5 up to 768 x 50304 and
+4096 x 4096, at most 5.8e-6 on the 1280-wide shapes)."""
 
 import numpy as np
 import pytest
@@ -15,7 +17,7 @@ from tests.lm_testutil import host_tensor, rel_fro, stored_values
 
 pytestmark = pytest.mark.gpu
 
-TOL = {"bf16": 2e-2, "f32": 1e-5, "f32tc": 5e-5}
+TOL = {"bf16": 2e-2, "f32": 1e-5, "f32tc": 2e-5}
 
 
 def _prec(L, precision):

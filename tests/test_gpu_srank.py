@@ -101,7 +101,7 @@ def test_mixed_steps_match_oracle_fp32_ns(precision):
     matrix takes the branch the rule selects on its current buffer; weights of
     Lion-selected matrices and of the vector bit-exact against the same-order
     float32 step, of Muon-selected matrices within the fp32 NS tolerance (1e-5
-    CUDA cores, 5e-5 three-piece tensor cores)
+    CUDA cores, 2e-5 three-piece tensor cores)
     carried into W; momentum bit-exact.  (The low-rank buffers are badly
     conditioned: storing their NS intermediates in bf16 alone moves the
     output by 30-45%, so the bf16 path is checked against the plain Muon
@@ -135,7 +135,7 @@ def test_mixed_steps_match_oracle_fp32_ns(precision):
                 w_ref = O.round_to_storage(O.muon_update(W[i].astype(np.float64), gh, cfg), "bf16")
                 o = O.ns_polynomial(gh, 5, *O.NS_QUINTIC, 1e-7)
                 d = rel_fro(O.ns_polynomial_schedule_storage(gh, (O.NS_QUINTIC,) * 5, 1e-7, "f32"), o)
-                tau = max(1e-5 if precision == 0 else 5e-5, 1.5 * d)
+                tau = max(1e-5 if precision == 0 else 2e-5, 1.5 * d)
                 r_w = eta_M * 0.2 * np.sqrt(max(s)) * tau * np.linalg.norm(o) / np.linalg.norm(w_ref)
                 assert rel_fro(wg, w_ref) <= 1e-4 + r_w + np.sqrt(r_w * 2.0 ** -8), (s, rel_fro(wg, w_ref))
                 _, m_ref = O.lion_step_f32(W[i], G[i], M[i], 0.9, 0.99, 0.0, 0.0, w_dtype="f32")

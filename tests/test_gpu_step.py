@@ -2,7 +2,7 @@
 against the storage-modelled fp64 oracle: weights within 1e-3 relative
 (Frobenius) after 8 steps with the fp32 Newton-Schulz path, and within the
 bound the 2e-2 NS tolerance implies with the bf16 tensor-core path (and the
-5e-5 one with the three-piece tensor-core fp32 mode, ns_precision 2); momentum
+2e-5 one with the three-piece tensor-core mode, ns_precision 2); momentum
 bit-exact (same-order fp32 EMA); the Muon direction itself within the NS
 tolerance; plus the state-size invariant, status flags and argument errors."""
 
@@ -26,7 +26,7 @@ def _cfg_pair(**kw):
 
 
 NS_TOL_BF16 = 2e-2     # relative Frobenius tolerance of the bf16 NS output
-NS_TOL_F32TC = 5e-5    # the same for the three-piece tensor-core fp32 mode
+NS_TOL_F32TC = 2e-5    # the same for the three-piece tensor-core mode
 F32TC = 2              # LM_NS_F32_TC
 BF16_ULP = 2.0 ** -8   # relative spacing of bf16 values (upper bound)
 
@@ -58,7 +58,7 @@ def _bf16_ns_bounds(W0, grads, dtype, cfg: O.Config, steps, Wo, tau_ns=NS_TOL_BF
     bf16 spacing), which adds sqrt(r u) in relative Frobenius terms.  The
     bound per parameter is 1e-3 + r + sqrt(r u) (the last term for bf16).
     tau_ns, storage, floor: the same bound for another NS mode (the
-    three-piece fp32 mode: 5e-5, fp32 storage, floor 1e-6 for fp32 W)."""
+    three-piece mode: 2e-5, fp32 storage, floor 1e-6 for fp32 W)."""
     P = [stored_values(host_tensor(w, dtype)) for w in W0]
     M = [np.zeros_like(p) for p in P]
     acc = [0.0] * len(P)

@@ -1,10 +1,15 @@
 """lm_msign_ns_noalloc, the Newton-Schulz entry point for callers that cannot
-allocate device memory while they run (their memory is budgeted up front, or
-cudaMalloc/cudaFree are too costly where they call from).  It works in a
-fixed in-library scratch area instead of allocating, so these tests check,
-through the C ABI, that two calls in a row give the same result as the
-allocating lm_msign_ns within the NS tolerances (2e-2 bf16, 1e-5 fp32), and
-that a matrix too large for the scratch area is refused.
+allocate device memory while they run: a program whose device memory is all
+handed out up front by its own allocator, or a latency-critical loop where
+cudaMalloc/cudaFree (and cudaFree's device synchronisation) are not
+acceptable.  It works in a fixed in-library scratch area instead of
+allocating.  Through the C ABI these tests check that calls in a row (a
+larger matrix, then smaller ones that reuse what the first left in the
+scratch area) match the fp64 oracle recurrence within the NS tolerances
+(2e-2 bf16, 1e-5 fp32) and the allocating lm_msign_ns within the same, for
+0, 1 and 5 iterations and for an input dtype other than the precision; that
+a matrix close to the 64 MiB limit runs and one beyond it is refused; and
+that the call's status word reads clean.
 
 The file name sorts last so that a run stopping at its first failure has
 already run every other test."""
@@ -14,6 +19,7 @@ import ctypes
 import numpy as np
 import pytest
 
+import oracle as O
 from paper_2605_19811_gb300 import synth
 from tests.lm_testutil import host_tensor, rel_fro, stored_values
 
@@ -37,18 +43,33 @@ def _call(entry, x, precision, steps=5):
     return stored_values(out)
 
 
-@pytest.mark.parametrize("precision", [1, 0])
-def test_noalloc_matches_allocating_entry_point_two_calls(precision):
-    in_dtype = "bf16" if precision == 1 else "f32"
-    # a larger call first, then a smaller one with different padding, so the
-    # second call runs on scratch the first one left behind
-    for shape, seed in (((640, 1500), 1), ((300, 200), 2)):
-        x = host_tensor(synth.draw_matrix(shape, seed=seed), in_dtype).cuda()
-        want = _call("lm_msign_ns", x, precision)
-        got = _call("lm_msign_ns_noalloc", x, precision)
+@pytest.mark.parametrize("precision,in_dtype", [(1, "bf16"), (0, "f32"), (0, "bf16"), (1, "f32")])
+@pytest.mark.parametrize("steps", [5, 1, 0])
+def test_noalloc_matches_oracle_and_allocating_entry_point(precision, in_dtype, steps):
+    from paper_2605_19811_gb300 import lionmuon as L
+    # a larger call first, then smaller ones with other padding, so the later
+    # calls run on scratch the first one left behind
+    for shape, seed in (((640, 1500), 1), ((300, 200), 2), ((1000, 130), 3)):
+        xh = host_tensor(synth.draw_matrix(shape, seed=seed), in_dtype)
+        x = xh.cuda()
+        got = _call("lm_msign_ns_noalloc", x, precision, steps)
+        want = O.ns_polynomial(stored_values(xh), steps, *QUINTIC, 1e-7)
+        alloc = _call("lm_msign_ns", x, precision, steps)
         assert got.shape == want.shape
         assert np.all(np.isfinite(got))
         assert rel_fro(got, want) <= TOL[precision]
+        assert rel_fro(alloc, want) <= TOL[precision]
+        assert rel_fro(got, alloc) <= TOL[precision]
+        assert L.msign_ns_noalloc_status() == (0, 0)
+
+
+def test_noalloc_near_scratch_limit():
+    """2048 x 5120 in bf16 needs (2 * 2048 * 5120 + 2 * 2048^2) * 2 bytes plus
+    tables, about 56 MiB: it fits."""
+    xh = host_tensor(synth.draw_matrix((2048, 5120), seed=4), "bf16")
+    got = _call("lm_msign_ns_noalloc", xh.cuda(), 1)
+    want = O.ns_polynomial(stored_values(xh), 5, *QUINTIC, 1e-7)
+    assert rel_fro(got, want) <= TOL[1]
 
 
 def test_noalloc_rejects_matrix_beyond_scratch_limit():
