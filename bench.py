@@ -559,6 +559,7 @@ def run_ours(args):
     ns_ms, ns_launches = prof["ns_gemm"]
     lion_ms, lion_launches = prof["lion"]
     ns_mats = own_mats if sharded else mats      # sharded: this rank's Newton-Schulz work
+    traffic_ok = args.set == "gpt_720m" and not sharded and not srank
     fl = ns_flops_sym(ns_mats) * n_muon
     # The burst peak applies to a kernel timed in a short region, the
     # sustained one (the power cap's) to one inside a seconds-long loop.
@@ -590,7 +591,8 @@ def run_ours(args):
             bound, kernel = "alu", "ns_simt_kernel"
             peak_kind = f"fp32 FMA, derived: {sms} SMs x 128 lanes x 2 FLOP x {mhz:.0f} MHz"
         # the recorded ncu traffic is the bf16 workload's
-        traffic = kernel_traffic(kernel) if args.precision != "f32tc" else None
+        # the recorded traffic is that of the 720M set's bf16 launches on one GPU
+        traffic = kernel_traffic(kernel) if traffic_ok and args.precision == "bf16" else None
         dense = sum(5 * (4.0 * min(m, n) ** 2 * max(m, n) + 2.0 * min(m, n) ** 3) for m, n in ns_mats) * n_muon
         # per phase: GRAM s^2 l, POLY s^3 (the symmetric products once), APPLY 2 s^2 l per iteration
         ph_fl = {"ns_gram": sum(min(a, b) ** 2 * max(a, b) for a, b in ns_mats),
@@ -622,7 +624,7 @@ def run_ours(args):
         gbs = bytes_moved / (lion_ms / 1e3) / 1e9
         pk = peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
         lion_roof = {"bound": "hbm", "achieved": gbs, "peak": pk, "unit": "GB/s", "frac": gbs / pk,
-                     "traffic": kernel_traffic("lion_kernel"), "kernel": "lion_kernel",
+                     "traffic": kernel_traffic("lion_kernel") if traffic_ok else None, "kernel": "lion_kernel",
                      # per full-set launch (one per Lion step); the vector-only launches of the
                      # Muon steps (0.02% of the parameters) are inside the sum
                      "per_launch_ms": lion_ms / max(n_lion, 1),

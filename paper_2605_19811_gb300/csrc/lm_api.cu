@@ -250,6 +250,12 @@ static const char* const kFamilyNames[LM_KERNEL_FAMILIES] = {
     "lion", "momentum_norm", "ns_gram", "ns_poly", "ns_apply", "finalize", "other", "adamw", "srank"};
 
 constexpr int64_t kLionChunk = 32768;   // elements per Lion work chunk
+// Three-piece mode: Gram tiles longer than this many 64-deep K blocks (1536)
+// are split along K, whatever the balance (the parts are added in fp32): the
+// tensor cores' fp32 accumulation error grows with the MMAs summed into one
+// accumulator.  Measured on a 720M-set Muon step: the largest direction error
+// 2.5e-5 at 96 blocks, 1.2e-5 at 48, 8.8e-6 at 32, 8.4e-6 at 24.
+constexpr int kGramCapF32TC = 24;
 constexpr uint64_t kRingWaitNs = 2000000000ull;   // the power-iteration ring's waits: 2 s unless set shorter
 
 struct LionTable {
@@ -531,8 +537,8 @@ static void layout_ns(std::vector<NsGroup>& groups, lm_dtype xdt, int nmat, Aren
       if (ph == NS_GRAM) {
         int nparts = 0;
         if (xdt == LM_BF16) {
-          // three-piece mode: no fp32 accumulation over more than 96 K blocks (6144)
-          split_gram_tiles(groups, g0, t, kTcBK, tc_max_pairs(), targets, nparts, pieces == 3 ? 96 : 0);
+          // three-piece mode: no fp32 accumulation over more than kGramCapF32TC K blocks
+          split_gram_tiles(groups, g0, t, kTcBK, tc_max_pairs(), targets, nparts, pieces == 3 ? kGramCapF32TC : 0);
         } else {
           int dev = 0, sms = 0;
           cudaGetDevice(&dev);

@@ -136,11 +136,9 @@ def test_stress_7b_muon_then_lion():
 def test_720m_three_piece_mode_directions():
     """The 720M-shaped set with ns_precision = LM_NS_F32_TC and fp32
     parameters and gradients (so that W's storage does not hide the NS error):
-    after one Muon step of the whole set, the hidden matrices' directions
-    within 1e-5 of the fp64 iteration and the 50304-row embedding's (its Gram
-    products sum 50304 terms) within the mode's 2e-5 (measured 1.24e-5)."""
+    after one Muon step of the whole set, the directions of the first, a middle
+    and the last matrix of every hidden shape and of the embedding within
+    1e-5 of the fp64 iteration (measured at most 8.4e-6)."""
     from paper_2605_19811_gb300 import lionmuon as L
-    _muon_then_lion("gpt_720m", 1, [(1280, 3840), (1280, 1280), (1280, 5120), (5120, 1280)],
+    _muon_then_lion("gpt_720m", 1, [(1280, 3840), (1280, 1280), (1280, 5120), (5120, 1280), (50304, 1280)],
                     dtype="f32", precision=L.LM_NS_F32_TC, tol=1e-5, lion=False)
-    _muon_then_lion("gpt_720m", 1, [(50304, 1280)], dtype="f32", precision=L.LM_NS_F32_TC, tol=2e-5,
-                    lion=False)

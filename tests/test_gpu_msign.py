@@ -109,16 +109,25 @@ MIXED_TABLE = ((3.0, -3.2, 1.2), (2.0, -1.5, 0.45), (1.875, -1.25, 0.375))
 
 
 def table_tolerance(x, table, precision):
-    """NS tolerance for a coefficient table: the stated one (2e-2 bf16,
-    1e-5 fp32), or 1.5 times the distance that storing the intermediates in
-    the path's precision alone puts between the oracle's storage-modelled
-    recurrence and its exact one, whichever is larger.  Aggressive first
-    polynomials (the minimax tables start near 8.5 x) amplify rounding of
-    small singular values; the storage-modelled oracle measures by how much
-    for this input, independently of the GPU."""
-    storage = "bf16" if precision == "bf16" else "f32"   # the three-piece mode stores fp32 exactly
-    d = rel_fro(O.ns_polynomial_schedule_storage(x, table, 1e-7, storage), O.ns_polynomial_schedule(x, table, 1e-7))
-    return max(TOL[precision], 1.5 * d)
+    """NS tolerance for a coefficient table.  bf16: the stated 2e-2, or 1.5
+    times the distance that storing the intermediates in bf16 alone puts
+    between the oracle's storage-modelled recurrence and its exact one,
+    whichever is larger (aggressive first polynomials, the minimax tables
+    start near 8.5 x, amplify rounding of small singular values; the
+    storage-modelled oracle measures by how much for this input, independently
+    of the GPU).  The fp32 modes: the stated tolerance, which holds for the
+    constant quintic, times the factor by which the table amplifies fp32-size
+    roundings more than the quintic does on the same input (the ratio of the
+    two storage-modelled distances in fp32; about 2 for Polar Express), or 1.5
+    times the table's own fp32 distance, whichever is larger."""
+    if precision == "bf16":
+        d = rel_fro(O.ns_polynomial_schedule_storage(x, table, 1e-7, "bf16"), O.ns_polynomial_schedule(x, table, 1e-7))
+        return max(TOL[precision], 1.5 * d)
+    quintic = [O.NS_QUINTIC] * 5
+    d = rel_fro(O.ns_polynomial_schedule_storage(x, table, 1e-7, "f32"), O.ns_polynomial_schedule(x, table, 1e-7))
+    dq = rel_fro(O.ns_polynomial_schedule_storage(x, quintic, 1e-7, "f32"),
+                 O.ns_polynomial_schedule(x, quintic, 1e-7))
+    return max(TOL[precision] * max(1.0, d / dq), 1.5 * d)
 
 
 def _table(name):
