@@ -136,7 +136,10 @@ def test_small_gpt_8_steps(period, precision):
                                for gs in grads], shapes, 0.99, steps)
     tol = (1e-3 if precision == 0 else _f32tc_bounds(W0, grads, "bf16", ocfg, steps, Wo) if precision == F32TC
            else _bf16_ns_bounds(W0, grads, "bf16", ocfg, steps, Wo))
-    _check(Wg, Wo, Mg, Mo, tol)
+    worst = _check(Wg, Wo, Mg, Mo, tol)
+    # the measured relative weight error per parameter, beside its bound (-s shows it)
+    print(f"P={period} ns_precision={precision}: " +
+          "; ".join(f"{tuple(s)} {e:.2e} <= {tl:.2e}" for s, (e, tl) in zip(shapes, worst)))
     assert flags == 0
 
 
