@@ -219,15 +219,17 @@ class ClockSampler:
 # CPU oracle timing (cpu_baseline leg and --impl reference)
 # ---------------------------------------------------------------------------
 
-def oracle_sample(name, period, budget_s=12.0):
-    """Time the oracle on a bounded sample of the workload and scale it to the
-    period-averaged ms/step of the whole set.  Returns (ms_per_step, info)."""
+def oracle_times(name, period, which=None):
+    """Time the oracle: a Lion step on a 4 M-element vector sample, and a full
+    fp64 Muon step (momentum, K_NS = 5 NS iterations, parameter update) of one
+    matrix of each shape in ``which`` (every distinct matrix shape of the set,
+    embedding included, if None).  Returns (Lion seconds per element,
+    {shape: Muon-step seconds})."""
     import numpy as np
     import oracle as O
-    ps, shapes, mats, numel, mat_elems = workload(name)
+    _, _, mats, _, _ = workload(name)
     cfg = O.Config(period=period)
     rng = np.random.default_rng(0)
-    # Lion branch on a vector sample
     n = 4_000_000
     W = rng.standard_normal(n) * 0.02
     G = rng.standard_normal(n) * 1e-3
@@ -235,37 +237,43 @@ def oracle_sample(name, period, budget_s=12.0):
     t0 = time.perf_counter()
     O.lionmuon_param_step(W, G, M, 1, cfg)
     lion_per_elem = (time.perf_counter() - t0) / n
-    # Muon branch on one matrix of each of the two smallest distinct shapes
-    shapes_u = sorted({(min(a, b), max(a, b)) for a, b in mats}, key=lambda x: x[0] * x[0] * x[1])
-    samples = []
-    spent = time.perf_counter() - t0
-    for s, l in shapes_u[:2]:
-        Wm = rng.standard_normal((s, l)) * 0.02
-        Gm = rng.standard_normal((s, l)) * 1e-3
-        Mm = np.zeros((s, l))
+    del W, G, M
+    times = {}
+    for a, b in (sorted(set(mats)) if which is None else which):
+        Wm = rng.standard_normal((a, b)) * 0.02
+        Gm = rng.standard_normal((a, b)) * 1e-3
+        Mm = np.zeros((a, b))
         t1 = time.perf_counter()
         O.lionmuon_param_step(Wm, Gm, Mm, 0, cfg)
-        dt = time.perf_counter() - t1
-        samples.append((s, l, dt))
-        spent += dt
-        if spent > budget_s:
-            break
-    # t(matrix) = alpha * NS flops + beta * elements, fitted on the samples
-    if len(samples) >= 2:
-        A = np.array([[5 * (4.0 * s * s * l + 2.0 * s ** 3), s * l] for s, l, _ in samples])
-        y = np.array([dt for _, _, dt in samples])
-        alpha, beta = np.linalg.lstsq(A, y, rcond=None)[0]
-        alpha, beta = max(alpha, 0.0), max(beta, 0.0)
-    else:
-        s, l, dt = samples[0]
-        alpha, beta = dt / (5 * (4.0 * s * s * l + 2.0 * s ** 3)), 0.0
-    t_muon = sum(alpha * 5 * (4.0 * min(a, b) ** 2 * max(a, b) + 2.0 * min(a, b) ** 3) + beta * a * b
-                 for a, b in mats) + lion_per_elem * (numel - mat_elems)
+        times[(a, b)] = time.perf_counter() - t1
+        del Wm, Gm, Mm
+    return lion_per_elem, times
+
+
+def oracle_estimate(name, period, lion_per_elem, times):
+    """Period-averaged ms/step of the whole set from sampled oracle times: each
+    shape's Muon-step time once per matrix of that shape, the Lion time once
+    per element (vectors take the Lion step on Muon steps too)."""
+    _, _, mats, numel, mat_elems = workload(name)
+    t_muon = lion_per_elem * (numel - mat_elems) + sum(times[tuple(m)] for m in mats)
     t_lion = lion_per_elem * numel
-    per_step = (t_muon + (period - 1) * t_lion) / period if period > 0 else t_lion
-    info = {"lion_sample_elems": n, "muon_samples": [f"{s}x{l}" for s, l, _ in samples],
-            "extrapolated": True}
-    return per_step * 1e3, info
+    return 1e3 * ((t_muon + (period - 1) * t_lion) / period if period > 0 else t_lion)
+
+
+def oracle_sample(name, period):
+    """(ms_per_step, description) of the oracle on the bounded sample of
+    oracle_times over every matrix shape."""
+    lion, times = oracle_times(name, period)
+    _, _, mats, _, _ = workload(name)
+    return oracle_estimate(name, period, lion, times), shape_counts(mats, times)
+
+
+def shape_counts(mats, times):
+    """'rows x cols (x count)' for each sampled shape."""
+    counts = {}
+    for m in mats:
+        counts[tuple(m)] = counts.get(tuple(m), 0) + 1
+    return ", ".join(f"{a}x{b} (x{counts[(a, b)]})" for a, b in sorted(times))
 
 
 def cpu_cores():
@@ -298,17 +306,27 @@ def dist_env():
 
 
 def run_reference(args):
+    """The oracle timed on the host cores: all matrix shapes once (before the
+    warm-up steps), then per step the Lion sample and one shape's Muon step in
+    turn, so that the whole run stays within a few minutes; a step's value is
+    the estimate from the latest time of every shape."""
     rank, world, local = dist_env()
     if rank != 0:
         return 0
     ps, shapes, mats, numel, mat_elems = workload(args.set)
+    lion, times = oracle_times(args.set, args.period)
+    value = oracle_estimate(args.set, args.period, lion, times)
+    desc = shape_counts(mats, times)
+    order = sorted(times)
     vals = []
-    info = None
     for i in range(args.warmup + args.steps):
-        v, info = oracle_sample(args.set, args.period, budget_s=6.0)
+        which = [order[i % len(order)]] if order else []
+        lion, t1 = oracle_times(args.set, args.period, which=which)
+        times.update(t1)
+        v = oracle_estimate(args.set, args.period, lion, times)
         if i >= args.warmup:
             vals.append(v)
-    value = statistics.median(vals)
+    value = statistics.median(vals) if vals else value
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "ms/step",
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
@@ -317,9 +335,11 @@ def run_reference(args):
         "config": {"workload": args.set, "params": numel, "matrices": len(mats), "period": args.period,
                    "ns_steps": 5},
         "cpu_baseline": {"value": value, "unit": "ms/step", "cores": cpu_cores(), "kind": "oracle",
-                         "sample": ("each step times the fp64 oracle on a 4M-element Lion sample and "
-                                    f"full Muon steps of {info['muon_samples']}, scaled to the whole set "
-                                    "by elements and NS FLOPs (extrapolated)")},
+                         "sample": ("fp64 oracle: a full Muon step of one matrix of every shape "
+                                    f"({desc}), timed once, then per step a 4M-element Lion step and "
+                                    "one shape's Muon step in turn; each shape's latest time counted "
+                                    "once per matrix of that shape, the Lion time per element "
+                                    "(extrapolated)")},
         "e2e": {"value": value, "unit": "ms/step", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -645,11 +665,11 @@ def run_ours(args):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
-        v, info = oracle_sample(args.set, P, budget_s=15.0)
+        v, desc = oracle_sample(args.set, P)
         cpu = {"value": v, "unit": "ms/step", "cores": cpu_cores(), "kind": "oracle",
-               "sample": ("fp64 oracle on a 4M-element Lion sample and full Muon steps of "
-                          f"{info['muon_samples']}, scaled to the whole set by elements and NS FLOPs "
-                          "(extrapolated)")}
+               "sample": ("fp64 oracle on a 4M-element Lion step and a full Muon step of one matrix of "
+                          f"every shape, {desc}; each shape's time counted once per matrix of that shape, "
+                          "the Lion time per element (extrapolated)")}
 
     if rank == 0:
         line = {

@@ -1,7 +1,7 @@
 """Host-side logic of the multi-rank bench harness with gloo on the CPU
 (world size 2): the max-over-ranks timing reduction, and the reference arm
-printing only on rank 0.  Every rank is an independent replica of the
-optimizer step (no data-path collective), so this is all the exchange there is."""
+printing only on rank 0.  (The layer-sharded exchange itself is covered by
+test_shard.py.)"""
 
 import io
 import os
@@ -29,7 +29,8 @@ def _worker(rank, world, port, q):
     dist.init_process_group("gloo", rank=rank, world_size=world)
     got = bench.max_over_ranks(1.5 + rank, world, "cpu")
     # the reference arm runs and prints on rank 0 only
-    bench.oracle_sample = lambda name, period, budget_s=0: (42.0, {"muon_samples": ["1x1"]})
+    bench.oracle_times = lambda name, period, which=None: (0.0, {})
+    bench.oracle_estimate = lambda name, period, lion, times: 42.0
 
     class A:
         gpus, steps, warmup, set, period = world, 1, 0, "gpt2_124m", 2
