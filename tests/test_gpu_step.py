@@ -165,6 +165,50 @@ def test_muon_step_direction_within_ns_tolerance(precision, tau):
     assert flags == 0
 
 
+@pytest.mark.parametrize("precision,tau", [(1, NS_TOL_BF16), (0, 1e-5), (F32TC, NS_TOL_F32TC)])
+def test_muon_step_degenerate_gradients(precision, tau):
+    """The method's degenerate inputs on a Muon step (Algorithm 1, Muon
+    branch).  A zero gradient: G_hat = 0, X_0 = 0 / (0 + eps) = 0, every NS
+    output is 0 and the step is pure decay.  Rank-one gradients s u v^T, wide,
+    tall and square: the exact NS output is phi^5(x) u v^T / (|u| |v|), but
+    NS raises any singular value near 0 about 480-fold over five quintic
+    iterations, so the rounding of X_0 alone fills the null space with
+    directions that differ from run to run (the oracle's storage model puts a
+    bf16 result 117% and an fp32 one 1.7e-5 away from the exact output).  What
+    is unique is checked: the component u^T O v along the input's singular
+    pair, within the NS tolerance of the oracle's (the storage model: at most
+    2.2e-3 bf16, 1e-8 fp32); the rest must be a valid NS output, every
+    singular value within the quintic's range [0, 1.2024].  Momentum
+    bit-exact; no status flag."""
+    shapes = [(192, 640), (640, 192), (256, 256), (200, 72), (72, 200)]
+    rng = np.random.default_rng(21)
+    W0 = [rng.standard_normal(s).astype(np.float32) for s in shapes]
+    u = [rng.standard_normal(s[0]) for s in shapes]
+    v = [rng.standard_normal(s[1]) for s in shapes]
+    scale = [0.0, 1.0, 1e-3, 1.0, 1e-3]
+    G = [(c * np.outer(a, b)).astype(np.float32) for c, a, b in zip(scale, u, v)]
+    eta, lam = 1.0, 0.1
+    gcfg, _ = _cfg_pair(eta_muon=eta, weight_decay=lam, period=1, ns_precision=precision)
+    Wg, Mg, flags = run_trajectory_gpu(W0, [G], "f32", gcfg, 1)
+    assert flags == 0
+    for w0, g, w1, m1, shp, a, b in zip(W0, G, Wg, Mg, shapes, u, v):
+        w0 = w0.astype(np.float64)
+        s = 0.2 * np.sqrt(max(shp))
+        o_gpu = (w0 - w1 - eta * lam * w0) / (eta * s)
+        # fp32 storage of W moves the recovered direction by |W| 2^-24 / (eta s) per entry
+        slack = 4 * np.linalg.norm(w0) * 2.0 ** -24 / (eta * s)
+        if not g.any():
+            assert np.linalg.norm(o_gpu) <= slack
+        else:
+            o_ref = O.ns_polynomial(0.1 * g.astype(np.float64), 5, *O.NS_QUINTIC, 1e-7)
+            uh, vh = a / np.linalg.norm(a), b / np.linalg.norm(b)
+            p_gpu, p_ref = uh @ o_gpu @ vh, uh @ o_ref @ vh
+            assert abs(p_gpu - p_ref) <= tau * abs(p_ref) + slack, (shp, p_gpu, p_ref)
+            assert np.linalg.norm(o_gpu, 2) <= 1.2024 + 1e-2 + slack
+        _, m_ref = O.lion_step_f32(np.zeros_like(g), g, np.zeros_like(g), 0.9, 0.99, 0.0, 0.0, w_dtype="f32")
+        np.testing.assert_array_equal(m1.astype(np.float32).view(np.uint32), m_ref.view(np.uint32))
+
+
 def test_p_infinity_matrices_take_lion_steps_bit_exact():
     """period = 0 (P = infinity): every parameter, matrices included, takes
     the Lion step; bit-exact against the same-order oracle."""

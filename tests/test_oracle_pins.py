@@ -478,3 +478,20 @@ def test_storage_mode_sign_decision_matches_f32_lion():
     # the larger addend
     mag = np.maximum(np.abs(m), np.abs(g)).astype(np.float32)
     assert np.all(np.abs(M[0] - m32.astype(np.float64)) <= 2 * np.spacing(mag).astype(np.float64))
+
+
+def test_quintic_iterates_stay_within_its_range():
+    """The published quintic phi(x) = a x + b x^3 + c x^5 maps [0, 1] into
+    [0, 1.2024] (its maximum on [0, 1], at x^2 = (3|b| - sqrt(9 b^2 - 20 a c))
+    / (10 c), is 1.20237) and keeps [0, 1.2024] there, so every singular
+    value of an NS output lies in [0, 1.2024]: the validity bound the GPU
+    tests apply to rank-deficient inputs."""
+    a, b, c = O.NS_QUINTIC
+    x2 = (-3 * b - np.sqrt(9 * b * b - 20 * a * c)) / (10 * c)
+    xm = np.sqrt(x2)
+    peak = a * xm + b * xm ** 3 + c * xm ** 5
+    assert 1.2023 < peak < 1.2025
+    x = np.linspace(0.0, 1.0, 200001)
+    for _ in range(5):
+        x = a * x + b * x ** 3 + c * x ** 5
+        assert x.min() >= 0.0 and x.max() <= peak + 1e-12
