@@ -491,10 +491,12 @@ def run_ours(args):
     # device-to-device copy snapshots the parameters (W is updated in place
     # by step t+1), and the snapshot is read back to the host while step t+1
     # runs.  Warm-up steps run through the same pipeline before the timed
-    # region, as in a training loop that reuses its buffers.  (Sharded, the
-    # exchange of a Muon step belongs to NCCL and is not in this pipeline.)
+    # region, as in a training loop that reuses its buffers.  Sharded, a
+    # Muon step's exchange is enqueued on the compute stream after the step
+    # and before the snapshot, so the parameters read back are the exchanged
+    # ones.
     e2e = None
-    if not args.no_e2e and not sharded:
+    if not args.no_e2e:
         g_host = torch.empty(flat_bytes // 2, dtype=torch.bfloat16, pin_memory=True)
         w_host = torch.empty(flat_bytes // 2, dtype=torch.bfloat16, pin_memory=True)
         g_host.copy_(gflat)
@@ -528,6 +530,9 @@ def run_ours(args):
                         ev_in[nb].record(s_h2d)
                 s_cmp.wait_event(ev_in[b])
                 opt.step_descs(gdescs[b], n, t0 + i, sh_cmp)
+                if ex is not None and shard.is_muon_step(t0 + i, P):
+                    with torch.cuda.stream(s_cmp):
+                        ex.run()
                 ev_used[b].record(s_cmp)
                 if i >= 2:                  # the snapshot buffer's previous read-back is done
                     s_cmp.wait_event(ev_out[sb])
@@ -560,7 +565,10 @@ def run_ours(args):
                "what": "pinned-host gradients copied in and updated parameters copied out every step, "
                        "through lm_step; the gradient copies and the read-back of a device snapshot of "
                        "the parameters overlap the steps (three gradient and two snapshot buffers); "
-                       "the same pipeline runs untimed warm-up steps first"}
+                       "the same pipeline runs untimed warm-up steps first"
+                       + ("; layer-sharded: each rank copies the full gradient set in and reads the exchanged "
+                          "parameters back, the NCCL exchange of each Muon step inside the timed region"
+                          if sharded else "")}
     clk = clocks.stop()
     flags = opt.status()
     took_last = opt.selection()[0] if srank else None
