@@ -58,6 +58,9 @@ def parse_args():
     ap.add_argument("--srank-iters", type=int, default=5)
     ap.add_argument("--vector-rule", choices=["lion", "adamw"], default="lion",
                     help="1-D parameters: the Lion step, or the AdamW fallback of Section 3")
+    ap.add_argument("--ns-table", choices=["quintic", "polar_express", "chebyshev3"], default="quintic",
+                    help="Newton-Schulz coefficients: the constant quintic, or a per-iteration minimax table "
+                         "(degree 5 Polar Express, degree 3 Chebyshev-type)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-graph", action="store_true",
                     help="skip timing the same steps replayed from CUDA graphs")
@@ -81,14 +84,26 @@ def workload(name):
     return ps, shapes, mats, numel, mat_elems
 
 
-def ns_flops_sym(mats, steps=5):
+def ns_flops_sym(mats, steps=5, poly_steps=None):
     """Algorithmic FLOPs of NS_K per Muon step, symmetric products counted
-    once: per iteration 3 s^2 l + s^3 per matrix (s = min, l = max)."""
+    once: per iteration 3 s^2 l + s^3 per matrix (s = min, l = max), the s^3
+    of A A only in the poly_steps iterations whose c is not 0 (all of them
+    if None)."""
+    poly_steps = steps if poly_steps is None else poly_steps
     tot = 0.0
     for a, b in mats:
         s, l = min(a, b), max(a, b)
-        tot += steps * (3.0 * s * s * l + 1.0 * s ** 3)
+        tot += steps * 3.0 * s * s * l + poly_steps * 1.0 * s ** 3
     return tot
+
+
+def ns_table(name):
+    """(table or None, iterations with c != 0) for --ns-table."""
+    from paper_2605_19811_gb300 import ns_coeffs
+    if name == "quintic":
+        return None, 5
+    table = {"polar_express": ns_coeffs.polar_express, "chebyshev3": ns_coeffs.chebyshev_cubic}[name](5)
+    return table, sum(1 for t in table if t[2] != 0.0)
 
 
 def cublas_ns_context(mats, dev, reps=5):
@@ -398,6 +413,9 @@ def run_ours(args):
     extra = {"vector_rule": L.LM_VECTOR_ADAMW} if args.vector_rule == "adamw" else {}
     if sharded:
         extra.update(shard_rank=rank, shard_world=world)
+    table, poly_steps = ns_table(args.ns_table)
+    if table is not None:
+        extra["ns_coeffs"] = table
     if srank:
         opt = L.LionMuon(params, period=P, ns_precision=prec, schedule=L.LM_SCHEDULE_STABLE_RANK,
                          srank_alpha=args.srank_alpha, srank_iters=args.srank_iters, **extra)
@@ -587,8 +605,8 @@ def run_ours(args):
     ns_ms, ns_launches = prof["ns_gemm"]
     lion_ms, lion_launches = prof["lion"]
     ns_mats = own_mats if sharded else mats      # sharded: this rank's Newton-Schulz work
-    traffic_ok = args.set == "gpt_720m" and not sharded and not srank
-    fl = ns_flops_sym(ns_mats) * n_muon
+    traffic_ok = args.set == "gpt_720m" and not sharded and not srank and args.ns_table == "quintic"
+    fl = ns_flops_sym(ns_mats, 5, poly_steps) * n_muon
     # The burst peak applies to a kernel timed in a short region, the
     # sustained one (the power cap's) to one inside a seconds-long loop.
     pk_burst = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
@@ -600,7 +618,8 @@ def run_ours(args):
     roof = None
     if ns_ms > 0 and n_muon > 0:
         achieved = fl / (ns_ms / 1e3) / 1e12
-        flops_note = "symmetric count 3 s^2 l + s^3 per matrix per NS iteration"
+        flops_note = ("symmetric count 3 s^2 l + s^3 per matrix per NS iteration"
+                      + (f" (s^3 in the {poly_steps} iterations with c != 0)" if poly_steps != 5 else ""))
         if args.precision == "bf16":
             pk = pk_bf16
             bound, kernel, peak_kind = "tensor", "ns_tc_kernel", bf16_kind
@@ -621,7 +640,8 @@ def run_ours(args):
         # the recorded ncu traffic is the bf16 workload's
         # the recorded traffic is that of the 720M set's bf16 launches on one GPU
         traffic = kernel_traffic(kernel) if traffic_ok and args.precision == "bf16" else None
-        dense = sum(5 * (4.0 * min(m, n) ** 2 * max(m, n) + 2.0 * min(m, n) ** 3) for m, n in ns_mats) * n_muon
+        dense = sum(5 * 4.0 * min(m, n) ** 2 * max(m, n) + poly_steps * 2.0 * min(m, n) ** 3
+                    for m, n in ns_mats) * n_muon
         # per phase: GRAM s^2 l, POLY s^3 (the symmetric products once), APPLY 2 s^2 l per iteration
         ph_fl = {"ns_gram": sum(min(a, b) ** 2 * max(a, b) for a, b in ns_mats),
                  "ns_poly": sum(min(a, b) ** 3 for a, b in ns_mats),
@@ -631,7 +651,7 @@ def run_ours(args):
         for k, f1 in ph_fl.items():
             ms_k, n_k = prof[k]
             if ms_k > 0:
-                tf = mult * 5 * f1 * n_muon / (ms_k / 1e3) / 1e12
+                tf = mult * (poly_steps if k == "ns_poly" else 5) * f1 * n_muon / (ms_k / 1e3) / 1e12
                 phases[k] = {"ms_per_launch": ms_k / max(n_k, 1), "tflops": tf,
                              **({"frac": tf / pk} if bound == "tensor" else {})}
         roof = {"bound": bound, "achieved": achieved, "peak": pk, "unit": "TFLOP/s",
@@ -688,6 +708,7 @@ def run_ours(args):
             "data": "synthetic",
             "config": {"workload": args.set, "params": numel, "matrices": len(mats),
                        "period": None if srank else P, "ns_steps": 5, "ns_precision": args.precision,
+                       **({"ns_table": args.ns_table} if args.ns_table != "quintic" else {}),
                        **({"vector_rule": "adamw"} if args.vector_rule == "adamw" else {}),
                        **({"schedule": "stable_rank", "srank_alpha": args.srank_alpha,
                            "srank_iters": args.srank_iters,
@@ -702,8 +723,8 @@ def run_ours(args):
                                        "steps on every GPU)") if sharded else "one GPU"},
             **({"exchange": {"bytes_received_per_muon_step_rank0": ex.received_bytes(0),
                              "broadcasts_per_muon_step": len(ex.items),
-                             "ns_tflop_per_muon_step_rank0": ns_flops_sym(own_mats) / 1e12,
-                             "ns_tflop_per_muon_step_total": ns_flops_sym(mats) / 1e12}} if sharded else {}),
+                             "ns_tflop_per_muon_step_rank0": ns_flops_sym(own_mats, 5, poly_steps) / 1e12,
+                             "ns_tflop_per_muon_step_total": ns_flops_sym(mats, 5, poly_steps) / 1e12}} if sharded else {}),
             "roofline": srank_roof if srank else roof, "roofline_lion": lion_roof,
             **({"roofline_ns": roof} if srank else {}),
             "kernel_ms_per_step": fam_ms,

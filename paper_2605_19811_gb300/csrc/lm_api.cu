@@ -719,13 +719,18 @@ static lm_status run_ns(const NsEngine& E, int steps, const NsCoeffs* coeffs, un
     for (const NsBatch& b : E.batches)
       for (int ph = 0; ph < 3; ++ph) {
         const NsCoeffs co = coeffs[it];
+        // an iteration without the A^2 term (c = 0, a cubic): B = b A is not
+        // formed; the tensor-core APPLY reads A and scales by b instead
+        const bool from_a = E.xdt == LM_BF16 && co.c == 0.f && !b.wide[NS_POLY] && !b.wide[NS_APPLY];
+        if (ph == NS_POLY && from_a) continue;
         const bool split = E.xdt == LM_BF16 && ph == NS_GRAM && b.nsplit > 0;
         cudaError_t e = timed(P, LM_KERNEL_NS_GRAM + ph, st, [&]() {
           if (E.xdt == LM_BF16) {
             cudaError_t r = launch_ns_tc((NsPhase)ph, it, b.ng, E.groups.data() + b.g0, E.maps.data() + b.g0, b.tiles[ph],
                                b.ntiles[ph], b.offsets[ph], b.npairs[ph], E.d_norm2, co, flags,
                                it == steps - 1 ? fuse : nullptr, st, active, split ? E.d_split_ws : nullptr,
-                               E.pieces, it == steps - 1 ? 1 : 0, b.wide[ph], E.pdl, E.wait_ns);
+                               E.pieces, it == steps - 1 ? 1 : 0, b.wide[ph], E.pdl, E.wait_ns,
+                               ph == NS_APPLY && from_a);
             if (r == cudaSuccess && split)
               r = launch_ns_split_finish(b.split_targets, b.nsplit, E.d_split_ws, flags, st);
             return r;

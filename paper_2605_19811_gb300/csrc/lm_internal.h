@@ -213,14 +213,17 @@ struct FuseFinal {
 constexpr uint64_t kDefaultWaitNs = 5000000000ull;   // 5 s
 uint64_t env_wait_limit_ns();   // LM_WAIT_LIMIT_NS if set to a positive integer, else kDefaultWaitNs
 // offsets: NULL (round robin over tiles) or npairs + 1 range starts;
-// fuse: NULL, or the parameter write of the last APPLY phase.
+// fuse: NULL, or the parameter write of the last APPLY phase;
+// apply_from_a: an APPLY of an iteration whose c is 0, whose POLY launch was
+// left out (B = b A): it reads A and scales its product by b (one-block
+// tiles only).
 cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* groups,
                          const TcGroupMaps* maps, const NsTile* tiles, int ntiles,
                          const int* offsets, int npairs, const double* norm2, NsCoeffs co,
                          unsigned* flags, const FuseFinal* fuse, cudaStream_t st,
                          const unsigned char* active = nullptr, float* split_ws = nullptr, int pieces = 1,
                          int final_f32 = 0, bool wide = false, bool pdl = false,
-                         uint64_t wait_ns = kDefaultWaitNs);
+                         uint64_t wait_ns = kDefaultWaitNs, bool apply_from_a = false);
 // split_ws: non-NULL only for a Gram launch whose tiles include split-K parts.
 // pieces = 3: fp32 operands as three bf16 pieces (no split tiles, no fused
 // parameter write); final_f32: this APPLY writes fp32 X to NsGroup::Xf.

@@ -104,7 +104,7 @@ __device__ __forceinline__ void plan_push(TilePlan& P, int kb_end, bool a_mn, bo
   P.seg[P.nseg++] = OpSeg{kb_end, a_mn, b_mn, ma, mb};
 }
 __device__ __forceinline__ TilePlan tile_plan(int phase, const NsGroup& g, const TcGroupMaps& mp, int cur,
-                                              const NsTile& t) {
+                                              const NsTile& t, bool from_a = false) {
   TilePlan P;
   P.nseg = 0;
   P.kb_start = 0;
@@ -123,12 +123,18 @@ __device__ __forceinline__ TilePlan tile_plan(int phase, const NsGroup& g, const
     plan_push(P, ka, true, true, &mp.amn, &mp.amn);
     plan_push(P, kn, false, true, &mp.a, &mp.amn);
     plan_push(P, P.nk, false, false, &mp.a, &mp.a);
-  } else if (!g.tall) {              // rows tm of B, X MN-major
-    plan_push(P, ka, true, true, &mp.bmn, &mp.xmn[cur]);
-    plan_push(P, P.nk, false, true, &mp.b, &mp.xmn[cur]);
+    return P;
+  }
+  // APPLY: the left operand is B, or A where B = b A was not formed (the
+  // same upper-tile storage)
+  const CUtensorMap* lmn = from_a ? &mp.amn : &mp.bmn;
+  const CUtensorMap* lk = from_a ? &mp.a : &mp.b;
+  if (!g.tall) {                     // rows tm of B, X MN-major
+    plan_push(P, ka, true, true, lmn, &mp.xmn[cur]);
+    plan_push(P, P.nk, false, true, lk, &mp.xmn[cur]);
   } else {                           // rows of X K-major, rows tn of B
-    plan_push(P, kn, false, true, &mp.xk[cur], &mp.bmn);
-    plan_push(P, P.nk, false, false, &mp.xk[cur], &mp.b);
+    plan_push(P, kn, false, true, &mp.xk[cur], lmn);
+    plan_push(P, P.nk, false, false, &mp.xk[cur], lk);
   }
   return P;
 }
@@ -247,10 +253,13 @@ __device__ __forceinline__ void split3(float v, float& h, float& m, float& l) {
 // memory, coalesced through the warp's transpose tile stg: lane l reads and
 // writes 16 bytes of row l / 4 + 8 k (k = 0 .. 3), so a warp access covers 8
 // rows x 64 bytes of one plane.
+//   kacc: APPLY's factor on the accumulator (1, or b where B = b A was not
+//   formed).
 //   aux: the A (POLY) or X (APPLY) element, hi + mid + lo; out: the result's
 //   pieces, or fp32 in out_f32 (last APPLY).  base: element (r0, j0) of the
 //   matrix in plane 0; ld: row length; plane: elements per piece.
 __device__ __forceinline__ void piece_chunk(const uint32_t (&r)[32], int phase, const NsCoeffs& co, float nscale,
+                                            float kacc,
                                             const __nv_bfloat16* aux, __nv_bfloat16* out, float* out_f32,
                                             size_t plane, size_t base, size_t ld, bool row_ok, int j0, int ncols,
                                             float (*stg)[33], int lane) {
@@ -287,7 +296,7 @@ __device__ __forceinline__ void piece_chunk(const uint32_t (&r)[32], int phase, 
     float o;
     if (phase == NS_GRAM) o = acc * nscale;
     else if (phase == NS_POLY) o = co.b * v[e] + co.c * acc;
-    else o = (co.a * v[e] + acc) * nscale;
+    else o = __fmaf_rn(co.a, v[e], kacc * acc) * nscale;   // kacc = 1: exactly a v + acc, one rounding
     stg[lane][e] = (row_ok && j0 + e < ncols) ? o : 0.f;
   }
   __syncwarp();
@@ -419,7 +428,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         const NsTile t = p.tiles[w];
         if (kMasked && !tile_active(p, t)) continue;
         const NsGroup& g = p.groups[t.group];
-        const TilePlan P = tile_plan(phase, g, p.maps[t.group], cur, t);
+        const TilePlan P = tile_plan(phase, g, p.maps[t.group], cur, t, p.apply_from_a != 0);
         const int row_a = t.tm * BM + (int)rank * kHalf;
         const int col_b = t.tn * BN + (int)rank * kHalf;
         int kb0 = P.kb_start;
@@ -454,7 +463,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         const NsTile t = p.tiles[w];
         if (kMasked && !tile_active(p, t)) continue;
         const NsGroup& g = p.groups[t.group];
-        const TilePlan P = tile_plan(phase, g, p.maps[t.group], cur, t);
+        const TilePlan P = tile_plan(phase, g, p.maps[t.group], cur, t, p.apply_from_a != 0);
         if (!mbar_wait(&accempty[ab], aph ^ 1u, abort_flag, wait_ns)) {
           give_up();
           break;
@@ -561,6 +570,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       }
       tc_fence_after();
 
+      // APPLY: X' = a X + B X, or a X + b (A X) where B = b A was not formed
+      const float kacc = p.apply_from_a ? p.co.b : 1.f;
       float nscale = 1.f;
       if (p.iter == 0) {
         const float n = (float)sqrt(p.norm2[g.first_mat + t.mat]) + p.co.eps;
@@ -602,7 +613,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           __nv_bfloat16* out = static_cast<__nv_bfloat16*>(phase == NS_GRAM ? g.A : (phase == NS_POLY ? g.B : g.X[cur ^ 1]));
           float* out_f32 = (phase == NS_APPLY && p.final_f32) ? static_cast<float*>(g.Xf) : nullptr;
           float (*stg)[33] = reinterpret_cast<float (*)[33]>(auxbuf) + (warp - 2) * 32;
-          piece_chunk(r, phase, p.co, nscale, aux, out, out_f32, plane, base, ld, i < nrows, j0, ncols, stg, lane);
+          piece_chunk(r, phase, p.co, nscale, kacc, aux, out, out_f32, plane, base, ld, i < nrows, j0, ncols, stg,
+                      lane);
           continue;
         }
         if (split) {
@@ -644,7 +656,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           float o;
           if (phase == NS_GRAM) o = acc * nscale;
           else if (phase == NS_POLY) o = p.co.b * v[e] + p.co.c * acc;
-          else o = (p.co.a * v[e] + acc) * nscale;
+          else o = __fmaf_rn(p.co.a, v[e], kacc * acc) * nscale;   // the same rounding as ns_wide_kernel
           v[e] = (i < nrows && j < ncols) ? o : 0.f;
         }
 #pragma unroll
@@ -909,8 +921,9 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
                          const int* offsets, int npairs, const double* norm2, NsCoeffs co,
                          unsigned* flags, const FuseFinal* fuse, cudaStream_t st,
                          const unsigned char* active, float* split_ws, int pieces, int final_f32, bool wide,
-                         bool pdl, uint64_t wait_ns) {
+                         bool pdl, uint64_t wait_ns, bool apply_from_a) {
   if (ntiles <= 0) return cudaSuccess;
+  if (apply_from_a && (ph != NS_APPLY || wide)) return cudaErrorInvalidValue;
   if (ngroups < 1 || ngroups > kMaxGroupsTc) return cudaErrorInvalidValue;
   if (pieces != 1 && pieces != 3) return cudaErrorInvalidValue;
   if (pieces == 3 && (fuse != nullptr || wide)) return cudaErrorInvalidValue;
@@ -942,6 +955,7 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
   prm.iter = iter;
   prm.norm2 = norm2;
   prm.co = co;
+  prm.apply_from_a = apply_from_a ? 1 : 0;
   prm.flags = flags;
   if (fuse != nullptr && ph == NS_APPLY) prm.fuse = *fuse;
   prm.active = active;

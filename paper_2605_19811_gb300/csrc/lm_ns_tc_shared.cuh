@@ -32,6 +32,8 @@ struct TcParams {
   float* split_ws;               // fp32 workspace of split Gram tiles (256 x 256 each)
   int final_f32;                 // three-piece operands: this APPLY writes fp32 X to NsGroup::Xf
   uint64_t wait_ns;              // limit of every bounded wait of the roles
+  int apply_from_a;              // APPLY of an iteration with c = 0: B = b A was not formed,
+                                 // the left operand is A and the accumulator is scaled by b
 };
 
 // Launch of the wide-tile kernel (lm_ns_wide.cu); grid = 2 x CTA pairs.

@@ -503,7 +503,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
               float o;
               if (phase == NS_GRAM) o = acc * nscale;
               else if (phase == NS_POLY) o = p.co.b * v[e] + p.co.c * acc;
-              else o = (p.co.a * v[e] + acc) * nscale;
+              else o = __fmaf_rn(p.co.a, v[e], acc) * nscale;   // the same rounding as ns_tc_kernel
               v[e] = (i_row < nrows && j0 + e < ncols) ? o : 0.f;
             }
 #pragma unroll

@@ -106,6 +106,8 @@ def test_msign_repeat_calls_identical():
 
 
 MIXED_TABLE = ((3.0, -3.2, 1.2), (2.0, -1.5, 0.45), (1.875, -1.25, 0.375))
+# cubic (c = 0: no polynomial launch, APPLY reads A) and quintic iterations in turn
+CUBIC_QUINTIC_TABLE = ((1.5, -0.5, 0.0), QUINTIC, (1.5, -0.5, 0.0), QUINTIC, (1.5, -0.5, 0.0))
 
 
 def table_tolerance(x, table, precision):
@@ -133,11 +135,11 @@ def table_tolerance(x, table, precision):
 def _table(name):
     from paper_2605_19811_gb300 import ns_coeffs as C
     return {"polar_express": C.polar_express(5, 1e-3), "chebyshev_cubic": C.chebyshev_cubic(6, 1e-3),
-            "mixed": MIXED_TABLE}[name]
+            "mixed": MIXED_TABLE, "cubic_quintic": CUBIC_QUINTIC_TABLE}[name]
 
 
 @pytest.mark.parametrize("precision", ["bf16", "f32", "f32tc"])
-@pytest.mark.parametrize("name", ["polar_express", "chebyshev_cubic", "mixed"])
+@pytest.mark.parametrize("name", ["polar_express", "chebyshev_cubic", "mixed", "cubic_quintic"])
 @pytest.mark.parametrize("shape", [(256, 768), (768, 256), (300, 130), (64, 64)])
 def test_msign_coefficient_table_parity(precision, name, shape):
     """Iteration-dependent coefficients (lm_msign_ns_coeffs) against the
@@ -167,16 +169,19 @@ def test_msign_coefficient_table_argument_errors():
         L.msign_ns_coeffs(x, out, [(1.0, 0.0, 0.0)] * 65)
 
 
+@pytest.mark.parametrize("coeffs", [QUINTIC, (1.5, -0.5, 0.0)])
 @pytest.mark.parametrize("precision", ["bf16", "f32tc"])
 @pytest.mark.parametrize("shape", [(200, 20000), (20000, 200), (768, 50304)])
-def test_msign_parity_long_k_split_gram(shape, precision):
+def test_msign_parity_long_k_split_gram(shape, precision, coeffs):
     """A matrix whose Gram tiles are far longer than a CTA pair's share of
     the launch: the Gram phase splits them along K into parts that add fp32
     partial sums (split-K; in the three-piece mode the finish kernel writes
-    the sum as three bf16 planes); the result must match the oracle."""
+    the sum as three bf16 planes); the result must match the oracle.  With
+    the cubic (c = 0) no polynomial launch runs and APPLY reads the A the
+    finish kernel wrote."""
     xh = host_tensor(synth.draw_matrix(shape, seed=5 + shape[0]), "bf16" if precision == "bf16" else "f32")
-    got = _msign(xh, precision)
-    want = O.ns_polynomial(stored_values(xh), 5, *QUINTIC, 1e-7)
+    got = _msign(xh, precision, coeffs=coeffs)
+    want = O.ns_polynomial(stored_values(xh), 5, *coeffs, 1e-7)
     assert rel_fro(got, want) <= TOL[precision]
 
 

@@ -334,13 +334,16 @@ def test_fused_parameter_write_matches_finalize_kernel_bit_exact():
         np.testing.assert_array_equal(a, b)
 
 
+@pytest.mark.parametrize("table_name", ["polar_express", "chebyshev_cubic"])
 @pytest.mark.parametrize("precision", [1, 0, F32TC])
-def test_small_gpt_8_steps_polar_express_table(precision):
+def test_small_gpt_8_steps_polar_express_table(precision, table_name):
     """Whole steps with an iteration-dependent NS table (the degree-5 minimax
-    schedule from l_0 = 1e-3): weights after 8 steps against the
+    schedule from l_0 = 1e-3, or the degree-3 one, whose iterations have
+    c = 0 and run without the polynomial launch, the parameter write fused
+    into an APPLY that reads A): weights after 8 steps against the
     storage-modelled oracle run with the same table."""
     from paper_2605_19811_gb300 import ns_coeffs as C
-    table = C.polar_express(5, 1e-3)
+    table = {"polar_express": C.polar_express, "chebyshev_cubic": C.chebyshev_cubic}[table_name](5, 1e-3)
     steps = 8
     shapes = SMALL_GPT.shapes
     W0, grads = make_problem(shapes, "student_t", steps)
