@@ -29,14 +29,14 @@ QUINTIC = (3.4445, -4.7750, 2.0315)
 TOL = {1: 2e-2, 0: 1e-5}   # LM_BF16, LM_F32
 
 
-def _call(entry, x, precision, steps=5):
+def _call(entry, x, precision, steps=5, coeffs=QUINTIC):
     import torch
     from paper_2605_19811_gb300 import lionmuon as L
     lib = L.load_library()
     out = torch.empty(x.shape, dtype=torch.float32, device="cuda")
     di, do = L.tensor_desc(x), L.tensor_desc(out)
     fn = getattr(lib, entry)
-    st = fn(ctypes.byref(di), ctypes.byref(do), steps, *QUINTIC, 1e-7, precision,
+    st = fn(ctypes.byref(di), ctypes.byref(do), steps, *coeffs, 1e-7, precision,
             ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
     assert st == 0, (entry, st, lib.lm_last_error())
     torch.cuda.synchronize()
@@ -61,6 +61,21 @@ def test_noalloc_matches_oracle_and_allocating_entry_point(precision, in_dtype, 
         assert rel_fro(alloc, want) <= TOL[precision]
         assert rel_fro(got, alloc) <= TOL[precision]
         assert L.msign_ns_noalloc_status() == (0, 0)
+
+
+@pytest.mark.parametrize("precision,in_dtype", [(1, "bf16"), (0, "f32")])
+def test_noalloc_cubic_matches_oracle(precision, in_dtype):
+    """The classic cubic (c = 0: the tensor-core path runs no polynomial
+    launch and APPLY reads A) through both entry points, wide and tall."""
+    cubic = (1.5, -0.5, 0.0)
+    for shape, seed in (((384, 1100), 6), ((900, 256), 7)):
+        xh = host_tensor(synth.draw_matrix(shape, seed=seed), in_dtype)
+        x = xh.cuda()
+        got = _call("lm_msign_ns_noalloc", x, precision, 8, cubic)
+        alloc = _call("lm_msign_ns", x, precision, 8, cubic)
+        want = O.ns_polynomial(stored_values(xh), 8, *cubic, 1e-7)
+        assert rel_fro(got, want) <= TOL[precision]
+        assert rel_fro(alloc, want) <= TOL[precision]
 
 
 def test_noalloc_near_scratch_limit():
