@@ -86,6 +86,11 @@ typedef struct {
  *                       for bit, slower on the GPT-style parameter sets
  *   LM_PDL=0            no programmatic dependent launch between the
  *                       Newton-Schulz launches (same results)
+ *   LM_NS_FOLD=0        bf16 Newton-Schulz keeps a X as a separate term of
+ *                       X' = a X + B X; by default an iteration with |a| < 4
+ *                       folds a into the diagonal of the stored B (results
+ *                       within the same tolerance, slightly closer to the
+ *                       fp64 iteration for the constant quintic)
  *   LM_WAIT_LIMIT_NS=n  limit of every bounded device wait in ns (default 5 s;
  *                       also read by lm_msign_ns and lm_msign_ns_noalloc).  A
  *                       wait that runs out raises LM_FLAG_TIMEOUT; every kernel

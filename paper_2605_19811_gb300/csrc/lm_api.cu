@@ -234,6 +234,8 @@ struct Arena {
 //                      (or LM_NS_TILES=narrow) is one-block tiles.  The
 //                      results are the same bit for bit
 //   LM_PDL=0           no programmatic dependent launch between NS launches
+//   LM_NS_FOLD=0       keep a X as a separate term of APPLY instead of folding
+//                      a into B's diagonal
 //   LM_WAIT_LIMIT_NS=n limit of every bounded device wait (default 5 s; a
 //                      short limit makes waits give up, for failure tests)
 static bool env_is(const char* name, const char* value) {
@@ -387,6 +389,7 @@ struct NsEngine {
   double* d_norm2 = nullptr;
   float* d_split_ws = nullptr;       // fp32 partial sums of split Gram tiles
   bool pdl = true;                   // programmatic dependent launch between NS launches
+  bool fold = true;                  // fold a into B's diagonal where |a| < 4 (bf16 operands)
   uint64_t wait_ns = kDefaultWaitNs; // limit of the kernels' bounded waits
 };
 
@@ -723,6 +726,15 @@ static lm_status run_ns(const NsEngine& E, int steps, const NsCoeffs* coeffs, un
         // formed; the tensor-core APPLY reads A and scales by b instead
         const bool from_a = E.xdt == LM_BF16 && co.c == 0.f && !b.wide[NS_POLY] && !b.wide[NS_APPLY];
         if (ph == NS_POLY && from_a) continue;
+        // an iteration whose |a| is below 4: POLY stores B' = a I + B and APPLY
+        // computes X' = B' X with no X tile in its epilogue (bf16 operands,
+        // one-block tiles).  On the constant quintic this also lowers the
+        // error against the fp64 iteration (bf16 msign: 6.2e-3 against 8.3e-3
+        // on 1280 x 5120, 6.5e-3 against 1.0e-2 on 768 x 50304); a larger a
+        // (the first minimax iterations, 8.47) would round the diagonal too
+        // coarsely.
+        const bool fold = E.fold && E.xdt == LM_BF16 && E.pieces == 1 && !from_a && std::fabs(co.a) < 4.f &&
+                          !b.wide[NS_POLY] && !b.wide[NS_APPLY];
         const bool split = E.xdt == LM_BF16 && ph == NS_GRAM && b.nsplit > 0;
         cudaError_t e = timed(P, LM_KERNEL_NS_GRAM + ph, st, [&]() {
           if (E.xdt == LM_BF16) {
@@ -730,7 +742,7 @@ static lm_status run_ns(const NsEngine& E, int steps, const NsCoeffs* coeffs, un
                                b.ntiles[ph], b.offsets[ph], b.npairs[ph], E.d_norm2, co, flags,
                                it == steps - 1 ? fuse : nullptr, st, active, split ? E.d_split_ws : nullptr,
                                E.pieces, it == steps - 1 ? 1 : 0, b.wide[ph], E.pdl, E.wait_ns,
-                               ph == NS_APPLY && from_a);
+                               ph == NS_APPLY && from_a, ph != NS_GRAM && fold);
             if (r == cudaSuccess && split)
               r = launch_ns_split_finish(b.split_targets, b.nsplit, E.d_split_ws, flags, st);
             return r;
@@ -1065,6 +1077,7 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
   NsLayout L;
   layout_ns(s->ns.groups, s->ns.xdt, s->nmat, ar, L, s->ns.batches, s->ns.pieces, env_tiles_mode());
   s->ns.pdl = !env_is("LM_PDL", "0");
+  s->ns.fold = !env_is("LM_NS_FOLD", "0");
   s->ns.wait_ns = env_wait_limit_ns();
   const size_t off_mats = ar.add((size_t)std::max(s->nmat, 1) * sizeof(MatDesc));
   std::vector<MatDesc> mats(s->nmat);
@@ -1787,6 +1800,7 @@ static lm_status msign_impl(const lm_tensor* in, lm_tensor* out, int steps, cons
   NsLayout L;
   layout_ns(E.groups, E.xdt, 1, ar, L, E.batches, E.pieces, env_tiles_mode());
   E.pdl = !env_is("LM_PDL", "0");
+  E.fold = !env_is("LM_NS_FOLD", "0");
   E.wait_ns = env_wait_limit_ns();
   const size_t off_mat = ar.add(sizeof(MatDesc));
   MatDesc d;

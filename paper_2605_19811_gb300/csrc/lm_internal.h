@@ -223,7 +223,7 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
                          unsigned* flags, const FuseFinal* fuse, cudaStream_t st,
                          const unsigned char* active = nullptr, float* split_ws = nullptr, int pieces = 1,
                          int final_f32 = 0, bool wide = false, bool pdl = false,
-                         uint64_t wait_ns = kDefaultWaitNs, bool apply_from_a = false);
+                         uint64_t wait_ns = kDefaultWaitNs, bool apply_from_a = false, bool fold_a = false);
 // split_ws: non-NULL only for a Gram launch whose tiles include split-K parts.
 // pieces = 3: fp32 operands as three bf16 pieces (no split tiles, no fused
 // parameter write); final_f32: this APPLY writes fp32 X to NsGroup::Xf.

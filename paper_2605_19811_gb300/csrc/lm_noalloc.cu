@@ -19,6 +19,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <mutex>
 
@@ -283,15 +284,20 @@ extern "C" lm_status lm_msign_ns_noalloc(const lm_tensor* in, lm_tensor* out, in
   e = launch_momentum_norm(xdt, in->dtype, ba.d_mat, ba.d_chunks, n_et, nullptr, mk, 1, stream);
   if (e != cudaSuccess) return set_error(LM_ERR_CUDA, cudaGetErrorString(e));
   const NsCoeffs co{(float)a, (float)b, (float)c, (float)eps};
-  // c = 0 (a cubic): B = b A is not formed, APPLY reads A and scales by b
+  // c = 0 (a cubic): B = b A is not formed, APPLY reads A and scales by b;
+  // otherwise, where |a| < 4, a is folded into B's diagonal (as lm_msign_ns
+  // does, unless LM_NS_FOLD=0)
   const bool from_a = xdt == LM_BF16 && co.c == 0.f;
+  const char* fold_env = std::getenv("LM_NS_FOLD");
+  const bool fold = xdt == LM_BF16 && !from_a && std::fabs(co.a) < 4.f &&
+                    !(fold_env != nullptr && std::strcmp(fold_env, "0") == 0);
   for (int it = 0; it < steps; ++it)
     for (int ph = 0; ph < 3; ++ph) {
       if (ph == NS_POLY && from_a) continue;
       if (xdt == LM_BF16)
         e = launch_ns_tc((NsPhase)ph, it, 1, &g, &maps, ba.d_tiles[ph], ntiles[ph], nullptr, 0,
                          d.norm2, co, ba.d_flags, nullptr, stream, nullptr, nullptr, 1, 0, false, false,
-                         env_wait_limit_ns(), ph == NS_APPLY && from_a);
+                         env_wait_limit_ns(), ph == NS_APPLY && from_a, ph != NS_GRAM && fold);
       else
         e = launch_ns_simt((NsPhase)ph, it, 1, ba.d_group, ba.d_tiles[ph], ntiles[ph], d.norm2, co,
                            stream, nullptr, nullptr, ba.d_flags);

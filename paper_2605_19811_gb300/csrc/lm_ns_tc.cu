@@ -364,7 +364,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   const int cur = p.iter & 1;
   const uint32_t rank = cluster_rank();          // 0: MMA issuer of the pair
   const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
-  const bool aux_phase = kP == 1 && phase != NS_GRAM;   // epilogue reads the A (POLY) or X (APPLY) tile
+  // epilogue reads the A (POLY) or X (APPLY) tile; an APPLY whose B has a
+  // folded into its diagonal needs no X tile
+  const bool aux_phase = kP == 1 && phase != NS_GRAM && !(phase == NS_APPLY && p.fold_a);
   // this pair's tiles: a host-balanced range, or round robin
   int w_begin = p.offsets ? p.offsets[pair] : pair;
   const int w_end = p.offsets ? p.offsets[pair + 1] : p.ntiles;
@@ -655,8 +657,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           const int j = j0 + e;
           float o;
           if (phase == NS_GRAM) o = acc * nscale;
-          else if (phase == NS_POLY) o = p.co.b * v[e] + p.co.c * acc;
-          else o = __fmaf_rn(p.co.a, v[e], kacc * acc) * nscale;   // the same rounding as ns_wide_kernel
+          else if (phase == NS_POLY) {
+            o = p.co.b * v[e] + p.co.c * acc;
+            if (p.fold_a && i == j) o += p.co.a;   // B' = a I + B
+          } else if (p.fold_a) {
+            o = acc * nscale;                      // X' = B' X
+          } else {
+            o = __fmaf_rn(p.co.a, v[e], kacc * acc) * nscale;   // the same rounding as ns_wide_kernel
+          }
           v[e] = (i < nrows && j < ncols) ? o : 0.f;
         }
 #pragma unroll
@@ -921,9 +929,10 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
                          const int* offsets, int npairs, const double* norm2, NsCoeffs co,
                          unsigned* flags, const FuseFinal* fuse, cudaStream_t st,
                          const unsigned char* active, float* split_ws, int pieces, int final_f32, bool wide,
-                         bool pdl, uint64_t wait_ns, bool apply_from_a) {
+                         bool pdl, uint64_t wait_ns, bool apply_from_a, bool fold_a) {
   if (ntiles <= 0) return cudaSuccess;
   if (apply_from_a && (ph != NS_APPLY || wide)) return cudaErrorInvalidValue;
+  if (fold_a && (ph == NS_GRAM || wide || pieces != 1 || apply_from_a)) return cudaErrorInvalidValue;
   if (ngroups < 1 || ngroups > kMaxGroupsTc) return cudaErrorInvalidValue;
   if (pieces != 1 && pieces != 3) return cudaErrorInvalidValue;
   if (pieces == 3 && (fuse != nullptr || wide)) return cudaErrorInvalidValue;
@@ -956,6 +965,7 @@ cudaError_t launch_ns_tc(NsPhase ph, int iter, int ngroups, const NsGroup* group
   prm.norm2 = norm2;
   prm.co = co;
   prm.apply_from_a = apply_from_a ? 1 : 0;
+  prm.fold_a = fold_a ? 1 : 0;
   prm.flags = flags;
   if (fuse != nullptr && ph == NS_APPLY) prm.fuse = *fuse;
   prm.active = active;

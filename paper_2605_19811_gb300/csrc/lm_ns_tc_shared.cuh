@@ -34,6 +34,7 @@ struct TcParams {
   uint64_t wait_ns;              // limit of every bounded wait of the roles
   int apply_from_a;              // APPLY of an iteration with c = 0: B = b A was not formed,
                                  // the left operand is A and the accumulator is scaled by b
+  int fold_a;                    // POLY adds a to B's diagonal (B' = a I + B); APPLY is X' = B' X
 };
 
 // Launch of the wide-tile kernel (lm_ns_wide.cu); grid = 2 x CTA pairs.

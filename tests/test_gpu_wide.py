@@ -10,7 +10,9 @@ schedule's masked launches and split-K Gram tiles.  The two-block results are
 also checked against the fp64 oracle recurrence (Section 2's iteration) at
 the bf16 tolerance, 2e-2.  LM_NS_TILES chooses the tiles and LM_PDL=0 turns
 programmatic launch off; both are read when a state is created or an msign
-call starts."""
+call starts.  The two-block kernel keeps a X as a separate term of APPLY, so
+these tests run the one-block kernel with LM_NS_FOLD=0 as well (the folded
+form is checked against the oracle elsewhere)."""
 
 import numpy as np
 import pytest
@@ -22,6 +24,11 @@ from tests.lm_testutil import bits, host_tensor, rel_fro, stored_values
 pytestmark = pytest.mark.gpu
 
 QUINTIC = O.NS_QUINTIC
+
+
+@pytest.fixture(autouse=True)
+def _unfolded(monkeypatch):
+    monkeypatch.setenv("LM_NS_FOLD", "0")
 
 
 def _msign_bf16(xh, steps=5, coeffs=QUINTIC):
