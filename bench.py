@@ -234,7 +234,7 @@ class ClockSampler:
 # CPU oracle timing (cpu_baseline leg and --impl reference)
 # ---------------------------------------------------------------------------
 
-def oracle_times(name, period, which=None):
+def oracle_times(name, period, which=None, table=None):
     """Time the oracle: a Lion step on a 4 M-element vector sample, and a full
     fp64 Muon step (momentum, K_NS = 5 NS iterations, parameter update) of one
     matrix of each shape in ``which`` (every distinct matrix shape of the set,
@@ -243,7 +243,7 @@ def oracle_times(name, period, which=None):
     import numpy as np
     import oracle as O
     _, _, mats, _, _ = workload(name)
-    cfg = O.Config(period=period)
+    cfg = O.Config(period=period, ns_coeffs=table)
     rng = np.random.default_rng(0)
     n = 4_000_000
     W = rng.standard_normal(n) * 0.02
@@ -275,10 +275,10 @@ def oracle_estimate(name, period, lion_per_elem, times):
     return 1e3 * ((t_muon + (period - 1) * t_lion) / period if period > 0 else t_lion)
 
 
-def oracle_sample(name, period):
+def oracle_sample(name, period, table=None):
     """(ms_per_step, description) of the oracle on the bounded sample of
     oracle_times over every matrix shape."""
-    lion, times = oracle_times(name, period)
+    lion, times = oracle_times(name, period, table=table)
     _, _, mats, _, _ = workload(name)
     return oracle_estimate(name, period, lion, times), shape_counts(mats, times)
 
@@ -329,14 +329,15 @@ def run_reference(args):
     if rank != 0:
         return 0
     ps, shapes, mats, numel, mat_elems = workload(args.set)
-    lion, times = oracle_times(args.set, args.period)
+    table, _ = ns_table(args.ns_table)
+    lion, times = oracle_times(args.set, args.period, table=table)
     value = oracle_estimate(args.set, args.period, lion, times)
     desc = shape_counts(mats, times)
     order = sorted(times)
     vals = []
     for i in range(args.warmup + args.steps):
         which = [order[i % len(order)]] if order else []
-        lion, t1 = oracle_times(args.set, args.period, which=which)
+        lion, t1 = oracle_times(args.set, args.period, which=which, table=table)
         times.update(t1)
         v = oracle_estimate(args.set, args.period, lion, times)
         if i >= args.warmup:
@@ -693,7 +694,7 @@ def run_ours(args):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
-        v, desc = oracle_sample(args.set, P)
+        v, desc = oracle_sample(args.set, P, table)
         cpu = {"value": v, "unit": "ms/step", "cores": cpu_cores(), "kind": "oracle",
                "sample": ("fp64 oracle on a 4M-element Lion step and a full Muon step of one matrix of "
                           f"every shape, {desc}; each shape's time counted once per matrix of that shape, "

@@ -29,11 +29,11 @@ def _worker(rank, world, port, q):
     dist.init_process_group("gloo", rank=rank, world_size=world)
     got = bench.max_over_ranks(1.5 + rank, world, "cpu")
     # the reference arm runs and prints on rank 0 only
-    bench.oracle_times = lambda name, period, which=None: (0.0, {})
+    bench.oracle_times = lambda name, period, which=None, table=None: (0.0, {})
     bench.oracle_estimate = lambda name, period, lion, times: 42.0
 
     class A:
-        gpus, steps, warmup, set, period = world, 1, 0, "gpt2_124m", 2
+        gpus, steps, warmup, set, period, ns_table = world, 1, 0, "gpt2_124m", 2, "quintic"
     buf = io.StringIO()
     with redirect_stdout(buf):
         rc = bench.run_reference(A)
