@@ -765,20 +765,34 @@ __global__ void __launch_bounds__(256) ns_split_finish_kernel(const NsSplitTarge
   if (lm_stopped(flags)) return;
   const NsSplitTarget T = targets[blockIdx.y];
   __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(T.a_tile);
-  for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < BM * BN; e += gridDim.x * blockDim.x) {
+  // four consecutive elements of a row per thread and trip (the tile's
+  // column extent is a multiple of 128): 16-byte loads of every part, 8-byte
+  // stores per plane; each element's parts are still added in part order
+  for (int e = (blockIdx.x * blockDim.x + threadIdx.x) * 4; e < BM * BN; e += gridDim.x * blockDim.x * 4) {
     const int r = e / BN, c = e % BN;
     if (r >= T.nr || c >= T.nc) continue;
-    float sum = 0.f;
-    for (int k = 0; k < T.nparts; ++k) sum += ws[(size_t)(T.first + k) * (BM * BN) + e];
+    float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
+    const float* part = ws + (size_t)T.first * (BM * BN) + e;
+#pragma unroll 4
+    for (int k = 0; k < T.nparts; ++k) {
+      const float4 v = __ldg(reinterpret_cast<const float4*>(part + (size_t)k * (BM * BN)));
+      sum.x += v.x;
+      sum.y += v.y;
+      sum.z += v.z;
+      sum.w += v.w;
+    }
     const size_t o = (size_t)r * T.ld + c;
     if (T.plane == 0) {
-      dst[o] = __float2bfloat16_rn(sum);
+      *reinterpret_cast<uint2*>(dst + o) = make_uint2(pack_bf2(sum.x, sum.y), pack_bf2(sum.z, sum.w));
     } else {   // three bf16 planes
-      float h, m, l;
-      split3(sum, h, m, l);
-      dst[o] = __float2bfloat16_rn(h);
-      dst[T.plane + o] = __float2bfloat16_rn(m);
-      dst[2 * T.plane + o] = __float2bfloat16_rn(l);
+      float h[4], m[4], l[4];
+      split3(sum.x, h[0], m[0], l[0]);
+      split3(sum.y, h[1], m[1], l[1]);
+      split3(sum.z, h[2], m[2], l[2]);
+      split3(sum.w, h[3], m[3], l[3]);
+      *reinterpret_cast<uint2*>(dst + o) = make_uint2(pack_bf2(h[0], h[1]), pack_bf2(h[2], h[3]));
+      *reinterpret_cast<uint2*>(dst + T.plane + o) = make_uint2(pack_bf2(m[0], m[1]), pack_bf2(m[2], m[3]));
+      *reinterpret_cast<uint2*>(dst + 2 * T.plane + o) = make_uint2(pack_bf2(l[0], l[1]), pack_bf2(l[2], l[3]));
     }
   }
 }
