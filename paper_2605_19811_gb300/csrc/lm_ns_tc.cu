@@ -28,9 +28,14 @@
 //   warp 1    TMEM allocator (both CTAs) + MMA issuer (CTA 0, one lane)
 //   warps 2-9 epilogue: tcgen05.ld from TMEM, fused polynomial combination,
 //             results written into shared memory (over the aux tile) and
-//             stored by TMA, one 64-column box at a time; each TMEM lane
-//             quadrant is served by two warps, one per half of the tile's
-//             columns
+//             stored by TMA, one 64-column box at a time.  Warps 2-5 (one
+//             per TMEM lane quadrant and SM sub-partition) cover the whole
+//             tile; warps 6-9 only work in a launch that also writes the
+//             parameters, where each quadrant takes two warps, one per half
+//             of the tile's columns (the W loads there are latency-bound).
+//             Eight epilogue warps elsewhere measured 4% slower per Muon
+//             step: two of them share each sub-partition's issue slots with
+//             the producer or the MMA issuer.
 //   warp 10   aux loader: TMA of the tile the POLY/APPLY epilogue combines
 //             with the accumulator (A or X), issued while the main loop runs
 // The last APPLY of a Muon step can also apply the parameter update
@@ -367,6 +372,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   // epilogue reads the A (POLY) or X (APPLY) tile; an APPLY whose B has a
   // folded into its diagonal needs no X tile
   const bool aux_phase = kP == 1 && phase != NS_GRAM && !(phase == NS_APPLY && p.fold_a);
+  // Active epilogue warps: one per TMEM lane quadrant (and SM sub-partition)
+  // except where the epilogue also writes the parameters.
+  const int nepi = (kP == 1 && !(phase == NS_APPLY && p.fuse.mats != nullptr)) ? 4 : kEpiWarps;
   // this pair's tiles: a host-balanced range, or round robin
   int w_begin = p.offsets ? p.offsets[pair] : pair;
   const int w_end = p.offsets ? p.offsets[pair + 1] : p.ntiles;
@@ -395,10 +403,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     }
     for (int b = 0; b < kAccBufs; ++b) {
       mbar_init(&accfull[b], 1);
-      mbar_init(&accempty[b], 2 * kEpiWarps);
+      mbar_init(&accempty[b], 2 * nepi);
     }
     mbar_init(aux_full, 1);
-    mbar_init(aux_empty, kEpiWarps);
+    mbar_init(aux_empty, nepi);
     mbar_init(done, 1);
     log->n = 0;
     *abort_flag = 0;
@@ -535,8 +543,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     }
   } else {
     // ------------------------------ epilogue -------------------------------
-    // Thread (quadrant q, lane) owns one row of this CTA's half tile and the
-    // 128 columns [half*128, half*128 + 128) of it, in four 32-column chunks.
+    // Thread (quadrant q, lane) owns one row of this CTA's half tile and
+    // 128 (nepi = 8) or all 256 (nepi = 4) of its columns, in 32-column chunks.
     // Results go into auxbuf (over the aux values, if any) in the 128-byte
     // swizzled box layout and leave by TMA stores, 32 rows x 64 columns each.
     // A warp stores each 64-column box as soon as its two chunks are written
@@ -545,13 +553,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     // starve the operand loads (measured: 2846 -> 1568 cycles per APPLY tile
     // of the MMA issuer waiting for operands; APPLY 2% faster).
     const int q = warp & 3;                   // TMEM lane quadrant of this warp
-    const int half = (warp - 2) >> 2;         // which 128 columns of the tile
+    const int half0 = nepi == 8 ? (warp - 2) >> 2 : 0;   // first 128 columns of the tile it covers
+    const int nhalves = 8 / nepi;
     const int row = q * 32 + lane;            // row of this CTA's half tile
     const uint32_t acc_empty0 = peer_addr(&accempty[0], 0);
     const uint32_t acc_empty1 = peer_addr(&accempty[kAccRing - 1], 0);
     int ab = 0;
     uint32_t aph = 0, xph = 0;
-    for (int w = w_begin; w < w_end; w += w_step) {
+    for (int w = (warp - 2 < nepi) ? w_begin : w_end; w < w_end; w += w_step) {
       const NsTile t = p.tiles[w];
       if (kMasked && !tile_active(p, t)) continue;
       const NsGroup& g = p.groups[t.group];
@@ -589,11 +598,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const int i = r0 + lane;
       const bool warp_in = r0 < row_lim;        // rows past the padded matrix are skipped
       const bool split = kSplit && phase == NS_GRAM && t.slot != 0;
-      if (fused && lane == 0 && q == 0 && half == 0 && rank == 0 && t.tm == 0 && t.tn == 0 &&
+      if (fused && lane == 0 && q == 0 && half0 == 0 && rank == 0 && t.tm == 0 && t.tn == 0 &&
           !isfinite((float)sqrt(p.norm2[g.first_mat + t.mat])))
         atomicOr(p.flags, LM_FLAG_NONFINITE);
-      for (int c4 = 0; c4 < 4; ++c4) {
-        const int ch = half * 4 + c4;
+      for (int c4 = 0; c4 < 4 * nhalves; ++c4) {
+        const int ch = half0 * 4 + c4;
         uint32_t r[32];
         __syncwarp();   // tcgen05.ld is warp-collective: reconverge first
         tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * BN + ch * 32), r);
@@ -651,21 +660,32 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             }
           }
         }
+        // One loop per phase (the branches are uniform), and the padding mask
+        // only on chunks that reach past the true extent: the element loop with
+        // all of them inside measured 2% slower per Muon step (issue slots
+        // shared with the producer and MMA-issuer warps).
+        if (phase == NS_POLY) {
 #pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          const float acc = __uint_as_float(r[e]);
-          const int j = j0 + e;
-          float o;
-          if (phase == NS_GRAM) o = acc * nscale;
-          else if (phase == NS_POLY) {
-            o = p.co.b * v[e] + p.co.c * acc;
-            if (p.fold_a && i == j) o += p.co.a;   // B' = a I + B
-          } else if (p.fold_a) {
-            o = acc * nscale;                      // X' = B' X
-          } else {
-            o = __fmaf_rn(p.co.a, v[e], kacc * acc) * nscale;   // the same rounding as ns_wide_kernel
+          for (int e = 0; e < 32; ++e) v[e] = p.co.b * v[e] + p.co.c * __uint_as_float(r[e]);
+          if (p.fold_a && t.tm == t.tn) {   // B' = a I + B
+#pragma unroll
+            for (int e = 0; e < 32; ++e)
+              if (i == j0 + e) v[e] += p.co.a;
           }
-          v[e] = (i < nrows && j < ncols) ? o : 0.f;
+        } else if (phase == NS_APPLY && !p.fold_a) {
+#pragma unroll
+          for (int e = 0; e < 32; ++e)
+            v[e] = __fmaf_rn(p.co.a, v[e], kacc * __uint_as_float(r[e])) * nscale;   // the same rounding as ns_wide_kernel
+        } else if (nscale != 1.f) {          // GRAM, or X' = B' X
+#pragma unroll
+          for (int e = 0; e < 32; ++e) v[e] = __uint_as_float(r[e]) * nscale;
+        } else {
+#pragma unroll
+          for (int e = 0; e < 32; ++e) v[e] = __uint_as_float(r[e]);
+        }
+        if (i >= nrows || j0 + 32 > ncols) {   // padding outside the true extent stays zero
+#pragma unroll
+          for (int e = 0; e < 32; ++e) v[e] = (i < nrows && j0 + e < ncols) ? v[e] : 0.f;
         }
 #pragma unroll
         for (int u = 0; u < 4; ++u)
@@ -698,39 +718,41 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         // Last APPLY: W <- W - eta_M (s X_K + lambda W), with X_K the bf16
         // values just written to auxbuf.  Half-warp h covers row 2k + h of the
         // warp's 32 rows, 16 lanes x 8 columns = 256 contiguous bytes of W.
-        if (warp_in && write_w) {
-          const int cc = lane & 15;
-          const int jc = t.tn * BN + half * 128 + cc * 8;
-          const unsigned char* box = auxbuf + (2 * half + (cc >> 3)) * kAuxBoxBytes;
-          const int ibase = t.tm * BM + (int)rank * kHalf + q * 32 + (lane >> 4);
-          __nv_bfloat16* wcol = static_cast<__nv_bfloat16*>(fd->w) + jc;
-          for (int k0 = 0; k0 < 16; k0 += kFuseBatch) {
-            uint4 wv[kFuseBatch], xv[kFuseBatch];
+        for (int half = half0; half < half0 + nhalves; ++half) {
+          if (warp_in && write_w) {
+            const int cc = lane & 15;
+            const int jc = t.tn * BN + half * 128 + cc * 8;
+            const unsigned char* box = auxbuf + (2 * half + (cc >> 3)) * kAuxBoxBytes;
+            const int ibase = t.tm * BM + (int)rank * kHalf + q * 32 + (lane >> 4);
+            __nv_bfloat16* wcol = static_cast<__nv_bfloat16*>(fd->w) + jc;
+            for (int k0 = 0; k0 < 16; k0 += kFuseBatch) {
+              uint4 wv[kFuseBatch], xv[kFuseBatch];
 #pragma unroll
-            for (int u = 0; u < kFuseBatch; ++u) {   // all loads of the batch first
-              const int rr = q * 32 + 2 * (k0 + u) + (lane >> 4);
-              const int ii = ibase + 2 * (k0 + u);
-              xv[u] = *reinterpret_cast<const uint4*>(box + rr * 128 + (((cc & 7) ^ (rr & 7)) << 4));
-              wv[u] = (ii < nrows && jc < ncols)
-                          ? *reinterpret_cast<const uint4*>(wcol + (int64_t)ii * fd->cols)
-                          : make_uint4(0u, 0u, 0u, 0u);
-            }
-#pragma unroll
-            for (int u = 0; u < kFuseBatch; ++u) {
-              const int ii = ibase + 2 * (k0 + u);
-              if (ii >= nrows || jc >= ncols) continue;
-              const uint32_t xw[4] = {xv[u].x, xv[u].y, xv[u].z, xv[u].w};
-              uint32_t ww[4] = {wv[u].x, wv[u].y, wv[u].z, wv[u].w};
-#pragma unroll
-              for (int e = 0; e < 4; ++e) {
-                const float w0 = bf_lo(ww[e]), w1 = bf_hi(ww[e]);
-                const float n0 = __fsub_rn(w0, __fmul_rn(p.fuse.eM, __fadd_rn(__fmul_rn(fd->shape_scale, bf_lo(xw[e])),
-                                                                             __fmul_rn(p.fuse.lam, w0))));
-                const float n1 = __fsub_rn(w1, __fmul_rn(p.fuse.eM, __fadd_rn(__fmul_rn(fd->shape_scale, bf_hi(xw[e])),
-                                                                             __fmul_rn(p.fuse.lam, w1))));
-                ww[e] = pack_bf2(n0, n1);
+              for (int u = 0; u < kFuseBatch; ++u) {   // all loads of the batch first
+                const int rr = q * 32 + 2 * (k0 + u) + (lane >> 4);
+                const int ii = ibase + 2 * (k0 + u);
+                xv[u] = *reinterpret_cast<const uint4*>(box + rr * 128 + (((cc & 7) ^ (rr & 7)) << 4));
+                wv[u] = (ii < nrows && jc < ncols)
+                            ? *reinterpret_cast<const uint4*>(wcol + (int64_t)ii * fd->cols)
+                            : make_uint4(0u, 0u, 0u, 0u);
               }
-              *reinterpret_cast<uint4*>(wcol + (int64_t)ii * fd->cols) = make_uint4(ww[0], ww[1], ww[2], ww[3]);
+#pragma unroll
+              for (int u = 0; u < kFuseBatch; ++u) {
+                const int ii = ibase + 2 * (k0 + u);
+                if (ii >= nrows || jc >= ncols) continue;
+                const uint32_t xw[4] = {xv[u].x, xv[u].y, xv[u].z, xv[u].w};
+                uint32_t ww[4] = {wv[u].x, wv[u].y, wv[u].z, wv[u].w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                  const float w0 = bf_lo(ww[e]), w1 = bf_hi(ww[e]);
+                  const float n0 = __fsub_rn(w0, __fmul_rn(p.fuse.eM, __fadd_rn(__fmul_rn(fd->shape_scale, bf_lo(xw[e])),
+                                                                               __fmul_rn(p.fuse.lam, w0))));
+                  const float n1 = __fsub_rn(w1, __fmul_rn(p.fuse.eM, __fadd_rn(__fmul_rn(fd->shape_scale, bf_hi(xw[e])),
+                                                                               __fmul_rn(p.fuse.lam, w1))));
+                  ww[e] = pack_bf2(n0, n1);
+                }
+                *reinterpret_cast<uint4*>(wcol + (int64_t)ii * fd->cols) = make_uint4(ww[0], ww[1], ww[2], ww[3]);
+              }
             }
           }
         }
