@@ -845,6 +845,7 @@ struct lm_state {
   int nmat = 0;
   MatDesc* d_mats = nullptr;
   bool fuse_final = false;   // parameter write in the last APPLY epilogue
+  CUtensorMap* d_wmaps = nullptr;   // TMA maps of every matrix's W (two each) for that write
   ElemChunk* d_echunks[2] = {nullptr, nullptr};   // chunks of bf16 / fp32 matrices
   int n_echunks[2] = {0, 0};
   NsEngine ns;
@@ -1080,6 +1081,9 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
   s->ns.fold = !env_is("LM_NS_FOLD", "0");
   s->ns.wait_ns = env_wait_limit_ns();
   const size_t off_mats = ar.add((size_t)std::max(s->nmat, 1) * sizeof(MatDesc));
+  // TMA maps of W for the parameter write in the last APPLY (bf16 tensor-core path)
+  const bool want_wmaps = s->ns.xdt == LM_BF16 && s->ns.pieces == 1 && s->nmat > 0;
+  const size_t off_wmaps = want_wmaps ? ar.add((size_t)s->nmat * 2 * sizeof(CUtensorMap)) : 0;
   std::vector<MatDesc> mats(s->nmat);
   // matrices are numbered in group order
   std::vector<int> mat_order;   // mat id -> index into mat_param
@@ -1326,6 +1330,13 @@ lm_status lm_create(const lm_tensor* params, int n, const lm_config* cfg, void* 
   s->fuse_final = s->ns.xdt == LM_BF16 && s->ns.pieces == 1 && cfg->ns_steps > 0 && s->nmat > 0;
   for (const MatDesc& d : mats)
     if (d.wdt != LM_BF16 || (d.cols & 7) != 0) s->fuse_final = false;
+  if (s->fuse_final) {
+    CUtensorMap* hm = reinterpret_cast<CUtensorMap*>(img.data() + off_wmaps);
+    for (int id = 0; id < s->nmat && s->fuse_final; ++id)
+      if (tc_encode_w_maps(mats[id].w, mats[id].rows, mats[id].cols, hm + 2 * id) != cudaSuccess)
+        s->fuse_final = false;   // finalize_kernel writes the parameters instead
+    s->d_wmaps = reinterpret_cast<CUtensorMap*>(base + off_wmaps);
+  }
   s->d_echunks[0] = reinterpret_cast<ElemChunk*>(base + off_echunks);
   s->d_echunks[1] = s->d_echunks[0] + s->n_echunks[0];
 
@@ -1562,7 +1573,7 @@ lm_status lm_step(lm_state* s, const lm_tensor* grads, int n, int64_t t, void* c
     if (e != cudaSuccess) return cuda_fail(e, "Lion kernel launch (mixed step)");
   }
   if (s->nmat > 0) {
-    const FuseFinal ff{s->d_mats, mk.eM, mk.lam};
+    const FuseFinal ff{s->d_mats, mk.eM, mk.lam, s->d_wmaps};
     if ((st = run_ns(s->ns, c.ns_steps, s->ns_co.data(), s->d_flags, stream, P, s->fuse_final ? &ff : nullptr,
                      mixed ? s->d_active : nullptr)) != LM_OK)
       return st;

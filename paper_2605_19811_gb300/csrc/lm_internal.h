@@ -206,7 +206,13 @@ cudaError_t launch_bounded_wait_probe(uint64_t limit_ns, unsigned* flags, cudaSt
 struct FuseFinal {
   const MatDesc* mats;
   float eM, lam;
+  // Two TMA maps per matrix (same index as mats), in device memory: W as
+  // 64 x 128 load boxes and 64 x 32 store boxes (tc_encode_w_maps).  Used
+  // where a is folded into B' (the APPLY then has no X tile to read).
+  const CUtensorMap* wmaps;
 };
+// The two W maps of FuseFinal::wmaps for one bf16 parameter (cols % 8 = 0).
+cudaError_t tc_encode_w_maps(void* w, int64_t rows, int64_t cols, CUtensorMap* maps);
 // Limit of a bounded device wait unless the state sets another
 // (LM_WAIT_LIMIT_NS at lm_create): a wait that runs out gives up and raises
 // LM_FLAG_TIMEOUT; every later kernel then does nothing until the flag is cleared.

@@ -40,9 +40,12 @@
 //             with the accumulator (A or X), issued while the main loop runs
 // The last APPLY of a Muon step can also apply the parameter update
 // W <- W - eta_M (s X_K + lambda W) (Algorithm 1, Muon branch) in its
-// epilogue: X_K goes to shared memory as bf16 as usual, then each warp reads
-// its 32 rows of W with coalesced 16-byte loads, updates and writes them, and
-// X_K itself is never stored.
+// epilogue, and X_K itself is never stored.  Where a is folded into B' (the
+// default), the aux loader brings the W tile by TMA, the epilogue updates it
+// in shared memory from the accumulator and stores it back by TMA (W tensor
+// maps per matrix in global memory).  Otherwise the aux tile is X, X_K goes
+// to shared memory as bf16, and each warp then reads its 32 rows of W with
+// coalesced 16-byte loads, updates and writes them.
 // Tiles are assigned to pairs on the host by a longest-first greedy balance
 // of their K lengths (a contiguous range per pair).
 // kAccBufs 256-column accumulators in TMEM (two let the epilogue of one tile
@@ -61,7 +64,7 @@ using namespace tc;    // PTX wrappers (lm_tc_ptx.cuh)
 using namespace tcs;   // constants, stop check and end-of-launch handshake (lm_ns_tc_shared.cuh)
 
 constexpr int kAccBufs = 2;                          // 256-column accumulators in TMEM
-constexpr int kFuseBatch = 4;   // W loads in flight per thread in the fused parameter write
+constexpr int kFuseBatch = 4;   // W loads in flight per thread in the global-memory parameter write
 constexpr int kTmemCols = kAccBufs * BN;
 // Shared-memory layout per operand precision.  kP = 1: bf16 operands, a
 // 5-stage ring of 32 KB per CTA and a 64 KB aux/staging buffer.  kP = 3:
@@ -371,10 +374,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
   // epilogue reads the A (POLY) or X (APPLY) tile; an APPLY whose B has a
   // folded into its diagonal needs no X tile
-  const bool aux_phase = kP == 1 && phase != NS_GRAM && !(phase == NS_APPLY && p.fold_a);
+  // The last APPLY of a Muon step may also write the parameters.  Where a is
+  // folded into B' its aux tile is the W tile, updated in shared memory and
+  // stored back by TMA; otherwise the aux tile is X and W is read from global
+  // memory after the tile (eight epilogue warps for the latency).
+  const bool fused_launch = phase == NS_APPLY && p.fuse.mats != nullptr;
+  const bool fuse_w_tile = kP == 1 && fused_launch && p.fold_a;
+  const bool aux_phase = kP == 1 && phase != NS_GRAM && (!(phase == NS_APPLY && p.fold_a) || fuse_w_tile);
   // Active epilogue warps: one per TMEM lane quadrant (and SM sub-partition)
-  // except where the epilogue also writes the parameters.
-  const int nepi = (kP == 1 && !(phase == NS_APPLY && p.fuse.mats != nullptr)) ? 4 : kEpiWarps;
+  // except in a parameter write that reads W from global memory.
+  const int nepi = (kP == 1 && !(fused_launch && !fuse_w_tile)) ? 4 : kEpiWarps;
   // this pair's tiles: a host-balanced range, or round robin
   int w_begin = p.offsets ? p.offsets[pair] : pair;
   const int w_end = p.offsets ? p.offsets[pair + 1] : p.ntiles;
@@ -512,8 +521,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     }
   } else if (warp == kAuxWarp) {
     // --------------------------- aux tile loader ---------------------------
-    // The epilogue of POLY needs the A tile, that of APPLY the X tile; both
-    // are loaded by TMA into auxbuf while the tile's main loop runs.
+    // The epilogue of POLY needs the A tile, that of APPLY the X tile (or the
+    // W tile of a parameter write); each is loaded by TMA into auxbuf while
+    // the tile's main loop runs.  W boxes past the parameter's extent read
+    // zeros.
     if (lane == 0 && aux_phase) {
       uint32_t xph = 0;
       int armed = -1;
@@ -523,6 +534,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         if (kMasked && !tile_active(p, t)) continue;
         const TcGroupMaps& mp = p.maps[t.group];
         const CUtensorMap* map = (phase == NS_POLY) ? &mp.a : &mp.xk[cur];
+        int zc = t.mat;
+        if (fuse_w_tile) {   // the W load map of this matrix (two maps per matrix: load, store)
+          map = p.fuse.wmaps + 2 * (p.groups[t.group].first_mat + t.mat);
+          zc = 0;
+        }
         if (!mbar_wait(aux_empty, xph ^ 1u, abort_flag, wait_ns)) {
           give_up();
           ok = false;
@@ -533,7 +549,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         const int row0 = t.tm * BM + (int)rank * kHalf;
 #pragma unroll
         for (int b = 0; b < 4; ++b)
-          tma_load_3d_local(auxbuf + b * kAuxBoxBytes, map, aux_full, t.tn * BN + 64 * b, row0, t.mat);
+          tma_load_3d_local(auxbuf + b * kAuxBoxBytes, map, aux_full, t.tn * BN + 64 * b, row0, zc);
         xph ^= 1u;
       }
       if (!ok && armed >= 0) {
@@ -664,7 +680,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         // only on chunks that reach past the true extent: the element loop with
         // all of them inside measured 2% slower per Muon step (issue slots
         // shared with the producer and MMA-issuer warps).
-        if (phase == NS_POLY) {
+        if (fuse_w_tile) {
+          // W <- W - eta_M (s X_K + lambda W) (Algorithm 1, Muon branch) on
+          // the W tile, with X_K = B' X rounded to bf16 as it would have been
+          // stored; entries past W's extent are not stored (TMA clips them)
+          const float ss = fd->shape_scale;
+#pragma unroll
+          for (int e = 0; e < 32; ++e) {
+            const float xk = __bfloat162float(__float2bfloat16_rn(__uint_as_float(r[e]) * nscale));
+            const float wo = v[e];
+            v[e] = __fsub_rn(wo, __fmul_rn(p.fuse.eM, __fadd_rn(__fmul_rn(ss, xk), __fmul_rn(p.fuse.lam, wo))));
+          }
+        } else if (phase == NS_POLY) {
 #pragma unroll
           for (int e = 0; e < 32; ++e) v[e] = p.co.b * v[e] + p.co.c * __uint_as_float(r[e]);
           if (p.fold_a && t.tm == t.tn) {   // B' = a I + B
@@ -683,7 +710,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int e = 0; e < 32; ++e) v[e] = __uint_as_float(r[e]);
         }
-        if (i >= nrows || j0 + 32 > ncols) {   // padding outside the true extent stays zero
+        if (!fuse_w_tile && (i >= nrows || j0 + 32 > ncols)) {   // padding outside the true extent stays zero
 #pragma unroll
           for (int e = 0; e < 32; ++e) v[e] = (i < nrows && j0 + e < ncols) ? v[e] : 0.f;
         }
@@ -692,15 +719,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           abox[(csub + u) ^ (row & 7)] =
               make_uint4(pack_bf2(v[u * 8 + 0], v[u * 8 + 1]), pack_bf2(v[u * 8 + 2], v[u * 8 + 3]),
                          pack_bf2(v[u * 8 + 4], v[u * 8 + 5]), pack_bf2(v[u * 8 + 6], v[u * 8 + 7]));
-        if (kP == 1 && !fused && (c4 & 1)) {
-          // box ch / 2 of this warp's 32 rows is complete: store it now
+        if (kP == 1 && (!fused || fuse_w_tile) && (c4 & 1)) {
+          // box ch / 2 of this warp's 32 rows is complete: store it now (a
+          // parameter write stores W boxes that reach into W, unless a wait
+          // of this step gave up)
           fence_proxy_async_smem();
           __syncwarp();
-          if (lane == 0) {
+          const int b = ch >> 1;
+          const int x0 = t.tn * BN + 64 * b;
+          if (lane == 0 && (!fused || (write_w && x0 < fd->cols && r0 < fd->rows))) {
             const TcGroupMaps& mp = p.maps[t.group];
             const CUtensorMap* dst = (phase == NS_GRAM) ? &mp.ast : (phase == NS_POLY ? &mp.bst : &mp.xst[cur ^ 1]);
-            const int b = ch >> 1;
-            tma_store_3d(dst, auxbuf + b * kAuxBoxBytes + q * 32 * 128, t.tn * BN + 64 * b, r0, t.mat);
+            if (fused) dst = p.fuse.wmaps + 2 * (g.first_mat + t.mat) + 1;
+            tma_store_3d(dst, auxbuf + b * kAuxBoxBytes + q * 32 * 128, x0, r0, fused ? 0 : t.mat);
             bulk_commit();
           }
         }
@@ -714,7 +745,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       }
       fence_proxy_async_smem();
       __syncwarp();
-      if (fused) {
+      if (fused && !fuse_w_tile) {
         // Last APPLY: W <- W - eta_M (s X_K + lambda W), with X_K the bf16
         // values just written to auxbuf.  Half-warp h covers row 2k + h of the
         // warp's 32 rows, 16 lanes x 8 columns = 256 contiguous bytes of W.
@@ -882,6 +913,16 @@ cudaError_t launch_bounded_wait_probe(uint64_t limit_ns, unsigned* flags, cudaSt
   count_launch();
   bounded_wait_probe_kernel<<<1, 32, 0, st>>>(limit_ns, flags);
   return cudaGetLastError();
+}
+
+cudaError_t tc_encode_w_maps(void* w, int64_t rows, int64_t cols, CUtensorMap* maps) {
+  // W (rows x cols bf16, row-major, cols % 8 = 0, 16-byte aligned) as a 3-D
+  // tensor of one matrix: loads of 64 x 128 boxes, stores of 64 x 32 boxes
+  if (rows <= 0 || cols <= 0 || (cols & 7) != 0 || (reinterpret_cast<uintptr_t>(w) & 15) != 0)
+    return cudaErrorInvalidValue;
+  cudaError_t e = encode_3d(&maps[0], w, (uint64_t)cols, (uint64_t)rows, 1, BK, kHalf);
+  if (e == cudaSuccess) e = encode_3d(&maps[1], w, (uint64_t)cols, (uint64_t)rows, 1, 64, 32);
+  return e;
 }
 
 int tc_pad_s(int s) { return (s + kHalf - 1) / kHalf * kHalf; }
