@@ -443,8 +443,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     // ------------------------------ producer ------------------------------
     if (lane == 0) {
       bool ok = true;
+      // the next tile's entry is loaded one tile ahead (its latency then
+      // falls inside the current tile, not between two tiles' MMAs)
+      NsTile tnext = w_begin < w_end ? p.tiles[w_begin] : NsTile{};
       for (int w = w_begin; ok && w < w_end; w += w_step) {
-        const NsTile t = p.tiles[w];
+        const NsTile t = tnext;
+        if (w + w_step < w_end) tnext = p.tiles[w + w_step];
         if (kMasked && !tile_active(p, t)) continue;
         const NsGroup& g = p.groups[t.group];
         const TilePlan P = tile_plan(phase, g, p.maps[t.group], cur, t, p.apply_from_a != 0);
@@ -478,8 +482,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       int ab = 0;
       uint32_t aph = 0;
       bool ok = true;
+      // the next tile's entry is loaded one tile ahead (its latency then
+      // falls inside the current tile, not between two tiles' MMAs)
+      NsTile tnext = w_begin < w_end ? p.tiles[w_begin] : NsTile{};
       for (int w = w_begin; ok && w < w_end; w += w_step) {
-        const NsTile t = p.tiles[w];
+        const NsTile t = tnext;
+        if (w + w_step < w_end) tnext = p.tiles[w + w_step];
         if (kMasked && !tile_active(p, t)) continue;
         const NsGroup& g = p.groups[t.group];
         const TilePlan P = tile_plan(phase, g, p.maps[t.group], cur, t, p.apply_from_a != 0);
