@@ -315,10 +315,14 @@ def test_fused_parameter_write_matches_finalize_kernel_bit_exact():
     last Newton-Schulz epilogue when every matrix is bf16 with a column count
     divisible by 8, and in a separate kernel otherwise; both evaluate the same
     float32 expression on the same bf16 X_K, so the weights agree bit for bit.
-    A 40 x 36 matrix added to the set switches the fusion off."""
+    A 40 x 36 matrix added to the set switches the fusion off.  The fused
+    write loads and stores W in 64-column boxes of 128 (load) or 32 (store)
+    rows: the shapes put box edges past W's last row and column, partly
+    (300 x 136: rows 288-299 of a 32-row box, columns 128-135 of a 64-column
+    box) and wholly (384 x 256, 136 x 520), in both orientations."""
     import torch
     from paper_2605_19811_gb300 import lionmuon as L
-    shapes = [(256, 384), (384, 256), (320, 320), (128,)]
+    shapes = [(256, 384), (384, 256), (320, 320), (300, 136), (136, 520), (128,)]
     W0, grads = make_problem(shapes + [(40, 36)], "student_t", 2)
     out = []
     for n in (len(shapes), len(shapes) + 1):
