@@ -228,13 +228,17 @@ __device__ __forceinline__ bool mma_range(int& stage, uint32_t& ph, uint8_t* sme
     tc_fence_after();
     const uint32_t sa = smem_u32(smem + (size_t)stage * L::kStageBytes);
     const uint32_t sb = same ? sa : sa + kP * kABytes;   // kBBytes == kABytes
+    // descriptors of the stage's K = 0 slices; a 16-deep K step adds its
+    // byte offset / 16 to the start-address field (bits 0-13: no carry, the
+    // shared-memory window is below 2^18 bytes)
+    const uint64_t a0 = AMN ? sw128_desc(sa, 64 * BK * 2, 1024) : sw128_desc(sa, 16, 1024);
+    const uint64_t b0 = BMN ? sw128_desc(sb, 64 * BK * 2, 1024) : sw128_desc(sb, 16, 1024);
 #pragma unroll
     for (int kk = 0; kk < BK / 16; ++kk) {
 #pragma unroll
       for (int m = 0; m < kProducts; ++m) {
-        const uint32_t pa = sa + qa[m] * kABytes, pb = sb + qb[m] * kBBytes;
-        const uint64_t adesc = AMN ? sw128_desc(pa + kk * 2048, 64 * BK * 2, 1024) : sw128_desc(pa + kk * 32, 16, 1024);
-        const uint64_t bdesc = BMN ? sw128_desc(pb + kk * 2048, 64 * BK * 2, 1024) : sw128_desc(pb + kk * 32, 16, 1024);
+        const uint64_t adesc = a0 + (uint64_t)((qa[m] * kABytes + kk * (AMN ? 2048 : 32)) >> 4);
+        const uint64_t bdesc = b0 + (uint64_t)((qb[m] * kBBytes + kk * (BMN ? 2048 : 32)) >> 4);
         const bool first = kb == kb_first && kk == 0 && m <= 1;   // first product into each accumulator
         umma_bf16(m == 0 ? d_tmem : d_cross, adesc, bdesc, idesc, first ? 0u : 1u);
       }
