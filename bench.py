@@ -638,7 +638,6 @@ def run_ours(args):
             pk = sms * 128 * 2 * mhz * 1e6 / 1e12
             bound, kernel = "alu", "ns_simt_kernel"
             peak_kind = f"fp32 FMA, derived: {sms} SMs x 128 lanes x 2 FLOP x {mhz:.0f} MHz"
-        # the recorded ncu traffic is the bf16 workload's
         # the recorded traffic is that of the 720M set's bf16 launches on one GPU
         traffic = kernel_traffic(kernel) if traffic_ok and args.precision == "bf16" else None
         dense = sum(5 * 4.0 * min(m, n) ** 2 * max(m, n) + poly_steps * 2.0 * min(m, n) ** 3
